@@ -1,0 +1,178 @@
+"""Seeded synthetic fork-decode workloads (inputs only, no attention arithmetic).
+
+The workloads stand in for the paper's serving load, which is not available
+here: reasoning traces of GLM-5.1 / DeepSeek-V4-Pro on KernelBench tasks
+(Section 8.1).  Their shape follows the paper's description of speculative
+generation: one long reasoning prefix per trace, K forks per fork event that
+share it (Algorithm 1), fork points between 14% and 70% of the trace
+(Section 4.2), and short private continuations per fork.
+
+This module is shared by the CUDA path's tests/benchmark and by the oracle's
+tests.  It only draws random numbers, rounds them to bf16, lays them out in
+the paged pool and builds block tables; it computes nothing of the method.
+
+Recipe (fixed per workload, seed = the workload's index unless overridden):
+  1. rng = numpy.random.default_rng(seed) (PCG64).
+  2. Integer lengths are drawn uniformly with inclusive bounds, in this order:
+     prefix lengths (per trace), fork counts (per trace), suffix lengths (per fork).
+  3. Logical pages: each trace's prefix needs ceil(P/B) pages, each fork's
+     suffix ceil(S/B) pages, plus ``sentinel_pages`` pages nobody references.
+     Physical ids are a seeded permutation of the pool when ``shuffle``.
+  4. K, V (and Q) values are float32 N(0,1) draws rounded to bf16
+     (round-to-nearest-even).  Slots past a sequence's length inside its last
+     page, and every sentinel page, hold a quiet NaN so that reading them is
+     detectable.
+"""
+
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, asdict
+
+import numpy as np
+
+BF16_QNAN = 0x7FC0
+
+
+@dataclass(frozen=True)
+class WorkloadSpec:
+    name: str
+    num_traces: int
+    prefix_len: tuple[int, int]       # inclusive uniform bounds per trace
+    forks: tuple[int, int]            # inclusive uniform bounds per trace
+    suffix_len: tuple[int, int]       # inclusive uniform bounds per fork
+    hq: int
+    hkv: int
+    dqk: int
+    dv: int
+    page_size: int
+    separate_v: bool = True           # False: V = first dv columns of K (latent KV)
+    shuffle: bool = True
+    seed: int = 0
+    sentinel_pages: int = 2
+
+    @property
+    def scale(self) -> float:
+        return 1.0 / math.sqrt(self.dqk)
+
+
+# The five workloads.  Sizes are the ones the fork-decode benchmark is quoted on.
+WORKLOADS = {
+    "tiny_p512_f4": WorkloadSpec(
+        "tiny_p512_f4", 1, (512, 512), (4, 4), (32, 32), hq=8, hkv=2, dqk=64, dv=64,
+        page_size=16, shuffle=False, seed=0),
+    "fork_p8k_f8": WorkloadSpec(
+        "fork_p8k_f8", 1, (8192, 8192), (8, 8), (64, 512), hq=64, hkv=8, dqk=128, dv=128,
+        page_size=16, seed=1),
+    "long_p32k_f16": WorkloadSpec(
+        "long_p32k_f16", 1, (32768, 32768), (16, 16), (256, 2048), hq=64, hkv=8, dqk=128,
+        dv=128, page_size=16, seed=2),
+    "ragged_t8": WorkloadSpec(
+        "ragged_t8", 8, (4096, 32768), (4, 16), (32, 1024), hq=64, hkv=8, dqk=128, dv=128,
+        page_size=16, seed=3),
+    "mla_p16k_f8": WorkloadSpec(
+        "mla_p16k_f8", 1, (16384, 16384), (8, 8), (128, 1024), hq=128, hkv=1, dqk=576,
+        dv=512, page_size=64, separate_v=False, seed=4),
+}
+WORKLOAD_ORDER = list(WORKLOADS)
+
+
+def round_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """float32 -> bf16 bit patterns, round-to-nearest-even (finite inputs)."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    lsb = (u >> np.uint32(16)) & np.uint32(1)
+    return ((u + np.uint32(0x7FFF) + lsb) >> np.uint32(16)).astype(np.uint16)
+
+
+def bf16_normal(rng: np.random.Generator, shape) -> np.ndarray:
+    return round_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32))
+
+
+def _uniform(rng, lo_hi, n):
+    lo, hi = lo_hi
+    return rng.integers(lo, hi + 1, size=n, dtype=np.int64)
+
+
+def make_workload(spec: WorkloadSpec | str, seed: int | None = None,
+                  fill_unused: str = "nan", **overrides) -> dict:
+    """Build the host-side workload dict (numpy arrays; bf16 as uint16 bits).
+
+    Keys: q, k_pages, v_pages (None for latent KV), prefix_table,
+    prefix_bt_offsets, prefix_lens, fork_offsets, suffix_table,
+    suffix_bt_offsets, suffix_lens, num_traces, total_forks, num_pages,
+    hq, hkv, dqk, dv, page_size, scale, name, sentinel_ids.
+    """
+    if isinstance(spec, str):
+        spec = WORKLOADS[spec]
+    if overrides:
+        spec = WorkloadSpec(**{**asdict(spec), **overrides})
+    rng = np.random.default_rng(spec.seed if seed is None else seed)
+    T, B = spec.num_traces, spec.page_size
+    prefix_lens = _uniform(rng, spec.prefix_len, T)
+    forks = _uniform(rng, spec.forks, T)
+    F = int(forks.sum())
+    suffix_lens = _uniform(rng, spec.suffix_len, F)
+    fork_offsets = np.concatenate([[0], np.cumsum(forks)]).astype(np.int64)
+
+    p_pages = -(-prefix_lens // B)
+    s_pages = -(-suffix_lens // B)
+    n_logical = int(p_pages.sum() + s_pages.sum())
+    num_pages = n_logical + spec.sentinel_pages
+    phys = rng.permutation(num_pages) if spec.shuffle else np.arange(num_pages)
+    phys = phys.astype(np.int32)
+    prefix_bt_offsets = np.concatenate([[0], np.cumsum(p_pages)]).astype(np.int32)
+    suffix_bt_offsets = np.concatenate([[0], np.cumsum(s_pages)]).astype(np.int32)
+    prefix_table = phys[: int(p_pages.sum())].copy()
+    suffix_table = phys[int(p_pages.sum()): n_logical].copy()
+    sentinel_ids = phys[n_logical:].copy()
+
+    k_pages = bf16_normal(rng, (num_pages, spec.hkv, B, spec.dqk))
+    v_pages = bf16_normal(rng, (num_pages, spec.hkv, B, spec.dv)) if spec.separate_v else None
+    q = bf16_normal(rng, (F, spec.hq, spec.dqk))
+
+    if fill_unused == "nan":
+        pools = [k_pages] + ([v_pages] if v_pages is not None else [])
+        for pool in pools:
+            pool[sentinel_ids] = BF16_QNAN
+            for lens, offs, table in ((prefix_lens, prefix_bt_offsets, prefix_table),
+                                      (suffix_lens, suffix_bt_offsets, suffix_table)):
+                for i, n in enumerate(lens):
+                    used = int(n) % B
+                    if used:
+                        last = table[offs[i + 1] - 1]
+                        pool[last, :, used:, :] = BF16_QNAN
+    return dict(
+        name=spec.name, q=q, k_pages=k_pages, v_pages=v_pages,
+        prefix_table=prefix_table, prefix_bt_offsets=prefix_bt_offsets,
+        prefix_lens=prefix_lens.astype(np.int32), fork_offsets=fork_offsets.astype(np.int32),
+        suffix_table=suffix_table, suffix_bt_offsets=suffix_bt_offsets,
+        suffix_lens=suffix_lens.astype(np.int32), num_traces=T, total_forks=F,
+        num_pages=num_pages, hq=spec.hq, hkv=spec.hkv, dqk=spec.dqk, dv=spec.dv,
+        page_size=B, scale=spec.scale, sentinel_ids=sentinel_ids,
+    )
+
+
+def algorithmic_bytes(w: dict) -> dict:
+    """Unique bytes one fork-decode call must move (counting only).
+
+    Prefix KV read once per trace, every suffix KV read once, Q read, O (bf16)
+    and LSE (fp32) written.  A latent KV pool (no separate V) reads each key
+    row once.  The F-fold prefix re-read a naive per-fork decode would make is
+    deliberately not counted.
+    """
+    kv_row = w["hkv"] * 2 * (w["dqk"] + (w["dv"] if w["v_pages"] is not None else 0))
+    prefix = int(np.sum(w["prefix_lens"])) * kv_row
+    suffix = int(np.sum(w["suffix_lens"])) * kv_row
+    q = w["total_forks"] * w["hq"] * w["dqk"] * 2
+    out = w["total_forks"] * w["hq"] * (w["dv"] * 2 + 4)
+    return dict(prefix=prefix, suffix=suffix, q=q, out=out, total=prefix + suffix + q + out)
+
+
+def algorithmic_flops(w: dict) -> dict:
+    """2 flops per multiply-add: QK^T over dqk plus PV over dv, per (row, key)."""
+    g = w["hq"] // w["hkv"]
+    fo = w["fork_offsets"]
+    prefix = sum(int(w["prefix_lens"][t]) * int(fo[t + 1] - fo[t]) for t in range(w["num_traces"]))
+    prefix *= w["hkv"] * g * 2 * (w["dqk"] + w["dv"])
+    suffix = int(np.sum(w["suffix_lens"])) * w["hkv"] * g * 2 * (w["dqk"] + w["dv"])
+    return dict(prefix=prefix, suffix=suffix, total=prefix + suffix)

@@ -1,0 +1,361 @@
+"""Pins for the fp64 oracle against facts fixed by mathematics, not by itself.
+
+Each test would fail under a plausible slip in the oracle (a dropped term, a
+wrong sign, a wrong head or page index, a transposed operand):
+  * closed forms: one key, all-equal scores, the hand-derived two-key case,
+    the empty key set;
+  * invariants: a constant added to every score, key order, page placement;
+  * library cross-checks: scipy.special.logsumexp / softmax on the scores;
+  * brute force: pure-Python loops straight from the pool on tiny workloads;
+  * the merge algebra: split + merge equals the unsplit attention.
+"""
+
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy.special import logsumexp, softmax
+
+import oracle
+from oracle import attention_rows, bf16_bits_to_f64, lse_merge
+from paper_2606_17518_gb300 import workloads as wl
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- bf16 widening
+def test_bf16_widening_known_patterns():
+    bits = np.array([0x3F80, 0xC000, 0x0000, 0x8000, 0x3E00, 0x7F80, 0x0001, 0x4049],
+                    dtype=np.uint16)
+    got = bf16_bits_to_f64(bits)
+    want = [1.0, -2.0, 0.0, -0.0, 0.125, math.inf, 2.0 ** -133, 3.140625]
+    assert got.tolist() == want
+    assert np.signbit(got[3])
+    assert np.isnan(bf16_bits_to_f64(np.array([0x7FC0], dtype=np.uint16)))[0]
+
+
+def test_workload_bf16_rounding_is_rne():
+    import torch
+    x = _rng(3).standard_normal(20000).astype(np.float32)
+    # halfway cases: low 16 bits exactly 0x8000
+    half = (np.arange(1, 200, dtype=np.uint32) << 16 | 0x8000).view(np.float32)
+    x = np.concatenate([x, half, -half])
+    mine = wl.round_to_bf16_bits(x)
+    ref = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(mine, ref)
+
+
+# ---------------------------------------------------------------- paging
+def test_gather_logical_brute_force():
+    rng = _rng(1)
+    pool = rng.integers(0, 2 ** 16, size=(7, 3, 4, 5), dtype=np.uint16)
+    table = np.array([5, 0, 6, 2], dtype=np.int32)
+    for length in (0, 1, 3, 4, 5, 13, 16):
+        for head in range(3):
+            got = oracle.gather_logical(pool, table, length, 4, head)
+            assert got.shape == (length, 5)
+            for j in range(length):
+                page, slot = table[j // 4], j % 4
+                want = bf16_bits_to_f64(pool[page, head, slot])
+                assert np.array_equal(got[j], want, equal_nan=True)
+
+
+# ---------------------------------------------------------------- closed forms
+def test_single_key_returns_its_value_row():
+    rng = _rng(2)
+    q = rng.standard_normal((3, 16))
+    k = rng.standard_normal((1, 16))
+    v = rng.standard_normal((1, 9))
+    o, lse = attention_rows(q, k, v, 0.37)
+    assert np.array_equal(o, np.repeat(v, 3, axis=0))
+    np.testing.assert_allclose(lse, 0.37 * (q @ k[0]), rtol=0, atol=1e-14)
+
+
+def test_zero_query_gives_mean_and_log_n():
+    rng = _rng(4)
+    for n in (1, 2, 7, 100):
+        k = rng.standard_normal((n, 8))
+        v = rng.standard_normal((n, 5))
+        o, lse = attention_rows(np.zeros((2, 8)), k, v, 0.5)
+        np.testing.assert_allclose(o, np.repeat(v.mean(axis=0, keepdims=True), 2, 0),
+                                   rtol=0, atol=1e-14)
+        np.testing.assert_allclose(lse, [math.log(n)] * 2, rtol=0, atol=1e-14)
+
+
+def test_two_key_golden_fixture():
+    vals = {}
+    with open(os.path.join(GOLDEN, "two_key_closed_form.txt")) as fh:
+        for line in fh:
+            if line.strip() and not line.startswith("#"):
+                name, *nums = line.split()
+                vals[name] = np.array([float(x) for x in nums])
+    o, lse = attention_rows(vals["q"][None], np.stack([vals["k0"], vals["k1"]]),
+                            np.stack([vals["v0"], vals["v1"]]), float(vals["scale"][0]))
+    np.testing.assert_allclose(o[0], vals["o"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(lse[0], vals["lse"][0], rtol=0, atol=1e-15)
+
+
+def test_empty_key_set():
+    o, lse = attention_rows(np.ones((2, 4)), np.zeros((0, 4)), np.zeros((0, 3)), 1.0)
+    assert np.array_equal(o, np.zeros((2, 3)))
+    assert np.all(lse == -np.inf)
+
+
+# ---------------------------------------------------------------- invariants
+def test_score_shift_changes_only_lse():
+    rng = _rng(5)
+    q = rng.standard_normal((1, 12))
+    k = rng.standard_normal((30, 12))
+    v = rng.standard_normal((30, 6))
+    scale, c = 0.3, 2.75
+    # moving every key by c/(scale |q|^2) * q adds exactly c to every score
+    k2 = k + (c / (scale * float(q[0] @ q[0]))) * q
+    o1, l1 = attention_rows(q, k, v, scale)
+    o2, l2 = attention_rows(q, k2, v, scale)
+    np.testing.assert_allclose(o2, o1, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(l2, l1 + c, rtol=0, atol=1e-12)
+
+
+def test_key_order_does_not_matter():
+    rng = _rng(6)
+    q = rng.standard_normal((4, 10))
+    k = rng.standard_normal((50, 10))
+    v = rng.standard_normal((50, 7))
+    perm = rng.permutation(50)
+    o1, l1 = attention_rows(q, k, v, 0.4)
+    o2, l2 = attention_rows(q, k[perm], v[perm], 0.4)
+    np.testing.assert_allclose(o2, o1, rtol=0, atol=1e-13)
+    np.testing.assert_allclose(l2, l1, rtol=0, atol=1e-13)
+
+
+def test_large_scores_stay_finite():
+    q = np.array([[1.0, 0.0]])
+    k = np.array([[1000.0, 0.0], [999.0, 0.0]])
+    v = np.array([[1.0], [0.0]])
+    o, lse = attention_rows(q, k, v, 1.0)
+    e = math.exp(-1.0)
+    np.testing.assert_allclose(o[0, 0], 1.0 / (1.0 + e), rtol=1e-15)
+    np.testing.assert_allclose(lse[0], 1000.0 + math.log1p(e), rtol=1e-15)
+    # a spread of 800 nats: exp of an unshifted or min-shifted score overflows fp64
+    k = np.array([[800.0, 0.0], [0.0, 0.0], [-5.0, 0.0]])
+    v = np.array([[2.0], [7.0], [9.0]])
+    o, lse = attention_rows(q, k, v, 1.0)
+    np.testing.assert_allclose(o[0, 0], 2.0, rtol=1e-15)
+    np.testing.assert_allclose(lse[0], 800.0, rtol=1e-15)
+
+
+def test_against_scipy_softmax_and_logsumexp():
+    rng = _rng(7)
+    q = rng.standard_normal((5, 24))
+    k = rng.standard_normal((77, 24))
+    v = rng.standard_normal((77, 11))
+    o, lse = attention_rows(q, k, v, 0.2)
+    s = 0.2 * np.einsum("rd,nd->rn", q, k)
+    np.testing.assert_allclose(lse, logsumexp(s, axis=1), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(o, softmax(s, axis=1) @ v, rtol=0, atol=1e-12)
+
+
+# ---------------------------------------------------------------- merge algebra
+def test_split_merge_equals_unsplit():
+    rng = _rng(8)
+    q = rng.standard_normal((6, 16))
+    k = rng.standard_normal((40, 16)) * 2
+    v = rng.standard_normal((40, 9))
+    o, lse = attention_rows(q, k, v, 0.25)
+    for cut in (0, 1, 17, 39, 40):
+        oa, la = attention_rows(q, k[:cut], v[:cut], 0.25)
+        ob, lb = attention_rows(q, k[cut:], v[cut:], 0.25)
+        om, lm = lse_merge(oa, la, ob, lb)
+        np.testing.assert_allclose(om, o, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lm, lse, rtol=0, atol=1e-12)
+    # merging is order independent
+    oa, la = attention_rows(q, k[:13], v[:13], 0.25)
+    ob, lb = attention_rows(q, k[13:], v[13:], 0.25)
+    o1, l1 = lse_merge(oa, la, ob, lb)
+    o2, l2 = lse_merge(ob, lb, oa, la)
+    np.testing.assert_allclose(o1, o2, rtol=0, atol=1e-14)
+    np.testing.assert_allclose(l1, l2, rtol=0, atol=1e-14)
+
+
+def test_merge_with_empty_part_is_identity():
+    rng = _rng(9)
+    o = rng.standard_normal((3, 4))
+    lse = rng.standard_normal(3)
+    empty_o = np.full((3, 4), 123.0)     # must be ignored, whatever it holds
+    empty_l = np.full(3, -np.inf)
+    for args in ((o, lse, empty_o, empty_l), (empty_o, empty_l, o, lse)):
+        om, lm = lse_merge(*args)
+        np.testing.assert_allclose(om, o, rtol=0, atol=1e-15)
+        np.testing.assert_allclose(lm, lse, rtol=0, atol=1e-15)
+    om, lm = lse_merge(empty_o, empty_l, empty_o, empty_l)
+    assert np.array_equal(om, np.zeros((3, 4))) and np.all(lm == -np.inf)
+
+
+def test_merge_weights_by_normaliser():
+    # parts with equal LSE average their outputs; a part 1 nat larger weighs e times more
+    oa, ob = np.array([[1.0, 0.0]]), np.array([[0.0, 1.0]])
+    om, lm = lse_merge(oa, np.array([0.5]), ob, np.array([1.5]))
+    e = math.e
+    np.testing.assert_allclose(om[0], [1 / (1 + e), e / (1 + e)], rtol=1e-15)
+    np.testing.assert_allclose(lm[0], 1.5 + math.log1p(1 / e), rtol=1e-15)
+
+
+# ---------------------------------------------------------------- whole workloads
+def _tiny(**kw):
+    base = dict(name="t", num_traces=2, prefix_len=(5, 37), forks=(1, 3), suffix_len=(0, 9),
+                hq=6, hkv=2, dqk=8, dv=4, page_size=4)
+    base.update(kw)
+    return wl.WorkloadSpec(**base)
+
+
+def _brute(w):
+    """Pure-Python loops from the pool, straight from the definition."""
+    nf, hq, g_size = w["total_forks"], w["hq"], w["hq"] // w["hkv"]
+    B, dv = w["page_size"], w["dv"]
+    o = np.zeros((nf, hq, dv))
+    lse = np.zeros((nf, hq))
+
+    def val(pool, page, g, slot, d):
+        bits = int(pool[page, g, slot, d])
+        return float(np.array([bits << 16], dtype=np.uint32).view(np.float32)[0])
+
+    for t in range(w["num_traces"]):
+        for f in range(w["fork_offsets"][t], w["fork_offsets"][t + 1]):
+            toks = []
+            pt = w["prefix_table"][w["prefix_bt_offsets"][t]:]
+            for j in range(w["prefix_lens"][t]):
+                toks.append((pt[j // B], j % B))
+            st = w["suffix_table"][w["suffix_bt_offsets"][f]:]
+            for j in range(w["suffix_lens"][f]):
+                toks.append((st[j // B], j % B))
+            for h in range(hq):
+                g = h // g_size
+                qrow = [float(np.array([int(x) << 16], dtype=np.uint32).view(np.float32)[0])
+                        for x in w["q"][f, h]]
+                if not toks:
+                    lse[f, h] = -math.inf
+                    continue
+                s = [w["scale"] * math.fsum(qrow[d] * val(w["k_pages"], p, g, sl, d)
+                                            for d in range(w["dqk"])) for p, sl in toks]
+                z = math.fsum(math.exp(x) for x in s)
+                lse[f, h] = math.log(z)
+                vp = w["v_pages"]
+                for d in range(dv):
+                    o[f, h, d] = math.fsum(
+                        math.exp(x - lse[f, h]) * (val(vp, p, g, sl, d) if vp is not None
+                                                   else val(w["k_pages"], p, g, sl, d))
+                        for x, (p, sl) in zip(s, toks))
+    return o, lse
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_fork_decode_brute_force(seed):
+    w = wl.make_workload(_tiny(), seed=seed)
+    o, lse = oracle.fork_attn_decode(w)
+    ob, lb = _brute(w)
+    np.testing.assert_allclose(lse, lb, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(o, ob, rtol=0, atol=1e-12)
+    assert np.all(np.isfinite(o))
+
+
+def test_fork_decode_brute_force_latent_kv():
+    w = wl.make_workload(_tiny(hq=4, hkv=1, dqk=10, dv=6, separate_v=False), seed=5)
+    assert w["v_pages"] is None
+    o, lse = oracle.fork_attn_decode(w)
+    ob, lb = _brute(w)
+    np.testing.assert_allclose(lse, lb, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(o, ob, rtol=0, atol=1e-12)
+
+
+def test_latent_kv_equals_explicit_value_pool():
+    w = wl.make_workload(_tiny(hq=4, hkv=1, dqk=10, dv=6, separate_v=False), seed=6)
+    w2 = dict(w)
+    w2["v_pages"] = np.ascontiguousarray(w["k_pages"][..., :6])
+    o1, l1 = oracle.fork_attn_decode(w)
+    o2, l2 = oracle.fork_attn_decode(w2)
+    assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
+
+
+@pytest.mark.parametrize("name", ["tiny_p512_f4"])
+def test_split_merge_equals_monolithic_workload(name):
+    w = wl.make_workload(name)
+    o, lse = oracle.fork_attn_decode(w)
+    o2, l2 = oracle.fork_attn_split_merge(w)
+    np.testing.assert_allclose(o2, o, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(l2, lse, rtol=0, atol=1e-12)
+
+
+def test_split_merge_with_empty_suffixes_and_prefixes():
+    w = wl.make_workload(_tiny(prefix_len=(0, 9), suffix_len=(0, 3)), seed=11)
+    assert (w["suffix_lens"] == 0).any() or (w["prefix_lens"] == 0).any()
+    o, lse = oracle.fork_attn_decode(w)
+    o2, l2 = oracle.fork_attn_split_merge(w)
+    np.testing.assert_allclose(o2, o, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(l2, lse, rtol=0, atol=1e-12)
+
+
+def test_page_placement_is_bit_invariant():
+    w = wl.make_workload(_tiny(), seed=3)
+    o1, l1 = oracle.fork_attn_decode(w)
+    perm = _rng(12).permutation(w["num_pages"]).astype(np.int32)
+    w2 = dict(w)
+    for key in ("k_pages", "v_pages"):
+        pool2 = np.empty_like(w[key])
+        pool2[perm] = w[key]                 # physical page p moves to perm[p]
+        w2[key] = pool2
+    w2["prefix_table"] = perm[w["prefix_table"]]
+    w2["suffix_table"] = perm[w["suffix_table"]]
+    o2, l2 = oracle.fork_attn_decode(w2)
+    assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
+
+
+def test_gqa_head_map_contiguous_groups():
+    """Query head h reads kv head h // G: changing kv head 1 changes exactly heads G..2G-1."""
+    w = wl.make_workload(_tiny(hq=6, hkv=3), seed=4)
+    o1, _ = oracle.fork_attn_decode(w)
+    w2 = dict(w)
+    w2["k_pages"] = w["k_pages"].copy()
+    w2["k_pages"][:, 1] = wl.bf16_normal(_rng(99), w["k_pages"][:, 1].shape)
+    o2, _ = oracle.fork_attn_decode(w2)
+    changed = np.any(o1 != o2, axis=(0, 2))
+    assert changed.tolist() == [False, False, True, True, False, False]
+
+
+def test_mha_special_case_matches_per_head_attention():
+    """G = 1 is ordinary multi-head decode: head h over kv head h alone."""
+    w = wl.make_workload(_tiny(hq=3, hkv=3), seed=8)
+    o, lse = oracle.fork_attn_decode(w)
+    f = w["total_forks"] - 1
+    t = int(np.searchsorted(w["fork_offsets"], f, side="right") - 1)
+    pt = w["prefix_table"][w["prefix_bt_offsets"][t]:w["prefix_bt_offsets"][t + 1]]
+    st = w["suffix_table"][w["suffix_bt_offsets"][f]:w["suffix_bt_offsets"][f + 1]]
+    for h in range(3):
+        k = np.concatenate([oracle.gather_logical(w["k_pages"], pt, w["prefix_lens"][t], 4, h),
+                            oracle.gather_logical(w["k_pages"], st, w["suffix_lens"][f], 4, h)])
+        v = np.concatenate([oracle.gather_logical(w["v_pages"], pt, w["prefix_lens"][t], 4, h),
+                            oracle.gather_logical(w["v_pages"], st, w["suffix_lens"][f], 4, h)])
+        s = w["scale"] * (k @ bf16_bits_to_f64(w["q"][f, h]))
+        np.testing.assert_allclose(lse[f, h], logsumexp(s), rtol=0, atol=1e-12)
+        np.testing.assert_allclose(o[f, h], softmax(s) @ v, rtol=0, atol=1e-12)
+
+
+def test_unused_slots_and_sentinels_are_never_read():
+    w = wl.make_workload(_tiny(), seed=7)
+    assert np.isnan(bf16_bits_to_f64(w["k_pages"][w["sentinel_ids"]])).all()
+    o, lse = oracle.fork_attn_decode(w)
+    assert np.all(np.isfinite(o)) and np.all(np.isfinite(lse))
+
+
+def test_rows_entry_matches_full():
+    w = wl.make_workload(_tiny(), seed=2)
+    o, lse = oracle.fork_attn_decode(w)
+    rows = [(w["total_forks"] - 1, 5), (0, 0), (0, 3)]
+    ro, rl = oracle.fork_attn_decode_rows(w, rows)
+    for i, (f, h) in enumerate(rows):
+        np.testing.assert_allclose(ro[i], o[f, h], rtol=0, atol=1e-14)
+        np.testing.assert_allclose(rl[i], lse[f, h], rtol=0, atol=1e-14)
