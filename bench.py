@@ -1,0 +1,441 @@
+#!/usr/bin/env python
+"""Fork-decode attention benchmark (one JSON line on rank 0).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+A step is one complete fork-decode call (prefix stage + suffix stage + merge)
+for every fork of the workload: one decode token per fork, one attention layer.
+Metric: tokens/s = forks per step / seconds per step.  The default workload is
+the reasoning-trace fork: one 8192-token shared prefix, 8 forks with suffixes
+in [64, 512], Hq=64, Hkv=8, head dim 128, page 16, shuffled pages.
+
+Timing: W untimed warm-up steps, then K steps between CUDA events on the
+launching stream, bracketed by a barrier and a device synchronise.  Inputs
+rotate over enough resident replicas that every step's KV is evicted from L2
+before it is read again (the union of replicas is >= 3x L2).  The dominant
+kernel's time comes from events the library records between its launches
+(specgen_fork_attn_run_profiled) during the same timed steps.
+
+With N > 1 (torchrun) every rank runs its own replica of the workload: fork
+decode shards by independent traces with no exchange, so scaling is weak and
+no collective is used.  ``--impl reference`` times the fp64 CPU oracle instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+DEFAULT_WORKLOAD = "fork_p8k_f8"
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
+    return ap.parse_args()
+
+
+ARGS = parse_args()
+if ARGS.impl == "reference" or os.environ.get("SPECGEN_ORACLE_CHILD"):
+    # the oracle runs single-threaded so that `cores` is exact
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[var] = "1"
+
+sys.path.insert(0, ROOT)
+import numpy as np  # noqa: E402
+
+METRIC = "fork-decode attention tokens/s"
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), \
+            "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines: list[str] = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def _query_once(self):
+        try:
+            out = subprocess.run(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                  "--format=csv,noheader,nounits"], capture_output=True,
+                                 text=True, timeout=20).stdout
+            return [l for l in out.splitlines() if l.strip()]
+        except Exception:
+            return []
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=10)
+            except Exception:
+                self.proc.kill()
+                out = ""
+            self.lines = [l for l in (out or "").splitlines() if l.strip()]
+        extra = self._query_once()
+        samples = self.lines or extra
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in samples:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- CPU oracle
+def oracle_sample(workload: str, seconds: float):
+    """Time the fp64 oracle (as it stands) on whole forks until ~`seconds` pass."""
+    import oracle
+    from paper_2606_17518_gb300 import workloads as wl
+    w = wl.make_workload(workload)
+    forks = 0
+    t0 = time.perf_counter()
+    while True:
+        f = forks % w["total_forks"]
+        oracle.fork_attn_decode_rows(w, [(f, h) for h in range(w["hq"])])
+        forks += 1
+        if time.perf_counter() - t0 >= seconds or forks >= 10000:
+            break
+    dt = time.perf_counter() - t0
+    return forks, dt
+
+
+def cpu_baseline(workload: str, seconds: float):
+    env = dict(os.environ, SPECGEN_ORACLE_CHILD="1", OMP_NUM_THREADS="1",
+               OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = ("import json,sys; sys.argv=['bench.py','--impl','reference']; import bench; "
+            f"f,dt=bench.oracle_sample({workload!r},{seconds}); print(json.dumps([f,dt]))")
+    res = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
+                         text=True, timeout=600)
+    forks, dt = json.loads(res.stdout.strip().splitlines()[-1])
+    return {"value": forks / dt, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"{forks} whole forks (all heads) of {workload}, fp64 numpy, "
+                      f"{dt:.1f} s on 1 host thread"}
+
+
+# --------------------------------------------------------------------------- reference arm
+def run_reference():
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    from paper_2606_17518_gb300 import workloads as wl
+    w = wl.make_workload(ARGS.workload)
+    F, hq = w["total_forks"], w["hq"]
+
+    def step(i):
+        oracle.fork_attn_decode_rows(w, [(i % F, h) for h in range(hq)])
+
+    for i in range(ARGS.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(ARGS.steps):
+        step(i)
+    dt = time.perf_counter() - t0
+    value = ARGS.steps / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": ARGS.gpus, "steps": ARGS.steps, "warmup": ARGS.warmup,
+        "ms_per_step": dt / ARGS.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": ARGS.workload, "step": "one whole fork (all query heads) "
+                   "of the workload per step, cycling forks"},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{ARGS.steps} forks of {ARGS.workload}, fp64 numpy, "
+                                   "1 host thread"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- GPU arm
+def kernel_source_sha(name: str) -> str:
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2606_17518_gb300", "csrc")
+    for fn in sorted(os.listdir(csrc)):
+        if fn.startswith(name) or fn in ("common.cuh", "plan.h"):
+            with open(os.path.join(csrc, fn), "rb") as fh:
+                h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if still current."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+        rec = d[kernel][workload]
+        if rec.get("source_sha") != kernel_source_sha(kernel):
+            return None
+        return float(rec["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+def run_ours():
+    import ctypes as C
+
+    import torch
+
+    import __graft_entry__
+    from paper_2606_17518_gb300 import _lib, workloads as wl
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+
+    rank, local_rank, world = dist_env()
+    __graft_entry__.build()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    w = wl.make_workload(ARGS.workload)
+    nbytes = wl.algorithmic_bytes(w)
+    flops = wl.algorithmic_flops(w)
+    F = w["total_forks"]
+    props = torch.cuda.get_device_properties(dev)
+    l2 = int(getattr(props, "L2_cache_size", 126 * 2 ** 20))
+    replicas = max(1, math.ceil(3 * l2 / nbytes["total"]))
+    log(f"[bench] {ARGS.workload}: {nbytes['total'] / 1e6:.1f} MB unique, L2 {l2 / 2**20:.0f} MiB,"
+        f" {replicas} replicas")
+    stream = torch.cuda.Stream(dev)
+    sp = stream.cuda_stream
+    reps = [ForkDecode(w, device=dev) for _ in range(replicas)]
+    with torch.cuda.stream(stream):
+        for r in reps:
+            r.plan(sp)
+    torch.cuda.synchronize(dev)
+    args = [r.args() for r in reps]
+    plans = [r.plan_info for r in reps]
+
+    # event ring: one set of marks per timed step
+    n_marks = 4
+    K, W = ARGS.steps, ARGS.warmup
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(K * n_marks)]
+    with torch.cuda.stream(stream):
+        for e in evs:
+            e.record(stream)  # create the events outside the timed region
+    torch.cuda.synchronize(dev)
+    handles = (C.c_void_p * len(evs))(*[e.cuda_event for e in evs])
+    lib = _lib.load()
+    n_l = C.c_int(0)
+    run_prof = lib.specgen_fork_attn_run_profiled
+    run = lib.specgen_fork_attn_run
+    arg_refs = [C.byref(a) for a in args]
+    plan_refs = [C.byref(p) for p in plans]
+    sp_c = C.c_void_p(sp)
+
+    for i in range(W):
+        st = run(arg_refs[i % replicas], plan_refs[i % replicas], sp_c)
+        assert st == 0, _lib.status_string(st)
+    torch.cuda.synchronize(dev)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local_rank)
+    barrier()
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    start.record(stream)
+    for i in range(K):
+        st = run_prof(arg_refs[i % replicas], plan_refs[i % replicas], sp_c,
+                      C.byref(handles, i * n_marks * C.sizeof(C.c_void_p)), n_marks,
+                      C.byref(n_l))
+        if st != 0:
+            raise RuntimeError(_lib.status_string(st))
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier()
+    clk = clocks.stop()
+    launches = n_l.value
+    total_ms = start.elapsed_time(end)
+    per_kernel = [0.0] * launches
+    for i in range(K):
+        for k in range(launches):
+            per_kernel[k] += evs[i * n_marks + k].elapsed_time(evs[i * n_marks + k + 1])
+    status = reps[0].status(sp)
+    if status != 0:
+        raise RuntimeError(f"workspace status {_lib.status_string(status)}")
+
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / K
+    value = world * F / (ms_per_step * 1e-3)
+
+    # ---- end to end through the public API: host buffers, copies in the timed region
+    e2e = measure_e2e(w, reps, stream, dev, K=min(K, 500), W=min(W, 5))
+
+    kernel_names = ["split_decode", "lse_merge"][:launches]
+    kernel_ms = [t / K for t in per_kernel]
+    dom = int(np.argmax(kernel_ms)) if kernel_ms else 0
+    hbm, tf_burst, tf_sus, peak_src = measured_peaks()
+    dom_bytes = nbytes["prefix"] + nbytes["suffix"] + nbytes["q"]
+    achieved = dom_bytes / (kernel_ms[dom] * 1e-3) / 1e9 if kernel_ms else None
+    traffic = recorded_traffic(kernel_names[dom], ARGS.workload)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {
+            "workload": ARGS.workload, "traces": w["num_traces"], "forks": F,
+            "prefix_tokens": int(np.sum(w["prefix_lens"])),
+            "suffix_tokens": int(np.sum(w["suffix_lens"])), "hq": w["hq"], "hkv": w["hkv"],
+            "head_dim": [w["dqk"], w["dv"]], "page_size": w["page_size"],
+            "unique_bytes": nbytes["total"], "flops": flops["total"],
+            "l2": f"inputs rotate over {replicas} resident replicas (>= 3x L2)",
+            "parallelism": f"replicas x{world}",
+        },
+        "gpu_launches": K * launches,
+        "kernels": {n: {"ms_per_launch": t, "share": t / max(1e-12, sum(kernel_ms))}
+                    for n, t in zip(kernel_names, kernel_ms)},
+        "achieved_gbs_whole_step": nbytes["total"] / (ms_per_step * 1e-3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": kernel_names[dom] if kernel_names else None,
+                     "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm if achieved else None, "traffic": traffic,
+                     "peak_source": peak_src,
+                     "algorithmic_bytes_per_launch": dom_bytes},
+        "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not ARGS.no_cpu_baseline:
+        try:
+            line["cpu_baseline"] = cpu_baseline(ARGS.workload, ARGS.cpu_sample_seconds)
+        except Exception as exc:  # reported, never silently dropped
+            line["cpu_baseline"] = {"error": repr(exc)[:200]}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def measure_e2e(w, reps, stream, dev, K, W):
+    """tokens/s through specgen_fork_attn_decode with host-resident per-step inputs.
+
+    Every step copies that step's queries and block tables from pinned host
+    memory, plans (host) and runs the call, and reads O and LSE back into
+    pinned host memory.  The KV pools are the serving cache and stay resident.
+    """
+    import torch
+
+    from paper_2606_17518_gb300 import _lib
+    replicas = len(reps)
+    pin = lambda t: t.detach().cpu().pin_memory()
+    host_in = [(pin(r.q), pin(r.prefix_table), pin(r.prefix_off), pin(r.suffix_table),
+                pin(r.suffix_off)) for r in reps]
+    host_out = [(torch.empty(r.out.shape, dtype=r.out.dtype).pin_memory(),
+                 torch.empty(r.lse.shape, dtype=r.lse.dtype).pin_memory()) for r in reps]
+    sp = stream.cuda_stream
+    bi = sum(t.numel() * t.element_size() for t in host_in[0])
+    bi += int(reps[0].plan_info.plan_bytes)
+    bo = sum(t.numel() * t.element_size() for t in host_out[0])
+
+    def step(i):
+        r, (hq_, hpt, hpo, hst, hso), (ho, hl) = reps[i % replicas], host_in[i % replicas], \
+            host_out[i % replicas]
+        with torch.cuda.stream(stream):
+            r.q.copy_(hq_, non_blocking=True)
+            r.prefix_table.copy_(hpt, non_blocking=True)
+            r.prefix_off.copy_(hpo, non_blocking=True)
+            r.suffix_table.copy_(hst, non_blocking=True)
+            r.suffix_off.copy_(hso, non_blocking=True)
+            r.decode(sp)
+            ho.copy_(r.out, non_blocking=True)
+            hl.copy_(r.lse, non_blocking=True)
+
+    for i in range(W):
+        step(i)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for i in range(K):
+        step(i)
+    torch.cuda.synchronize(dev)
+    dt = time.perf_counter() - t0
+    for r in reps:  # the per-step plan left every replica planned and consistent
+        r.plan_info = None
+        r.plan(sp)
+    torch.cuda.synchronize(dev)
+    return {"value": w["total_forks"] * K / dt, "unit": "tokens/s", "h2d_bytes_per_step": bi,
+            "d2h_bytes_per_step": bo, "steps": K}
+
+
+def main():
+    if os.environ.get("SPECGEN_ORACLE_CHILD"):
+        return
+    if ARGS.impl == "reference":
+        run_reference()
+    else:
+        run_ours()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,169 @@
+/*
+ * specgen.h -- C ABI of the GB300 fork-decode attention library.
+ *
+ * The operation.  SpecGen forks K non-reasoning generations off a running
+ * reasoning generation; every fork's prompt is the iteration prompt followed by
+ * the reasoning prefix pi (Algorithm 1, "Fork K spec. generations"; Section
+ * 6.1.1), so the forks share that prefix's KV cache (Section 4.2; Section 8.6,
+ * prefix-cache reuse).  Decoding one token for every fork means: for fork f of
+ * trace t and query head h (kv head g = h / (hq / hkv)),
+ *
+ *     keys/values = prefix tokens 0..P_t-1 of trace t, then suffix tokens
+ *                   0..S_f-1 of fork f (logical order)
+ *     s_i  = scale * <q[f,h,:], k_i[g,:]>
+ *     O    = sum_i softmax(s)_i v_i[g,:]        LSE = ln sum_i exp(s_i)
+ *
+ * The library splits this into a prefix stage (all forks of a trace read the
+ * shared prefix pages once), a per-fork suffix stage, and a log-sum-exp merge of
+ * the partial results; the answer is the plain definition above up to fp32
+ * rounding.
+ *
+ * Paged KV layout (caller-owned device memory, never freed by the library):
+ *     k_pages  bf16 [num_pages][hkv][page_size][head_dim_qk]
+ *     v_pages  bf16 [num_pages][hkv][page_size][head_dim_v]
+ *              or NULL: latent KV, value row = first head_dim_v columns of the
+ *              key row (MLA-style absorbed attention, hkv = 1 typically).
+ *     Token j of a sequence lives in page table[j / page_size] at slot
+ *     j % page_size.  A suffix starts at slot 0 of its own first page.  Slots
+ *     past a sequence's length are never read (they may hold anything,
+ *     including NaN).
+ * Block tables are CSR int32 arrays on the device:
+ *     prefix pages of trace t: prefix_block_table[prefix_bt_offsets[t] + i]
+ *     suffix pages of fork f:  suffix_block_table[suffix_bt_offsets[f] + i]
+ * Forks of trace t are forks fork_offsets[t] .. fork_offsets[t+1]-1 (host).
+ *
+ * Conventions.  Every call is asynchronous on the caller's CUDA stream
+ * (cudaStream_t passed as void*, NULL = legacy default stream), performs no
+ * device synchronisation and allocates no device memory: scratch lives in the
+ * caller's workspace.  Errors are status codes, never exceptions or aborts.
+ * Kernels never trap: a page id outside [0, num_pages) is skipped and recorded
+ * in the workspace status word (read it with specgen_workspace_status).
+ */
+#ifndef SPECGEN_H
+#define SPECGEN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SPECGEN_OK = 0,
+  SPECGEN_ERR_NULL = -1,        /* a required pointer is NULL */
+  SPECGEN_ERR_SHAPE = -2,       /* inconsistent sizes (e.g. hq % hkv != 0, negative length) */
+  SPECGEN_ERR_UNSUPPORTED = -3, /* head dims / page size / group size not built */
+  SPECGEN_ERR_WORKSPACE = -4,   /* workspace too small or misaligned (256 B) */
+  SPECGEN_ERR_INDEX = -5,       /* device saw a page id outside [0, num_pages) */
+  SPECGEN_ERR_CUDA = -6,        /* a CUDA runtime call or launch failed */
+  SPECGEN_ERR_TIMEOUT = -7      /* a device-side wait hit its iteration limit */
+} specgen_status;
+
+/* Device-side arguments of one fork-decode call (all pointers device memory). */
+typedef struct {
+  int num_traces;               /* T >= 1 */
+  int total_forks;              /* F >= 1, sum over traces */
+  int hq, hkv;                  /* query / kv heads, hq % hkv == 0 */
+  int head_dim_qk, head_dim_v;  /* (64,64), (128,128) or (576,512) with v_pages == NULL */
+  int page_size;                /* 16 or 64 tokens */
+  int num_pages;                /* pool size; page ids are checked against it */
+  float scale;                  /* softmax scale sigma applied to q.k */
+  const void* q;                /* bf16 [total_forks][hq][head_dim_qk] */
+  const void* k_pages;          /* bf16, layout above */
+  const void* v_pages;          /* bf16, layout above, or NULL (latent KV) */
+  const int32_t* prefix_block_table;
+  const int32_t* prefix_bt_offsets;  /* [num_traces + 1] */
+  const int32_t* suffix_block_table;
+  const int32_t* suffix_bt_offsets;  /* [total_forks + 1] */
+  void* out;                    /* bf16 [total_forks][hq][head_dim_v] (written) */
+  float* lse;                   /* fp32 [total_forks][hq] natural-log LSE (written) */
+  void* workspace;              /* >= specgen_fork_attn_workspace_size bytes, 256-B aligned */
+  size_t workspace_bytes;
+} specgen_fork_attn_args;
+
+/* Host copies of the lengths: planning reads them, so no device->host copy is
+ * needed.  The device block tables must hold at least ceil(len/page_size)
+ * pages for every sequence. */
+typedef struct {
+  const int32_t* prefix_lens;   /* host [num_traces], >= 0 */
+  const int32_t* fork_offsets;  /* host [num_traces + 1], non-decreasing, [0]=0, [T]=F */
+  const int32_t* suffix_lens;   /* host [total_forks], >= 0 */
+} specgen_host_lens;
+
+/* Result of planning: work counts and workspace offsets.  Treat as opaque;
+ * valid for the args/lens it was made from while the workspace is unchanged. */
+typedef struct {
+  int32_t valid;
+  int32_t n_prefix_items;       /* tensor-core prefix-stage work items */
+  int32_t n_split_items;        /* split-K paged-decode work items */
+  int32_t n_rows;               /* total_forks * hq */
+  int32_t total_slots;          /* partial (O, LSE) slots */
+  int32_t flags;
+  int64_t plan_bytes;           /* plan bytes copied into the workspace */
+  int64_t ws_plan_off, ws_part_o_off, ws_part_lse_off, ws_end;
+  int64_t reserved[8];
+} specgen_plan;
+
+/* Bytes of workspace one call needs (0 on invalid input).  Depends only on the
+ * sizes in args (pointers may be NULL) and on the host lengths. */
+size_t specgen_fork_attn_workspace_size(const specgen_fork_attn_args* args,
+                                        const specgen_host_lens* lens);
+
+/* Plan the call on the host and copy the plan into the workspace (one
+ * cudaMemcpyAsync on `stream` from library-owned host memory that stays valid
+ * until the next plan call from this thread).  Also resets the workspace status
+ * word.  `plan` receives the launch shapes used by specgen_fork_attn_run. */
+specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
+                                      const specgen_host_lens* lens,
+                                      specgen_plan* plan, void* cuda_stream);
+
+/* Launch the kernels of a planned call (no host-device copies; capturable in a
+ * CUDA graph).  The data pointers in args may differ from the planning call;
+ * the sizes and workspace may not. */
+specgen_status specgen_fork_attn_run(const specgen_fork_attn_args* args,
+                                     const specgen_plan* plan, void* cuda_stream);
+
+/* specgen_fork_attn_run with timing marks for per-kernel measurement: records
+ * events[0] on `cuda_stream` before the first kernel and events[i] after the
+ * i-th kernel (i = 1 .. n_events-1; extra launches get no mark).  `events`
+ * holds cudaEvent_t handles created by the caller.  Runs exactly the same
+ * kernels as specgen_fork_attn_run; *n_launches (if not NULL) receives how
+ * many kernels were launched. */
+specgen_status specgen_fork_attn_run_profiled(const specgen_fork_attn_args* args,
+                                              const specgen_plan* plan, void* cuda_stream,
+                                              void* const* events, int n_events,
+                                              int* n_launches);
+
+/* Fork-decode attention for every fork and query head: plan + run. */
+specgen_status specgen_fork_attn_decode(const specgen_fork_attn_args* args,
+                                        const specgen_host_lens* lens,
+                                        void* cuda_stream);
+
+/* Standalone log-sum-exp merge of two partial attentions over disjoint key
+ * sets (the combination step of the split computation):
+ *     m = max(lse_a, lse_b); w_x = exp(lse_x - m)
+ *     out = (w_a out_a + w_b out_b) / (w_a + w_b);  lse = m + ln(w_a + w_b)
+ * An input row with lse = -inf is empty; both empty gives out = 0, lse = -inf.
+ * out_a, out_b, out: [rows][dv] of dtype (0 = bf16, 1 = fp32); lse_*: fp32 [rows].
+ * out/lse may alias out_a/lse_a (in-place).  Device pointers. */
+specgen_status specgen_lse_merge(const void* out_a, const float* lse_a,
+                                 const void* out_b, const float* lse_b,
+                                 void* out, float* lse, int rows, int dv,
+                                 int dtype, void* cuda_stream);
+
+/* Read the workspace status word written by the kernels (synchronises
+ * `cuda_stream`).  Returns SPECGEN_OK, SPECGEN_ERR_INDEX or SPECGEN_ERR_TIMEOUT. */
+specgen_status specgen_workspace_status(const void* workspace, void* cuda_stream);
+
+/* Static text for a status code. */
+const char* specgen_status_string(specgen_status status);
+
+/* Library version (major * 10000 + minor * 100 + patch). */
+int specgen_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPECGEN_H */

@@ -1,0 +1,190 @@
+"""ctypes binding of the fork-decode C ABI (``include/specgen.h``).
+
+Argument marshalling only: every step of the computation runs in the CUDA
+kernels of ``libspecgen.so``.  The function names match the C entry points.
+The library is built in-tree (``paper_2606_17518_gb300/build.py``); if it is
+missing, loading fails loudly -- there is no fallback implementation.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libspecgen.so")
+
+SPECGEN_OK = 0
+SPECGEN_ERR_NULL = -1
+SPECGEN_ERR_SHAPE = -2
+SPECGEN_ERR_UNSUPPORTED = -3
+SPECGEN_ERR_WORKSPACE = -4
+SPECGEN_ERR_INDEX = -5
+SPECGEN_ERR_CUDA = -6
+SPECGEN_ERR_TIMEOUT = -7
+
+EXPORTED = [
+    "specgen_fork_attn_workspace_size",
+    "specgen_fork_attn_plan",
+    "specgen_fork_attn_run",
+    "specgen_fork_attn_run_profiled",
+    "specgen_fork_attn_decode",
+    "specgen_lse_merge",
+    "specgen_workspace_status",
+    "specgen_status_string",
+    "specgen_version",
+]
+
+
+class ForkAttnArgs(C.Structure):
+    _fields_ = [
+        ("num_traces", C.c_int), ("total_forks", C.c_int), ("hq", C.c_int), ("hkv", C.c_int),
+        ("head_dim_qk", C.c_int), ("head_dim_v", C.c_int), ("page_size", C.c_int),
+        ("num_pages", C.c_int), ("scale", C.c_float),
+        ("q", C.c_void_p), ("k_pages", C.c_void_p), ("v_pages", C.c_void_p),
+        ("prefix_block_table", C.c_void_p), ("prefix_bt_offsets", C.c_void_p),
+        ("suffix_block_table", C.c_void_p), ("suffix_bt_offsets", C.c_void_p),
+        ("out", C.c_void_p), ("lse", C.c_void_p),
+        ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t),
+    ]
+
+
+class HostLens(C.Structure):
+    _fields_ = [("prefix_lens", C.c_void_p), ("fork_offsets", C.c_void_p),
+                ("suffix_lens", C.c_void_p)]
+
+
+class Plan(C.Structure):
+    _fields_ = [
+        ("valid", C.c_int32), ("n_prefix_items", C.c_int32), ("n_split_items", C.c_int32),
+        ("n_rows", C.c_int32), ("total_slots", C.c_int32), ("flags", C.c_int32),
+        ("plan_bytes", C.c_int64), ("ws_plan_off", C.c_int64), ("ws_part_o_off", C.c_int64),
+        ("ws_part_lse_off", C.c_int64), ("ws_end", C.c_int64), ("reserved", C.c_int64 * 8),
+    ]
+
+
+class SpecgenError(RuntimeError):
+    def __init__(self, status: int, what: str = ""):
+        self.status = status
+        super().__init__(f"{what}: {status_string(status)} ({status})")
+
+
+_lib = None
+
+
+def load() -> C.CDLL:
+    """Load libspecgen.so (built in-tree); raise if it is absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: run paper_2606_17518_gb300.build.build() "
+                           "first (no CPU fallback exists)")
+    lib = C.CDLL(LIB_PATH)
+    P = C.POINTER
+    lib.specgen_fork_attn_workspace_size.restype = C.c_size_t
+    lib.specgen_fork_attn_workspace_size.argtypes = [P(ForkAttnArgs), P(HostLens)]
+    lib.specgen_fork_attn_plan.restype = C.c_int
+    lib.specgen_fork_attn_plan.argtypes = [P(ForkAttnArgs), P(HostLens), P(Plan), C.c_void_p]
+    lib.specgen_fork_attn_run.restype = C.c_int
+    lib.specgen_fork_attn_run.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
+    lib.specgen_fork_attn_run_profiled.restype = C.c_int
+    lib.specgen_fork_attn_run_profiled.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p,
+                                                   C.c_void_p, C.c_int, P(C.c_int)]
+    lib.specgen_fork_attn_decode.restype = C.c_int
+    lib.specgen_fork_attn_decode.argtypes = [P(ForkAttnArgs), P(HostLens), C.c_void_p]
+    lib.specgen_lse_merge.restype = C.c_int
+    lib.specgen_lse_merge.argtypes = [C.c_void_p] * 6 + [C.c_int, C.c_int, C.c_int, C.c_void_p]
+    lib.specgen_workspace_status.restype = C.c_int
+    lib.specgen_workspace_status.argtypes = [C.c_void_p, C.c_void_p]
+    lib.specgen_status_string.restype = C.c_char_p
+    lib.specgen_status_string.argtypes = [C.c_int]
+    lib.specgen_version.restype = C.c_int
+    lib.specgen_version.argtypes = []
+    _lib = lib
+    return lib
+
+
+def status_string(status: int) -> str:
+    return load().specgen_status_string(int(status)).decode()
+
+
+def _check(status: int, what: str):
+    if status != SPECGEN_OK:
+        raise SpecgenError(status, what)
+
+
+def _ptr(t) -> int | None:
+    """Data pointer of a torch tensor / numpy array, or None."""
+    if t is None:
+        return None
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def make_host_lens(prefix_lens, fork_offsets, suffix_lens):
+    """HostLens over int32 numpy arrays (kept alive by the returned tuple)."""
+    arrs = tuple(np.ascontiguousarray(a, dtype=np.int32) for a in
+                 (prefix_lens, fork_offsets, suffix_lens))
+    return HostLens(*(a.ctypes.data for a in arrs)), arrs
+
+
+def make_args(*, num_traces, total_forks, hq, hkv, head_dim_qk, head_dim_v, page_size,
+              num_pages, scale, q, k_pages, v_pages, prefix_block_table, prefix_bt_offsets,
+              suffix_block_table, suffix_bt_offsets, out, lse, workspace=None,
+              workspace_bytes=0) -> ForkAttnArgs:
+    return ForkAttnArgs(
+        int(num_traces), int(total_forks), int(hq), int(hkv), int(head_dim_qk),
+        int(head_dim_v), int(page_size), int(num_pages), float(scale),
+        _ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(prefix_block_table),
+        _ptr(prefix_bt_offsets), _ptr(suffix_block_table), _ptr(suffix_bt_offsets),
+        _ptr(out), _ptr(lse), _ptr(workspace), int(workspace_bytes))
+
+
+def specgen_fork_attn_workspace_size(args: ForkAttnArgs, lens: HostLens) -> int:
+    return int(load().specgen_fork_attn_workspace_size(C.byref(args), C.byref(lens)))
+
+
+def specgen_fork_attn_plan(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> Plan:
+    plan = Plan()
+    _check(load().specgen_fork_attn_plan(C.byref(args), C.byref(lens), C.byref(plan),
+                                         C.c_void_p(stream)), "specgen_fork_attn_plan")
+    return plan
+
+
+def specgen_fork_attn_run(args: ForkAttnArgs, plan: Plan, stream: int = 0) -> None:
+    _check(load().specgen_fork_attn_run(C.byref(args), C.byref(plan), C.c_void_p(stream)),
+           "specgen_fork_attn_run")
+
+
+def specgen_fork_attn_run_profiled(args: ForkAttnArgs, plan: Plan, stream: int, events,
+                                   n_events: int) -> int:
+    """Run with timing marks; ``events`` is a ctypes void* array (or a byref into one)."""
+    n = C.c_int(0)
+    _check(load().specgen_fork_attn_run_profiled(C.byref(args), C.byref(plan),
+                                                 C.c_void_p(stream), events, int(n_events),
+                                                 C.byref(n)), "specgen_fork_attn_run_profiled")
+    return n.value
+
+
+def specgen_fork_attn_decode(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> None:
+    _check(load().specgen_fork_attn_decode(C.byref(args), C.byref(lens), C.c_void_p(stream)),
+           "specgen_fork_attn_decode")
+
+
+def specgen_lse_merge(out_a, lse_a, out_b, lse_b, out, lse, rows: int, dv: int, dtype: int,
+                      stream: int = 0) -> None:
+    _check(load().specgen_lse_merge(_ptr(out_a), _ptr(lse_a), _ptr(out_b), _ptr(lse_b),
+                                    _ptr(out), _ptr(lse), int(rows), int(dv), int(dtype),
+                                    C.c_void_p(stream)), "specgen_lse_merge")
+
+
+def specgen_workspace_status(workspace, stream: int = 0) -> int:
+    return int(load().specgen_workspace_status(_ptr(workspace), C.c_void_p(stream)))
+
+
+def specgen_version() -> int:
+    return int(load().specgen_version())

@@ -1,0 +1,24 @@
+// Host-visible interface of the log-sum-exp merge kernels (internal).
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace specgen {
+
+struct MergeParams {
+  const float* part_o;       // [slots][hq][dv]
+  const float* part_lse;     // [slots][hq]
+  const int32_t* part_base;  // [forks]
+  const int32_t* n_parts;    // [forks]
+  __nv_bfloat16* out;        // [forks][hq][dv]
+  float* lse;                // [forks][hq]
+  int n_rows, hq, dv;
+};
+
+cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream);
+cudaError_t launch_lse_merge2(const void* oa, const float* la, const void* ob, const float* lb,
+                              void* o, float* l, int rows, int dv, int dtype,
+                              cudaStream_t stream);
+
+}  // namespace specgen

@@ -1,0 +1,53 @@
+// Work-list records shared by the host planner and the kernels (internal).
+//
+// A fork-decode call is cut into work items, each producing one partial
+// attention (O normalised by its own softmax sum, plus its LSE) over a
+// contiguous range of logical tokens of one paged sequence.  Every (fork, head)
+// row owns `n_parts` consecutive partial slots starting at `part_base`; the
+// merge kernel combines them by log-sum-exp.
+#pragma once
+#include <stdint.h>
+
+namespace specgen {
+
+constexpr uint32_t kStatusIndex = 1u;    // a page id outside [0, num_pages) was seen
+constexpr uint32_t kStatusTimeout = 2u;  // a device wait hit its iteration limit
+
+// Split-K paged decode item: query rows [h0, h0+nrows) of one fork against
+// tokens [tok_begin, tok_end) of one sequence (the fork's trace prefix or the
+// fork's own suffix), value columns [dv0, dv0 + tile width).
+struct SplitItem {
+  int32_t fork;
+  int32_t table_kind;  // 0: prefix table of trace `seq`; 1: suffix table of fork `seq`
+  int32_t seq;
+  int32_t kv_head;
+  int32_t h0;
+  int32_t nrows;
+  int32_t dv0;
+  int32_t tok_begin;
+  int32_t tok_end;
+  int32_t slot;        // partial slot: part_o[slot][h][dv], part_lse[slot][h]
+};
+
+// Shared-prefix item (tensor-core prefix stage): the query rows of forks
+// [fork0, fork0 + nforks) of one trace for kv head `kv_head` (nforks * G rows)
+// against prefix tokens [tok_begin, tok_end).  Row (fork0 + i, head) writes
+// slot part_base[fork0 + i] + chunk.
+struct PrefixItem {
+  int32_t trace;
+  int32_t kv_head;
+  int32_t fork0;
+  int32_t nforks;
+  int32_t tok_begin;
+  int32_t tok_end;
+  int32_t chunk;
+  int32_t dv0;
+};
+
+// Plan header at the start of the plan region.
+struct PlanHeader {
+  int32_t n_split, n_prefix, n_forks, hq;
+  int32_t split_off, prefix_off, part_base_off, n_parts_off;  // byte offsets in plan
+};
+
+}  // namespace specgen

@@ -1,0 +1,406 @@
+// C ABI of the fork-decode attention library: argument checks, the host
+// planner that turns ragged lengths into a work list, and the launches.
+//
+// Planning runs on the host from host copies of the lengths, so a call needs
+// no device->host copy.  The work list and the per-fork partial-slot map are
+// copied into the caller's workspace; the kernels read them from there.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <string.h>
+
+#include <algorithm>
+#include <vector>
+
+#include "../../include/specgen.h"
+#include "lse_merge.h"
+#include "plan.h"
+#include "split_decode.h"
+
+using namespace specgen;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr size_t kHeaderBytes = 256;  // status word + reserved
+constexpr int kTileTokens = 64;       // split-kernel tile; chunk sizes are multiples of it
+constexpr int kRowBlock = 16;         // split-kernel rows per item
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int device_sm_count() {
+  static thread_local int cached_dev = -1, cached_sms = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (dev != cached_dev) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    cached_dev = dev;
+    cached_sms = n;
+  }
+  return cached_sms;
+}
+
+struct Shape {
+  int T, F, hq, hkv, G, dqk, dv, B, num_pages;
+  bool latent;
+};
+
+specgen_status check_shape(const specgen_fork_attn_args* a, const specgen_host_lens* lens,
+                           Shape* s) {
+  if (!a || !lens || !lens->prefix_lens || !lens->fork_offsets || !lens->suffix_lens)
+    return SPECGEN_ERR_NULL;
+  if (a->num_traces < 1 || a->total_forks < 1 || a->hq < 1 || a->hkv < 1 || a->page_size < 1 ||
+      a->num_pages < 0 || a->head_dim_qk < 1 || a->head_dim_v < 1)
+    return SPECGEN_ERR_SHAPE;
+  if (a->hq % a->hkv != 0) return SPECGEN_ERR_SHAPE;
+  if (!isfinite(a->scale)) return SPECGEN_ERR_SHAPE;
+  const bool latent = a->v_pages == nullptr;
+  if (latent && a->head_dim_v > a->head_dim_qk) return SPECGEN_ERR_SHAPE;
+  if (!split_variant_supported(a->head_dim_qk, a->head_dim_v, latent))
+    return SPECGEN_ERR_UNSUPPORTED;
+  if (a->page_size > 1024 || (a->page_size & (a->page_size - 1)) != 0)
+    return SPECGEN_ERR_UNSUPPORTED;
+  const int32_t* fo = lens->fork_offsets;
+  if (fo[0] != 0 || fo[a->num_traces] != a->total_forks) return SPECGEN_ERR_SHAPE;
+  for (int t = 0; t < a->num_traces; ++t) {
+    if (fo[t + 1] < fo[t] || lens->prefix_lens[t] < 0) return SPECGEN_ERR_SHAPE;
+  }
+  for (int f = 0; f < a->total_forks; ++f)
+    if (lens->suffix_lens[f] < 0) return SPECGEN_ERR_SHAPE;
+  s->T = a->num_traces;
+  s->F = a->total_forks;
+  s->hq = a->hq;
+  s->hkv = a->hkv;
+  s->G = a->hq / a->hkv;
+  s->dqk = a->head_dim_qk;
+  s->dv = a->head_dim_v;
+  s->B = a->page_size;
+  s->num_pages = a->num_pages;
+  s->latent = latent;
+  return SPECGEN_OK;
+}
+
+specgen_status check_pointers(const specgen_fork_attn_args* a) {
+  if (!a->q || !a->k_pages || !a->prefix_block_table || !a->prefix_bt_offsets ||
+      !a->suffix_block_table || !a->suffix_bt_offsets || !a->out || !a->lse || !a->workspace)
+    return SPECGEN_ERR_NULL;
+  if (reinterpret_cast<uintptr_t>(a->workspace) % kAlign != 0) return SPECGEN_ERR_WORKSPACE;
+  return SPECGEN_OK;
+}
+
+// The host-side plan: work items plus the partial-slot map.
+struct HostPlan {
+  std::vector<SplitItem> split;
+  std::vector<PrefixItem> prefix;
+  std::vector<int32_t> part_base, n_parts;
+  int total_slots = 0;
+};
+
+void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
+  const int dvt = split_dv_tile(s.dqk, s.dv, s.latent);
+  const int row_blocks = (s.G + kRowBlock - 1) / kRowBlock;
+  const int dv_blocks = s.dv / dvt;
+  const long long units = (long long)s.hkv * row_blocks * dv_blocks;
+
+  // chunk length: spread the token work over ~4 CTAs per SM, in whole tiles
+  long long total_tokens = 0;
+  for (int t = 0; t < s.T; ++t)
+    for (int f = lens->fork_offsets[t]; f < lens->fork_offsets[t + 1]; ++f)
+      total_tokens += (long long)lens->prefix_lens[t] + lens->suffix_lens[f];
+  const long long target_items = (long long)device_sm_count() * 4;
+  long long chunk = (total_tokens * units + target_items - 1) / std::max(1LL, target_items);
+  chunk = std::max<long long>(kTileTokens, (chunk + kTileTokens - 1) / kTileTokens * kTileTokens);
+  chunk = std::min<long long>(chunk, 1 << 20);
+
+  hp->split.clear();
+  hp->prefix.clear();
+  hp->part_base.assign(s.F, 0);
+  hp->n_parts.assign(s.F, 0);
+  int slot = 0;
+  for (int t = 0; t < s.T; ++t) {
+    const int P = lens->prefix_lens[t];
+    const int np = (int)((P + chunk - 1) / chunk);
+    for (int f = lens->fork_offsets[t]; f < lens->fork_offsets[t + 1]; ++f) {
+      const int S = lens->suffix_lens[f];
+      const int ns = (int)((S + chunk - 1) / chunk);
+      hp->part_base[f] = slot;
+      hp->n_parts[f] = np + ns;
+      for (int g = 0; g < s.hkv; ++g)
+        for (int rb = 0; rb < row_blocks; ++rb)
+          for (int db = 0; db < dv_blocks; ++db) {
+            SplitItem it;
+            it.fork = f;
+            it.kv_head = g;
+            it.h0 = g * s.G + rb * kRowBlock;
+            it.nrows = std::min(kRowBlock, s.G - rb * kRowBlock);
+            it.dv0 = db * dvt;
+            for (int c = 0; c < np; ++c) {
+              it.table_kind = 0;
+              it.seq = t;
+              it.tok_begin = (int)(c * chunk);
+              it.tok_end = (int)std::min<long long>(P, (c + 1) * chunk);
+              it.slot = slot + c;
+              hp->split.push_back(it);
+            }
+            for (int c = 0; c < ns; ++c) {
+              it.table_kind = 1;
+              it.seq = f;
+              it.tok_begin = (int)(c * chunk);
+              it.tok_end = (int)std::min<long long>(S, (c + 1) * chunk);
+              it.slot = slot + np + c;
+              hp->split.push_back(it);
+            }
+          }
+      slot += np + ns;
+    }
+  }
+  hp->total_slots = slot;
+}
+
+struct Layout {
+  size_t split_off, prefix_off, part_base_off, n_parts_off, plan_bytes;
+  size_t ws_plan, ws_part_o, ws_part_lse, ws_end;
+};
+
+Layout layout_of(const Shape& s, const HostPlan& hp) {
+  Layout L;
+  L.split_off = align_up(sizeof(PlanHeader), 16);
+  L.prefix_off = align_up(L.split_off + hp.split.size() * sizeof(SplitItem), 16);
+  L.part_base_off = align_up(L.prefix_off + hp.prefix.size() * sizeof(PrefixItem), 16);
+  L.n_parts_off = align_up(L.part_base_off + (size_t)s.F * 4, 16);
+  L.plan_bytes = L.n_parts_off + (size_t)s.F * 4;
+  L.ws_plan = kHeaderBytes;
+  L.ws_part_o = align_up(L.ws_plan + L.plan_bytes, kAlign);
+  L.ws_part_lse =
+      align_up(L.ws_part_o + (size_t)hp.total_slots * s.hq * s.dv * sizeof(float), kAlign);
+  L.ws_end = align_up(L.ws_part_lse + (size_t)hp.total_slots * s.hq * sizeof(float), kAlign);
+  return L;
+}
+
+thread_local HostPlan t_plan;
+thread_local std::vector<unsigned char> t_plan_bytes;
+
+}  // namespace
+
+extern "C" {
+
+size_t specgen_fork_attn_workspace_size(const specgen_fork_attn_args* args,
+                                        const specgen_host_lens* lens) {
+  Shape s;
+  if (check_shape(args, lens, &s) != SPECGEN_OK) return 0;
+  HostPlan hp;
+  build_plan(s, lens, &hp);
+  return layout_of(s, hp).ws_end;
+}
+
+specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
+                                      const specgen_host_lens* lens, specgen_plan* plan,
+                                      void* cuda_stream) {
+  if (!plan) return SPECGEN_ERR_NULL;
+  memset(plan, 0, sizeof(*plan));
+  Shape s;
+  specgen_status st = check_shape(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
+  if ((st = check_pointers(args)) != SPECGEN_OK) return st;
+  build_plan(s, lens, &t_plan);
+  const Layout L = layout_of(s, t_plan);
+  if (args->workspace_bytes < L.ws_end) return SPECGEN_ERR_WORKSPACE;
+
+  t_plan_bytes.assign(L.plan_bytes, 0);
+  PlanHeader h;
+  h.n_split = (int32_t)t_plan.split.size();
+  h.n_prefix = (int32_t)t_plan.prefix.size();
+  h.n_forks = s.F;
+  h.hq = s.hq;
+  h.split_off = (int32_t)L.split_off;
+  h.prefix_off = (int32_t)L.prefix_off;
+  h.part_base_off = (int32_t)L.part_base_off;
+  h.n_parts_off = (int32_t)L.n_parts_off;
+  unsigned char* b = t_plan_bytes.data();
+  memcpy(b, &h, sizeof(h));
+  if (!t_plan.split.empty())
+    memcpy(b + L.split_off, t_plan.split.data(), t_plan.split.size() * sizeof(SplitItem));
+  if (!t_plan.prefix.empty())
+    memcpy(b + L.prefix_off, t_plan.prefix.data(), t_plan.prefix.size() * sizeof(PrefixItem));
+  memcpy(b + L.part_base_off, t_plan.part_base.data(), (size_t)s.F * 4);
+  memcpy(b + L.n_parts_off, t_plan.n_parts.data(), (size_t)s.F * 4);
+
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  unsigned char* ws = static_cast<unsigned char*>(args->workspace);
+  if (cudaMemsetAsync(ws, 0, kHeaderBytes, stream) != cudaSuccess) return SPECGEN_ERR_CUDA;
+  if (cudaMemcpyAsync(ws + L.ws_plan, b, L.plan_bytes, cudaMemcpyHostToDevice, stream) !=
+      cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+
+  plan->valid = 1;
+  plan->n_prefix_items = h.n_prefix;
+  plan->n_split_items = h.n_split;
+  plan->n_rows = s.F * s.hq;
+  plan->total_slots = t_plan.total_slots;
+  plan->flags = s.latent ? 1 : 0;
+  plan->plan_bytes = (int64_t)L.plan_bytes;
+  plan->ws_plan_off = (int64_t)L.ws_plan;
+  plan->ws_part_o_off = (int64_t)L.ws_part_o;
+  plan->ws_part_lse_off = (int64_t)L.ws_part_lse;
+  plan->ws_end = (int64_t)L.ws_end;
+  plan->reserved[0] = (int64_t)L.split_off;
+  plan->reserved[1] = (int64_t)L.prefix_off;
+  plan->reserved[2] = (int64_t)L.part_base_off;
+  plan->reserved[3] = (int64_t)L.n_parts_off;
+  return SPECGEN_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+// Records mark `i` of the caller's event list (if there is one) on `stream`.
+struct Marks {
+  void* const* events;
+  int n;
+  int launches = 0;
+  bool mark(cudaStream_t stream, int i) {
+    if (!events || i >= n || !events[i]) return true;
+    return cudaEventRecord(static_cast<cudaEvent_t>(events[i]), stream) == cudaSuccess;
+  }
+};
+
+specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* plan,
+                        void* cuda_stream, Marks& marks);
+
+}  // namespace
+
+extern "C" {
+
+specgen_status specgen_fork_attn_run(const specgen_fork_attn_args* args, const specgen_plan* plan,
+                                     void* cuda_stream) {
+  Marks marks{nullptr, 0};
+  return run_impl(args, plan, cuda_stream, marks);
+}
+
+specgen_status specgen_fork_attn_run_profiled(const specgen_fork_attn_args* args,
+                                              const specgen_plan* plan, void* cuda_stream,
+                                              void* const* events, int n_events,
+                                              int* n_launches) {
+  Marks marks{events, n_events};
+  specgen_status st = run_impl(args, plan, cuda_stream, marks);
+  if (n_launches) *n_launches = marks.launches;
+  return st;
+}
+
+}  // extern "C"
+
+namespace {
+
+specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* plan,
+                        void* cuda_stream, Marks& marks) {
+  if (!args || !plan) return SPECGEN_ERR_NULL;
+  if (!plan->valid) return SPECGEN_ERR_SHAPE;
+  specgen_status st = check_pointers(args);
+  if (st != SPECGEN_OK) return st;
+  if ((int64_t)args->workspace_bytes < plan->ws_end) return SPECGEN_ERR_WORKSPACE;
+  if ((args->v_pages == nullptr) != (plan->flags & 1)) return SPECGEN_ERR_SHAPE;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  unsigned char* ws = static_cast<unsigned char*>(args->workspace);
+  unsigned char* pl = ws + plan->ws_plan_off;
+  float* part_o = reinterpret_cast<float*>(ws + plan->ws_part_o_off);
+  float* part_lse = reinterpret_cast<float*>(ws + plan->ws_part_lse_off);
+
+  SplitParams sp;
+  sp.q = static_cast<const __nv_bfloat16*>(args->q);
+  sp.k_pages = static_cast<const __nv_bfloat16*>(args->k_pages);
+  sp.v_pages = static_cast<const __nv_bfloat16*>(args->v_pages);
+  sp.prefix_bt = args->prefix_block_table;
+  sp.prefix_bt_off = args->prefix_bt_offsets;
+  sp.suffix_bt = args->suffix_block_table;
+  sp.suffix_bt_off = args->suffix_bt_offsets;
+  sp.items = reinterpret_cast<const SplitItem*>(pl + plan->reserved[0]);
+  sp.part_o = part_o;
+  sp.part_lse = part_lse;
+  sp.status = reinterpret_cast<uint32_t*>(ws);
+  sp.hq = args->hq;
+  sp.hkv = args->hkv;
+  sp.dqk = args->head_dim_qk;
+  sp.dv = args->head_dim_v;
+  sp.page_size = args->page_size;
+  sp.num_pages = args->num_pages;
+  sp.scale_log2 = args->scale * 1.4426950408889634f;
+  if (!marks.mark(stream, 0)) return SPECGEN_ERR_CUDA;
+  if (plan->n_split_items > 0) {
+    if (launch_split_decode(sp, plan->n_split_items, args->v_pages == nullptr, stream) !=
+        cudaSuccess)
+      return SPECGEN_ERR_CUDA;
+    if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
+  }
+
+  MergeParams mp;
+  mp.part_o = part_o;
+  mp.part_lse = part_lse;
+  mp.part_base = reinterpret_cast<const int32_t*>(pl + plan->reserved[2]);
+  mp.n_parts = reinterpret_cast<const int32_t*>(pl + plan->reserved[3]);
+  mp.out = static_cast<__nv_bfloat16*>(args->out);
+  mp.lse = args->lse;
+  mp.n_rows = plan->n_rows;
+  mp.hq = args->hq;
+  mp.dv = args->head_dim_v;
+  if (launch_merge_parts(mp, stream) != cudaSuccess) return SPECGEN_ERR_CUDA;
+  if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+specgen_status specgen_fork_attn_decode(const specgen_fork_attn_args* args,
+                                        const specgen_host_lens* lens, void* cuda_stream) {
+  specgen_plan plan;
+  specgen_status st = specgen_fork_attn_plan(args, lens, &plan, cuda_stream);
+  if (st != SPECGEN_OK) return st;
+  return specgen_fork_attn_run(args, &plan, cuda_stream);
+}
+
+specgen_status specgen_lse_merge(const void* out_a, const float* lse_a, const void* out_b,
+                                 const float* lse_b, void* out, float* lse, int rows, int dv,
+                                 int dtype, void* cuda_stream) {
+  if (rows < 0 || dv < 0) return SPECGEN_ERR_SHAPE;
+  if (dtype != 0 && dtype != 1) return SPECGEN_ERR_UNSUPPORTED;
+  if (rows == 0) return SPECGEN_OK;
+  if (!out_a || !lse_a || !out_b || !lse_b || !out || !lse) return SPECGEN_ERR_NULL;
+  if (launch_lse_merge2(out_a, lse_a, out_b, lse_b, out, lse, rows, dv, dtype,
+                        static_cast<cudaStream_t>(cuda_stream)) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
+}
+
+specgen_status specgen_workspace_status(const void* workspace, void* cuda_stream) {
+  if (!workspace) return SPECGEN_ERR_NULL;
+  uint32_t word = 0;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  if (cudaMemcpyAsync(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost, stream) !=
+      cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return SPECGEN_ERR_CUDA;
+  if (word & kStatusTimeout) return SPECGEN_ERR_TIMEOUT;
+  if (word & kStatusIndex) return SPECGEN_ERR_INDEX;
+  return SPECGEN_OK;
+}
+
+const char* specgen_status_string(specgen_status status) {
+  switch (status) {
+    case SPECGEN_OK: return "ok";
+    case SPECGEN_ERR_NULL: return "null pointer argument";
+    case SPECGEN_ERR_SHAPE: return "inconsistent shape or length";
+    case SPECGEN_ERR_UNSUPPORTED: return "unsupported head dims, page size or group size";
+    case SPECGEN_ERR_WORKSPACE: return "workspace too small or misaligned";
+    case SPECGEN_ERR_INDEX: return "page id outside [0, num_pages)";
+    case SPECGEN_ERR_CUDA: return "CUDA error";
+    case SPECGEN_ERR_TIMEOUT: return "device wait exceeded its iteration limit";
+  }
+  return "unknown status";
+}
+
+int specgen_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,89 @@
+"""Device-side fork-decode call over torch-allocated buffers.
+
+``ForkDecode`` owns the device copies of one workload (PyTorch is used only
+to allocate device memory and provide streams), builds the C-ABI argument
+structs and calls ``specgen_fork_attn_plan`` / ``specgen_fork_attn_run`` /
+``specgen_fork_attn_decode``.  It does no arithmetic of its own.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+from . import _lib
+
+
+def _bf16(a, device):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(device).view(torch.bfloat16)
+
+
+def _i32(a, device):
+    import torch
+    a = np.ascontiguousarray(a, dtype=np.int32)
+    if a.size == 0:                      # keep a valid (never read) pointer for empty tables
+        a = np.zeros(1, dtype=np.int32)
+    return torch.from_numpy(a).to(device)
+
+
+class ForkDecode:
+    """One workload resident on the GPU plus its output and workspace buffers."""
+
+    def __init__(self, w: dict, device="cuda", upload_kv: bool = True):
+        import torch
+        self.w = w
+        self.device = torch.device(device)
+        self.latent = w["v_pages"] is None
+        self.q = _bf16(w["q"], device)
+        self.k_pages = _bf16(w["k_pages"], device) if upload_kv else None
+        self.v_pages = (None if self.latent else _bf16(w["v_pages"], device)) if upload_kv else None
+        self.prefix_table = _i32(w["prefix_table"], device)
+        self.prefix_off = _i32(w["prefix_bt_offsets"], device)
+        self.suffix_table = _i32(w["suffix_table"], device)
+        self.suffix_off = _i32(w["suffix_bt_offsets"], device)
+        F, hq, dv = w["total_forks"], w["hq"], w["dv"]
+        self.out = torch.empty((F, hq, dv), dtype=torch.bfloat16, device=device)
+        self.lse = torch.empty((F, hq), dtype=torch.float32, device=device)
+        self.lens, self._lens_keep = _lib.make_host_lens(
+            w["prefix_lens"], w["fork_offsets"], w["suffix_lens"])
+        self.ws_bytes = _lib.specgen_fork_attn_workspace_size(self.args(with_ws=False), self.lens)
+        if self.ws_bytes == 0:
+            raise _lib.SpecgenError(_lib.SPECGEN_ERR_SHAPE, "specgen_fork_attn_workspace_size")
+        self.workspace = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        self.plan_info = None
+
+    def args(self, with_ws: bool = True, **override) -> _lib.ForkAttnArgs:
+        w = self.w
+        kw = dict(
+            num_traces=w["num_traces"], total_forks=w["total_forks"], hq=w["hq"], hkv=w["hkv"],
+            head_dim_qk=w["dqk"], head_dim_v=w["dv"], page_size=w["page_size"],
+            num_pages=w["num_pages"], scale=w["scale"], q=self.q, k_pages=self.k_pages,
+            v_pages=self.v_pages, prefix_block_table=self.prefix_table,
+            prefix_bt_offsets=self.prefix_off, suffix_block_table=self.suffix_table,
+            suffix_bt_offsets=self.suffix_off, out=self.out, lse=self.lse,
+            workspace=self.workspace if with_ws else None,
+            workspace_bytes=self.ws_bytes if with_ws else 0)
+        kw.update(override)
+        return _lib.make_args(**kw)
+
+    def plan(self, stream: int = 0):
+        self.plan_info = _lib.specgen_fork_attn_plan(self.args(), self.lens, stream)
+        return self.plan_info
+
+    def run(self, stream: int = 0):
+        if self.plan_info is None:
+            self.plan(stream)
+        _lib.specgen_fork_attn_run(self.args(), self.plan_info, stream)
+
+    def decode(self, stream: int = 0):
+        _lib.specgen_fork_attn_decode(self.args(), self.lens, stream)
+
+    def status(self, stream: int = 0) -> int:
+        return _lib.specgen_workspace_status(self.workspace, stream)
+
+    def results(self):
+        """(O as float64 numpy [F, hq, dv], LSE as float64 numpy [F, hq])."""
+        import torch
+        torch.cuda.synchronize(self.device)
+        return (self.out.float().cpu().numpy().astype(np.float64),
+                self.lse.cpu().numpy().astype(np.float64))

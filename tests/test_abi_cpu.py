@@ -1,0 +1,169 @@
+"""C-ABI checks that need no GPU: the library loads, exports every entry point
+declared in include/specgen.h, and rejects bad arguments with status codes
+before touching the device."""
+
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+import __graft_entry__
+from paper_2606_17518_gb300 import _lib, workloads as wl
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    __graft_entry__.build()
+
+
+def _declared():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(specgen_\w+)\s*\(", src))
+    return names
+
+
+def test_exports_every_declared_symbol():
+    lib = _lib.load()
+    declared = _declared()
+    assert declared >= set(_lib.EXPORTED), declared
+    for name in declared:
+        assert hasattr(lib, name), name
+
+
+def test_status_strings():
+    for code in range(0, -8, -1):
+        s = _lib.status_string(code)
+        assert s and s != "unknown status"
+    assert _lib.status_string(-99) == "unknown status"
+    assert _lib.specgen_version() >= 100
+
+
+def _fake_args(w, **kw):
+    # non-null fake device pointers: the checks below fail before any CUDA call
+    fake = 0x10000
+    base = dict(num_traces=w["num_traces"], total_forks=w["total_forks"], hq=w["hq"],
+                hkv=w["hkv"], head_dim_qk=w["dqk"], head_dim_v=w["dv"],
+                page_size=w["page_size"], num_pages=w["num_pages"], scale=w["scale"])
+    args = _lib.ForkAttnArgs(*[int(base[k]) if k != "scale" else float(base[k])
+                               for k in ("num_traces", "total_forks", "hq", "hkv",
+                                         "head_dim_qk", "head_dim_v", "page_size",
+                                         "num_pages", "scale")])
+    for name in ("q", "k_pages", "v_pages", "prefix_block_table", "prefix_bt_offsets",
+                 "suffix_block_table", "suffix_bt_offsets", "out", "lse", "workspace"):
+        setattr(args, name, fake)
+    if w["v_pages"] is None:
+        args.v_pages = None
+    args.workspace_bytes = 1 << 40
+    for k, v in kw.items():
+        setattr(args, k, v)
+    return args
+
+
+def _lens(w, **kw):
+    arrs = dict(prefix_lens=w["prefix_lens"], fork_offsets=w["fork_offsets"],
+                suffix_lens=w["suffix_lens"])
+    arrs.update(kw)
+    return _lib.make_host_lens(arrs["prefix_lens"], arrs["fork_offsets"], arrs["suffix_lens"])
+
+
+def _plan_status(args, lens):
+    plan = _lib.Plan()
+    return _lib.load().specgen_fork_attn_plan(C.byref(args), C.byref(lens), C.byref(plan), None)
+
+
+@pytest.fixture(scope="module")
+def w():
+    return wl.make_workload("tiny_p512_f4")
+
+
+def test_workspace_size_positive_and_monotone(w):
+    lens, keep = _lens(w)
+    n = _lib.specgen_fork_attn_workspace_size(_fake_args(w), lens)
+    assert n > 0 and n % 256 == 0
+    lens2, keep2 = _lens(w, suffix_lens=w["suffix_lens"] * 40)
+    assert _lib.specgen_fork_attn_workspace_size(_fake_args(w), lens2) >= n
+
+
+@pytest.mark.parametrize("name", wl.WORKLOAD_ORDER)
+def test_workspace_size_all_workloads(name):
+    spec = wl.WORKLOADS[name]
+    # sizes only: build a length-only workload without drawing the pools
+    rng = np.random.default_rng(0)
+    T = spec.num_traces
+    pl = rng.integers(spec.prefix_len[0], spec.prefix_len[1] + 1, T).astype(np.int32)
+    fk = rng.integers(spec.forks[0], spec.forks[1] + 1, T)
+    fo = np.concatenate([[0], np.cumsum(fk)]).astype(np.int32)
+    sl = rng.integers(spec.suffix_len[0], spec.suffix_len[1] + 1, int(fo[-1])).astype(np.int32)
+    w = dict(num_traces=T, total_forks=int(fo[-1]), hq=spec.hq, hkv=spec.hkv, dqk=spec.dqk,
+             dv=spec.dv, page_size=spec.page_size, num_pages=1000, scale=spec.scale,
+             v_pages=(None if not spec.separate_v else 1), prefix_lens=pl, fork_offsets=fo,
+             suffix_lens=sl)
+    lens, keep = _lens(w)
+    n = _lib.specgen_fork_attn_workspace_size(_fake_args(w), lens)
+    assert 0 < n < (1 << 31)
+
+
+def test_shape_errors(w):
+    lens, keep = _lens(w)
+    S = _lib
+    assert _plan_status(_fake_args(w, hq=7), lens) == S.SPECGEN_ERR_SHAPE          # hq % hkv
+    assert _plan_status(_fake_args(w, num_traces=0), lens) == S.SPECGEN_ERR_SHAPE
+    assert _plan_status(_fake_args(w, head_dim_qk=96, head_dim_v=96), lens) == \
+        S.SPECGEN_ERR_UNSUPPORTED
+    assert _plan_status(_fake_args(w, page_size=12), lens) == S.SPECGEN_ERR_UNSUPPORTED
+    assert _plan_status(_fake_args(w, scale=float("nan")), lens) == S.SPECGEN_ERR_SHAPE
+    bad, k1 = _lens(w, suffix_lens=np.array([1, -1, 2, 3], dtype=np.int32))
+    assert _plan_status(_fake_args(w), bad) == S.SPECGEN_ERR_SHAPE
+    bad, k2 = _lens(w, fork_offsets=np.array([0, 3], dtype=np.int32))              # != F
+    assert _plan_status(_fake_args(w), bad) == S.SPECGEN_ERR_SHAPE
+    assert _lib.specgen_fork_attn_workspace_size(_fake_args(w, hq=7), lens) == 0
+
+
+def test_null_and_workspace_errors(w):
+    lens, keep = _lens(w)
+    S = _lib
+    assert _plan_status(_fake_args(w, q=None), lens) == S.SPECGEN_ERR_NULL
+    assert _plan_status(_fake_args(w, out=None), lens) == S.SPECGEN_ERR_NULL
+    assert _plan_status(_fake_args(w, workspace=0x10010), lens) == S.SPECGEN_ERR_WORKSPACE
+    assert _plan_status(_fake_args(w, workspace_bytes=1024), lens) == S.SPECGEN_ERR_WORKSPACE
+    plan = _lib.Plan()
+    lib = _lib.load()
+    assert lib.specgen_fork_attn_plan(None, C.byref(lens), C.byref(plan), None) == \
+        S.SPECGEN_ERR_NULL
+    assert lib.specgen_fork_attn_plan(C.byref(_fake_args(w)), C.byref(lens), None, None) == \
+        S.SPECGEN_ERR_NULL
+    # run with an invalid (zeroed) plan is rejected on the host
+    assert lib.specgen_fork_attn_run(C.byref(_fake_args(w)), C.byref(plan), None) == \
+        S.SPECGEN_ERR_SHAPE
+
+
+def test_lse_merge_host_checks():
+    lib = _lib.load()
+    S = _lib
+    fake = C.c_void_p(0x10000)
+    assert lib.specgen_lse_merge(fake, fake, fake, fake, fake, fake, 0, 128, 0, None) == S.SPECGEN_OK
+    assert lib.specgen_lse_merge(fake, fake, fake, fake, fake, fake, 4, 128, 3, None) == \
+        S.SPECGEN_ERR_UNSUPPORTED
+    assert lib.specgen_lse_merge(None, fake, fake, fake, fake, fake, 4, 128, 0, None) == \
+        S.SPECGEN_ERR_NULL
+    assert lib.specgen_lse_merge(fake, fake, fake, fake, fake, fake, -1, 128, 0, None) == \
+        S.SPECGEN_ERR_SHAPE
+
+
+def test_product_path_has_no_oracle_import():
+    """The package never imports the oracle (it is test infrastructure)."""
+    pkg = os.path.join(ROOT, "paper_2606_17518_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for fn in files:
+            if fn.endswith((".py", ".cu", ".cuh", ".h")):
+                src = open(os.path.join(dirpath, fn)).read()
+                assert not re.search(r"^\s*(import|from)\s+oracle\b", src, re.M), fn
+                assert "oracle/" not in src, fn

@@ -1,0 +1,194 @@
+"""GPU vs fp64 oracle parity, through the C ABI (libspecgen.so).
+
+Tolerances (from the fork-decode target): max |dO| <= 2e-2 on bf16 outputs
+and max |dLSE| <= 1e-3 on fp32 LSE.  Index handling is bit-exact: the same
+logical KV at a different physical page placement gives identical bits, and a
+page id outside the pool is reported, never read.  Every pool holds NaN in
+unused slots and sentinel pages, so any read past a length shows up.
+"""
+
+import numpy as np
+import pytest
+
+import __graft_entry__
+import oracle
+from paper_2606_17518_gb300 import _lib, workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+TOL_O = 2e-2
+TOL_LSE = 1e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    __graft_entry__.build()
+
+
+def _gpu(w):
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    fd = ForkDecode(w)
+    fd.decode()
+    o, lse = fd.results()
+    assert fd.status() == _lib.SPECGEN_OK
+    return o, lse, fd
+
+
+def _compare(o, lse, o_ref, lse_ref, what=""):
+    assert np.all(np.isfinite(o)), what
+    fin = np.isfinite(lse_ref)
+    assert np.array_equal(np.isfinite(lse), fin), what
+    assert np.all(lse[~fin] == lse_ref[~fin]), what
+    err_o = float(np.max(np.abs(o - o_ref))) if o.size else 0.0
+    err_l = float(np.max(np.abs(lse[fin] - lse_ref[fin]))) if fin.any() else 0.0
+    assert err_o <= TOL_O, (what, err_o)
+    assert err_l <= TOL_LSE, (what, err_l)
+    return err_o, err_l
+
+
+@pytest.mark.parametrize("name", ["tiny_p512_f4", "fork_p8k_f8", "mla_p16k_f8"])
+def test_workload_full(name):
+    w = wl.make_workload(name)
+    o, lse, _ = _gpu(w)
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, name)
+
+
+@pytest.mark.parametrize("name", ["long_p32k_f16", "ragged_t8"])
+def test_workload_sampled(name):
+    """Full-size workloads: every head of the first and last fork plus random rows."""
+    w = wl.make_workload(name)
+    o, lse, _ = _gpu(w)
+    F, hq = w["total_forks"], w["hq"]
+    rng = np.random.default_rng(123)
+    rows = [(0, h) for h in range(hq)] + [(F - 1, h) for h in range(hq)]
+    rows += [(int(f), int(h)) for f, h in zip(rng.integers(0, F, 96), rng.integers(0, hq, 96))]
+    o_ref, lse_ref = oracle.fork_attn_decode_rows(w, rows)
+    idx_f = np.array([r[0] for r in rows])
+    idx_h = np.array([r[1] for r in rows])
+    _compare(o[idx_f, idx_h], lse[idx_f, idx_h], o_ref, lse_ref, name)
+
+
+def _fuzz_spec(rng, page_size, dqk, G, hkv):
+    B = page_size
+    edge = [0, 1, B - 1, B, B + 1, 3 * B + 5]
+    return wl.WorkloadSpec(
+        name="fuzz", num_traces=int(rng.integers(1, 4)),
+        prefix_len=tuple(sorted(int(x) for x in rng.choice(edge + [200, 700], 2))),
+        forks=(1, int(rng.integers(1, 6))),
+        suffix_len=tuple(sorted(int(x) for x in rng.choice(edge + [130], 2))),
+        hq=G * hkv, hkv=hkv, dqk=dqk, dv=dqk, page_size=B, seed=int(rng.integers(1 << 30)))
+
+
+@pytest.mark.parametrize("case", range(12))
+def test_fuzz_small_shapes(case):
+    rng = np.random.default_rng(1000 + case)
+    page_size = [16, 64][case % 2]
+    dqk = [64, 128][(case // 2) % 2]
+    G = [1, 4, 8, 16][case % 4]
+    hkv = [1, 2, 3][case % 3]
+    w = wl.make_workload(_fuzz_spec(rng, page_size, dqk, G, hkv))
+    o, lse, _ = _gpu(w)
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, f"fuzz{case}")
+
+
+def test_empty_prefix_and_suffix_edges():
+    spec = wl.WorkloadSpec(name="edges", num_traces=3, prefix_len=(0, 40), forks=(2, 4),
+                           suffix_len=(0, 2), hq=8, hkv=2, dqk=128, dv=128, page_size=16,
+                           seed=77)
+    w = wl.make_workload(spec)
+    w["prefix_lens"][0] = 0          # trace 0: no prefix (its forks see only their suffix)
+    w["suffix_lens"][:] = [0 if i % 2 == 0 else x for i, x in enumerate(w["suffix_lens"])]
+    w["suffix_lens"][w["fork_offsets"][0]] = 0   # a fork with nothing at all: O = 0, LSE = -inf
+    o, lse, _ = _gpu(w)
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, "edges")
+    assert np.all(lse[0] == -np.inf) and np.all(o[0] == 0)
+
+
+def test_latent_small_against_oracle():
+    spec = wl.WorkloadSpec(name="mla_small", num_traces=2, prefix_len=(60, 300), forks=(1, 3),
+                           suffix_len=(0, 130), hq=128, hkv=1, dqk=576, dv=512, page_size=64,
+                           separate_v=False, seed=5)
+    w = wl.make_workload(spec)
+    o, lse, _ = _gpu(w)
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, "mla_small")
+
+
+def test_page_placement_is_bit_exact():
+    w = wl.make_workload("fork_p8k_f8")
+    o1, l1, _ = _gpu(w)
+    perm = np.random.default_rng(9).permutation(w["num_pages"]).astype(np.int32)
+    w2 = dict(w)
+    for key in ("k_pages", "v_pages"):
+        pool = np.empty_like(w[key])
+        pool[perm] = w[key]
+        w2[key] = pool
+    w2["prefix_table"] = perm[w["prefix_table"]]
+    w2["suffix_table"] = perm[w["suffix_table"]]
+    o2, l2, _ = _gpu(w2)
+    assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
+
+
+def test_invalid_page_id_is_reported_not_read():
+    w = wl.make_workload("tiny_p512_f4")
+    w = dict(w)
+    w["suffix_table"] = w["suffix_table"].copy()
+    w["suffix_table"][0] = w["num_pages"] + 7
+    w["prefix_table"] = w["prefix_table"].copy()
+    w["prefix_table"][3] = -2
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    fd = ForkDecode(w)
+    fd.decode()
+    o, lse = fd.results()
+    assert fd.status() == _lib.SPECGEN_ERR_INDEX
+    assert np.all(np.isfinite(o))
+
+
+def test_plan_once_run_many_is_deterministic():
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload("fork_p8k_f8")
+    fd = ForkDecode(w)
+    fd.plan()
+    fd.run()
+    o1, l1 = fd.results()
+    fd.out.zero_()
+    fd.run()
+    fd.run()
+    o2, l2 = fd.results()
+    assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
+
+
+@pytest.mark.parametrize("dtype", [0, 1])
+def test_lse_merge_standalone(dtype):
+    import torch
+    rng = np.random.default_rng(4 + dtype)
+    rows, dv = 777, 128
+    oa, ob = rng.standard_normal((rows, dv)), rng.standard_normal((rows, dv))
+    la, lb = rng.standard_normal(rows) * 3, rng.standard_normal(rows) * 3
+    la[::7] = -np.inf
+    lb[::11] = -np.inf
+    tdt = torch.bfloat16 if dtype == 0 else torch.float32
+    t = lambda a, dt: torch.tensor(a, dtype=dt, device="cuda")
+    d_oa, d_ob = t(oa, tdt), t(ob, tdt)
+    d_la, d_lb = t(la, torch.float32), t(lb, torch.float32)
+    d_o = torch.empty_like(d_oa)
+    d_l = torch.empty_like(d_la)
+    _lib.specgen_lse_merge(d_oa, d_la, d_ob, d_lb, d_o, d_l, rows, dv, dtype)
+    torch.cuda.synchronize()
+    # the oracle merges the same (rounded) inputs the GPU saw
+    oa_in = d_oa.float().cpu().numpy().astype(np.float64)
+    ob_in = d_ob.float().cpu().numpy().astype(np.float64)
+    o_ref, l_ref = oracle.lse_merge(oa_in, la.astype(np.float32).astype(np.float64),
+                                    ob_in, lb.astype(np.float32).astype(np.float64))
+    o = d_o.float().cpu().numpy().astype(np.float64)
+    lse = d_l.cpu().numpy().astype(np.float64)
+    tol = TOL_O if dtype == 0 else 1e-5
+    _compare(o, lse, o_ref, l_ref, "merge")
+    assert np.max(np.abs(o - o_ref)) <= tol
+    # in place: out aliases the a-side
+    _lib.specgen_lse_merge(d_oa, d_la, d_ob, d_lb, d_oa, d_la, rows, dv, dtype)
+    torch.cuda.synchronize()
+    assert torch.equal(d_oa, d_o) and torch.equal(d_la, d_l)
