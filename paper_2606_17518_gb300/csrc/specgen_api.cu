@@ -14,6 +14,7 @@
 #include "../../include/specgen.h"
 #include "lse_merge.h"
 #include "plan.h"
+#include "prefix_tc.h"
 #include "split_decode.h"
 
 using namespace specgen;
@@ -98,18 +99,38 @@ struct HostPlan {
 };
 
 void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
+  const int n_sm = device_sm_count();
+  const int32_t* fo = lens->fork_offsets;
+  const bool tc_prefix = prefix_tc_supported(s.dqk, s.dv, s.latent, s.B, s.G);
+
+  // ---- shared-prefix items (tensor cores): all forks of a trace x one kv head
+  // in one row tile (up to 128 rows), prefix cut into page-aligned chunks so
+  // that about one wave of CTAs (one per SM) covers every trace.
+  const int forks_per_item = std::max(1, 128 / s.G);
+  long long prefix_chunk = 0;
+  if (tc_prefix) {
+    long long work = 0;  // prefix tokens x kv heads x row tiles
+    for (int t = 0; t < s.T; ++t) {
+      const int nf = fo[t + 1] - fo[t];
+      if (nf == 0) continue;
+      work += (long long)lens->prefix_lens[t] * s.hkv * ((nf + forks_per_item - 1) / forks_per_item);
+    }
+    const int pg = prefix_tc_page_size();
+    prefix_chunk = (work + n_sm - 1) / std::max(1, n_sm);
+    prefix_chunk = std::max<long long>(pg, (prefix_chunk + pg - 1) / pg * pg);
+  }
+
+  // ---- split-K items: whatever the prefix kernel does not cover
   const int dvt = split_dv_tile(s.dqk, s.dv, s.latent);
   const int row_blocks = (s.G + kRowBlock - 1) / kRowBlock;
   const int dv_blocks = s.dv / dvt;
   const long long units = (long long)s.hkv * row_blocks * dv_blocks;
-
-  // chunk length: spread the token work over ~4 CTAs per SM, in whole tiles
-  long long total_tokens = 0;
+  long long split_tokens = 0;
   for (int t = 0; t < s.T; ++t)
-    for (int f = lens->fork_offsets[t]; f < lens->fork_offsets[t + 1]; ++f)
-      total_tokens += (long long)lens->prefix_lens[t] + lens->suffix_lens[f];
-  const long long target_items = (long long)device_sm_count() * 4;
-  long long chunk = (total_tokens * units + target_items - 1) / std::max(1LL, target_items);
+    for (int f = fo[t]; f < fo[t + 1]; ++f)
+      split_tokens += (tc_prefix ? 0LL : (long long)lens->prefix_lens[t]) + lens->suffix_lens[f];
+  const long long target_items = (long long)n_sm * 4;
+  long long chunk = (split_tokens * units + target_items - 1) / std::max(1LL, target_items);
   chunk = std::max<long long>(kTileTokens, (chunk + kTileTokens - 1) / kTileTokens * kTileTokens);
   chunk = std::min<long long>(chunk, 1 << 20);
 
@@ -120,8 +141,9 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   int slot = 0;
   for (int t = 0; t < s.T; ++t) {
     const int P = lens->prefix_lens[t];
-    const int np = (int)((P + chunk - 1) / chunk);
-    for (int f = lens->fork_offsets[t]; f < lens->fork_offsets[t + 1]; ++f) {
+    const long long pchunk = tc_prefix ? prefix_chunk : chunk;
+    const int np = (int)((P + pchunk - 1) / pchunk);
+    for (int f = fo[t]; f < fo[t + 1]; ++f) {
       const int S = lens->suffix_lens[f];
       const int ns = (int)((S + chunk - 1) / chunk);
       hp->part_base[f] = slot;
@@ -135,7 +157,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
             it.h0 = g * s.G + rb * kRowBlock;
             it.nrows = std::min(kRowBlock, s.G - rb * kRowBlock);
             it.dv0 = db * dvt;
-            for (int c = 0; c < np; ++c) {
+            for (int c = 0; !tc_prefix && c < np; ++c) {
               it.table_kind = 0;
               it.seq = t;
               it.tok_begin = (int)(c * chunk);
@@ -153,6 +175,22 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
             }
           }
       slot += np + ns;
+    }
+    if (tc_prefix && np > 0) {
+      for (int g = 0; g < s.hkv; ++g)
+        for (int f0 = fo[t]; f0 < fo[t + 1]; f0 += forks_per_item)
+          for (int c = 0; c < np; ++c) {
+            PrefixItem it;
+            it.trace = t;
+            it.kv_head = g;
+            it.fork0 = f0;
+            it.nforks = std::min(forks_per_item, fo[t + 1] - f0);
+            it.tok_begin = (int)(c * prefix_chunk);
+            it.tok_end = (int)std::min<long long>(P, (c + 1) * prefix_chunk);
+            it.chunk = c;
+            it.dv0 = 0;
+            hp->prefix.push_back(it);
+          }
     }
   }
   hp->total_slots = slot;
@@ -327,6 +365,28 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   sp.num_pages = args->num_pages;
   sp.scale_log2 = args->scale * 1.4426950408889634f;
   if (!marks.mark(stream, 0)) return SPECGEN_ERR_CUDA;
+  if (plan->n_prefix_items > 0) {
+    PrefixParams pp;
+    pp.q = sp.q;
+    pp.prefix_bt = args->prefix_block_table;
+    pp.prefix_bt_off = args->prefix_bt_offsets;
+    pp.items = reinterpret_cast<const PrefixItem*>(pl + plan->reserved[1]);
+    pp.part_base = reinterpret_cast<const int32_t*>(pl + plan->reserved[2]);
+    pp.part_o = part_o;
+    pp.part_lse = part_lse;
+    pp.status = sp.status;
+    pp.hq = args->hq;
+    pp.hkv = args->hkv;
+    pp.G = args->hq / args->hkv;
+    pp.dv = args->head_dim_v;
+    pp.page_size = args->page_size;
+    pp.num_pages = args->num_pages;
+    pp.scale_log2 = sp.scale_log2;
+    if (launch_prefix_tc(pp, args->k_pages, args->v_pages, plan->n_prefix_items,
+                         args->head_dim_qk, stream) != cudaSuccess)
+      return SPECGEN_ERR_CUDA;
+    if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
+  }
   if (plan->n_split_items > 0) {
     if (launch_split_decode(sp, plan->n_split_items, args->v_pages == nullptr, stream) !=
         cudaSuccess)
