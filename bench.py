@@ -333,11 +333,22 @@ def run_ours():
     # ---- end to end through the public API: host buffers, copies in the timed region
     e2e = measure_e2e(w, reps, stream, dev, K=min(K, 500), W=min(W, 5))
 
-    kernel_names = ["split_decode", "lse_merge"][:launches]
+    kernel_names = (["prefix_tc"] if plans[0].n_prefix_items > 0 else []) + \
+        (["split_decode"] if plans[0].n_split_items > 0 else []) + ["lse_merge"]
+    kernel_names = kernel_names[:launches]
     kernel_ms = [t / K for t in per_kernel]
     dom = int(np.argmax(kernel_ms)) if kernel_ms else 0
     hbm, tf_burst, tf_sus, peak_src = measured_peaks()
-    dom_bytes = nbytes["prefix"] + nbytes["suffix"] + nbytes["q"]
+    # algorithmic bytes of the dominant launch: what that kernel must read/write once
+    dom_name = kernel_names[dom] if kernel_names else None
+    if dom_name == "prefix_tc":
+        dom_bytes = nbytes["prefix"] + nbytes["q"]
+    elif dom_name == "split_decode" and plans[0].n_prefix_items > 0:
+        dom_bytes = nbytes["suffix"] + nbytes["q"]
+    elif dom_name == "split_decode":
+        dom_bytes = nbytes["prefix"] + nbytes["suffix"] + nbytes["q"]
+    else:
+        dom_bytes = nbytes["total"]
     achieved = dom_bytes / (kernel_ms[dom] * 1e-3) / 1e9 if kernel_ms else None
     traffic = recorded_traffic(kernel_names[dom], ARGS.workload)
 

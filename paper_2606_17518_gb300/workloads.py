@@ -176,3 +176,34 @@ def algorithmic_flops(w: dict) -> dict:
     prefix *= w["hkv"] * g * 2 * (w["dqk"] + w["dv"])
     suffix = int(np.sum(w["suffix_lens"])) * w["hkv"] * g * 2 * (w["dqk"] + w["dv"])
     return dict(prefix=prefix, suffix=suffix, total=prefix + suffix)
+
+
+def shard_traces(w: dict, rank: int, world: int) -> dict:
+    """The traces ``t`` with ``t % world == rank`` of a workload, re-indexed.
+
+    Fork decode has no exchange between traces (each trace's forks read only
+    that trace's prefix and their own suffixes), so ranks can take disjoint
+    sets of traces and run them with no collective.  The KV pools are shared
+    by reference: page ids keep pointing into the same pool.  Returns a
+    workload dict of the same form (possibly with zero traces).
+    """
+    traces = [t for t in range(w["num_traces"]) if t % world == rank]
+    fo, pbo, sbo = w["fork_offsets"], w["prefix_bt_offsets"], w["suffix_bt_offsets"]
+    forks = [f for t in traces for f in range(fo[t], fo[t + 1])]
+    pt = [w["prefix_table"][pbo[t]:pbo[t + 1]] for t in traces]
+    st = [w["suffix_table"][sbo[f]:sbo[f + 1]] for f in forks]
+    cat = lambda parts: (np.concatenate(parts).astype(np.int32) if parts
+                         else np.zeros(0, dtype=np.int32))
+    offs = lambda parts: np.concatenate([[0], np.cumsum([len(x) for x in parts])]).astype(np.int32)
+    out = dict(w)
+    out.update(
+        q=w["q"][forks] if forks else w["q"][:0],
+        prefix_table=cat(pt), prefix_bt_offsets=offs(pt),
+        prefix_lens=w["prefix_lens"][traces].astype(np.int32),
+        fork_offsets=offs([range(fo[t], fo[t + 1]) for t in traces]),
+        suffix_table=cat(st), suffix_bt_offsets=offs(st),
+        suffix_lens=w["suffix_lens"][forks].astype(np.int32),
+        num_traces=len(traces), total_forks=len(forks),
+        global_forks=np.array(forks, dtype=np.int64),
+    )
+    return out
