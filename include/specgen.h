@@ -68,7 +68,7 @@ typedef struct {
   int head_dim_qk, head_dim_v;  /* (64,64), (128,128) or (576,512) with v_pages == NULL */
   int page_size;                /* 16 or 64 tokens */
   int num_pages;                /* pool size; page ids are checked against it */
-  float scale;                  /* softmax scale sigma applied to q.k */
+  float scale;                  /* softmax scale sigma applied to q.k, finite and > 0 */
   const void* q;                /* bf16 [total_forks][hq][head_dim_qk] */
   const void* k_pages;          /* bf16, layout above */
   const void* v_pages;          /* bf16, layout above, or NULL (latent KV) */
@@ -95,14 +95,16 @@ typedef struct {
  * valid for the args/lens it was made from while the workspace is unchanged. */
 typedef struct {
   int32_t valid;
-  int32_t n_prefix_items;       /* tensor-core prefix-stage work items */
+  int32_t n_tc_items;           /* tensor-core work items (prefix and suffix chunks) */
+  int32_t n_tc_ctas;            /* persistent CTAs of the tensor-core kernel */
   int32_t n_split_items;        /* split-K paged-decode work items */
   int32_t n_rows;               /* total_forks * hq */
   int32_t total_slots;          /* partial (O, LSE) slots */
   int32_t flags;
+  int32_t reserved0;
   int64_t plan_bytes;           /* plan bytes copied into the workspace */
   int64_t ws_plan_off, ws_part_o_off, ws_part_lse_off, ws_end;
-  int64_t reserved[8];
+  int64_t offsets[8];           /* internal offsets inside the plan region */
 } specgen_plan;
 
 /* Bytes of workspace one call needs (0 on invalid input).  Depends only on the

@@ -1,0 +1,476 @@
+// Fork-decode attention on the 5th-generation tensor cores (tcgen05 + TMA).
+//
+// One persistent CTA per SM walks its list of TcItems.  An item is either a
+// chunk of a trace's shared prefix (the query rows of all the trace's forks for
+// one kv head, gathered into one M = nforks * G <= 128 row tile, so each prefix
+// page is fetched from HBM once for every fork) or a chunk of one fork's
+// private suffix (M = G rows).  Each item writes a partial (O / l, LSE) per row.
+//
+// Per 128-token tile t (8 pages of 16 tokens), with t counted across items:
+//   warp 0 (TMA)     K_t, V_t pages -> 2-stage shared-memory ring (two 64-column
+//                    boxes per page, 128B swizzle), byte-counted on full[t%2]
+//   warp 1 (MMA)     S_t = Q K_t^T -> TMEM S[t%2]   (M=128, N=16*pages, K=D)
+//                    O  += P_t V_t -> TMEM O         (M=128, N=D,  K=16*pages)
+//   warps 2-5        one thread per row (= TMEM lane): the 128 scores of the
+//                    tile in registers, masked where needed, running max kept
+//                    in log2 units; P_t = exp2(s*scale*log2e - m) to shared
+//                    memory as bf16 (128B-swizzled, K-major); the TMEM output
+//                    is rescaled only when a row's max grows by more than
+//                    2^8 (lazy rescaling), otherwise P may exceed 1.
+// S is double-buffered in TMEM so S_{t+1} runs while tile t is in softmax.
+// Warps whose 32 rows are all padding skip the softmax work.  Tokens past the
+// item, past the sequence or on an invalid page are masked to -inf, and value
+// rows past the sequence inside its last page are zeroed in shared memory
+// before the PV product, so nothing stored there (even NaN) reaches the output.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "fork_tc.h"
+#include "plan.h"
+#include "tc_common.cuh"
+
+namespace specgen {
+
+namespace {
+
+using namespace tc;
+
+constexpr int kPB = 16;                      // page size (tokens)
+constexpr int kTileTok = 128;                // tokens per tile
+constexpr int kPagesPerTile = kTileTok / kPB;
+constexpr uint32_t kPanelBytes = 128 * 128;  // 128 rows x 128 B (64 bf16 columns)
+constexpr int kThreads = 192;                // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
+constexpr uint32_t kTmemCols = 512;          // S0 [0,128) S1 [128,256) O [256, 256+D)
+constexpr uint32_t kTmemO = 256;
+constexpr float kRescaleLog2 = 8.0f;         // lazy-rescale threshold (factor 256)
+
+template <int D>
+struct Smem {
+  static constexpr int kPanels = D / 64;
+  static constexpr uint32_t kQ = kPanels * kPanelBytes;
+  static constexpr uint32_t kKV = kPanels * kPanelBytes;  // one K or V tile
+  static constexpr uint32_t kStage = 2 * kKV;
+  static constexpr uint32_t kP = 2 * kPanelBytes;         // 128 rows x 128 tokens
+  static constexpr uint32_t kOffKV = kQ;
+  static constexpr uint32_t kOffP = kOffKV + 2 * kStage;
+  static constexpr uint32_t kOffBar = kOffP + 2 * kP;
+  static constexpr uint32_t kBytes = kOffBar + 128 + 1024;  // + barriers + alignment slack
+};
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                             uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+               "r"(d)
+               : "memory");
+}
+
+struct ItemView {
+  const int32_t* table;
+  int ntiles, page0, M;
+};
+
+__device__ __forceinline__ ItemView view(const TcParams& p, const TcItem& it) {
+  ItemView v;
+  v.table = it.table_kind == 0 ? p.prefix_bt + p.prefix_bt_off[it.seq]
+                               : p.suffix_bt + p.suffix_bt_off[it.seq];
+  v.ntiles = (it.tok_end - it.tok_begin + kTileTok - 1) / kTileTok;
+  v.page0 = it.tok_begin / kPB;
+  v.M = it.nforks * p.G;
+  return v;
+}
+
+__device__ __forceinline__ int tile_tokens(const TcItem& it, int j) {
+  const int n = it.tok_end - (it.tok_begin + j * kTileTok);
+  return n < kTileTok ? n : kTileTok;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    fork_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tmk,
+                   const __grid_constant__ CUtensorMap tmv) {
+  using L = Smem<D>;
+  extern __shared__ unsigned char smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;  // 128B-swizzled tiles: 1024-B aligned
+  unsigned char* gbase = smem_raw + (base - raw);
+  const uint32_t sQ = base;
+  const uint32_t sKV = base + L::kOffKV;
+  const uint32_t sP = base + L::kOffP;
+  const uint32_t bar0 = base + L::kOffBar;
+  auto full = [&](int s) { return bar0 + 8u * s; };
+  auto empty = [&](int s) { return bar0 + 16u + 8u * s; };
+  auto s_full = [&](int b) { return bar0 + 32u + 8u * b; };
+  auto p_full = [&](int b) { return bar0 + 48u + 8u * b; };
+  const uint32_t o_full = bar0 + 64u;
+  const uint32_t q_ready = bar0 + 72u;
+  const uint32_t mma_done = bar0 + 80u;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 96);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + L::kOffBar + 100);
+  auto sK = [&](int s) { return sKV + s * L::kStage; };
+  auto sV = [&](int s) { return sKV + s * L::kStage + L::kKV; };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(full(i), 1);
+      mbar_init(empty(i), 1);
+      mbar_init(s_full(i), 1);
+      mbar_init(p_full(i), 128);
+    }
+    mbar_init(o_full, 1);
+    mbar_init(q_ready, 128);
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    mbar_init_fence();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int t = 0;  // tiles issued so far (across items)
+      bool ok = true;
+      for (int ii = it_begin; ok && ii < it_end; ++ii) {
+        const TcItem it = p.items[p.cta_items[ii]];
+        const ItemView v = view(p, it);
+        for (int j = 0; j < v.ntiles; ++j, ++t) {
+          const int s = t & 1;
+          if (!(ok = mbar_wait(empty(s), ((t >> 1) & 1) ^ 1, abort_flag, p.status))) break;
+          const int np = (tile_tokens(it, j) + kPB - 1) / kPB;
+          int pages[kPagesPerTile];  // fetch the tile's page ids before issuing any copy
+#pragma unroll
+          for (int pg = 0; pg < kPagesPerTile; ++pg)
+            pages[pg] = pg < np ? v.table[v.page0 + j * kPagesPerTile + pg] : 0;
+          mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
+#pragma unroll
+          for (int pg = 0; pg < kPagesPerTile; ++pg) {
+            if (pg >= np) break;
+            const int page = pages[pg];
+            if (page < 0 || page >= p.num_pages) atomicOr(p.status, kStatusIndex);  // zero-filled
+#pragma unroll
+            for (int pn = 0; pn < L::kPanels; ++pn) {
+              const uint32_t off = pn * kPanelBytes + pg * (kPB * 128u);
+              tma_load_4d(sK(s) + off, &tmk, pn * 64, 0, it.kv_head, page, full(s));
+              tma_load_4d(sV(s) + off, &tmv, pn * 64, 0, it.kv_head, page, full(s));
+            }
+          }
+        }
+      }
+      // never leave a copy in flight into this CTA's shared memory
+      for (int u = t - 2 < 0 ? 0 : t - 2; u < t; ++u) mbar_wait_drain(full(u & 1), (u >> 1) & 1, p.status);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int t = 0;
+      bool ok = true;
+      for (int ii = it_begin; ok && ii < it_end; ++ii) {
+        const TcItem it = p.items[p.cta_items[ii]];
+        const ItemView v = view(p, it);
+        if (!(ok = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status))) break;
+        tc_fence_after();
+        for (int j = 0; j <= v.ntiles; ++j) {
+          if (j < v.ntiles) {
+            const int u = t + j, s = u & 1;
+            if (!(ok = mbar_wait(full(s), (u >> 1) & 1, abort_flag, p.status))) break;
+            tc_fence_after();
+            const int np = (tile_tokens(it, j) + kPB - 1) / kPB;
+            const uint32_t idesc = idesc_bf16(128, np * kPB, false);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32u;
+              mma_bf16(tmem + (uint32_t)s * 128u, smem_desc_sw128(sQ + off, 16, 1024),
+                       smem_desc_sw128(sK(s) + off, 16, 1024), idesc, kk > 0 ? 1u : 0u);
+            }
+            mma_commit(s_full(s));
+          }
+          if (j >= 1) {
+            const int u = t + j - 1, b = u & 1;
+            if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
+            tc_fence_after();
+            const int np = (tile_tokens(it, j - 1) + kPB - 1) / kPB;
+            constexpr uint32_t idesc = idesc_bf16(128, D, true);
+            for (int kk = 0; kk < np; ++kk) {  // one page (16 tokens) per k-step
+              const uint64_t a = smem_desc_sw128(sP + b * L::kP + (kk >> 2) * kPanelBytes +
+                                                     (kk & 3) * 32u, 16, 1024);
+              const uint64_t vd = smem_desc_sw128(sV(b) + kk * (kPB * 128u), kPanelBytes, 1024);
+              mma_bf16(tmem + kTmemO, a, vd, idesc, (j > 1 || kk > 0) ? 1u : 0u);
+            }
+            mma_commit(o_full);
+            mma_commit(empty(b));
+          }
+        }
+        t += v.ntiles;
+      }
+      // every MMA issued by this thread has finished before TMEM is released
+      mma_commit(mma_done);
+      mbar_wait_drain(mma_done, 0, p.status);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax warps
+    const int q4 = warp & 3;
+    const int row = q4 * 32 + lane;
+    const int tid = threadIdx.x - 64;  // 0..127
+    const uint32_t lane_addr = (uint32_t)(q4 * 32) << 16;
+    const uint32_t s_base = tmem + lane_addr;
+    const uint32_t o_base = tmem + lane_addr + kTmemO;
+    const float sl2 = p.scale_log2;
+    int t = 0;
+    bool ok = true;
+    for (int ii = it_begin; ok && ii < it_end; ++ii) {
+      const TcItem it = p.items[p.cta_items[ii]];
+      const ItemView v = view(p, it);
+      const bool warp_live = q4 * 32 < v.M;  // some real row in this warp
+      const bool row_ok = row < v.M;
+      const int fl = row / p.G, gi = row % p.G;
+      const int head = it.kv_head * p.G + gi;
+
+      // Q rows -> shared memory (128B-swizzled K-major); padding rows are zero
+      if (warp_live) {
+        const uint4* src = reinterpret_cast<const uint4*>(
+            p.q + ((size_t)(it.fork0 + (row_ok ? fl : 0)) * p.hq + (row_ok ? head : 0)) * D);
+#pragma unroll
+        for (int c = 0; c < D / 8; ++c) {
+          uint4 q = row_ok ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+          st_shared_v4(sQ + (c >> 3) * kPanelBytes + row * 128u + (((c & 7) ^ (row & 7)) << 4),
+                       q.x, q.y, q.z, q.w);
+        }
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(q_ready);
+
+      float m = -INFINITY, l = 0.f;  // running max (log2 units) and sum of this row
+      for (int j = 0; j < v.ntiles; ++j) {
+        const int u = t + j, b = u & 1;
+        const bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
+        if (__any_sync(0xffffffffu, !w)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int nt = tile_tokens(it, j);
+        const int np = (nt + kPB - 1) / kPB;
+        bool rescale = false;
+        float alpha = 1.f;
+        if (warp_live) {
+          uint32_t pv = 0;  // valid pages of this tile
+#pragma unroll
+          for (int pg = 0; pg < kPagesPerTile; ++pg) {
+            if (pg < np) {
+              const int page = v.table[v.page0 + j * kPagesPerTile + pg];
+              if (page >= 0 && page < p.num_pages) pv |= 1u << pg;
+            }
+          }
+          float s[kTileTok];
+          {
+            uint32_t r[16];
+#pragma unroll
+            for (int c = 0; c < kTileTok / 16; ++c) {
+              tmem_ld16(s_base + (uint32_t)b * 128u + c * 16u, r);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 16; ++i) s[c * 16 + i] = __uint_as_float(r[i]);
+            }
+          }
+          const bool full_tile = nt == kTileTok && pv == 0xFFu;
+          if (!full_tile) {
+#pragma unroll
+            for (int i = 0; i < kTileTok; ++i)
+              if (!(i < nt && ((pv >> (i / kPB)) & 1u))) s[i] = -INFINITY;
+          }
+          float mx = s[0];
+#pragma unroll
+          for (int i = 1; i < kTileTok; ++i) mx = fmaxf(mx, s[i]);
+          const float m_tile = mx * sl2;  // scale > 0
+          if (m_tile > m + kRescaleLog2 || (m == -INFINITY && m_tile != -INFINITY)) {
+            alpha = m == -INFINITY ? 0.f : fast_exp2(m - m_tile);
+            rescale = m != -INFINITY;
+            l *= alpha;
+            m = m_tile;
+          }
+          const float sub = m == -INFINITY ? 0.f : m;
+          float psum = 0.f;
+          const uint32_t prow = sP + b * L::kP + row * 128u;
+#pragma unroll
+          for (int c = 0; c < kTileTok / 8; ++c) {  // 8 columns = one 16-byte chunk
+            uint32_t pk[4];
+#pragma unroll
+            for (int i = 0; i < 8; i += 2) {
+              const float p0 = fast_exp2(fmaf(s[c * 8 + i], sl2, -sub));
+              const float p1 = fast_exp2(fmaf(s[c * 8 + i + 1], sl2, -sub));
+              psum += p0 + p1;
+              pk[i >> 1] = pack_bf16x2(p0, p1);
+            }
+            st_shared_v4(prow + (c >> 3) * kPanelBytes + (((c & 7) ^ (row & 7)) << 4), pk[0],
+                         pk[1], pk[2], pk[3]);
+          }
+          l += psum;
+        }
+        // value rows past the sequence inside its last page: zero them before PV
+        if (j == v.ntiles - 1 && (nt % kPB) != 0) {
+          const int pg = np - 1, first = nt % kPB;
+          const int units = (kPB - first) * L::kPanels * 8;
+          for (int x = tid; x < units; x += 128) {
+            const int rr = first + x / (L::kPanels * 8);
+            const int rem = x % (L::kPanels * 8);
+            st_shared_v4(sV(b) + (rem >> 3) * kPanelBytes + (pg * kPB + rr) * 128u +
+                             ((rem & 7) << 4), 0u, 0u, 0u, 0u);
+          }
+        }
+        // the previous PV must be done before the output is rescaled
+        if (j >= 1) {
+          const bool w2 = mbar_wait(o_full, (u - 1) & 1, abort_flag, p.status);
+          if (__any_sync(0xffffffffu, !w2)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          if (__any_sync(0xffffffffu, rescale)) {
+            const float a = rescale ? alpha : 1.f;
+#pragma unroll
+            for (int c = 0; c < D / 16; ++c) {
+              uint32_t r[16];
+              tmem_ld16(o_base + c * 16u, r);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * a);
+              tmem_st16(o_base + c * 16u, r);
+            }
+            tmem_wait_st();
+          }
+        }
+        tc_fence_before();
+        fence_proxy_async_smem();
+        mbar_arrive(p_full(b));
+      }
+      if (!ok) break;
+      // final output of the item: wait for the last PV, read O, normalise
+      {
+        const int u = t + v.ntiles - 1;
+        const bool w = mbar_wait(o_full, u & 1, abort_flag, p.status);
+        if (__any_sync(0xffffffffu, !w)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (warp_live) {
+          const int fork = it.fork0 + (row_ok ? fl : 0);
+          const size_t prow_out = (size_t)(p.part_base[fork] + it.part) * p.hq + head;
+          float4* dst = reinterpret_cast<float4*>(p.part_o + prow_out * p.dv);
+          const float inv = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+          for (int c = 0; c < D / 16; ++c) {
+            uint32_t r[16];
+            tmem_ld16(o_base + c * 16u, r);
+            tmem_wait_ld();
+            if (row_ok) {
+#pragma unroll
+              for (int i = 0; i < 16; i += 4)
+                dst[c * 4 + i / 4] = make_float4(
+                    __uint_as_float(r[i]) * inv, __uint_as_float(r[i + 1]) * inv,
+                    __uint_as_float(r[i + 2]) * inv, __uint_as_float(r[i + 3]) * inv);
+            }
+          }
+          if (row_ok) p.part_lse[prow_out] = m == -INFINITY ? -INFINITY : (m + log2f(l)) * kLn2;
+        }
+      }
+      t += v.ntiles;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// Paged pool [num_pages][hkv][page][D] bf16 as a 4-D tensor (D, page, hkv, pages);
+// one box = 64 columns x one page of one head, 128-byte swizzled.
+bool make_pool_map(CUtensorMap* map, const void* pool, int D, int page, int hkv, int num_pages) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc || !pool || num_pages < 1) return false;
+  const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)page, (cuuint64_t)hkv,
+                              (cuuint64_t)num_pages};
+  const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)page * D * 2,
+                                 (cuuint64_t)hkv * page * D * 2};
+  const cuuint32_t box[4] = {64, (cuuint32_t)page, 1, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(pool), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap& mv, int grid,
+                     cudaStream_t stream) {
+  constexpr int smem = (int)Smem<D>::kBytes;
+  static_assert(smem <= 232448, "fork_tc kernel shared memory exceeds 227 KB");
+  auto kern = fork_tc_kernel<D>;
+  static thread_local int configured = -1;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (configured != dev) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    configured = dev;
+  }
+  kern<<<grid, kThreads, smem, stream>>>(p, mk, mv);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G) {
+  return !latent && dqk == dv && (dqk == 64 || dqk == 128) && page_size == kPB && G <= 128;
+}
+
+int fork_tc_tile_tokens() { return kTileTok; }
+int fork_tc_page_size() { return kPB; }
+
+cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
+                           int dqk, cudaStream_t stream) {
+  if (grid == 0) return cudaSuccess;
+  CUtensorMap mk, mv;
+  if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
+      !make_pool_map(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
+    return cudaErrorInvalidValue;
+  if (dqk == 128) return launch_d<128>(p, mk, mv, grid, stream);
+  if (dqk == 64) return launch_d<64>(p, mk, mv, grid, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace specgen

@@ -1,0 +1,34 @@
+// Host-visible interface of the tensor-core fork-decode kernel (internal).
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "plan.h"
+
+namespace specgen {
+
+struct TcParams {
+  const __nv_bfloat16* q;
+  const int32_t* prefix_bt;
+  const int32_t* prefix_bt_off;
+  const int32_t* suffix_bt;
+  const int32_t* suffix_bt_off;
+  const TcItem* items;
+  const int32_t* cta_items;    // item indices, grouped per CTA
+  const int32_t* cta_offsets;  // [grid + 1] into cta_items
+  const int32_t* part_base;    // [forks] first partial slot of each fork
+  float* part_o;               // [slots][hq][dv]
+  float* part_lse;             // [slots][hq]
+  uint32_t* status;
+  int hq, hkv, G, dv, num_pages;
+  float scale_log2;            // softmax scale * log2(e), > 0
+};
+
+bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G);
+int fork_tc_tile_tokens();
+int fork_tc_page_size();
+cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
+                           int dqk, cudaStream_t stream);
+
+}  // namespace specgen

@@ -29,25 +29,25 @@ struct SplitItem {
   int32_t slot;        // partial slot: part_o[slot][h][dv], part_lse[slot][h]
 };
 
-// Shared-prefix item (tensor-core prefix stage): the query rows of forks
-// [fork0, fork0 + nforks) of one trace for kv head `kv_head` (nforks * G rows)
-// against prefix tokens [tok_begin, tok_end).  Row (fork0 + i, head) writes
-// slot part_base[fork0 + i] + chunk.
-struct PrefixItem {
-  int32_t trace;
+// Tensor-core item (shared prefix or one fork's suffix): the query rows of
+// forks [fork0, fork0 + nforks) for kv head `kv_head` (nforks * G <= 128 rows)
+// against tokens [tok_begin, tok_end) of one paged sequence.  Row (fork, head)
+// writes partial slot part_base[fork] + part.
+struct TcItem {
+  int32_t table_kind;  // 0: prefix table of trace `seq`; 1: suffix table of fork `seq`
+  int32_t seq;
   int32_t kv_head;
   int32_t fork0;
   int32_t nforks;
   int32_t tok_begin;
   int32_t tok_end;
-  int32_t chunk;
-  int32_t dv0;
+  int32_t part;
 };
 
 // Plan header at the start of the plan region.
 struct PlanHeader {
-  int32_t n_split, n_prefix, n_forks, hq;
-  int32_t split_off, prefix_off, part_base_off, n_parts_off;  // byte offsets in plan
+  int32_t n_split, n_tc, n_tc_ctas, n_forks;
+  int32_t split_off, tc_off, cta_items_off, cta_offsets_off, part_base_off, n_parts_off;
 };
 
 }  // namespace specgen

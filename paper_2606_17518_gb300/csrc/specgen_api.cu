@@ -9,12 +9,14 @@
 #include <string.h>
 
 #include <algorithm>
+#include <queue>
+#include <utility>
 #include <vector>
 
 #include "../../include/specgen.h"
 #include "lse_merge.h"
 #include "plan.h"
-#include "prefix_tc.h"
+#include "fork_tc.h"
 #include "split_decode.h"
 
 using namespace specgen;
@@ -55,7 +57,7 @@ specgen_status check_shape(const specgen_fork_attn_args* a, const specgen_host_l
       a->num_pages < 0 || a->head_dim_qk < 1 || a->head_dim_v < 1)
     return SPECGEN_ERR_SHAPE;
   if (a->hq % a->hkv != 0) return SPECGEN_ERR_SHAPE;
-  if (!isfinite(a->scale)) return SPECGEN_ERR_SHAPE;
+  if (!isfinite(a->scale) || !(a->scale > 0.f)) return SPECGEN_ERR_SHAPE;
   const bool latent = a->v_pages == nullptr;
   if (latent && a->head_dim_v > a->head_dim_qk) return SPECGEN_ERR_SHAPE;
   if (!split_variant_supported(a->head_dim_qk, a->head_dim_v, latent))
@@ -90,37 +92,118 @@ specgen_status check_pointers(const specgen_fork_attn_args* a) {
   return SPECGEN_OK;
 }
 
-// The host-side plan: work items plus the partial-slot map.
+// The host-side plan: work items, their CTA assignment, and the partial-slot map.
 struct HostPlan {
   std::vector<SplitItem> split;
-  std::vector<PrefixItem> prefix;
+  std::vector<TcItem> tc;
+  std::vector<int32_t> cta_items, cta_offsets;
   std::vector<int32_t> part_base, n_parts;
   int total_slots = 0;
 };
 
+// Longest-processing-time-first assignment of items to `n_cta` persistent CTAs:
+// items in decreasing cost, each to the currently least-loaded CTA.
+void assign_lpt(const std::vector<long long>& cost, int n_cta, std::vector<int32_t>* cta_items,
+                std::vector<int32_t>* cta_offsets) {
+  const int n = (int)cost.size();
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return cost[a] > cost[b]; });
+  typedef std::pair<long long, int> Load;  // (load, cta)
+  std::priority_queue<Load, std::vector<Load>, std::greater<Load>> heap;
+  for (int c = 0; c < n_cta; ++c) heap.push(Load(0, c));
+  std::vector<std::vector<int32_t>> lists(n_cta);
+  for (int i : order) {
+    Load top = heap.top();
+    heap.pop();
+    lists[top.second].push_back(i);
+    heap.push(Load(top.first + cost[i], top.second));
+  }
+  cta_items->clear();
+  cta_offsets->assign(1, 0);
+  for (int c = 0; c < n_cta; ++c) {
+    cta_items->insert(cta_items->end(), lists[c].begin(), lists[c].end());
+    cta_offsets->push_back((int32_t)cta_items->size());
+  }
+}
+
 void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   const int n_sm = device_sm_count();
   const int32_t* fo = lens->fork_offsets;
-  const bool tc_prefix = prefix_tc_supported(s.dqk, s.dv, s.latent, s.B, s.G);
+  const bool tc = fork_tc_supported(s.dqk, s.dv, s.latent, s.B, s.G);
+  hp->split.clear();
+  hp->tc.clear();
+  hp->cta_items.clear();
+  hp->cta_offsets.assign(1, 0);
+  hp->part_base.assign(s.F, 0);
+  hp->n_parts.assign(s.F, 0);
+  int slot = 0;
 
-  // ---- shared-prefix items (tensor cores): all forks of a trace x one kv head
-  // in one row tile (up to 128 rows), prefix cut into page-aligned chunks so
-  // that about one wave of CTAs (one per SM) covers every trace.
-  const int forks_per_item = std::max(1, 128 / s.G);
-  long long prefix_chunk = 0;
-  if (tc_prefix) {
-    long long work = 0;  // prefix tokens x kv heads x row tiles
+  if (tc) {
+    // Tensor-core path: the prefix of each trace is cut into chunks whose query
+    // rows are all forks of the trace (up to 128 rows per item); every suffix is
+    // cut into chunks of the same length.  The chunk length spreads the total
+    // token work over one persistent CTA per SM.
+    const int pg = fork_tc_page_size();
+    const int forks_per_item = std::max(1, 128 / s.G);
+    long long work = 0;
     for (int t = 0; t < s.T; ++t) {
       const int nf = fo[t + 1] - fo[t];
-      if (nf == 0) continue;
       work += (long long)lens->prefix_lens[t] * s.hkv * ((nf + forks_per_item - 1) / forks_per_item);
+      for (int f = fo[t]; f < fo[t + 1]; ++f) work += (long long)lens->suffix_lens[f] * s.hkv;
     }
-    const int pg = prefix_tc_page_size();
-    prefix_chunk = (work + n_sm - 1) / std::max(1, n_sm);
-    prefix_chunk = std::max<long long>(pg, (prefix_chunk + pg - 1) / pg * pg);
+    long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
+    chunk = std::max<long long>(fork_tc_tile_tokens(), (chunk + pg - 1) / pg * pg);
+    std::vector<long long> cost;
+    const long long item_overhead = 64;  // token-equivalents per item (Q load, output write)
+    for (int t = 0; t < s.T; ++t) {
+      const int P = lens->prefix_lens[t];
+      const int np = (int)((P + chunk - 1) / chunk);
+      for (int f = fo[t]; f < fo[t + 1]; ++f) {
+        const int S = lens->suffix_lens[f];
+        const int ns = (int)((S + chunk - 1) / chunk);
+        hp->part_base[f] = slot;
+        hp->n_parts[f] = np + ns;
+        slot += np + ns;
+        for (int g = 0; g < s.hkv; ++g)
+          for (int c = 0; c < ns; ++c) {
+            TcItem it;
+            it.table_kind = 1;
+            it.seq = f;
+            it.kv_head = g;
+            it.fork0 = f;
+            it.nforks = 1;
+            it.tok_begin = (int)(c * chunk);
+            it.tok_end = (int)std::min<long long>(S, (c + 1) * chunk);
+            it.part = np + c;
+            hp->tc.push_back(it);
+            cost.push_back(it.tok_end - it.tok_begin + item_overhead);
+          }
+      }
+      for (int g = 0; g < s.hkv; ++g)
+        for (int f0 = fo[t]; f0 < fo[t + 1]; f0 += forks_per_item)
+          for (int c = 0; c < np; ++c) {
+            TcItem it;
+            it.table_kind = 0;
+            it.seq = t;
+            it.kv_head = g;
+            it.fork0 = f0;
+            it.nforks = std::min(forks_per_item, fo[t + 1] - f0);
+            it.tok_begin = (int)(c * chunk);
+            it.tok_end = (int)std::min<long long>(P, (c + 1) * chunk);
+            it.part = c;
+            hp->tc.push_back(it);
+            cost.push_back(it.tok_end - it.tok_begin + item_overhead);
+          }
+    }
+    const int n_cta = (int)std::min<size_t>((size_t)n_sm, hp->tc.size());
+    assign_lpt(cost, n_cta, &hp->cta_items, &hp->cta_offsets);
+    hp->total_slots = slot;
+    return;
   }
 
-  // ---- split-K items: whatever the prefix kernel does not cover
+  // Split-K path (shapes the tensor-core kernel does not cover): every fork
+  // reads its trace's prefix and its own suffix in chunks of whole tiles.
   const int dvt = split_dv_tile(s.dqk, s.dv, s.latent);
   const int row_blocks = (s.G + kRowBlock - 1) / kRowBlock;
   const int dv_blocks = s.dv / dvt;
@@ -128,21 +211,14 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   long long split_tokens = 0;
   for (int t = 0; t < s.T; ++t)
     for (int f = fo[t]; f < fo[t + 1]; ++f)
-      split_tokens += (tc_prefix ? 0LL : (long long)lens->prefix_lens[t]) + lens->suffix_lens[f];
+      split_tokens += (long long)lens->prefix_lens[t] + lens->suffix_lens[f];
   const long long target_items = (long long)n_sm * 4;
   long long chunk = (split_tokens * units + target_items - 1) / std::max(1LL, target_items);
   chunk = std::max<long long>(kTileTokens, (chunk + kTileTokens - 1) / kTileTokens * kTileTokens);
   chunk = std::min<long long>(chunk, 1 << 20);
-
-  hp->split.clear();
-  hp->prefix.clear();
-  hp->part_base.assign(s.F, 0);
-  hp->n_parts.assign(s.F, 0);
-  int slot = 0;
   for (int t = 0; t < s.T; ++t) {
     const int P = lens->prefix_lens[t];
-    const long long pchunk = tc_prefix ? prefix_chunk : chunk;
-    const int np = (int)((P + pchunk - 1) / pchunk);
+    const int np = (int)((P + chunk - 1) / chunk);
     for (int f = fo[t]; f < fo[t + 1]; ++f) {
       const int S = lens->suffix_lens[f];
       const int ns = (int)((S + chunk - 1) / chunk);
@@ -157,55 +233,36 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
             it.h0 = g * s.G + rb * kRowBlock;
             it.nrows = std::min(kRowBlock, s.G - rb * kRowBlock);
             it.dv0 = db * dvt;
-            for (int c = 0; !tc_prefix && c < np; ++c) {
-              it.table_kind = 0;
-              it.seq = t;
-              it.tok_begin = (int)(c * chunk);
-              it.tok_end = (int)std::min<long long>(P, (c + 1) * chunk);
+            for (int c = 0; c < np + ns; ++c) {
+              const bool pre = c < np;
+              const int cc = pre ? c : c - np;
+              const int len = pre ? P : S;
+              it.table_kind = pre ? 0 : 1;
+              it.seq = pre ? t : f;
+              it.tok_begin = (int)(cc * chunk);
+              it.tok_end = (int)std::min<long long>(len, (cc + 1) * chunk);
               it.slot = slot + c;
-              hp->split.push_back(it);
-            }
-            for (int c = 0; c < ns; ++c) {
-              it.table_kind = 1;
-              it.seq = f;
-              it.tok_begin = (int)(c * chunk);
-              it.tok_end = (int)std::min<long long>(S, (c + 1) * chunk);
-              it.slot = slot + np + c;
               hp->split.push_back(it);
             }
           }
       slot += np + ns;
-    }
-    if (tc_prefix && np > 0) {
-      for (int g = 0; g < s.hkv; ++g)
-        for (int f0 = fo[t]; f0 < fo[t + 1]; f0 += forks_per_item)
-          for (int c = 0; c < np; ++c) {
-            PrefixItem it;
-            it.trace = t;
-            it.kv_head = g;
-            it.fork0 = f0;
-            it.nforks = std::min(forks_per_item, fo[t + 1] - f0);
-            it.tok_begin = (int)(c * prefix_chunk);
-            it.tok_end = (int)std::min<long long>(P, (c + 1) * prefix_chunk);
-            it.chunk = c;
-            it.dv0 = 0;
-            hp->prefix.push_back(it);
-          }
     }
   }
   hp->total_slots = slot;
 }
 
 struct Layout {
-  size_t split_off, prefix_off, part_base_off, n_parts_off, plan_bytes;
+  size_t split_off, tc_off, cta_items_off, cta_offsets_off, part_base_off, n_parts_off, plan_bytes;
   size_t ws_plan, ws_part_o, ws_part_lse, ws_end;
 };
 
 Layout layout_of(const Shape& s, const HostPlan& hp) {
   Layout L;
   L.split_off = align_up(sizeof(PlanHeader), 16);
-  L.prefix_off = align_up(L.split_off + hp.split.size() * sizeof(SplitItem), 16);
-  L.part_base_off = align_up(L.prefix_off + hp.prefix.size() * sizeof(PrefixItem), 16);
+  L.tc_off = align_up(L.split_off + hp.split.size() * sizeof(SplitItem), 16);
+  L.cta_items_off = align_up(L.tc_off + hp.tc.size() * sizeof(TcItem), 16);
+  L.cta_offsets_off = align_up(L.cta_items_off + hp.cta_items.size() * 4, 16);
+  L.part_base_off = align_up(L.cta_offsets_off + hp.cta_offsets.size() * 4, 16);
   L.n_parts_off = align_up(L.part_base_off + (size_t)s.F * 4, 16);
   L.plan_bytes = L.n_parts_off + (size_t)s.F * 4;
   L.ws_plan = kHeaderBytes;
@@ -248,21 +305,26 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   t_plan_bytes.assign(L.plan_bytes, 0);
   PlanHeader h;
   h.n_split = (int32_t)t_plan.split.size();
-  h.n_prefix = (int32_t)t_plan.prefix.size();
+  h.n_tc = (int32_t)t_plan.tc.size();
+  h.n_tc_ctas = (int32_t)t_plan.cta_offsets.size() - 1;
   h.n_forks = s.F;
-  h.hq = s.hq;
   h.split_off = (int32_t)L.split_off;
-  h.prefix_off = (int32_t)L.prefix_off;
+  h.tc_off = (int32_t)L.tc_off;
+  h.cta_items_off = (int32_t)L.cta_items_off;
+  h.cta_offsets_off = (int32_t)L.cta_offsets_off;
   h.part_base_off = (int32_t)L.part_base_off;
   h.n_parts_off = (int32_t)L.n_parts_off;
   unsigned char* b = t_plan_bytes.data();
   memcpy(b, &h, sizeof(h));
-  if (!t_plan.split.empty())
-    memcpy(b + L.split_off, t_plan.split.data(), t_plan.split.size() * sizeof(SplitItem));
-  if (!t_plan.prefix.empty())
-    memcpy(b + L.prefix_off, t_plan.prefix.data(), t_plan.prefix.size() * sizeof(PrefixItem));
-  memcpy(b + L.part_base_off, t_plan.part_base.data(), (size_t)s.F * 4);
-  memcpy(b + L.n_parts_off, t_plan.n_parts.data(), (size_t)s.F * 4);
+  auto put = [&](size_t off, const void* src, size_t bytes) {
+    if (bytes) memcpy(b + off, src, bytes);
+  };
+  put(L.split_off, t_plan.split.data(), t_plan.split.size() * sizeof(SplitItem));
+  put(L.tc_off, t_plan.tc.data(), t_plan.tc.size() * sizeof(TcItem));
+  put(L.cta_items_off, t_plan.cta_items.data(), t_plan.cta_items.size() * 4);
+  put(L.cta_offsets_off, t_plan.cta_offsets.data(), t_plan.cta_offsets.size() * 4);
+  put(L.part_base_off, t_plan.part_base.data(), (size_t)s.F * 4);
+  put(L.n_parts_off, t_plan.n_parts.data(), (size_t)s.F * 4);
 
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   unsigned char* ws = static_cast<unsigned char*>(args->workspace);
@@ -272,7 +334,8 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
     return SPECGEN_ERR_CUDA;
 
   plan->valid = 1;
-  plan->n_prefix_items = h.n_prefix;
+  plan->n_tc_items = h.n_tc;
+  plan->n_tc_ctas = h.n_tc_ctas;
   plan->n_split_items = h.n_split;
   plan->n_rows = s.F * s.hq;
   plan->total_slots = t_plan.total_slots;
@@ -282,10 +345,12 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   plan->ws_part_o_off = (int64_t)L.ws_part_o;
   plan->ws_part_lse_off = (int64_t)L.ws_part_lse;
   plan->ws_end = (int64_t)L.ws_end;
-  plan->reserved[0] = (int64_t)L.split_off;
-  plan->reserved[1] = (int64_t)L.prefix_off;
-  plan->reserved[2] = (int64_t)L.part_base_off;
-  plan->reserved[3] = (int64_t)L.n_parts_off;
+  plan->offsets[0] = (int64_t)L.split_off;
+  plan->offsets[1] = (int64_t)L.tc_off;
+  plan->offsets[2] = (int64_t)L.cta_items_off;
+  plan->offsets[3] = (int64_t)L.cta_offsets_off;
+  plan->offsets[4] = (int64_t)L.part_base_off;
+  plan->offsets[5] = (int64_t)L.n_parts_off;
   return SPECGEN_OK;
 }
 
@@ -353,7 +418,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   sp.prefix_bt_off = args->prefix_bt_offsets;
   sp.suffix_bt = args->suffix_block_table;
   sp.suffix_bt_off = args->suffix_bt_offsets;
-  sp.items = reinterpret_cast<const SplitItem*>(pl + plan->reserved[0]);
+  sp.items = reinterpret_cast<const SplitItem*>(pl + plan->offsets[0]);
   sp.part_o = part_o;
   sp.part_lse = part_lse;
   sp.status = reinterpret_cast<uint32_t*>(ws);
@@ -365,25 +430,28 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   sp.num_pages = args->num_pages;
   sp.scale_log2 = args->scale * 1.4426950408889634f;
   if (!marks.mark(stream, 0)) return SPECGEN_ERR_CUDA;
-  if (plan->n_prefix_items > 0) {
-    PrefixParams pp;
-    pp.q = sp.q;
-    pp.prefix_bt = args->prefix_block_table;
-    pp.prefix_bt_off = args->prefix_bt_offsets;
-    pp.items = reinterpret_cast<const PrefixItem*>(pl + plan->reserved[1]);
-    pp.part_base = reinterpret_cast<const int32_t*>(pl + plan->reserved[2]);
-    pp.part_o = part_o;
-    pp.part_lse = part_lse;
-    pp.status = sp.status;
-    pp.hq = args->hq;
-    pp.hkv = args->hkv;
-    pp.G = args->hq / args->hkv;
-    pp.dv = args->head_dim_v;
-    pp.page_size = args->page_size;
-    pp.num_pages = args->num_pages;
-    pp.scale_log2 = sp.scale_log2;
-    if (launch_prefix_tc(pp, args->k_pages, args->v_pages, plan->n_prefix_items,
-                         args->head_dim_qk, stream) != cudaSuccess)
+  if (plan->n_tc_ctas > 0) {
+    TcParams tp;
+    tp.q = sp.q;
+    tp.prefix_bt = args->prefix_block_table;
+    tp.prefix_bt_off = args->prefix_bt_offsets;
+    tp.suffix_bt = args->suffix_block_table;
+    tp.suffix_bt_off = args->suffix_bt_offsets;
+    tp.items = reinterpret_cast<const TcItem*>(pl + plan->offsets[1]);
+    tp.cta_items = reinterpret_cast<const int32_t*>(pl + plan->offsets[2]);
+    tp.cta_offsets = reinterpret_cast<const int32_t*>(pl + plan->offsets[3]);
+    tp.part_base = reinterpret_cast<const int32_t*>(pl + plan->offsets[4]);
+    tp.part_o = part_o;
+    tp.part_lse = part_lse;
+    tp.status = sp.status;
+    tp.hq = args->hq;
+    tp.hkv = args->hkv;
+    tp.G = args->hq / args->hkv;
+    tp.dv = args->head_dim_v;
+    tp.num_pages = args->num_pages;
+    tp.scale_log2 = sp.scale_log2;
+    if (launch_fork_tc(tp, args->k_pages, args->v_pages, plan->n_tc_ctas, args->head_dim_qk,
+                       stream) != cudaSuccess)
       return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
   }
@@ -397,8 +465,8 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   MergeParams mp;
   mp.part_o = part_o;
   mp.part_lse = part_lse;
-  mp.part_base = reinterpret_cast<const int32_t*>(pl + plan->reserved[2]);
-  mp.n_parts = reinterpret_cast<const int32_t*>(pl + plan->reserved[3]);
+  mp.part_base = reinterpret_cast<const int32_t*>(pl + plan->offsets[4]);
+  mp.n_parts = reinterpret_cast<const int32_t*>(pl + plan->offsets[5]);
   mp.out = static_cast<__nv_bfloat16*>(args->out);
   mp.lse = args->lse;
   mp.n_rows = plan->n_rows;

@@ -120,6 +120,7 @@ def test_shape_errors(w):
         S.SPECGEN_ERR_UNSUPPORTED
     assert _plan_status(_fake_args(w, page_size=12), lens) == S.SPECGEN_ERR_UNSUPPORTED
     assert _plan_status(_fake_args(w, scale=float("nan")), lens) == S.SPECGEN_ERR_SHAPE
+    assert _plan_status(_fake_args(w, scale=-0.125), lens) == S.SPECGEN_ERR_SHAPE
     bad, k1 = _lens(w, suffix_lens=np.array([1, -1, 2, 3], dtype=np.int32))
     assert _plan_status(_fake_args(w), bad) == S.SPECGEN_ERR_SHAPE
     bad, k2 = _lens(w, fork_offsets=np.array([0, 3], dtype=np.int32))              # != F
