@@ -103,9 +103,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto empty = [&](int s) { return bar0 + 16u + 8u * s; };
   auto s_full = [&](int b) { return bar0 + 32u + 8u * b; };
   auto p_full = [&](int b) { return bar0 + 48u + 8u * b; };
-  const uint32_t o_full = bar0 + 64u;
-  const uint32_t q_ready = bar0 + 72u;
-  const uint32_t mma_done = bar0 + 80u;
+  // PV_u done -> o_full[u%2]: one barrier per tile parity, so that a consumer
+  // that is up to one tile behind never sees a barrier two phases ahead
+  auto o_full = [&](int b) { return bar0 + 64u + 8u * b; };
+  const uint32_t q_ready = bar0 + 80u;
+  const uint32_t mma_done = bar0 + 88u;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 96);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + L::kOffBar + 100);
   auto sK = [&](int s) { return sKV + s * L::kStage; };
@@ -121,7 +123,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(s_full(i), 1);
       mbar_init(p_full(i), 128);
     }
-    mbar_init(o_full, 1);
+    mbar_init(o_full(0), 1);
+    mbar_init(o_full(1), 1);
     mbar_init(q_ready, 128);
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -207,7 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const uint64_t vd = smem_desc_sw128(sV(b) + kk * (kPB * 128u), kPanelBytes, 1024);
               mma_bf16(tmem + kTmemO, a, vd, idesc, (j > 1 || kk > 0) ? 1u : 0u);
             }
-            mma_commit(o_full);
+            mma_commit(o_full(b));
             mma_commit(empty(b));
           }
         }
@@ -226,7 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t s_base = tmem + lane_addr;
     const uint32_t o_base = tmem + lane_addr + kTmemO;
     const float sl2 = p.scale_log2;
-    int t = 0;
+    int t = 0, oc = 0;  // tiles done; next o_full phase to consume
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
       const TcItem it = p.items[p.cta_items[ii]];
@@ -252,6 +255,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_arrive(q_ready);
 
       float m = -INFINITY, l = 0.f;  // running max (log2 units) and sum of this row
+      // page ids of the next tile are fetched one tile ahead
+      int next_pages[kPagesPerTile];
+      auto fetch_pages = [&](int j) {
+        const int np = (tile_tokens(it, j) + kPB - 1) / kPB;
+#pragma unroll
+        for (int pg = 0; pg < kPagesPerTile; ++pg)
+          next_pages[pg] = pg < np ? v.table[v.page0 + j * kPagesPerTile + pg] : 0;
+      };
+      if (warp_live) fetch_pages(0);
       for (int j = 0; j < v.ntiles; ++j) {
         const int u = t + j, b = u & 1;
         const bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
@@ -260,6 +272,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
+        // S_u completing implies PV_{u-2} completed (same issuing thread, in
+        // order): consume those o_full phases without stalling
+        while (oc <= u - 2) {
+          mbar_wait(o_full(oc & 1), (oc >> 1) & 1, abort_flag, p.status);
+          ++oc;
+        }
         const int nt = tile_tokens(it, j);
         const int np = (nt + kPB - 1) / kPB;
         bool rescale = false;
@@ -267,21 +285,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (warp_live) {
           uint32_t pv = 0;  // valid pages of this tile
 #pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg) {
-            if (pg < np) {
-              const int page = v.table[v.page0 + j * kPagesPerTile + pg];
-              if (page >= 0 && page < p.num_pages) pv |= 1u << pg;
-            }
-          }
+          for (int pg = 0; pg < kPagesPerTile; ++pg)
+            if (pg < np && next_pages[pg] >= 0 && next_pages[pg] < p.num_pages) pv |= 1u << pg;
+          if (j + 1 < v.ntiles) fetch_pages(j + 1);
           float s[kTileTok];
           {
-            uint32_t r[16];
+            uint32_t r0[32], r1[32], r2[32], r3[32];
+            const uint32_t sa = s_base + (uint32_t)b * 128u;
+            tmem_ld32(sa, r0);
+            tmem_ld32(sa + 32u, r1);
+            tmem_ld32(sa + 64u, r2);
+            tmem_ld32(sa + 96u, r3);
+            tmem_wait_ld();
 #pragma unroll
-            for (int c = 0; c < kTileTok / 16; ++c) {
-              tmem_ld16(s_base + (uint32_t)b * 128u + c * 16u, r);
-              tmem_wait_ld();
-#pragma unroll
-              for (int i = 0; i < 16; ++i) s[c * 16 + i] = __uint_as_float(r[i]);
+            for (int i = 0; i < 32; ++i) {
+              s[i] = __uint_as_float(r0[i]);
+              s[32 + i] = __uint_as_float(r1[i]);
+              s[64 + i] = __uint_as_float(r2[i]);
+              s[96 + i] = __uint_as_float(r3[i]);
             }
           }
           const bool full_tile = nt == kTileTok && pv == 0xFFu;
@@ -290,10 +311,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < kTileTok; ++i)
               if (!(i < nt && ((pv >> (i / kPB)) & 1u))) s[i] = -INFINITY;
           }
-          float mx = s[0];
+          float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
 #pragma unroll
-          for (int i = 1; i < kTileTok; ++i) mx = fmaxf(mx, s[i]);
-          const float m_tile = mx * sl2;  // scale > 0
+          for (int i = 4; i < kTileTok; i += 4) {
+            mx0 = fmaxf(mx0, s[i]);
+            mx1 = fmaxf(mx1, s[i + 1]);
+            mx2 = fmaxf(mx2, s[i + 2]);
+            mx3 = fmaxf(mx3, s[i + 3]);
+          }
+          const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;  // scale > 0
           if (m_tile > m + kRescaleLog2 || (m == -INFINITY && m_tile != -INFINITY)) {
             alpha = m == -INFINITY ? 0.f : fast_exp2(m - m_tile);
             rescale = m != -INFINITY;
@@ -301,7 +327,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             m = m_tile;
           }
           const float sub = m == -INFINITY ? 0.f : m;
-          float psum = 0.f;
+          float ps0 = 0.f, ps1 = 0.f;
           const uint32_t prow = sP + b * L::kP + row * 128u;
 #pragma unroll
           for (int c = 0; c < kTileTok / 8; ++c) {  // 8 columns = one 16-byte chunk
@@ -310,13 +336,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 8; i += 2) {
               const float p0 = fast_exp2(fmaf(s[c * 8 + i], sl2, -sub));
               const float p1 = fast_exp2(fmaf(s[c * 8 + i + 1], sl2, -sub));
-              psum += p0 + p1;
+              ps0 += p0;
+              ps1 += p1;
               pk[i >> 1] = pack_bf16x2(p0, p1);
             }
             st_shared_v4(prow + (c >> 3) * kPanelBytes + (((c & 7) ^ (row & 7)) << 4), pk[0],
                          pk[1], pk[2], pk[3]);
           }
-          l += psum;
+          l += ps0 + ps1;
         }
         // value rows past the sequence inside its last page: zero them before PV
         if (j == v.ntiles - 1 && (nt % kPB) != 0) {
@@ -329,27 +356,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                              ((rem & 7) << 4), 0u, 0u, 0u, 0u);
           }
         }
-        // the previous PV must be done before the output is rescaled
-        if (j >= 1) {
-          const bool w2 = mbar_wait(o_full, (u - 1) & 1, abort_flag, p.status);
+        // a row whose max grew: the previous PV must be done, then rescale O in TMEM
+        if (j >= 1 && __any_sync(0xffffffffu, rescale)) {
+          bool w2 = true;
+          while (oc <= u - 1) {
+            w2 = w2 && mbar_wait(o_full(oc & 1), (oc >> 1) & 1, abort_flag, p.status);
+            ++oc;
+          }
           if (__any_sync(0xffffffffu, !w2)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          if (__any_sync(0xffffffffu, rescale)) {
-            const float a = rescale ? alpha : 1.f;
+          const float a = rescale ? alpha : 1.f;
 #pragma unroll
-            for (int c = 0; c < D / 16; ++c) {
-              uint32_t r[16];
-              tmem_ld16(o_base + c * 16u, r);
-              tmem_wait_ld();
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld32(o_base + c * 32u, r);
+            tmem_wait_ld();
 #pragma unroll
-              for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * a);
-              tmem_st16(o_base + c * 16u, r);
-            }
-            tmem_wait_st();
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * a);
+            tmem_st16(o_base + c * 32u, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+            tmem_st16(o_base + c * 32u + 16u, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
           }
+          tmem_wait_st();
         }
         tc_fence_before();
         fence_proxy_async_smem();
@@ -359,7 +389,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       // final output of the item: wait for the last PV, read O, normalise
       {
         const int u = t + v.ntiles - 1;
-        const bool w = mbar_wait(o_full, u & 1, abort_flag, p.status);
+        bool w = true;
+        while (oc <= u) {
+          w = w && mbar_wait(o_full(oc & 1), (oc >> 1) & 1, abort_flag, p.status);
+          ++oc;
+        }
         if (__any_sync(0xffffffffu, !w)) {
           ok = false;
           break;
@@ -371,14 +405,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           float4* dst = reinterpret_cast<float4*>(p.part_o + prow_out * p.dv);
           const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll
-          for (int c = 0; c < D / 16; ++c) {
-            uint32_t r[16];
-            tmem_ld16(o_base + c * 16u, r);
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld32(o_base + c * 32u, r);
             tmem_wait_ld();
             if (row_ok) {
 #pragma unroll
-              for (int i = 0; i < 16; i += 4)
-                dst[c * 4 + i / 4] = make_float4(
+              for (int i = 0; i < 32; i += 4)
+                dst[c * 8 + i / 4] = make_float4(
                     __uint_as_float(r[i]) * inv, __uint_as_float(r[i + 1]) * inv,
                     __uint_as_float(r[i + 2]) * inv, __uint_as_float(r[i + 3]) * inv);
             }

@@ -17,7 +17,7 @@ namespace specgen {
 
 namespace {
 
-constexpr int kMergeWarps = 8;
+constexpr int kMergeWarps = 4;
 
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
@@ -25,48 +25,87 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// One warp per (fork, head) row.  Lane i holds the LSE (and then the weight) of
+// part i, so the max and the normaliser are two warp reductions; the weighted
+// sum then streams the parts' rows with four independent loads in flight.
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_parts_kernel(const MergeParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x * kMergeWarps + warp;
   if (row >= p.n_rows) return;
   const int f = row / p.hq, h = row % p.hq;
   const int base = p.part_base[f], n = p.n_parts[f];
+  __nv_bfloat16* out = p.out + (size_t)row * p.dv;
 
   float m = -INFINITY;
   for (int i = lane; i < n; i += 32) m = fmaxf(m, p.part_lse[(size_t)(base + i) * p.hq + h]);
   m = warp_max(m);
-
-  __nv_bfloat16* out = p.out + (size_t)row * p.dv;
   if (m == -INFINITY) {  // no keys at all: O = 0, LSE = -inf
     for (int c = lane; c < p.dv; c += 32) out[c] = __float2bfloat16_rn(0.f);
     if (lane == 0) p.lse[row] = -INFINITY;
     return;
   }
   float wsum = 0.f;
-  for (int i = 0; i < n; ++i) {
-    float li = p.part_lse[(size_t)(base + i) * p.hq + h];
+  for (int i0 = 0; i0 < n; i0 += 32) {
+    const int i = i0 + lane;
+    const float li = i < n ? p.part_lse[(size_t)(base + i) * p.hq + h] : -INFINITY;
     wsum += li == -INFINITY ? 0.f : fast_exp2((li - m) * kLog2e);
   }
+  wsum = warp_sum(wsum);
   const float inv = 1.f / wsum;
-  for (int c4 = lane; c4 < p.dv / 4; c4 += 32) {
+  // every lane runs every iteration (the shuffles need the full warp); lanes
+  // past the row's last column load nothing and store nothing
+  for (int c0 = 0; c0 < p.dv / 4; c0 += 32) {
+    const int c4 = c0 + lane;
+    const bool active = c4 < p.dv / 4;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int i = 0; i < n; ++i) {
-      const size_t prow = (size_t)(base + i) * p.hq + h;
-      float li = p.part_lse[prow];
-      if (li == -INFINITY) continue;
-      float w = fast_exp2((li - m) * kLog2e);
-      float4 v = reinterpret_cast<const float4*>(p.part_o + prow * p.dv)[c4];
-      acc.x += w * v.x;
-      acc.y += w * v.y;
-      acc.z += w * v.z;
-      acc.w += w * v.w;
+    for (int i0 = 0; i0 < n; i0 += 32) {
+      const int i = i0 + lane;
+      const float li = i < n ? p.part_lse[(size_t)(base + i) * p.hq + h] : -INFINITY;
+      const float wl = li == -INFINITY ? 0.f : fast_exp2((li - m) * kLog2e);
+      const int cnt = n - i0 < 32 ? n - i0 : 32;
+      int k = 0;
+      for (; k + 4 <= cnt; k += 4) {
+        float w[4];
+        float4 v[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          w[e] = __shfl_sync(0xffffffffu, wl, k + e);
+          v[e] = active ? reinterpret_cast<const float4*>(
+                              p.part_o + ((size_t)(base + i0 + k + e) * p.hq + h) * p.dv)[c4]
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          if (w[e] == 0.f) continue;  // empty part: its row may hold anything
+          acc.x += w[e] * v[e].x;
+          acc.y += w[e] * v[e].y;
+          acc.z += w[e] * v[e].z;
+          acc.w += w[e] * v[e].w;
+        }
+      }
+      for (; k < cnt; ++k) {
+        const float we = __shfl_sync(0xffffffffu, wl, k);
+        if (we == 0.f || !active) continue;
+        const float4 v = reinterpret_cast<const float4*>(
+            p.part_o + ((size_t)(base + i0 + k) * p.hq + h) * p.dv)[c4];
+        acc.x += we * v.x;
+        acc.y += we * v.y;
+        acc.z += we * v.z;
+        acc.w += we * v.w;
+      }
     }
     __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
     __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
     uint2 packed;
     packed.x = *reinterpret_cast<uint32_t*>(&lo);
     packed.y = *reinterpret_cast<uint32_t*>(&hi);
-    reinterpret_cast<uint2*>(out)[c4] = packed;
+    if (active) reinterpret_cast<uint2*>(out)[c4] = packed;
   }
   if (lane == 0) p.lse[row] = m + log2f(wsum) * kLn2;
 }
