@@ -38,25 +38,29 @@ namespace {
 using namespace tc;
 
 constexpr int kPB = 16;                      // page size (tokens)
-constexpr int kTileTok = 128;                // tokens per tile
-constexpr int kPagesPerTile = kTileTok / kPB;
 constexpr uint32_t kPanelBytes = 128 * 128;  // 128 rows x 128 B (64 bf16 columns)
 constexpr int kThreads = 192;                // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
-constexpr uint32_t kTmemCols = 512;          // S0 [0,128) S1 [128,256) O [256, 256+D)
+constexpr uint32_t kTmemCols = 512;          // S0 [0,TT) S1 [TT,2TT) O [256, 256+D)
 constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleLog2 = 8.0f;         // lazy-rescale threshold (factor 256)
+constexpr int kMaxStages = 8;
+constexpr int kTile = 64;                    // tokens per pipeline tile (4 pages)
 
-template <int D>
+// Shared memory of one CTA: Q (M x D), a ring of `ST` (K, V) stages of TT
+// tokens, and two P buffers (M x TT); every operand tile is built of 128-row x
+// 128-byte panels (64 bf16 columns), 1024-byte aligned.
+template <int D, int TT, int ST>
 struct Smem {
   static constexpr int kPanels = D / 64;
+  static constexpr uint32_t kRowsTile = TT * 128u;        // one 64-column panel of TT rows
   static constexpr uint32_t kQ = kPanels * kPanelBytes;
-  static constexpr uint32_t kKV = kPanels * kPanelBytes;  // one K or V tile
+  static constexpr uint32_t kKV = kPanels * kRowsTile;    // one K or V tile
   static constexpr uint32_t kStage = 2 * kKV;
-  static constexpr uint32_t kP = 2 * kPanelBytes;         // 128 rows x 128 tokens
+  static constexpr uint32_t kP = (TT / 64) * kPanelBytes; // 128 rows x TT tokens
   static constexpr uint32_t kOffKV = kQ;
-  static constexpr uint32_t kOffP = kOffKV + 2 * kStage;
+  static constexpr uint32_t kOffP = kOffKV + ST * kStage;
   static constexpr uint32_t kOffBar = kOffP + 2 * kP;
-  static constexpr uint32_t kBytes = kOffBar + 128 + 1024;  // + barriers + alignment slack
+  static constexpr uint32_t kBytes = kOffBar + 256 + 1024;  // + barriers + alignment slack
 };
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
@@ -71,26 +75,30 @@ struct ItemView {
   int ntiles, page0, M;
 };
 
+template <int TT>
 __device__ __forceinline__ ItemView view(const TcParams& p, const TcItem& it) {
   ItemView v;
   v.table = it.table_kind == 0 ? p.prefix_bt + p.prefix_bt_off[it.seq]
                                : p.suffix_bt + p.suffix_bt_off[it.seq];
-  v.ntiles = (it.tok_end - it.tok_begin + kTileTok - 1) / kTileTok;
+  v.ntiles = (it.tok_end - it.tok_begin + TT - 1) / TT;
   v.page0 = it.tok_begin / kPB;
   v.M = it.nforks * p.G;
   return v;
 }
 
+template <int TT>
 __device__ __forceinline__ int tile_tokens(const TcItem& it, int j) {
-  const int n = it.tok_end - (it.tok_begin + j * kTileTok);
-  return n < kTileTok ? n : kTileTok;
+  const int n = it.tok_end - (it.tok_begin + j * TT);
+  return n < TT ? n : TT;
 }
 
-template <int D>
+template <int D, int TT, int ST>
 __global__ void __launch_bounds__(kThreads, 1)
     fork_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tmk,
                    const __grid_constant__ CUtensorMap tmv) {
-  using L = Smem<D>;
+  using L = Smem<D, TT, ST>;
+  constexpr int kTileTok = TT;
+  constexpr int kPagesPerTile = TT / kPB;
   extern __shared__ unsigned char smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // 128B-swizzled tiles: 1024-B aligned
@@ -99,17 +107,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sKV = base + L::kOffKV;
   const uint32_t sP = base + L::kOffP;
   const uint32_t bar0 = base + L::kOffBar;
+  // barrier block: full[ST] empty[ST] s_full[2] p_full[2] o_full[2] q_ready mma_done
   auto full = [&](int s) { return bar0 + 8u * s; };
-  auto empty = [&](int s) { return bar0 + 16u + 8u * s; };
-  auto s_full = [&](int b) { return bar0 + 32u + 8u * b; };
-  auto p_full = [&](int b) { return bar0 + 48u + 8u * b; };
+  auto empty = [&](int s) { return bar0 + 8u * (kMaxStages + s); };
+  auto s_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + b); };
+  auto p_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 2 + b); };
   // PV_u done -> o_full[u%2]: one barrier per tile parity, so that a consumer
   // that is up to one tile behind never sees a barrier two phases ahead
-  auto o_full = [&](int b) { return bar0 + 64u + 8u * b; };
-  const uint32_t q_ready = bar0 + 80u;
-  const uint32_t mma_done = bar0 + 88u;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 96);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + L::kOffBar + 100);
+  auto o_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 4 + b); };
+  const uint32_t q_ready = bar0 + 8u * (2 * kMaxStages + 6);
+  const uint32_t mma_done = bar0 + 8u * (2 * kMaxStages + 7);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 8));
+  volatile int* abort_flag =
+      reinterpret_cast<volatile int*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 8) + 4);
   auto sK = [&](int s) { return sKV + s * L::kStage; };
   auto sV = [&](int s) { return sKV + s * L::kStage + L::kKV; };
 
@@ -117,9 +127,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < ST; ++i) {
       mbar_init(full(i), 1);
       mbar_init(empty(i), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(s_full(i), 1);
       mbar_init(p_full(i), 128);
     }
@@ -146,11 +158,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int ii = it_begin; ok && ii < it_end; ++ii) {
         const TcItem it = p.items[p.cta_items[ii]];
-        const ItemView v = view(p, it);
+        const ItemView v = view<TT>(p, it);
         for (int j = 0; j < v.ntiles; ++j, ++t) {
-          const int s = t & 1;
-          if (!(ok = mbar_wait(empty(s), ((t >> 1) & 1) ^ 1, abort_flag, p.status))) break;
-          const int np = (tile_tokens(it, j) + kPB - 1) / kPB;
+          const int s = t % ST;
+          if (!(ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status))) break;
+          const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
           int pages[kPagesPerTile];  // fetch the tile's page ids before issuing any copy
 #pragma unroll
           for (int pg = 0; pg < kPagesPerTile; ++pg)
@@ -163,7 +175,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (page < 0 || page >= p.num_pages) atomicOr(p.status, kStatusIndex);  // zero-filled
 #pragma unroll
             for (int pn = 0; pn < L::kPanels; ++pn) {
-              const uint32_t off = pn * kPanelBytes + pg * (kPB * 128u);
+              const uint32_t off = pn * L::kRowsTile + pg * (kPB * 128u);
               tma_load_4d(sK(s) + off, &tmk, pn * 64, 0, it.kv_head, page, full(s));
               tma_load_4d(sV(s) + off, &tmv, pn * 64, 0, it.kv_head, page, full(s));
             }
@@ -171,7 +183,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       // never leave a copy in flight into this CTA's shared memory
-      for (int u = t - 2 < 0 ? 0 : t - 2; u < t; ++u) mbar_wait_drain(full(u & 1), (u >> 1) & 1, p.status);
+      for (int u = t - ST < 0 ? 0 : t - ST; u < t; ++u)
+        mbar_wait_drain(full(u % ST), (u / ST) & 1, p.status);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -180,38 +193,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int ii = it_begin; ok && ii < it_end; ++ii) {
         const TcItem it = p.items[p.cta_items[ii]];
-        const ItemView v = view(p, it);
+        const ItemView v = view<TT>(p, it);
         if (!(ok = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status))) break;
         tc_fence_after();
         for (int j = 0; j <= v.ntiles; ++j) {
           if (j < v.ntiles) {
-            const int u = t + j, s = u & 1;
-            if (!(ok = mbar_wait(full(s), (u >> 1) & 1, abort_flag, p.status))) break;
+            const int u = t + j, s = u % ST, b = u & 1;
+            if (!(ok = mbar_wait(full(s), (u / ST) & 1, abort_flag, p.status))) break;
             tc_fence_after();
-            const int np = (tile_tokens(it, j) + kPB - 1) / kPB;
+            const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
             const uint32_t idesc = idesc_bf16(128, np * kPB, false);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32u;
-              mma_bf16(tmem + (uint32_t)s * 128u, smem_desc_sw128(sQ + off, 16, 1024),
-                       smem_desc_sw128(sK(s) + off, 16, 1024), idesc, kk > 0 ? 1u : 0u);
+              const uint32_t qoff = (kk >> 2) * kPanelBytes + (kk & 3) * 32u;
+              const uint32_t koff = (kk >> 2) * L::kRowsTile + (kk & 3) * 32u;
+              mma_bf16(tmem + (uint32_t)b * TT, smem_desc_sw128(sQ + qoff, 16, 1024),
+                       smem_desc_sw128(sK(s) + koff, 16, 1024), idesc, kk > 0 ? 1u : 0u);
             }
-            mma_commit(s_full(s));
+            mma_commit(s_full(b));
           }
           if (j >= 1) {
-            const int u = t + j - 1, b = u & 1;
+            const int u = t + j - 1, b = u & 1, s = u % ST;
             if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
             tc_fence_after();
-            const int np = (tile_tokens(it, j - 1) + kPB - 1) / kPB;
+            const int np = (tile_tokens<TT>(it, j - 1) + kPB - 1) / kPB;
             constexpr uint32_t idesc = idesc_bf16(128, D, true);
             for (int kk = 0; kk < np; ++kk) {  // one page (16 tokens) per k-step
               const uint64_t a = smem_desc_sw128(sP + b * L::kP + (kk >> 2) * kPanelBytes +
                                                      (kk & 3) * 32u, 16, 1024);
-              const uint64_t vd = smem_desc_sw128(sV(b) + kk * (kPB * 128u), kPanelBytes, 1024);
+              const uint64_t vd =
+                  smem_desc_sw128(sV(s) + kk * (kPB * 128u), L::kRowsTile, 1024);
               mma_bf16(tmem + kTmemO, a, vd, idesc, (j > 1 || kk > 0) ? 1u : 0u);
             }
             mma_commit(o_full(b));
-            mma_commit(empty(b));
+            mma_commit(empty(s));
           }
         }
         t += v.ntiles;
@@ -233,7 +248,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
       const TcItem it = p.items[p.cta_items[ii]];
-      const ItemView v = view(p, it);
+      const ItemView v = view<TT>(p, it);
       const bool warp_live = q4 * 32 < v.M;  // some real row in this warp
       const bool row_ok = row < v.M;
       const int fl = row / p.G, gi = row % p.G;
@@ -258,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // page ids of the next tile are fetched one tile ahead
       int next_pages[kPagesPerTile];
       auto fetch_pages = [&](int j) {
-        const int np = (tile_tokens(it, j) + kPB - 1) / kPB;
+        const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
 #pragma unroll
         for (int pg = 0; pg < kPagesPerTile; ++pg)
           next_pages[pg] = pg < np ? v.table[v.page0 + j * kPagesPerTile + pg] : 0;
@@ -278,7 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_wait(o_full(oc & 1), (oc >> 1) & 1, abort_flag, p.status);
           ++oc;
         }
-        const int nt = tile_tokens(it, j);
+        const int nt = tile_tokens<TT>(it, j);
         const int np = (nt + kPB - 1) / kPB;
         bool rescale = false;
         float alpha = 1.f;
@@ -290,22 +305,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (j + 1 < v.ntiles) fetch_pages(j + 1);
           float s[kTileTok];
           {
-            uint32_t r0[32], r1[32], r2[32], r3[32];
-            const uint32_t sa = s_base + (uint32_t)b * 128u;
-            tmem_ld32(sa, r0);
-            tmem_ld32(sa + 32u, r1);
-            tmem_ld32(sa + 64u, r2);
-            tmem_ld32(sa + 96u, r3);
+            uint32_t r[kTileTok / 32][32];
+            const uint32_t sa = s_base + (uint32_t)b * TT;
+#pragma unroll
+            for (int c = 0; c < kTileTok / 32; ++c) tmem_ld32(sa + c * 32u, r[c]);
             tmem_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              s[i] = __uint_as_float(r0[i]);
-              s[32 + i] = __uint_as_float(r1[i]);
-              s[64 + i] = __uint_as_float(r2[i]);
-              s[96 + i] = __uint_as_float(r3[i]);
-            }
+            for (int c = 0; c < kTileTok / 32; ++c)
+#pragma unroll
+              for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[c][i]);
           }
-          const bool full_tile = nt == kTileTok && pv == 0xFFu;
+          const bool full_tile = nt == kTileTok && pv == (1u << kPagesPerTile) - 1u;
           if (!full_tile) {
 #pragma unroll
             for (int i = 0; i < kTileTok; ++i)
@@ -352,7 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int x = tid; x < units; x += 128) {
             const int rr = first + x / (L::kPanels * 8);
             const int rem = x % (L::kPanels * 8);
-            st_shared_v4(sV(b) + (rem >> 3) * kPanelBytes + (pg * kPB + rr) * 128u +
+            st_shared_v4(sV(u % ST) + (rem >> 3) * L::kRowsTile + (pg * kPB + rr) * 128u +
                              ((rem & 7) << 4), 0u, 0u, 0u, 0u);
           }
         }
@@ -467,12 +477,13 @@ bool make_pool_map(CUtensorMap* map, const void* pool, int D, int page, int hkv,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D>
+template <int D, int TT, int ST>
 cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap& mv, int grid,
                      cudaStream_t stream) {
-  constexpr int smem = (int)Smem<D>::kBytes;
+  constexpr int smem = (int)Smem<D, TT, ST>::kBytes;
   static_assert(smem <= 232448, "fork_tc kernel shared memory exceeds 227 KB");
-  auto kern = fork_tc_kernel<D>;
+  static_assert(ST <= kMaxStages && (TT == 64 || TT == 128), "unsupported pipeline shape");
+  auto kern = fork_tc_kernel<D, TT, ST>;
   static thread_local int configured = -1;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -492,7 +503,7 @@ bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G) {
   return !latent && dqk == dv && (dqk == 64 || dqk == 128) && page_size == kPB && G <= 128;
 }
 
-int fork_tc_tile_tokens() { return kTileTok; }
+int fork_tc_tile_tokens() { return kTile; }
 int fork_tc_page_size() { return kPB; }
 
 cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
@@ -502,8 +513,8 @@ cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v
   if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
       !make_pool_map(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
     return cudaErrorInvalidValue;
-  if (dqk == 128) return launch_d<128>(p, mk, mv, grid, stream);
-  if (dqk == 64) return launch_d<64>(p, mk, mv, grid, stream);
+  if (dqk == 128) return launch_d<128, kTile, 5>(p, mk, mv, grid, stream);
+  if (dqk == 64) return launch_d<64, kTile, 6>(p, mk, mv, grid, stream);
   return cudaErrorInvalidValue;
 }
 
