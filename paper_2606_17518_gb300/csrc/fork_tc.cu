@@ -153,39 +153,53 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      int t = 0;  // tiles issued so far (across items)
-      bool ok = true;
-      for (int ii = it_begin; ok && ii < it_end; ++ii) {
-        const TcItem it = p.items[p.cta_items[ii]];
-        const ItemView v = view<TT>(p, it);
-        for (int j = 0; j < v.ntiles; ++j, ++t) {
-          const int s = t % ST;
-          if (!(ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status))) break;
+    // The whole warp fetches page ids 32 at a time (one coalesced load, one
+    // batch ahead); lane 0 waits for free stages and issues the copies.
+    int t = 0;  // tiles issued so far (across items)
+    bool ok = true;
+    for (int ii = it_begin; ok && ii < it_end; ++ii) {
+      const TcItem it = p.items[p.cta_items[ii]];
+      const ItemView v = view<TT>(p, it);
+      const int npages = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
+      int cur = lane < npages ? v.table[v.page0 + lane] : 0;
+      for (int pb = 0; ok && pb < npages; pb += 32) {
+        const int nxt = pb + 32 + lane < npages ? v.table[v.page0 + pb + 32 + lane] : 0;
+        const int batch_pages = npages - pb < 32 ? npages - pb : 32;
+        for (int tp = 0; tp < batch_pages; tp += kPagesPerTile, ++t) {
+          const int j = (pb + tp) / kPagesPerTile;  // tile index within the item
           const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
-          int pages[kPagesPerTile];  // fetch the tile's page ids before issuing any copy
+          int pages[kPagesPerTile];
 #pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg)
-            pages[pg] = pg < np ? v.table[v.page0 + j * kPagesPerTile + pg] : 0;
-          mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
+          for (int pg = 0; pg < kPagesPerTile; ++pg) pages[pg] = __shfl_sync(0xffffffffu, cur, tp + pg);
+          const int s = t % ST;
+          if (lane == 0) {
+            ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
+            if (ok) {
+              mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
 #pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg) {
-            if (pg >= np) break;
-            const int page = pages[pg];
-            if (page < 0 || page >= p.num_pages) atomicOr(p.status, kStatusIndex);  // zero-filled
+              for (int pg = 0; pg < kPagesPerTile; ++pg) {
+                if (pg >= np) break;
+                const int page = pages[pg];
+                if (page < 0 || page >= p.num_pages) atomicOr(p.status, kStatusIndex);  // zero-filled
 #pragma unroll
-            for (int pn = 0; pn < L::kPanels; ++pn) {
-              const uint32_t off = pn * L::kRowsTile + pg * (kPB * 128u);
-              tma_load_4d(sK(s) + off, &tmk, pn * 64, 0, it.kv_head, page, full(s));
-              tma_load_4d(sV(s) + off, &tmv, pn * 64, 0, it.kv_head, page, full(s));
+                for (int pn = 0; pn < L::kPanels; ++pn) {
+                  const uint32_t off = pn * L::kRowsTile + pg * (kPB * 128u);
+                  tma_load_4d(sK(s) + off, &tmk, pn * 64, 0, it.kv_head, page, full(s));
+                  tma_load_4d(sV(s) + off, &tmv, pn * 64, 0, it.kv_head, page, full(s));
+                }
+              }
             }
           }
+          ok = __shfl_sync(0xffffffffu, ok, 0);
+          if (!ok) break;
         }
+        cur = nxt;
       }
-      // never leave a copy in flight into this CTA's shared memory
+    }
+    // never leave a copy in flight into this CTA's shared memory
+    if (lane == 0)
       for (int u = t - ST < 0 ? 0 : t - ST; u < t; ++u)
         mbar_wait_drain(full(u % ST), (u / ST) & 1, p.status);
-    }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -270,15 +284,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_arrive(q_ready);
 
       float m = -INFINITY, l = 0.f;  // running max (log2 units) and sum of this row
-      // page ids of the next tile are fetched one tile ahead
-      int next_pages[kPagesPerTile];
-      auto fetch_pages = [&](int j) {
-        const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
-#pragma unroll
-        for (int pg = 0; pg < kPagesPerTile; ++pg)
-          next_pages[pg] = pg < np ? v.table[v.page0 + j * kPagesPerTile + pg] : 0;
+      // page ids: 32 per coalesced warp load, one batch ahead (lane i holds page pb + i)
+      const int npages_item = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
+      auto load_batch = [&](int pb) {
+        return pb + lane < npages_item ? v.table[v.page0 + pb + lane] : 0;
       };
-      if (warp_live) fetch_pages(0);
+      int cur_pages = load_batch(0), nxt_pages = load_batch(32);
       for (int j = 0; j < v.ntiles; ++j) {
         const int u = t + j, b = u & 1;
         const bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
@@ -295,14 +306,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const int nt = tile_tokens<TT>(it, j);
         const int np = (nt + kPB - 1) / kPB;
+        const int tp0 = (j * kPagesPerTile) & 31;  // first page of this tile within the batch
+        if (j > 0 && tp0 == 0) {                     // entering the next batch of 32 pages
+          cur_pages = nxt_pages;
+          nxt_pages = load_batch(j * kPagesPerTile + 32);
+        }
         bool rescale = false;
         float alpha = 1.f;
         if (warp_live) {
           uint32_t pv = 0;  // valid pages of this tile
 #pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg)
-            if (pg < np && next_pages[pg] >= 0 && next_pages[pg] < p.num_pages) pv |= 1u << pg;
-          if (j + 1 < v.ntiles) fetch_pages(j + 1);
+          for (int pg = 0; pg < kPagesPerTile; ++pg) {
+            const int page = __shfl_sync(0xffffffffu, cur_pages, (tp0 + pg) & 31);
+            if (pg < np && page >= 0 && page < p.num_pages) pv |= 1u << pg;
+          }
           float s[kTileTok];
           {
             uint32_t r[kTileTok / 32][32];
