@@ -38,28 +38,24 @@ namespace {
 using namespace tc;
 
 constexpr int kPB = 16;                      // page size (tokens)
-constexpr uint32_t kPanelBytes = 128 * 128;  // 128 rows x 128 B (64 bf16 columns)
 constexpr int kThreads = 192;                // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
-constexpr uint32_t kTmemCols = 512;          // S0 [0,TT) S1 [TT,2TT) O [256, 256+D)
-constexpr uint32_t kTmemO = 256;
+constexpr uint32_t kTmemCols = 512;          // S0 [0,TT) S1 [TT,2TT) Q [256,..) O [384,..)
+constexpr uint32_t kTmemQ = 256;
+constexpr uint32_t kTmemO = 384;
 constexpr float kRescaleLog2 = 8.0f;         // lazy-rescale threshold (factor 256)
 constexpr int kMaxStages = 8;
 constexpr int kTile = 64;                    // tokens per pipeline tile (4 pages)
 
-// Shared memory of one CTA: Q (M x D), a ring of `ST` (K, V) stages of TT
-// tokens, and two P buffers (M x TT); every operand tile is built of 128-row x
-// 128-byte panels (64 bf16 columns), 1024-byte aligned.
+// Shared memory of one CTA: a ring of `ST` (K, V) stages of TT tokens.  Each
+// K or V tile is D/64 panels of TT rows x 128 bytes (64 bf16 columns,
+// 128B-swizzled by TMA), 1024-byte aligned.  Q and P live in tensor memory.
 template <int D, int TT, int ST>
 struct Smem {
   static constexpr int kPanels = D / 64;
   static constexpr uint32_t kRowsTile = TT * 128u;        // one 64-column panel of TT rows
-  static constexpr uint32_t kQ = kPanels * kPanelBytes;
   static constexpr uint32_t kKV = kPanels * kRowsTile;    // one K or V tile
   static constexpr uint32_t kStage = 2 * kKV;
-  static constexpr uint32_t kP = (TT / 64) * kPanelBytes; // 128 rows x TT tokens
-  static constexpr uint32_t kOffKV = kQ;
-  static constexpr uint32_t kOffP = kOffKV + ST * kStage;
-  static constexpr uint32_t kOffBar = kOffP + 2 * kP;
+  static constexpr uint32_t kOffBar = ST * kStage;
   static constexpr uint32_t kBytes = kOffBar + 256 + 1024;  // + barriers + alignment slack
 };
 
@@ -97,15 +93,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     fork_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tmk,
                    const __grid_constant__ CUtensorMap tmv) {
   using L = Smem<D, TT, ST>;
-  constexpr int kTileTok = TT;
   constexpr int kPagesPerTile = TT / kPB;
   extern __shared__ unsigned char smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // 128B-swizzled tiles: 1024-B aligned
   unsigned char* gbase = smem_raw + (base - raw);
-  const uint32_t sQ = base;
-  const uint32_t sKV = base + L::kOffKV;
-  const uint32_t sP = base + L::kOffP;
   const uint32_t bar0 = base + L::kOffBar;
   // barrier block: full[ST] empty[ST] s_full[2] p_full[2] o_full[2] q_ready mma_done
   auto full = [&](int s) { return bar0 + 8u * s; };
@@ -120,8 +112,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 8));
   volatile int* abort_flag =
       reinterpret_cast<volatile int*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 8) + 4);
-  auto sK = [&](int s) { return sKV + s * L::kStage; };
-  auto sV = [&](int s) { return sKV + s * L::kStage + L::kKV; };
+  auto sK = [&](int s) { return base + s * L::kStage; };
+  auto sV = [&](int s) { return base + s * L::kStage + L::kKV; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
@@ -134,9 +126,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(s_full(i), 1);
       mbar_init(p_full(i), 128);
+      mbar_init(o_full(i), 1);
     }
-    mbar_init(o_full(0), 1);
-    mbar_init(o_full(1), 1);
     mbar_init(q_ready, 128);
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -154,7 +145,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     // The whole warp fetches page ids 32 at a time (one coalesced load, one
-    // batch ahead); lane 0 waits for free stages and issues the copies.
+    // batch ahead).  Lane 0 waits for a free stage; then lanes 0..2*D/64-1
+    // each issue one box of every page (K and V, one 64-column panel each), so
+    // a page's boxes leave in one instruction.
+    constexpr int kIssuers = 2 * L::kPanels;
+    const bool issuer = lane < kIssuers;
+    const bool is_v = lane >= L::kPanels;
+    const int pn = is_v ? lane - L::kPanels : lane;
+    const void* tmap = is_v ? static_cast<const void*>(&tmv) : static_cast<const void*>(&tmk);
     int t = 0;  // tiles issued so far (across items)
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
@@ -170,28 +168,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
           int pages[kPagesPerTile];
 #pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg) pages[pg] = __shfl_sync(0xffffffffu, cur, tp + pg);
+          for (int pg = 0; pg < kPagesPerTile; ++pg)
+            pages[pg] = __shfl_sync(0xffffffffu, cur, tp + pg);
           const int s = t % ST;
           if (lane == 0) {
             ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
-            if (ok) {
-              mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
-#pragma unroll
-              for (int pg = 0; pg < kPagesPerTile; ++pg) {
-                if (pg >= np) break;
-                const int page = pages[pg];
-                if (page < 0 || page >= p.num_pages) atomicOr(p.status, kStatusIndex);  // zero-filled
-#pragma unroll
-                for (int pn = 0; pn < L::kPanels; ++pn) {
-                  const uint32_t off = pn * L::kRowsTile + pg * (kPB * 128u);
-                  tma_load_4d(sK(s) + off, &tmk, pn * 64, 0, it.kv_head, page, full(s));
-                  tma_load_4d(sV(s) + off, &tmv, pn * 64, 0, it.kv_head, page, full(s));
-                }
-              }
-            }
+            if (ok) mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
           }
           ok = __shfl_sync(0xffffffffu, ok, 0);
           if (!ok) break;
+          if (issuer) {
+            const uint32_t dst = (is_v ? sV(s) : sK(s)) + pn * L::kRowsTile;
+#pragma unroll
+            for (int pg = 0; pg < kPagesPerTile; ++pg) {
+              if (pg >= np) break;
+              tma_load_4d(dst + pg * (kPB * 128u), tmap, pn * 64, 0, it.kv_head, pages[pg], full(s));
+            }
+          }
+          if (lane == 0)
+            for (int pg = 0; pg < np; ++pg)
+              if (pages[pg] < 0 || pages[pg] >= p.num_pages)
+                atomicOr(p.status, kStatusIndex);  // TMA zero-fills out-of-range pages
         }
         cur = nxt;
       }
@@ -211,7 +208,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status))) break;
         tc_fence_after();
         for (int j = 0; j <= v.ntiles; ++j) {
-          if (j < v.ntiles) {
+          if (j < v.ntiles) {  // S_u = Q K_u^T (A = Q from TMEM, B = K tile)
             const int u = t + j, s = u % ST, b = u & 1;
             if (!(ok = mbar_wait(full(s), (u / ST) & 1, abort_flag, p.status))) break;
             tc_fence_after();
@@ -219,25 +216,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t idesc = idesc_bf16(128, np * kPB, false);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t qoff = (kk >> 2) * kPanelBytes + (kk & 3) * 32u;
               const uint32_t koff = (kk >> 2) * L::kRowsTile + (kk & 3) * 32u;
-              mma_bf16(tmem + (uint32_t)b * TT, smem_desc_sw128(sQ + qoff, 16, 1024),
-                       smem_desc_sw128(sK(s) + koff, 16, 1024), idesc, kk > 0 ? 1u : 0u);
+              mma_bf16_ts(tmem + (uint32_t)b * TT, tmem + kTmemQ + kk * 8u,
+                          smem_desc_sw128(sK(s) + koff, 16, 1024), idesc, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
           }
-          if (j >= 1) {
+          if (j >= 1) {  // O += P_u V_u (A = P from TMEM over S_u, B = V tile)
             const int u = t + j - 1, b = u & 1, s = u % ST;
             if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
             tc_fence_after();
             const int np = (tile_tokens<TT>(it, j - 1) + kPB - 1) / kPB;
             constexpr uint32_t idesc = idesc_bf16(128, D, true);
             for (int kk = 0; kk < np; ++kk) {  // one page (16 tokens) per k-step
-              const uint64_t a = smem_desc_sw128(sP + b * L::kP + (kk >> 2) * kPanelBytes +
-                                                     (kk & 3) * 32u, 16, 1024);
               const uint64_t vd =
                   smem_desc_sw128(sV(s) + kk * (kPB * 128u), L::kRowsTile, 1024);
-              mma_bf16(tmem + kTmemO, a, vd, idesc, (j > 1 || kk > 0) ? 1u : 0u);
+              mma_bf16_ts(tmem + kTmemO, tmem + (uint32_t)b * TT + kk * 8u, vd, idesc,
+                          (j > 1 || kk > 0) ? 1u : 0u);
             }
             mma_commit(o_full(b));
             mma_commit(empty(s));
@@ -268,18 +263,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int fl = row / p.G, gi = row % p.G;
       const int head = it.kv_head * p.G + gi;
 
-      // Q rows -> shared memory (128B-swizzled K-major); padding rows are zero
+      // Q row -> tensor memory (lane = row, two bf16 per column); padding rows are zero
       if (warp_live) {
         const uint4* src = reinterpret_cast<const uint4*>(
             p.q + ((size_t)(it.fork0 + (row_ok ? fl : 0)) * p.hq + (row_ok ? head : 0)) * D);
 #pragma unroll
-        for (int c = 0; c < D / 8; ++c) {
-          uint4 q = row_ok ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
-          st_shared_v4(sQ + (c >> 3) * kPanelBytes + row * 128u + (((c & 7) ^ (row & 7)) << 4),
-                       q.x, q.y, q.z, q.w);
+        for (int c = 0; c < D / 64; ++c) {
+          uint32_t r[32];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const uint4 q = row_ok ? __ldg(src + c * 8 + e) : make_uint4(0, 0, 0, 0);
+            r[4 * e] = q.x;
+            r[4 * e + 1] = q.y;
+            r[4 * e + 2] = q.z;
+            r[4 * e + 3] = q.w;
+          }
+          tmem_st32(s_base + kTmemQ + c * 32u, r);
         }
+        tmem_wait_st();
       }
-      fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(q_ready);
 
@@ -320,27 +322,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int page = __shfl_sync(0xffffffffu, cur_pages, (tp0 + pg) & 31);
             if (pg < np && page >= 0 && page < p.num_pages) pv |= 1u << pg;
           }
-          float s[kTileTok];
+          float s[TT];
           {
-            uint32_t r[kTileTok / 32][32];
+            uint32_t r[TT / 32][32];
             const uint32_t sa = s_base + (uint32_t)b * TT;
 #pragma unroll
-            for (int c = 0; c < kTileTok / 32; ++c) tmem_ld32(sa + c * 32u, r[c]);
+            for (int c = 0; c < TT / 32; ++c) tmem_ld32(sa + c * 32u, r[c]);
             tmem_wait_ld();
 #pragma unroll
-            for (int c = 0; c < kTileTok / 32; ++c)
+            for (int c = 0; c < TT / 32; ++c)
 #pragma unroll
               for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[c][i]);
           }
-          const bool full_tile = nt == kTileTok && pv == (1u << kPagesPerTile) - 1u;
+          const bool full_tile = nt == TT && pv == (1u << kPagesPerTile) - 1u;
           if (!full_tile) {
 #pragma unroll
-            for (int i = 0; i < kTileTok; ++i)
+            for (int i = 0; i < TT; ++i)
               if (!(i < nt && ((pv >> (i / kPB)) & 1u))) s[i] = -INFINITY;
           }
           float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
 #pragma unroll
-          for (int i = 4; i < kTileTok; i += 4) {
+          for (int i = 4; i < TT; i += 4) {
             mx0 = fmaxf(mx0, s[i]);
             mx1 = fmaxf(mx1, s[i + 1]);
             mx2 = fmaxf(mx2, s[i + 2]);
@@ -355,21 +357,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const float sub = m == -INFINITY ? 0.f : m;
           float ps0 = 0.f, ps1 = 0.f;
-          const uint32_t prow = sP + b * L::kP + row * 128u;
+          // P_u (bf16 pairs) over the first TT/2 columns of S_u's TMEM buffer
 #pragma unroll
-          for (int c = 0; c < kTileTok / 8; ++c) {  // 8 columns = one 16-byte chunk
-            uint32_t pk[4];
+          for (int c = 0; c < TT / 64; ++c) {
+            uint32_t pk[32];
 #pragma unroll
-            for (int i = 0; i < 8; i += 2) {
-              const float p0 = fast_exp2(fmaf(s[c * 8 + i], sl2, -sub));
-              const float p1 = fast_exp2(fmaf(s[c * 8 + i + 1], sl2, -sub));
+            for (int i = 0; i < 32; ++i) {
+              const float p0 = fast_exp2(fmaf(s[c * 64 + 2 * i], sl2, -sub));
+              const float p1 = fast_exp2(fmaf(s[c * 64 + 2 * i + 1], sl2, -sub));
               ps0 += p0;
               ps1 += p1;
-              pk[i >> 1] = pack_bf16x2(p0, p1);
+              pk[i] = pack_bf16x2(p0, p1);
             }
-            st_shared_v4(prow + (c >> 3) * kPanelBytes + (((c & 7) ^ (row & 7)) << 4), pk[0],
-                         pk[1], pk[2], pk[3]);
+            tmem_st32(s_base + (uint32_t)b * TT + c * 32u, pk);
           }
+          tmem_wait_st();
           l += ps0 + ps1;
         }
         // value rows past the sequence inside its last page: zero them before PV
@@ -382,6 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             st_shared_v4(sV(u % ST) + (rem >> 3) * L::kRowsTile + (pg * kPB + rr) * 128u +
                              ((rem & 7) << 4), 0u, 0u, 0u, 0u);
           }
+          fence_proxy_async_smem();
         }
         // a row whose max grew: the previous PV must be done, then rescale O in TMEM
         if (j >= 1 && __any_sync(0xffffffffu, rescale)) {
@@ -403,13 +406,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * a);
-            tmem_st16(o_base + c * 32u, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-            tmem_st16(o_base + c * 32u + 16u, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+            tmem_st32(o_base + c * 32u, r);
           }
           tmem_wait_st();
         }
         tc_fence_before();
-        fence_proxy_async_smem();
         mbar_arrive(p_full(b));
       }
       if (!ok) break;
@@ -446,6 +447,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (row_ok) p.part_lse[prow_out] = m == -INFINITY ? -INFINITY : (m + log2f(l)) * kLn2;
         }
+        // the next item's Q overwrites this item's Q in TMEM only after this point
+        tc_fence_before();
       }
       t += v.ntiles;
     }
@@ -530,8 +533,8 @@ cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v
   if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
       !make_pool_map(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
     return cudaErrorInvalidValue;
-  if (dqk == 128) return launch_d<128, kTile, 5>(p, mk, mv, grid, stream);
-  if (dqk == 64) return launch_d<64, kTile, 6>(p, mk, mv, grid, stream);
+  if (dqk == 128) return launch_d<128, kTile, 6>(p, mk, mv, grid, stream);
+  if (dqk == 64) return launch_d<64, kTile, 8>(p, mk, mv, grid, stream);
   return cudaErrorInvalidValue;
 }
 
