@@ -38,25 +38,29 @@ namespace {
 using namespace tc;
 
 constexpr int kPB = 16;                      // page size (tokens)
-constexpr int kThreads = 192;                // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
-constexpr uint32_t kTmemCols = 512;          // S0 [0,TT) S1 [TT,2TT) Q [256,..) O [384,..)
-constexpr uint32_t kTmemQ = 256;
-constexpr uint32_t kTmemO = 384;
+constexpr int kWG = 2;                       // softmax warpgroups (alternating tiles)
+constexpr int kThreads = 64 + 128 * kWG;     // warp 0 TMA, warp 1 MMA, 4 warps per softmax group
+constexpr uint32_t kTmemCols = 512;          // S[0] [0,TT) S[1] [TT,2TT) O[0] [256,..) O[1] [384,..)
+constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleLog2 = 8.0f;         // lazy-rescale threshold (factor 256)
 constexpr int kMaxStages = 8;
-constexpr int kTile = 64;                    // tokens per pipeline tile (4 pages)
+constexpr int kTile = 128;                   // tokens per pipeline tile (8 pages)
 
-// Shared memory of one CTA: a ring of `ST` (K, V) stages of TT tokens.  Each
-// K or V tile is D/64 panels of TT rows x 128 bytes (64 bf16 columns,
-// 128B-swizzled by TMA), 1024-byte aligned.  Q and P live in tensor memory.
+// Shared memory of one CTA: Q (128 rows x D) and a ring of `ST` (K, V) stages of
+// TT tokens.  Every operand tile is made of 64-column panels (128-byte rows,
+// 128B-swizzled), 1024-byte aligned.  P lives in tensor memory.
 template <int D, int TT, int ST>
 struct Smem {
   static constexpr int kPanels = D / 64;
+  static constexpr uint32_t kQPanel = 128 * 128u;         // 128 rows x 128 B
+  static constexpr uint32_t kQ = kPanels * kQPanel;
   static constexpr uint32_t kRowsTile = TT * 128u;        // one 64-column panel of TT rows
   static constexpr uint32_t kKV = kPanels * kRowsTile;    // one K or V tile
   static constexpr uint32_t kStage = 2 * kKV;
-  static constexpr uint32_t kOffBar = ST * kStage;
-  static constexpr uint32_t kBytes = kOffBar + 256 + 1024;  // + barriers + alignment slack
+  static constexpr uint32_t kOffKV = kQ;
+  static constexpr uint32_t kOffBar = kOffKV + ST * kStage;
+  static constexpr uint32_t kOffML = kOffBar + 256;        // 128 x (m, l) of the second group
+  static constexpr uint32_t kBytes = kOffML + 128 * 8 + 1024;
 };
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
@@ -65,7 +69,6 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
                "r"(d)
                : "memory");
 }
-
 struct ItemView {
   const int32_t* table;
   int ntiles, page0, M;
@@ -94,26 +97,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                    const __grid_constant__ CUtensorMap tmv) {
   using L = Smem<D, TT, ST>;
   constexpr int kPagesPerTile = TT / kPB;
+  static_assert(32 % kPagesPerTile == 0, "a batch of 32 page ids holds whole tiles");
   extern __shared__ unsigned char smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // 128B-swizzled tiles: 1024-B aligned
   unsigned char* gbase = smem_raw + (base - raw);
+  const uint32_t sQ = base;
   const uint32_t bar0 = base + L::kOffBar;
   // barrier block: full[ST] empty[ST] s_full[2] p_full[2] o_full[2] q_ready mma_done
   auto full = [&](int s) { return bar0 + 8u * s; };
   auto empty = [&](int s) { return bar0 + 8u * (kMaxStages + s); };
   auto s_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + b); };
   auto p_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 2 + b); };
-  // PV_u done -> o_full[u%2]: one barrier per tile parity, so that a consumer
-  // that is up to one tile behind never sees a barrier two phases ahead
   auto o_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 4 + b); };
   const uint32_t q_ready = bar0 + 8u * (2 * kMaxStages + 6);
   const uint32_t mma_done = bar0 + 8u * (2 * kMaxStages + 7);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 8));
+  const uint32_t ml_ready = bar0 + 8u * (2 * kMaxStages + 8);  // group 1's (m, l) written
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 9));
   volatile int* abort_flag =
-      reinterpret_cast<volatile int*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 8) + 4);
-  auto sK = [&](int s) { return base + s * L::kStage; };
-  auto sV = [&](int s) { return base + s * L::kStage + L::kKV; };
+      reinterpret_cast<volatile int*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 9) + 4);
+  float2* ml1 = reinterpret_cast<float2*>(gbase + L::kOffML);  // second group's (m, l) per row
+  auto sK = [&](int s) { return base + L::kOffKV + s * L::kStage; };
+  auto sV = [&](int s) { return base + L::kOffKV + s * L::kStage + L::kKV; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
@@ -130,6 +135,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(q_ready, 128);
     mbar_init(mma_done, 1);
+    mbar_init(ml_ready, 128);
     *abort_flag = 0;
     mbar_init_fence();
   }
@@ -146,8 +152,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ TMA producer
     // The whole warp fetches page ids 32 at a time (one coalesced load, one
     // batch ahead).  Lane 0 waits for a free stage; then lanes 0..2*D/64-1
-    // each issue one box of every page (K and V, one 64-column panel each), so
-    // a page's boxes leave in one instruction.
+    // each issue one box of every page (K and V, one 64-column panel each).
     constexpr int kIssuers = 2 * L::kPanels;
     const bool issuer = lane < kIssuers;
     const bool is_v = lane >= L::kPanels;
@@ -208,7 +213,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status))) break;
         tc_fence_after();
         for (int j = 0; j <= v.ntiles; ++j) {
-          if (j < v.ntiles) {  // S_u = Q K_u^T (A = Q from TMEM, B = K tile)
+          if (j < v.ntiles) {  // S_u = Q K_u^T -> S[u%2]
             const int u = t + j, s = u % ST, b = u & 1;
             if (!(ok = mbar_wait(full(s), (u / ST) & 1, abort_flag, p.status))) break;
             tc_fence_after();
@@ -216,23 +221,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t idesc = idesc_bf16(128, np * kPB, false);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t qoff = (kk >> 2) * L::kQPanel + (kk & 3) * 32u;
               const uint32_t koff = (kk >> 2) * L::kRowsTile + (kk & 3) * 32u;
-              mma_bf16_ts(tmem + (uint32_t)b * TT, tmem + kTmemQ + kk * 8u,
-                          smem_desc_sw128(sK(s) + koff, 16, 1024), idesc, kk > 0 ? 1u : 0u);
+              mma_bf16(tmem + (uint32_t)b * TT, smem_desc_sw128(sQ + qoff, 16, 1024),
+                       smem_desc_sw128(sK(s) + koff, 16, 1024), idesc, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
           }
-          if (j >= 1) {  // O += P_u V_u (A = P from TMEM over S_u, B = V tile)
-            const int u = t + j - 1, b = u & 1, s = u % ST;
+          if (j >= 1) {  // O[u%2] += P_u V_u (P_u in TMEM over S_u)
+            const int jj = j - 1, u = t + jj, b = u & 1, s = u % ST;
             if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
             tc_fence_after();
-            const int np = (tile_tokens<TT>(it, j - 1) + kPB - 1) / kPB;
+            const int np = (tile_tokens<TT>(it, jj) + kPB - 1) / kPB;
             constexpr uint32_t idesc = idesc_bf16(128, D, true);
+            const uint32_t o_tmem = tmem + kTmemO + (uint32_t)(jj & 1) * 128u;
             for (int kk = 0; kk < np; ++kk) {  // one page (16 tokens) per k-step
               const uint64_t vd =
                   smem_desc_sw128(sV(s) + kk * (kPB * 128u), L::kRowsTile, 1024);
-              mma_bf16_ts(tmem + kTmemO, tmem + (uint32_t)b * TT + kk * 8u, vd, idesc,
-                          (j > 1 || kk > 0) ? 1u : 0u);
+              mma_bf16_ts(o_tmem, tmem + (uint32_t)b * TT + kk * 8u, vd, idesc,
+                          (jj >= 2 || kk > 0) ? 1u : 0u);
             }
             mma_commit(o_full(b));
             mma_commit(empty(s));
@@ -245,15 +252,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_drain(mma_done, 0, p.status);
     }
   } else {
-    // ------------------------------------------------------------ softmax warps
+    // ------------------------------------------------------------ softmax groups
+    // Group g (warps 2+4g .. 5+4g) takes the tiles j = g, g+2, ... of every item
+    // with its own running max/sum and its own TMEM output O[g]; group 0 merges
+    // the two halves at the end of the item.
+    const int grp = (warp - 2) >> 2;
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
-    const int tid = threadIdx.x - 64;  // 0..127
+    const int gtid = (threadIdx.x - 64) & 127;  // 0..127 within the group
     const uint32_t lane_addr = (uint32_t)(q4 * 32) << 16;
     const uint32_t s_base = tmem + lane_addr;
-    const uint32_t o_base = tmem + lane_addr + kTmemO;
+    const uint32_t o_mine = tmem + lane_addr + kTmemO + (uint32_t)grp * 128u;
     const float sl2 = p.scale_log2;
-    int t = 0, oc = 0;  // tiles done; next o_full phase to consume
+    int t = 0;
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
       const TcItem it = p.items[p.cta_items[ii]];
@@ -263,36 +274,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int fl = row / p.G, gi = row % p.G;
       const int head = it.kv_head * p.G + gi;
 
-      // Q row -> tensor memory (lane = row, two bf16 per column); padding rows are zero
-      if (warp_live) {
+      if (grp == 0) {
+        // Q row -> shared memory, 128B-swizzled K-major panels; padding rows are zero
         const uint4* src = reinterpret_cast<const uint4*>(
             p.q + ((size_t)(it.fork0 + (row_ok ? fl : 0)) * p.hq + (row_ok ? head : 0)) * D);
+        if (warp_live) {
 #pragma unroll
-        for (int c = 0; c < D / 64; ++c) {
-          uint32_t r[32];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const uint4 q = row_ok ? __ldg(src + c * 8 + e) : make_uint4(0, 0, 0, 0);
-            r[4 * e] = q.x;
-            r[4 * e + 1] = q.y;
-            r[4 * e + 2] = q.z;
-            r[4 * e + 3] = q.w;
+          for (int c = 0; c < D / 8; ++c) {
+            const uint4 q = row_ok ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+            st_shared_v4(sQ + (c >> 3) * L::kQPanel + row * 128u + (((c & 7) ^ (row & 7)) << 4),
+                         q.x, q.y, q.z, q.w);
           }
-          tmem_st32(s_base + kTmemQ + c * 32u, r);
         }
-        tmem_wait_st();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(q_ready);
+      } else {
+        // group 1 starts an item only after group 0 has finished merging the
+        // previous one (group 0 arrives on q_ready after that merge)
+        const bool w = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status);
+        if (__any_sync(0xffffffffu, !w)) {
+          ok = false;
+          break;
+        }
       }
-      tc_fence_before();
-      mbar_arrive(q_ready);
 
-      float m = -INFINITY, l = 0.f;  // running max (log2 units) and sum of this row
-      // page ids: 32 per coalesced warp load, one batch ahead (lane i holds page pb + i)
+      float m = -INFINITY, l = 0.f;  // this group's running max (log2 units) and sum
+      // page ids: 32 per coalesced warp load (lane i holds page pb + i), one batch ahead
       const int npages_item = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
       auto load_batch = [&](int pb) {
         return pb + lane < npages_item ? v.table[v.page0 + pb + lane] : 0;
       };
+      int cur_batch = 0;
       int cur_pages = load_batch(0), nxt_pages = load_batch(32);
-      for (int j = 0; j < v.ntiles; ++j) {
+      for (int j = grp; j < v.ntiles; j += 2) {
         const int u = t + j, b = u & 1;
         const bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
         if (__any_sync(0xffffffffu, !w)) {
@@ -300,21 +315,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-        // S_u completing implies PV_{u-2} completed (same issuing thread, in
-        // order): consume those o_full phases without stalling
-        while (oc <= u - 2) {
-          mbar_wait(o_full(oc & 1), (oc >> 1) & 1, abort_flag, p.status);
-          ++oc;
-        }
+        // S_u done implies every earlier MMA is done, in particular PV_{u-2}
+        // (this group's previous tile): consume that o_full phase now
+        if (j >= 2) mbar_wait(o_full(b), ((u - 2) >> 1) & 1, abort_flag, p.status);
         const int nt = tile_tokens<TT>(it, j);
         const int np = (nt + kPB - 1) / kPB;
-        const int tp0 = (j * kPagesPerTile) & 31;  // first page of this tile within the batch
-        if (j > 0 && tp0 == 0) {                     // entering the next batch of 32 pages
+        const int batch = (j * kPagesPerTile) >> 5;
+        while (cur_batch < batch) {  // at most one step per visited tile
           cur_pages = nxt_pages;
-          nxt_pages = load_batch(j * kPagesPerTile + 32);
+          ++cur_batch;
+          nxt_pages = load_batch(cur_batch * 32 + 32);
         }
-        bool rescale = false;
-        float alpha = 1.f;
+        const int tp0 = (j * kPagesPerTile) & 31;
         if (warp_live) {
           uint32_t pv = 0;  // valid pages of this tile
 #pragma unroll
@@ -349,6 +361,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mx3 = fmaxf(mx3, s[i + 3]);
           }
           const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;  // scale > 0
+          bool rescale = false;
+          float alpha = 1.f;
           if (m_tile > m + kRescaleLog2 || (m == -INFINITY && m_tile != -INFINITY)) {
             alpha = m == -INFINITY ? 0.f : fast_exp2(m - m_tile);
             rescale = m != -INFINITY;
@@ -371,14 +385,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tmem_st32(s_base + (uint32_t)b * TT + c * 32u, pk);
           }
-          tmem_wait_st();
           l += ps0 + ps1;
+          // a row whose max grew: rescale this group's output (its previous PV is done)
+          if (j >= 2 && __any_sync(0xffffffffu, rescale)) {
+            const float a = rescale ? alpha : 1.f;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+              uint32_t r[32];
+              tmem_ld32(o_mine + c * 32u, r);
+              tmem_wait_ld();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * a);
+              tmem_st32(o_mine + c * 32u, r);
+            }
+          }
+          tmem_wait_st();
         }
         // value rows past the sequence inside its last page: zero them before PV
         if (j == v.ntiles - 1 && (nt % kPB) != 0) {
           const int pg = np - 1, first = nt % kPB;
           const int units = (kPB - first) * L::kPanels * 8;
-          for (int x = tid; x < units; x += 128) {
+          for (int x = gtid; x < units; x += 128) {
             const int rr = first + x / (L::kPanels * 8);
             const int rem = x % (L::kPanels * 8);
             st_shared_v4(sV(u % ST) + (rem >> 3) * L::kRowsTile + (pg * kPB + rr) * 128u +
@@ -386,70 +413,65 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           fence_proxy_async_smem();
         }
-        // a row whose max grew: the previous PV must be done, then rescale O in TMEM
-        if (j >= 1 && __any_sync(0xffffffffu, rescale)) {
-          bool w2 = true;
-          while (oc <= u - 1) {
-            w2 = w2 && mbar_wait(o_full(oc & 1), (oc >> 1) & 1, abort_flag, p.status);
-            ++oc;
-          }
-          if (__any_sync(0xffffffffu, !w2)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const float a = rescale ? alpha : 1.f;
-#pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t r[32];
-            tmem_ld32(o_base + c * 32u, r);
-            tmem_wait_ld();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * a);
-            tmem_st32(o_base + c * 32u, r);
-          }
-          tmem_wait_st();
-        }
         tc_fence_before();
         mbar_arrive(p_full(b));
       }
       if (!ok) break;
-      // final output of the item: wait for the last PV, read O, normalise
-      {
-        const int u = t + v.ntiles - 1;
-        bool w = true;
-        while (oc <= u) {
-          w = w && mbar_wait(o_full(oc & 1), (oc >> 1) & 1, abort_flag, p.status);
-          ++oc;
-        }
-        if (__any_sync(0xffffffffu, !w)) {
-          ok = false;
-          break;
-        }
+      // ---- end of item: wait for this group's last PV, then merge the groups
+      const int last = grp + ((v.ntiles - 1 - grp) >> 1) * 2;  // this group's last tile (if any)
+      const bool has = grp < v.ntiles;
+      if (has) {
+        const int u = t + last, b = u & 1;
+        const bool w = mbar_wait(o_full(b), (u >> 1) & 1, abort_flag, p.status);
+        if (__any_sync(0xffffffffu, !w)) ok = false;
         tc_fence_after();
-        if (warp_live) {
+      }
+      if (grp == 1) {
+        ml1[row] = make_float2(has ? m : -INFINITY, has ? l : 0.f);
+        tc_fence_before();
+        mbar_arrive(ml_ready);
+      } else {
+        const bool w = mbar_wait(ml_ready, (ii - it_begin) & 1, abort_flag, p.status);
+        if (__any_sync(0xffffffffu, !w)) ok = false;
+        tc_fence_after();
+        if (ok && warp_live) {
+          const float2 o1 = ml1[row];
+          const float mm = fmaxf(m, o1.x);
+          const float w0 = m == -INFINITY ? 0.f : fast_exp2(m - mm);
+          const float w1 = o1.x == -INFINITY ? 0.f : fast_exp2(o1.x - mm);
+          const float lsum = l * w0 + o1.y * w1;
+          const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
           const int fork = it.fork0 + (row_ok ? fl : 0);
           const size_t prow_out = (size_t)(p.part_base[fork] + it.part) * p.hq + head;
           float4* dst = reinterpret_cast<float4*>(p.part_o + prow_out * p.dv);
-          const float inv = l > 0.f ? 1.f / l : 0.f;
+          const uint32_t o0 = tmem + lane_addr + kTmemO, o1a = o0 + 128u;
 #pragma unroll
           for (int c = 0; c < D / 32; ++c) {
-            uint32_t r[32];
-            tmem_ld32(o_base + c * 32u, r);
+            uint32_t r0[32], r1[32];
+            tmem_ld32(o0 + c * 32u, r0);
+            tmem_ld32(o1a + c * 32u, r1);
             tmem_wait_ld();
             if (row_ok) {
 #pragma unroll
-              for (int i = 0; i < 32; i += 4)
-                dst[c * 8 + i / 4] = make_float4(
-                    __uint_as_float(r[i]) * inv, __uint_as_float(r[i + 1]) * inv,
-                    __uint_as_float(r[i + 2]) * inv, __uint_as_float(r[i + 3]) * inv);
+              for (int i = 0; i < 32; i += 4) {
+                float x[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  // an unused output buffer (weight 0) may hold anything: never multiply it
+                  const float a0 = w0 == 0.f ? 0.f : __uint_as_float(r0[i + e]) * w0;
+                  const float a1 = w1 == 0.f ? 0.f : __uint_as_float(r1[i + e]) * w1;
+                  x[e] = (a0 + a1) * inv;
+                }
+                dst[c * 8 + i / 4] = make_float4(x[0], x[1], x[2], x[3]);
+              }
             }
           }
-          if (row_ok) p.part_lse[prow_out] = m == -INFINITY ? -INFINITY : (m + log2f(l)) * kLn2;
+          if (row_ok)
+            p.part_lse[prow_out] = mm == -INFINITY ? -INFINITY : (mm + log2f(lsum)) * kLn2;
         }
-        // the next item's Q overwrites this item's Q in TMEM only after this point
         tc_fence_before();
       }
+      if (__any_sync(0xffffffffu, !ok)) ok = false;
       t += v.ntiles;
     }
   }
@@ -503,6 +525,7 @@ cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap
   constexpr int smem = (int)Smem<D, TT, ST>::kBytes;
   static_assert(smem <= 232448, "fork_tc kernel shared memory exceeds 227 KB");
   static_assert(ST <= kMaxStages && (TT == 64 || TT == 128), "unsupported pipeline shape");
+  static_assert(kTmemO + 128u * kWG <= kTmemCols && 2 * TT <= (int)kTmemO, "TMEM layout");
   auto kern = fork_tc_kernel<D, TT, ST>;
   static thread_local int configured = -1;
   int dev = 0;
@@ -533,8 +556,8 @@ cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v
   if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
       !make_pool_map(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
     return cudaErrorInvalidValue;
-  if (dqk == 128) return launch_d<128, kTile, 6>(p, mk, mv, grid, stream);
-  if (dqk == 64) return launch_d<64, kTile, 8>(p, mk, mv, grid, stream);
+  if (dqk == 128) return launch_d<128, kTile, 3>(p, mk, mv, grid, stream);
+  if (dqk == 64) return launch_d<64, kTile, 4>(p, mk, mv, grid, stream);
   return cudaErrorInvalidValue;
 }
 
