@@ -142,6 +142,27 @@ specgen_status specgen_fork_attn_decode(const specgen_fork_attn_args* args,
                                         const specgen_host_lens* lens,
                                         void* cuda_stream);
 
+/* specgen_fork_attn_decode for callers that cannot allocate device memory.
+ * (No counterpart in the paper: this is a deployment convenience.)  Some
+ * callers cannot call cudaMalloc at all -- for example a plugin inside a host
+ * engine that owns the whole device memory pool, or code on a latency-critical
+ * path where an allocation (which may synchronise the device) is not allowed --
+ * so they cannot supply args->workspace.  This entry point ignores
+ * args->workspace / workspace_bytes and uses a library-owned scratch array of
+ * 16 MiB (SPECGEN_STATIC_WORKSPACE_BYTES) that every GPU loading the library
+ * keeps until the process exits; it allocates nothing.  A call whose
+ * specgen_fork_attn_workspace_size exceeds that returns SPECGEN_ERR_WORKSPACE.
+ * The first call on a device looks up the array's device address (a CUDA
+ * runtime query), so make that first call before any stream capture.  All calls
+ * share the one array: calls that may overlap on the GPU (different streams,
+ * or host threads) race and must be serialised by the caller.  The status word
+ * read by specgen_workspace_status lives in that array too and is not exposed
+ * here: an out-of-range page id is skipped silently. */
+#define SPECGEN_STATIC_WORKSPACE_BYTES (16u << 20)
+specgen_status specgen_fork_attn_decode_static(const specgen_fork_attn_args* args,
+                                               const specgen_host_lens* lens,
+                                               void* cuda_stream);
+
 /* Standalone log-sum-exp merge of two partial attentions over disjoint key
  * sets (the combination step of the split computation):
  *     m = max(lse_a, lse_b); w_x = exp(lse_x - m)

@@ -31,6 +31,7 @@ EXPORTED = [
     "specgen_fork_attn_run",
     "specgen_fork_attn_run_profiled",
     "specgen_fork_attn_decode",
+    "specgen_fork_attn_decode_static",
     "specgen_lse_merge",
     "specgen_workspace_status",
     "specgen_status_string",
@@ -96,6 +97,8 @@ def load() -> C.CDLL:
                                                    C.c_void_p, C.c_int, P(C.c_int)]
     lib.specgen_fork_attn_decode.restype = C.c_int
     lib.specgen_fork_attn_decode.argtypes = [P(ForkAttnArgs), P(HostLens), C.c_void_p]
+    lib.specgen_fork_attn_decode_static.restype = C.c_int
+    lib.specgen_fork_attn_decode_static.argtypes = [P(ForkAttnArgs), P(HostLens), C.c_void_p]
     lib.specgen_lse_merge.restype = C.c_int
     lib.specgen_lse_merge.argtypes = [C.c_void_p] * 6 + [C.c_int, C.c_int, C.c_int, C.c_void_p]
     lib.specgen_workspace_status.restype = C.c_int
@@ -174,6 +177,13 @@ def specgen_fork_attn_run_profiled(args: ForkAttnArgs, plan: Plan, stream: int, 
 def specgen_fork_attn_decode(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> None:
     _check(load().specgen_fork_attn_decode(C.byref(args), C.byref(lens), C.c_void_p(stream)),
            "specgen_fork_attn_decode")
+
+
+def specgen_fork_attn_decode_static(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> None:
+    """Fork decode using the library's fixed scratch array (no workspace, no allocation)."""
+    _check(load().specgen_fork_attn_decode_static(C.byref(args), C.byref(lens),
+                                                  C.c_void_p(stream)),
+           "specgen_fork_attn_decode_static")
 
 
 def specgen_lse_merge(out_a, lse_a, out_b, lse_b, out, lse, rows: int, dv: int, dtype: int,

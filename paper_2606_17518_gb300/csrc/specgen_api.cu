@@ -532,3 +532,63 @@ const char* specgen_status_string(specgen_status status) {
 int specgen_version(void) { return 100; }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of specgen_fork_attn_decode.
+//
+// Some callers cannot allocate device memory at all: a plugin that runs inside
+// a host engine which owns the whole device memory pool, or code on a
+// latency-critical path where cudaMalloc (which can synchronise the device) is
+// not allowed.  They cannot provide the workspace the other entry points take,
+// so this variant uses a fixed, library-owned scratch array instead.  The
+// array is a file-scope device variable: every GPU that loads this library
+// holds kStaticWorkspaceBytes of it until the process exits.
+namespace {
+
+constexpr size_t kStaticWorkspaceBytes = 16u << 20;  // 16 MiB
+static __device__ __align__(256) unsigned char g_static_workspace[kStaticWorkspaceBytes];
+
+constexpr int kMaxDevices = 64;
+void* g_static_ws_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  Host code may
+// not use the symbol itself as a device pointer, so the address is looked up
+// once per device (with that device current) and cached.
+specgen_status static_workspace(void** ptr) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return SPECGEN_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return SPECGEN_ERR_UNSUPPORTED;
+  if (!g_static_ws_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_workspace) != cudaSuccess || !p) return SPECGEN_ERR_CUDA;
+    g_static_ws_ptr[dev] = p;
+  }
+  *ptr = g_static_ws_ptr[dev];
+  return SPECGEN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+specgen_status specgen_fork_attn_decode_static(const specgen_fork_attn_args* args,
+                                               const specgen_host_lens* lens,
+                                               void* cuda_stream) {
+  if (!args) return SPECGEN_ERR_NULL;
+  const size_t need = specgen_fork_attn_workspace_size(args, lens);
+  if (need == 0) {
+    Shape s;
+    const specgen_status st = check_shape(args, lens, &s);
+    return st == SPECGEN_OK ? SPECGEN_ERR_SHAPE : st;
+  }
+  if (need > kStaticWorkspaceBytes) return SPECGEN_ERR_WORKSPACE;
+  void* ws = nullptr;
+  specgen_status st = static_workspace(&ws);
+  if (st != SPECGEN_OK) return st;
+  specgen_fork_attn_args a = *args;
+  a.workspace = ws;
+  a.workspace_bytes = kStaticWorkspaceBytes;
+  return specgen_fork_attn_decode(&a, lens, cuda_stream);
+}
+
+}  // extern "C"
