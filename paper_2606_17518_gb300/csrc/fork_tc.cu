@@ -122,6 +122,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
+  // let the merge grid (a programmatic dependent) get launched early; it waits
+  // for this grid's completion before it reads anything
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < ST; ++i) {

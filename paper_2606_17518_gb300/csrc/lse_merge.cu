@@ -17,7 +17,6 @@ namespace specgen {
 
 namespace {
 
-constexpr int kMergeWarps = 4;
 
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
@@ -31,83 +30,81 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// One warp per (fork, head) row.  Lane i holds the LSE (and then the weight) of
-// part i, so the max and the normaliser are two warp reductions; the weighted
-// sum then streams the parts' rows with four independent loads in flight.
-__global__ void __launch_bounds__(kMergeWarps * 32) merge_parts_kernel(const MergeParams p) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row = blockIdx.x * kMergeWarps + warp;
+// One thread per (row, 4-column slice): every thread reads the LSE of all of its
+// row's parts (the 32 threads of a row read the same words) and the parts'
+// float4 slices, all loads independent, so a row costs about two memory round
+// trips.  With programmatic dependent launch the grid starts while the kernel
+// producing the partials is still running and waits for it here.
+constexpr int kMergeThreads = 128;  // small blocks can sit beside a running tensor-core CTA
+
+__global__ void __launch_bounds__(kMergeThreads) merge_parts_kernel(const MergeParams p) {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  const int c4n = p.dv / 4;
+  const int gid = blockIdx.x * kMergeThreads + threadIdx.x;
+  const int row = gid / c4n, c4 = gid % c4n;
   if (row >= p.n_rows) return;
   const int f = row / p.hq, h = row % p.hq;
   const int base = p.part_base[f], n = p.n_parts[f];
-  __nv_bfloat16* out = p.out + (size_t)row * p.dv;
-
+  const float* lse_p = p.part_lse + (size_t)base * p.hq + h;
   float m = -INFINITY;
-  for (int i = lane; i < n; i += 32) m = fmaxf(m, p.part_lse[(size_t)(base + i) * p.hq + h]);
-  m = warp_max(m);
+  int i = 0;
+  for (; i + 8 <= n; i += 8) {
+    float v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = lse_p[(size_t)(i + e) * p.hq];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) m = fmaxf(m, v[e]);
+  }
+  for (; i < n; ++i) m = fmaxf(m, lse_p[(size_t)i * p.hq]);
+  __nv_bfloat16* out = p.out + (size_t)row * p.dv;
   if (m == -INFINITY) {  // no keys at all: O = 0, LSE = -inf
-    for (int c = lane; c < p.dv; c += 32) out[c] = __float2bfloat16_rn(0.f);
-    if (lane == 0) p.lse[row] = -INFINITY;
+    reinterpret_cast<uint2*>(out)[c4] = make_uint2(0u, 0u);
+    if (c4 == 0) p.lse[row] = -INFINITY;
     return;
   }
+  const float4* o_p = reinterpret_cast<const float4*>(p.part_o + ((size_t)base * p.hq + h) * p.dv) + c4;
+  const size_t o_stride = (size_t)p.hq * p.dv / 4;  // float4s between consecutive parts
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   float wsum = 0.f;
-  for (int i0 = 0; i0 < n; i0 += 32) {
-    const int i = i0 + lane;
-    const float li = i < n ? p.part_lse[(size_t)(base + i) * p.hq + h] : -INFINITY;
-    wsum += li == -INFINITY ? 0.f : fast_exp2((li - m) * kLog2e);
-  }
-  wsum = warp_sum(wsum);
-  const float inv = 1.f / wsum;
-  // every lane runs every iteration (the shuffles need the full warp); lanes
-  // past the row's last column load nothing and store nothing
-  for (int c0 = 0; c0 < p.dv / 4; c0 += 32) {
-    const int c4 = c0 + lane;
-    const bool active = c4 < p.dv / 4;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int i0 = 0; i0 < n; i0 += 32) {
-      const int i = i0 + lane;
-      const float li = i < n ? p.part_lse[(size_t)(base + i) * p.hq + h] : -INFINITY;
-      const float wl = li == -INFINITY ? 0.f : fast_exp2((li - m) * kLog2e);
-      const int cnt = n - i0 < 32 ? n - i0 : 32;
-      int k = 0;
-      for (; k + 4 <= cnt; k += 4) {
-        float w[4];
-        float4 v[4];
+  i = 0;
+  for (; i + 4 <= n; i += 4) {
+    float li[4];
+    float4 v[4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          w[e] = __shfl_sync(0xffffffffu, wl, k + e);
-          v[e] = active ? reinterpret_cast<const float4*>(
-                              p.part_o + ((size_t)(base + i0 + k + e) * p.hq + h) * p.dv)[c4]
-                        : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          if (w[e] == 0.f) continue;  // empty part: its row may hold anything
-          acc.x += w[e] * v[e].x;
-          acc.y += w[e] * v[e].y;
-          acc.z += w[e] * v[e].z;
-          acc.w += w[e] * v[e].w;
-        }
-      }
-      for (; k < cnt; ++k) {
-        const float we = __shfl_sync(0xffffffffu, wl, k);
-        if (we == 0.f || !active) continue;
-        const float4 v = reinterpret_cast<const float4*>(
-            p.part_o + ((size_t)(base + i0 + k) * p.hq + h) * p.dv)[c4];
-        acc.x += we * v.x;
-        acc.y += we * v.y;
-        acc.z += we * v.z;
-        acc.w += we * v.w;
-      }
+    for (int e = 0; e < 4; ++e) {
+      li[e] = lse_p[(size_t)(i + e) * p.hq];
+      v[e] = o_p[(size_t)(i + e) * o_stride];
     }
-    __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-    __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-    uint2 packed;
-    packed.x = *reinterpret_cast<uint32_t*>(&lo);
-    packed.y = *reinterpret_cast<uint32_t*>(&hi);
-    if (active) reinterpret_cast<uint2*>(out)[c4] = packed;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      if (li[e] == -INFINITY) continue;  // empty part: its row may hold anything
+      const float w = fast_exp2((li[e] - m) * kLog2e);
+      wsum += w;
+      acc.x += w * v[e].x;
+      acc.y += w * v[e].y;
+      acc.z += w * v[e].z;
+      acc.w += w * v[e].w;
+    }
   }
-  if (lane == 0) p.lse[row] = m + log2f(wsum) * kLn2;
+  for (; i < n; ++i) {
+    const float li = lse_p[(size_t)i * p.hq];
+    if (li == -INFINITY) continue;
+    const float w = fast_exp2((li - m) * kLog2e);
+    const float4 v = o_p[(size_t)i * o_stride];
+    wsum += w;
+    acc.x += w * v.x;
+    acc.y += w * v.y;
+    acc.z += w * v.z;
+    acc.w += w * v.w;
+  }
+  const float inv = 1.f / wsum;
+  __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+  __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+  uint2 packed;
+  packed.x = *reinterpret_cast<uint32_t*>(&lo);
+  packed.y = *reinterpret_cast<uint32_t*>(&hi);
+  reinterpret_cast<uint2*>(out)[c4] = packed;
+  if (c4 == 0) p.lse[row] = m + log2f(wsum) * kLn2;
 }
 
 template <typename T>
@@ -154,11 +151,20 @@ __global__ void __launch_bounds__(256) lse_merge2_kernel(const T* oa, const floa
 
 }  // namespace
 
-cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream) {
+cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool after_dependent) {
   if (p.n_rows == 0) return cudaSuccess;
-  const int blocks = (p.n_rows + kMergeWarps - 1) / kMergeWarps;
-  merge_parts_kernel<<<blocks, kMergeWarps * 32, 0, stream>>>(p);
-  return cudaGetLastError();
+  const long long threads = (long long)p.n_rows * (p.dv / 4);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((threads + kMergeThreads - 1) / kMergeThreads));
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = after_dependent ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, merge_parts_kernel, p);
 }
 
 cudaError_t launch_lse_merge2(const void* oa, const float* la, const void* ob, const float* lb,

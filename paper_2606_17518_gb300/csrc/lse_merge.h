@@ -16,7 +16,10 @@ struct MergeParams {
   int n_rows, hq, dv;
 };
 
-cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream);
+// after_dependent: launch as a programmatic dependent of the previous kernel on
+// the stream (which must trigger griddepcontrol.launch_dependents); the merge
+// waits for that kernel's completion before reading the partials.
+cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool after_dependent);
 cudaError_t launch_lse_merge2(const void* oa, const float* la, const void* ob, const float* lb,
                               void* o, float* l, int rows, int dv, int dtype,
                               cudaStream_t stream);

@@ -472,7 +472,8 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   mp.n_rows = plan->n_rows;
   mp.hq = args->hq;
   mp.dv = args->head_dim_v;
-  if (launch_merge_parts(mp, stream) != cudaSuccess) return SPECGEN_ERR_CUDA;
+  if (launch_merge_parts(mp, stream, plan->n_tc_ctas > 0 && plan->n_split_items == 0) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
   if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
   return SPECGEN_OK;
 }
