@@ -275,49 +275,65 @@ def run_ours():
     args = [r.args() for r in reps]
     plans = [r.plan_info for r in reps]
 
-    # event ring: one set of marks per timed step
+    # Timed steps replay CUDA graphs (one graph per step slot, each one call of
+    # the library for one replica) so that host launch latency never starves
+    # the GPU.  Inside every graph the library records event marks between its
+    # kernels; after the timed region each slot's marks hold the times of its
+    # last replay, giving per-kernel durations over the last n_slots steps.
     n_marks = 4
     K, W = ARGS.steps, ARGS.warmup
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(K * n_marks)]
-    with torch.cuda.stream(stream):
-        for e in evs:
-            e.record(stream)  # create the events outside the timed region
-    torch.cuda.synchronize(dev)
-    handles = (C.c_void_p * len(evs))(*[e.cuda_event for e in evs])
+    n_slots = max(replicas, min(K, 64))
     lib = _lib.load()
     n_l = C.c_int(0)
     run_prof = lib.specgen_fork_attn_run_profiled
-    run = lib.specgen_fork_attn_run
     arg_refs = [C.byref(a) for a in args]
     plan_refs = [C.byref(p) for p in plans]
     sp_c = C.c_void_p(sp)
-
-    for i in range(W):
-        st = run(arg_refs[i % replicas], plan_refs[i % replicas], sp_c)
+    for i in range(2):  # first calls configure the kernels outside any capture
+        st = lib.specgen_fork_attn_run(arg_refs[i % replicas], plan_refs[i % replicas], sp_c)
         assert st == 0, _lib.status_string(st)
+    torch.cuda.synchronize(dev)
+    slot_events, graphs = [], []
+    for g in range(n_slots):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_marks)]
+        with torch.cuda.stream(stream):
+            for e in evs:
+                e.record(stream)  # create the CUDA events before the capture
+        torch.cuda.synchronize(dev)
+        handles = (C.c_void_p * n_marks)(*[e.cuda_event for e in evs])
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            st = run_prof(arg_refs[g % replicas], plan_refs[g % replicas], sp_c, handles,
+                          n_marks, C.byref(n_l))
+        if st != 0:
+            raise RuntimeError(_lib.status_string(st))
+        slot_events.append(evs)
+        graphs.append(graph)
+    torch.cuda.synchronize(dev)
+    for i in range(W):
+        graphs[i % n_slots].replay()
     torch.cuda.synchronize(dev)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local_rank)
     barrier()
     torch.cuda.synchronize(dev)
     clocks.start()
-    start.record(stream)
-    for i in range(K):
-        st = run_prof(arg_refs[i % replicas], plan_refs[i % replicas], sp_c,
-                      C.byref(handles, i * n_marks * C.sizeof(C.c_void_p)), n_marks,
-                      C.byref(n_l))
-        if st != 0:
-            raise RuntimeError(_lib.status_string(st))
-    end.record(stream)
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for i in range(K):
+            graphs[i % n_slots].replay()
+        end.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
     clk = clocks.stop()
     launches = n_l.value
     total_ms = start.elapsed_time(end)
+    sampled = min(K, n_slots)
     per_kernel = [0.0] * launches
-    for i in range(K):
+    for g in range(sampled):
         for k in range(launches):
-            per_kernel[k] += evs[i * n_marks + k].elapsed_time(evs[i * n_marks + k + 1])
+            per_kernel[k] += slot_events[g][k].elapsed_time(slot_events[g][k + 1])
+    per_kernel = [x * K / sampled for x in per_kernel]  # scale the sample to K steps
     status = reps[0].status(sp)
     if status != 0:
         raise RuntimeError(f"workspace status {_lib.status_string(status)}")
@@ -360,6 +376,8 @@ def run_ours():
             "head_dim": [w["dqk"], w["dv"]], "page_size": w["page_size"],
             "unique_bytes": nbytes["total"], "flops": flops["total"],
             "l2": f"inputs rotate over {replicas} resident replicas (>= 3x L2)",
+            "timing": f"CUDA-graph replay per step; per-kernel times from the last "
+                      f"{min(K, n_slots)} timed steps",
             "parallelism": f"replicas x{world}",
         },
         "gpu_launches": K * launches,

@@ -365,6 +365,13 @@ struct Marks {
   int launches = 0;
   bool mark(cudaStream_t stream, int i) {
     if (!events || i >= n || !events[i]) return true;
+    // inside a stream capture the mark must be an external event-record node so
+    // that it still records a time stamp when the graph is replayed
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) return false;
+    if (cs == cudaStreamCaptureStatusActive)
+      return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(events[i]), stream,
+                                      cudaEventRecordExternal) == cudaSuccess;
     return cudaEventRecord(static_cast<cudaEvent_t>(events[i]), stream) == cudaSuccess;
   }
 };
