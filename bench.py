@@ -275,14 +275,15 @@ def run_ours():
     args = [r.args() for r in reps]
     plans = [r.plan_info for r in reps]
 
-    # Timed steps replay CUDA graphs (one graph per step slot, each one call of
-    # the library for one replica) so that host launch latency never starves
-    # the GPU.  Inside every graph the library records event marks between its
-    # kernels; after the timed region each slot's marks hold the times of its
-    # last replay, giving per-kernel durations over the last n_slots steps.
+    # Timed steps replay CUDA graphs.  Each graph holds `per_graph` consecutive
+    # steps (one library call each, on rotating replicas) so that host launch
+    # overhead never starves the GPU; inside every step the library records
+    # event marks between its kernels (external record nodes), so after the
+    # timed region each graph's marks hold the per-kernel times of its last
+    # replay.  K is covered exactly: full graphs plus one remainder graph.
     n_marks = 4
     K, W = ARGS.steps, ARGS.warmup
-    n_slots = max(replicas, min(K, 64))
+    per_graph = max(1, min(16, K))
     lib = _lib.load()
     n_l = C.c_int(0)
     run_prof = lib.specgen_fork_attn_run_profiled
@@ -293,25 +294,34 @@ def run_ours():
         st = lib.specgen_fork_attn_run(arg_refs[i % replicas], plan_refs[i % replicas], sp_c)
         assert st == 0, _lib.status_string(st)
     torch.cuda.synchronize(dev)
-    slot_events, graphs = [], []
-    for g in range(n_slots):
-        evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_marks)]
+
+    def make_graph(first_step, n_steps):
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_marks)]
+               for _ in range(n_steps)]
         with torch.cuda.stream(stream):
-            for e in evs:
-                e.record(stream)  # create the CUDA events before the capture
+            for row in evs:
+                for e in row:
+                    e.record(stream)  # create the CUDA events before the capture
         torch.cuda.synchronize(dev)
-        handles = (C.c_void_p * n_marks)(*[e.cuda_event for e in evs])
+        handles = [(C.c_void_p * n_marks)(*[e.cuda_event for e in row]) for row in evs]
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=stream):
-            st = run_prof(arg_refs[g % replicas], plan_refs[g % replicas], sp_c, handles,
-                          n_marks, C.byref(n_l))
+            for k in range(n_steps):
+                r = (first_step + k) % replicas
+                st = run_prof(arg_refs[r], plan_refs[r], sp_c, handles[k], n_marks, C.byref(n_l))
+                if st != 0:
+                    break
         if st != 0:
             raise RuntimeError(_lib.status_string(st))
-        slot_events.append(evs)
-        graphs.append(graph)
-    torch.cuda.synchronize(dev)
-    for i in range(W):
-        graphs[i % n_slots].replay()
+        return graph, evs
+
+    n_full, rem = divmod(K, per_graph)
+    n_distinct = max(1, min(n_full, 8))
+    full_graphs = [make_graph(g * per_graph, per_graph) for g in range(n_distinct)] if n_full else []
+    rem_graph = make_graph(0, rem) if rem else None
+    schedule = [full_graphs[i % n_distinct] for i in range(n_full)] + ([rem_graph] if rem else [])
+    for i in range(max(1, (W + per_graph - 1) // per_graph)):
+        schedule[i % len(schedule)][0].replay()
     torch.cuda.synchronize(dev)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local_rank)
@@ -320,20 +330,23 @@ def run_ours():
     clocks.start()
     with torch.cuda.stream(stream):
         start.record(stream)
-        for i in range(K):
-            graphs[i % n_slots].replay()
+        for graph, _ in schedule:
+            graph.replay()
         end.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
     clk = clocks.stop()
     launches = n_l.value
     total_ms = start.elapsed_time(end)
-    sampled = min(K, n_slots)
+    sampled_graphs = full_graphs + ([rem_graph] if rem_graph else [])
+    sampled = sum(len(evs) for _, evs in sampled_graphs)
     per_kernel = [0.0] * launches
-    for g in range(sampled):
-        for k in range(launches):
-            per_kernel[k] += slot_events[g][k].elapsed_time(slot_events[g][k + 1])
+    for _, evs in sampled_graphs:
+        for row in evs:
+            for k in range(launches):
+                per_kernel[k] += row[k].elapsed_time(row[k + 1])
     per_kernel = [x * K / sampled for x in per_kernel]  # scale the sample to K steps
+    n_slots = sampled
     status = reps[0].status(sp)
     if status != 0:
         raise RuntimeError(f"workspace status {_lib.status_string(status)}")
@@ -376,8 +389,8 @@ def run_ours():
             "head_dim": [w["dqk"], w["dv"]], "page_size": w["page_size"],
             "unique_bytes": nbytes["total"], "flops": flops["total"],
             "l2": f"inputs rotate over {replicas} resident replicas (>= 3x L2)",
-            "timing": f"CUDA-graph replay per step; per-kernel times from the last "
-                      f"{min(K, n_slots)} timed steps",
+            "timing": f"CUDA graphs of {per_graph} steps; per-kernel times from the last "
+                      f"replay of each graph ({n_slots} timed steps)",
             "parallelism": f"replicas x{world}",
         },
         "gpu_launches": K * launches,
