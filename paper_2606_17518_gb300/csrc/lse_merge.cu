@@ -153,6 +153,18 @@ __global__ void __launch_bounds__(256) lse_merge2_kernel(const T* oa, const floa
 
 cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool after_dependent) {
   if (p.n_rows == 0) return cudaSuccess;
+  // keep the SMs in the shared-memory-heavy configuration of the kernels around
+  // this one, so that no L1/shared-memory reconfiguration is needed between them
+  static thread_local int configured = -1;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (configured != dev) {
+    e = cudaFuncSetAttribute(merge_parts_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             (int)cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+    configured = dev;
+  }
   const long long threads = (long long)p.n_rows * (p.dv / 4);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)((threads + kMergeThreads - 1) / kMergeThreads));
