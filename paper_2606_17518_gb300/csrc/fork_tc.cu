@@ -340,7 +340,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           packed.x = *reinterpret_cast<uint32_t*>(&lo);
           packed.y = *reinterpret_cast<uint32_t*>(&hi);
           reinterpret_cast<uint2*>(p.out + orow * p.dv)[c4] = packed;
-          if (c4 == 0) p.lse[orow] = mm == -INFINITY ? -INFINITY : (mm + log2f(ws)) * kLn2;
+          if (c4 == 0) p.lse[orow] = mm == -INFINITY ? -INFINITY : mm + log2f(ws) * kLn2;
         }
       }
     };
