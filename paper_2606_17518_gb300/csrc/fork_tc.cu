@@ -28,6 +28,7 @@
 
 #include "common.cuh"
 #include "fork_tc.h"
+#include "merge_row.cuh"
 #include "plan.h"
 #include "tc_common.cuh"
 
@@ -311,36 +312,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int idx = gtid; idx < p.G * c4n; idx += 128) {
           const int r = idx / c4n, c4 = idx % c4n;
           const int h = it.kv_head * p.G + r;
-          const float* lse_p = p.part_lse + (size_t)base * p.hq + h;
-          const float4* o_p =
-              reinterpret_cast<const float4*>(p.part_o + ((size_t)base * p.hq + h) * p.dv) + c4;
-          const size_t o_stride = (size_t)p.hq * p.dv / 4;
-          float mm = -INFINITY;
-          for (int i = 0; i < n; ++i) mm = fmaxf(mm, __ldcg(lse_p + (size_t)i * p.hq));
-          float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-          float ws = 0.f;
-          if (mm != -INFINITY) {
-            for (int i = 0; i < n; ++i) {
-              const float li = __ldcg(lse_p + (size_t)i * p.hq);
-              const float4 vv = __ldcg(o_p + (size_t)i * o_stride);
-              if (li == -INFINITY) continue;  // an empty part may hold anything
-              const float wgt = fast_exp2((li - mm) * kLog2e);
-              ws += wgt;
-              acc.x += wgt * vv.x;
-              acc.y += wgt * vv.y;
-              acc.z += wgt * vv.z;
-              acc.w += wgt * vv.w;
-            }
-          }
-          const float inv = ws > 0.f ? 1.f / ws : 0.f;
+          const RowMerge mr = merge_row(
+              p.part_lse + (size_t)base * p.hq + h, (size_t)p.hq,
+              reinterpret_cast<const float4*>(p.part_o + ((size_t)base * p.hq + h) * p.dv) + c4,
+              (size_t)p.hq * p.dv / 4, n);
           const size_t orow = (size_t)fork * p.hq + h;
-          __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-          __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-          uint2 packed;
-          packed.x = *reinterpret_cast<uint32_t*>(&lo);
-          packed.y = *reinterpret_cast<uint32_t*>(&hi);
-          reinterpret_cast<uint2*>(p.out + orow * p.dv)[c4] = packed;
-          if (c4 == 0) p.lse[orow] = mm == -INFINITY ? -INFINITY : mm + log2f(ws) * kLn2;
+          store_merged(mr, p.out + orow * p.dv, c4, p.lse + orow, c4 == 0);
         }
       }
     };

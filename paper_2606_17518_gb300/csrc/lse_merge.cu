@@ -12,6 +12,7 @@
 
 #include "common.cuh"
 #include "lse_merge.h"
+#include "merge_row.cuh"
 
 namespace specgen {
 
@@ -45,66 +46,11 @@ __global__ void __launch_bounds__(kMergeThreads) merge_parts_kernel(const MergeP
   if (row >= p.n_rows) return;
   const int f = row / p.hq, h = row % p.hq;
   const int base = p.part_base[f], n = p.n_parts[f];
-  const float* lse_p = p.part_lse + (size_t)base * p.hq + h;
-  float m = -INFINITY;
-  int i = 0;
-  for (; i + 8 <= n; i += 8) {
-    float v[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = lse_p[(size_t)(i + e) * p.hq];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) m = fmaxf(m, v[e]);
-  }
-  for (; i < n; ++i) m = fmaxf(m, lse_p[(size_t)i * p.hq]);
-  __nv_bfloat16* out = p.out + (size_t)row * p.dv;
-  if (m == -INFINITY) {  // no keys at all: O = 0, LSE = -inf
-    reinterpret_cast<uint2*>(out)[c4] = make_uint2(0u, 0u);
-    if (c4 == 0) p.lse[row] = -INFINITY;
-    return;
-  }
-  const float4* o_p = reinterpret_cast<const float4*>(p.part_o + ((size_t)base * p.hq + h) * p.dv) + c4;
-  const size_t o_stride = (size_t)p.hq * p.dv / 4;  // float4s between consecutive parts
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  float wsum = 0.f;
-  i = 0;
-  for (; i + 4 <= n; i += 4) {
-    float li[4];
-    float4 v[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      li[e] = lse_p[(size_t)(i + e) * p.hq];
-      v[e] = o_p[(size_t)(i + e) * o_stride];
-    }
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      if (li[e] == -INFINITY) continue;  // empty part: its row may hold anything
-      const float w = fast_exp2((li[e] - m) * kLog2e);
-      wsum += w;
-      acc.x += w * v[e].x;
-      acc.y += w * v[e].y;
-      acc.z += w * v[e].z;
-      acc.w += w * v[e].w;
-    }
-  }
-  for (; i < n; ++i) {
-    const float li = lse_p[(size_t)i * p.hq];
-    if (li == -INFINITY) continue;
-    const float w = fast_exp2((li - m) * kLog2e);
-    const float4 v = o_p[(size_t)i * o_stride];
-    wsum += w;
-    acc.x += w * v.x;
-    acc.y += w * v.y;
-    acc.z += w * v.z;
-    acc.w += w * v.w;
-  }
-  const float inv = 1.f / wsum;
-  __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-  __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-  uint2 packed;
-  packed.x = *reinterpret_cast<uint32_t*>(&lo);
-  packed.y = *reinterpret_cast<uint32_t*>(&hi);
-  reinterpret_cast<uint2*>(out)[c4] = packed;
-  if (c4 == 0) p.lse[row] = m + log2f(wsum) * kLn2;
+  const RowMerge mr = merge_row(
+      p.part_lse + (size_t)base * p.hq + h, (size_t)p.hq,
+      reinterpret_cast<const float4*>(p.part_o + ((size_t)base * p.hq + h) * p.dv) + c4,
+      (size_t)p.hq * p.dv / 4, n);
+  store_merged(mr, p.out + (size_t)row * p.dv, c4, p.lse + row, c4 == 0);
 }
 
 template <typename T>
