@@ -28,7 +28,6 @@
 
 #include "common.cuh"
 #include "fork_tc.h"
-#include "merge_row.cuh"
 #include "plan.h"
 #include "tc_common.cuh"
 
@@ -61,8 +60,7 @@ struct Smem {
   static constexpr uint32_t kOffKV = kQ;
   static constexpr uint32_t kOffBar = kOffKV + ST * kStage;
   static constexpr uint32_t kOffML = kOffBar + 256;        // 128 x (m, l) of the second group
-  static constexpr uint32_t kOffMerge = kOffML + 128 * 8;  // 128 fork ids to merge
-  static constexpr uint32_t kBytes = kOffMerge + 128 * 4 + 1024;
+  static constexpr uint32_t kBytes = kOffML + 128 * 8 + 1024;
 };
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
@@ -115,12 +113,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t q_ready = bar0 + 8u * (2 * kMaxStages + 6);
   const uint32_t mma_done = bar0 + 8u * (2 * kMaxStages + 7);
   const uint32_t ml_ready = bar0 + 8u * (2 * kMaxStages + 8);  // group 1's (m, l) written
-  const uint32_t parts_done = bar0 + 8u * (2 * kMaxStages + 9);  // group 0 wrote its partials
-  const uint32_t tickets_done = bar0 + 8u * (2 * kMaxStages + 10);  // merge list is ready
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 11));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 9));
   volatile int* abort_flag =
-      reinterpret_cast<volatile int*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 11) + 4);
-  int* merge_list = reinterpret_cast<int*>(gbase + L::kOffMerge);  // per fork of the item
+      reinterpret_cast<volatile int*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 9) + 4);
   float2* ml1 = reinterpret_cast<float2*>(gbase + L::kOffML);  // second group's (m, l) per row
   auto sK = [&](int s) { return base + L::kOffKV + s * L::kStage; };
   auto sV = [&](int s) { return base + L::kOffKV + s * L::kStage + L::kKV; };
@@ -144,8 +139,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_ready, 128);
     mbar_init(mma_done, 1);
     mbar_init(ml_ready, 128);
-    mbar_init(parts_done, 128);
-    mbar_init(tickets_done, 128);
     *abort_flag = 0;
     mbar_init_fence();
   }
@@ -276,51 +269,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float sl2 = p.scale_log2;
     int t = 0;
     bool ok = true;
-
-    // Fused merge (group 0 only).  Every (fork, kv head) group owns n_parts
-    // partial slots written by different items, possibly on different CTAs.
-    // After this item's partials are written and fenced, the first row of each
-    // fork takes a ticket; the CTA that takes a group's last ticket merges the
-    // group's partials into the final output and resets its counter.
-    auto merge_finished_groups = [&](const TcItem& it, int M, int local_item, bool all_ok) {
-      __threadfence();  // this thread's partial row is visible device-wide
-      const uint32_t ph = (uint32_t)local_item & 1u;
-      mbar_arrive(parts_done);
-      bool w = mbar_wait(parts_done, ph, abort_flag, p.status);
-      const int nf = it.nforks;
-      if (gtid < nf) {
-        const int fork = it.fork0 + gtid;
-        int winner = -1;
-        if (w && all_ok) {
-          int32_t* cnt = p.tickets + (size_t)fork * p.hkv + it.kv_head;
-          if (atomicAdd(cnt, 1) == p.n_parts[fork] - 1) {
-            *cnt = 0;  // ready for the next call
-            winner = fork;
-          }
-        }
-        merge_list[gtid] = winner;
-      }
-      __threadfence();
-      mbar_arrive(tickets_done);
-      w = mbar_wait(tickets_done, ph, abort_flag, p.status) && w;
-      if (!w || !all_ok) return;
-      const int c4n = p.dv / 4;
-      for (int k = 0; k < nf; ++k) {
-        const int fork = merge_list[k];
-        if (fork < 0) continue;
-        const int base = p.part_base[fork], n = p.n_parts[fork];
-        for (int idx = gtid; idx < p.G * c4n; idx += 128) {
-          const int r = idx / c4n, c4 = idx % c4n;
-          const int h = it.kv_head * p.G + r;
-          const RowMerge mr = merge_row(
-              p.part_lse + (size_t)base * p.hq + h, (size_t)p.hq,
-              reinterpret_cast<const float4*>(p.part_o + ((size_t)base * p.hq + h) * p.dv) + c4,
-              (size_t)p.hq * p.dv / 4, n);
-          const size_t orow = (size_t)fork * p.hq + h;
-          store_merged(mr, p.out + orow * p.dv, c4, p.lse + orow, c4 == 0);
-        }
-      }
-    };
 
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
       const TcItem it = p.items[p.cta_items[ii]];
@@ -526,7 +474,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             p.part_lse[prow_out] = mm == -INFINITY ? -INFINITY : (mm + log2f(lsum)) * kLn2;
         }
         tc_fence_before();
-        if (p.fused_merge) merge_finished_groups(it, v.M, ii - it_begin, ok);
       }
       if (__any_sync(0xffffffffu, !ok)) ok = false;
       t += v.ntiles;

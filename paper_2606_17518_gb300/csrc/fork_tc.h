@@ -18,13 +18,8 @@ struct TcParams {
   const int32_t* cta_items;    // item indices, grouped per CTA
   const int32_t* cta_offsets;  // [grid + 1] into cta_items
   const int32_t* part_base;    // [forks] first partial slot of each fork
-  const int32_t* n_parts;      // [forks] partial slots of each fork
   float* part_o;               // [slots][hq][dv]
   float* part_lse;             // [slots][hq]
-  int32_t* tickets;            // [forks][hkv] parts written so far (zero between calls)
-  __nv_bfloat16* out;          // [forks][hq][dv] final output (fused merge)
-  float* lse;                  // [forks][hq] final LSE (fused merge)
-  int fused_merge;             // 1: the CTA writing a group's last part merges it
   uint32_t* status;
   int hq, hkv, G, dv, num_pages;
   float scale_log2;            // softmax scale * log2(e), > 0

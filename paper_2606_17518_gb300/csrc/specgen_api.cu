@@ -253,7 +253,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
 
 struct Layout {
   size_t split_off, tc_off, cta_items_off, cta_offsets_off, part_base_off, n_parts_off, plan_bytes;
-  size_t ws_tickets, ws_plan, ws_part_o, ws_part_lse, ws_end;
+  size_t ws_plan, ws_part_o, ws_part_lse, ws_end;
 };
 
 Layout layout_of(const Shape& s, const HostPlan& hp) {
@@ -265,8 +265,7 @@ Layout layout_of(const Shape& s, const HostPlan& hp) {
   L.part_base_off = align_up(L.cta_offsets_off + hp.cta_offsets.size() * 4, 16);
   L.n_parts_off = align_up(L.part_base_off + (size_t)s.F * 4, 16);
   L.plan_bytes = L.n_parts_off + (size_t)s.F * 4;
-  L.ws_tickets = kHeaderBytes;  // [forks][hkv] int32 merge tickets, zeroed with the header
-  L.ws_plan = align_up(L.ws_tickets + (size_t)s.F * s.hkv * 4, kAlign);
+  L.ws_plan = kHeaderBytes;
   L.ws_part_o = align_up(L.ws_plan + L.plan_bytes, kAlign);
   L.ws_part_lse =
       align_up(L.ws_part_o + (size_t)hp.total_slots * s.hq * s.dv * sizeof(float), kAlign);
@@ -340,12 +339,7 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   plan->n_split_items = h.n_split;
   plan->n_rows = s.F * s.hq;
   plan->total_slots = t_plan.total_slots;
-  // the tensor-core kernel merges the partials itself unless some fork has no
-  // key at all (that row would never be written by a work item)
-  bool all_forks_have_parts = true;
-  for (int f = 0; f < s.F; ++f) all_forks_have_parts = all_forks_have_parts && t_plan.n_parts[f] > 0;
-  const bool fused = h.n_tc > 0 && all_forks_have_parts;
-  plan->flags = (s.latent ? 1 : 0) | (fused ? 2 : 0);
+  plan->flags = s.latent ? 1 : 0;
   plan->plan_bytes = (int64_t)L.plan_bytes;
   plan->ws_plan_off = (int64_t)L.ws_plan;
   plan->ws_part_o_off = (int64_t)L.ws_part_o;
@@ -357,7 +351,6 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   plan->offsets[3] = (int64_t)L.cta_offsets_off;
   plan->offsets[4] = (int64_t)L.part_base_off;
   plan->offsets[5] = (int64_t)L.n_parts_off;
-  plan->offsets[6] = (int64_t)L.ws_tickets;
   return SPECGEN_OK;
 }
 
@@ -455,13 +448,8 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     tp.cta_items = reinterpret_cast<const int32_t*>(pl + plan->offsets[2]);
     tp.cta_offsets = reinterpret_cast<const int32_t*>(pl + plan->offsets[3]);
     tp.part_base = reinterpret_cast<const int32_t*>(pl + plan->offsets[4]);
-    tp.n_parts = reinterpret_cast<const int32_t*>(pl + plan->offsets[5]);
     tp.part_o = part_o;
     tp.part_lse = part_lse;
-    tp.tickets = reinterpret_cast<int32_t*>(ws + plan->offsets[6]);
-    tp.out = static_cast<__nv_bfloat16*>(args->out);
-    tp.lse = args->lse;
-    tp.fused_merge = (plan->flags & 2) ? 1 : 0;
     tp.status = sp.status;
     tp.hq = args->hq;
     tp.hkv = args->hkv;
@@ -481,7 +469,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
   }
 
-  if (!(plan->flags & 2)) {  // merge pass (the tensor-core kernel did not merge)
+  {  // merge pass: combine every row's partials
     MergeParams mp;
     mp.part_o = part_o;
     mp.part_lse = part_lse;
