@@ -362,7 +362,8 @@ def run_ours():
     # ---- end to end through the public API: host buffers, copies in the timed region
     e2e = measure_e2e(w, reps, stream, dev, K=min(K, 500), W=min(W, 5))
 
-    kernel_names = (["fork_tc"] if plans[0].n_tc_items > 0 else []) + \
+    tc_name = "mla_tc" if w["v_pages"] is None else "fork_tc"
+    kernel_names = ([tc_name] if plans[0].n_tc_items > 0 else []) + \
         (["split_decode"] if plans[0].n_split_items > 0 else []) + ["lse_merge"]
     kernel_names = kernel_names[:launches]
     kernel_ms = [t / K for t in per_kernel]
@@ -370,7 +371,7 @@ def run_ours():
     hbm, tf_burst, tf_sus, peak_src = measured_peaks()
     # algorithmic bytes of the dominant launch: what that kernel must read/write once
     dom_name = kernel_names[dom] if kernel_names else None
-    if dom_name in ("fork_tc", "split_decode"):
+    if dom_name in ("fork_tc", "mla_tc", "split_decode"):
         # the kernel that reads the KV: unique prefix + every suffix + Q
         dom_bytes = nbytes["prefix"] + nbytes["suffix"] + nbytes["q"]
     else:

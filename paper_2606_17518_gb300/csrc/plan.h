@@ -42,6 +42,7 @@ struct TcItem {
   int32_t tok_begin;
   int32_t tok_end;
   int32_t part;
+  int32_t dv0;         // first value column this item produces (latent KV: 0 or 256)
 };
 
 // Plan header at the start of the plan region.

@@ -17,6 +17,7 @@
 #include "lse_merge.h"
 #include "plan.h"
 #include "fork_tc.h"
+#include "mla_tc.h"
 #include "split_decode.h"
 
 using namespace specgen;
@@ -176,6 +177,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
             it.tok_begin = (int)(c * chunk);
             it.tok_end = (int)std::min<long long>(S, (c + 1) * chunk);
             it.part = np + c;
+            it.dv0 = 0;
             hp->tc.push_back(it);
             cost.push_back(it.tok_end - it.tok_begin + item_overhead);
           }
@@ -192,6 +194,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
             it.tok_begin = (int)(c * chunk);
             it.tok_end = (int)std::min<long long>(P, (c + 1) * chunk);
             it.part = c;
+            it.dv0 = 0;
             hp->tc.push_back(it);
             cost.push_back(it.tok_end - it.tok_begin + item_overhead);
           }
@@ -202,7 +205,54 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
     return;
   }
 
-  // Split-K path (shapes the tensor-core kernel does not cover): every fork
+  if (mla_tc_supported(s.dqk, s.dv, s.latent, s.B, s.hq, s.hkv)) {
+    // Latent-KV tensor-core path: one item = one fork's 128 heads x one value
+    // half x a chunk of its prefix or suffix; chunks are whole tiles.
+    const int tt = mla_tc_tile_tokens();
+    long long work = 0;
+    for (int t = 0; t < s.T; ++t)
+      for (int f = fo[t]; f < fo[t + 1]; ++f)
+        work += 2LL * ((long long)lens->prefix_lens[t] + lens->suffix_lens[f]);
+    long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
+    chunk = std::max<long long>(4 * tt, (chunk + tt - 1) / tt * tt);
+    std::vector<long long> cost;
+    const long long item_overhead = 64;
+    for (int t = 0; t < s.T; ++t) {
+      const int P = lens->prefix_lens[t];
+      const int np = (int)((P + chunk - 1) / chunk);
+      for (int f = fo[t]; f < fo[t + 1]; ++f) {
+        const int S = lens->suffix_lens[f];
+        const int ns = (int)((S + chunk - 1) / chunk);
+        hp->part_base[f] = slot;
+        hp->n_parts[f] = np + ns;
+        slot += np + ns;
+        for (int c = 0; c < np + ns; ++c)
+          for (int half = 0; half < 2; ++half) {
+            const bool pre = c < np;
+            const int cc = pre ? c : c - np;
+            const int len = pre ? P : S;
+            TcItem it;
+            it.table_kind = pre ? 0 : 1;
+            it.seq = pre ? t : f;
+            it.kv_head = 0;
+            it.fork0 = f;
+            it.nforks = 1;
+            it.tok_begin = (int)(cc * chunk);
+            it.tok_end = (int)std::min<long long>(len, (cc + 1) * chunk);
+            it.part = c;
+            it.dv0 = half * 256;
+            hp->tc.push_back(it);
+            cost.push_back(it.tok_end - it.tok_begin + item_overhead);
+          }
+      }
+    }
+    const int n_cta = (int)std::min<size_t>((size_t)n_sm, hp->tc.size());
+    assign_lpt(cost, n_cta, &hp->cta_items, &hp->cta_offsets);
+    hp->total_slots = slot;
+    return;
+  }
+
+  // Split-K path (shapes the tensor-core kernels do not cover): every fork
   // reads its trace's prefix and its own suffix in chunks of whole tiles.
   const int dvt = split_dv_tile(s.dqk, s.dv, s.latent);
   const int row_blocks = (s.G + kRowBlock - 1) / kRowBlock;
@@ -457,9 +507,30 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     tp.dv = args->head_dim_v;
     tp.num_pages = args->num_pages;
     tp.scale_log2 = sp.scale_log2;
-    if (launch_fork_tc(tp, args->k_pages, args->v_pages, plan->n_tc_ctas, args->head_dim_qk,
-                       stream) != cudaSuccess)
-      return SPECGEN_ERR_CUDA;
+    cudaError_t e;
+    if (args->v_pages == nullptr) {
+      MlaParams mp;
+      mp.q = tp.q;
+      mp.prefix_bt = tp.prefix_bt;
+      mp.prefix_bt_off = tp.prefix_bt_off;
+      mp.suffix_bt = tp.suffix_bt;
+      mp.suffix_bt_off = tp.suffix_bt_off;
+      mp.items = tp.items;
+      mp.cta_items = tp.cta_items;
+      mp.cta_offsets = tp.cta_offsets;
+      mp.part_base = tp.part_base;
+      mp.part_o = part_o;
+      mp.part_lse = part_lse;
+      mp.status = tp.status;
+      mp.hq = args->hq;
+      mp.num_pages = args->num_pages;
+      mp.scale_log2 = tp.scale_log2;
+      e = launch_mla_tc(mp, args->k_pages, plan->n_tc_ctas, stream);
+    } else {
+      e = launch_fork_tc(tp, args->k_pages, args->v_pages, plan->n_tc_ctas, args->head_dim_qk,
+                         stream);
+    }
+    if (e != cudaSuccess) return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
   }
   if (plan->n_split_items > 0) {
