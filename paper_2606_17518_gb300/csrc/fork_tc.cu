@@ -208,6 +208,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
+      // descriptors are built once; every MMA only adds a constant offset
+      // (in 16-byte units) to the start-address field
+      const uint64_t dq = smem_desc_sw128(sQ, 16, 1024);
+      const uint64_t dk0 = smem_desc_sw128(sK(0), 16, 1024);
+      const uint64_t dv0 = smem_desc_sw128(sV(0), L::kRowsTile, 1024);
+      constexpr uint64_t kStageDesc = L::kStage >> 4;
+      constexpr uint32_t idesc_pv = idesc_bf16(128, D, true);
       int t = 0;
       bool ok = true;
       for (int ii = it_begin; ok && ii < it_end; ++ii) {
@@ -222,12 +229,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
             const uint32_t idesc = idesc_bf16(128, np * kPB, false);
+            const uint64_t dk = dk0 + (uint64_t)s * kStageDesc;
+            const uint32_t d_s = tmem + (uint32_t)b * TT;
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t qoff = (kk >> 2) * L::kQPanel + (kk & 3) * 32u;
-              const uint32_t koff = (kk >> 2) * L::kRowsTile + (kk & 3) * 32u;
-              mma_bf16(tmem + (uint32_t)b * TT, smem_desc_sw128(sQ + qoff, 16, 1024),
-                       smem_desc_sw128(sK(s) + koff, 16, 1024), idesc, kk > 0 ? 1u : 0u);
+              const uint64_t qo = ((kk >> 2) * L::kQPanel + (kk & 3) * 32u) >> 4;
+              const uint64_t ko = ((kk >> 2) * L::kRowsTile + (kk & 3) * 32u) >> 4;
+              mma_bf16(d_s, dq + qo, dk + ko, idesc, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
           }
@@ -236,13 +244,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
             tc_fence_after();
             const int np = (tile_tokens<TT>(it, jj) + kPB - 1) / kPB;
-            constexpr uint32_t idesc = idesc_bf16(128, D, true);
+            const uint64_t dv = dv0 + (uint64_t)s * kStageDesc;
             const uint32_t o_tmem = tmem + kTmemO + (uint32_t)(jj & 1) * 128u;
-            for (int kk = 0; kk < np; ++kk) {  // one page (16 tokens) per k-step
-              const uint64_t vd =
-                  smem_desc_sw128(sV(s) + kk * (kPB * 128u), L::kRowsTile, 1024);
-              mma_bf16_ts(o_tmem, tmem + (uint32_t)b * TT + kk * 8u, vd, idesc,
-                          (jj >= 2 || kk > 0) ? 1u : 0u);
+            const uint32_t p_tmem = tmem + (uint32_t)b * TT;
+            const uint32_t acc0 = jj >= 2 ? 1u : 0u;
+            if (np == kPagesPerTile) {
+#pragma unroll
+              for (int kk = 0; kk < kPagesPerTile; ++kk)  // one page (16 tokens) per k-step
+                mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
+                            idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
+            } else {
+              for (int kk = 0; kk < np; ++kk)
+                mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
+                            idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
             }
             mma_commit(o_full(b));
             mma_commit(empty(s));

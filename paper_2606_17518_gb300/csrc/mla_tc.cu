@@ -11,13 +11,11 @@
 // item produces one half of the value columns (dv0 = 0 or 256); the score tile
 // is computed for each half.  Per 32-token tile t (half a page):
 //   warp 0 (TMA)   nine boxes of 32 rows x 64 columns (128B swizzle) -> 2-stage ring
-//   warp 1 (MMA)   S_t = Q K_t^T as four independent accumulators (K split in
-//                  four 144-column pieces, issued interleaved so the tensor pipe
-//                  is not serialised on one accumulator), then
+//   warp 1 (MMA)   S_t = Q K_t^T (36 k-steps, N = 32), then
 //                  O += P_t V_t[:, dv0:dv0+256] (A = P in TMEM, N = 256)
-//   warps 2-5      one thread per head: sum of the four score pieces, masked,
-//                  online softmax in log2 units with lazy rescaling, P back to
-//                  TMEM as bf16 pairs.
+//   warps 2-5      one thread per head: the tile's scores, masked, online
+//                  softmax in log2 units with lazy rescaling, P back to TMEM
+//                  as bf16 pairs.
 // Value rows past a sequence inside its last tile are zeroed in shared memory
 // before the PV product; every wait is bounded.
 #include <cuda.h>
@@ -42,10 +40,9 @@ constexpr int kPage = 64;
 constexpr int kTT = 32;                      // tokens per tile (half a page)
 constexpr int kST = 2;                       // pipeline stages
 constexpr int kPanels = kDqk / 64;           // 9 column panels of 64
-constexpr int kChains = 4;                   // independent score accumulators
-constexpr int kStepsPerChain = kDqk / 16 / kChains;  // 9 k-steps each
+constexpr int kSteps = kDqk / 16;            // 36 k-steps of 16 for the scores
 constexpr int kThreads = 192;                // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
-constexpr uint32_t kTmemCols = 512;          // S[0] [0,128) S[1] [128,256) O [256,512)
+constexpr uint32_t kTmemCols = 512;          // S[0] [0,32) S[1] [32,64) O [256,512)
 constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr uint32_t kQPanel = 128 * 128u;     // 128 rows x 128 B
@@ -159,14 +156,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
+      // descriptors are built once; every MMA adds a constant offset to them
+      const uint64_t dq = smem_desc_sw128(sQ, 16, 1024);
+      const uint64_t dk0 = smem_desc_sw128(sK(0), 16, 1024);
+      const uint64_t dvb0 = smem_desc_sw128(sK(0), kKPanel, 1024);
+      constexpr uint64_t kStageDesc = kStage >> 4;
+      constexpr uint32_t idesc_s = idesc_bf16(128, kTT, false);
+      constexpr uint32_t idesc_pv = idesc_bf16(128, kDvHalf, true);
       int t = 0;
       bool ok = true;
-      const uint32_t idesc_s = idesc_bf16(128, kTT, false);
-      const uint32_t idesc_pv = idesc_bf16(128, kDvHalf, true);
       for (int ii = it_begin; ok && ii < it_end; ++ii) {
         const TcItem it = p.items[p.cta_items[ii]];
         const int ntiles = ntiles_of(it);
-        const int vpanel0 = it.dv0 / 64;
+        const uint64_t vpanel = (uint64_t)((it.dv0 / 64) * kKPanel) >> 4;
         if (!(ok = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status))) break;
         tc_fence_after();
         for (int j = 0; j <= ntiles; ++j) {
@@ -174,16 +176,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int u = t + j, s = u % kST, b = u & 1;
             if (!(ok = mbar_wait(full(s), (u / kST) & 1, abort_flag, p.status))) break;
             tc_fence_after();
+            const uint64_t dk = dk0 + (uint64_t)s * kStageDesc;
+            const uint32_t d_s = tmem + (uint32_t)b * kTT;
 #pragma unroll
-            for (int step = 0; step < kStepsPerChain; ++step) {
-#pragma unroll
-              for (int c = 0; c < kChains; ++c) {
-                const int kk = c * kStepsPerChain + step;
-                const uint32_t qoff = (kk >> 2) * kQPanel + (kk & 3) * 32u;
-                const uint32_t koff = (kk >> 2) * kKPanel + (kk & 3) * 32u;
-                mma_bf16(tmem + (uint32_t)b * 128u + c * 32u, smem_desc_sw128(sQ + qoff, 16, 1024),
-                         smem_desc_sw128(sK(s) + koff, 16, 1024), idesc_s, step > 0 ? 1u : 0u);
-              }
+            for (int kk = 0; kk < kSteps; ++kk) {
+              const uint64_t qo = ((kk >> 2) * kQPanel + (kk & 3) * 32u) >> 4;
+              const uint64_t ko = ((kk >> 2) * kKPanel + (kk & 3) * 32u) >> 4;
+              mma_bf16(d_s, dq + qo, dk + ko, idesc_s, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
           }
@@ -191,13 +190,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int u = t + j - 1, b = u & 1, s = u % kST;
             if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
             tc_fence_after();
+            const uint64_t dv = dvb0 + (uint64_t)s * kStageDesc + vpanel;
 #pragma unroll
-            for (int kk = 0; kk < kTT / 16; ++kk) {
-              const uint64_t vd =
-                  smem_desc_sw128(sK(s) + vpanel0 * kKPanel + kk * 2048u, kKPanel, 1024);
-              mma_bf16_ts(tmem + kTmemO, tmem + (uint32_t)b * 128u + kk * 8u, vd, idesc_pv,
+            for (int kk = 0; kk < kTT / 16; ++kk)
+              mma_bf16_ts(tmem + kTmemO, tmem + (uint32_t)b * kTT + kk * 8u,
+                          dv + (uint64_t)((kk * 2048u) >> 4), idesc_pv,
                           (j > 1 || kk > 0) ? 1u : 0u);
-            }
             mma_commit(o_full(b));
             mma_commit(empty(s));
           }
@@ -256,14 +254,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool page_ok = page >= 0 && page < p.num_pages;
         float s[kTT];
         {
-          uint32_t r[kChains][32];
-#pragma unroll
-          for (int c = 0; c < kChains; ++c) tmem_ld32(s_base + (uint32_t)b * 128u + c * 32u, r[c]);
+          uint32_t r[32];
+          tmem_ld32(s_base + (uint32_t)b * kTT, r);
           tmem_wait_ld();
 #pragma unroll
-          for (int i = 0; i < kTT; ++i)
-            s[i] = (__uint_as_float(r[0][i]) + __uint_as_float(r[1][i])) +
-                   (__uint_as_float(r[2][i]) + __uint_as_float(r[3][i]));
+          for (int i = 0; i < kTT; ++i) s[i] = __uint_as_float(r[i]);
         }
         if (nt < kTT || !page_ok) {
 #pragma unroll
@@ -296,7 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ps += p0 + p1;
             pk[i] = pack_bf16x2(p0, p1);
           }
-          tmem_st16(s_base + (uint32_t)b * 128u, pk);
+          tmem_st16(s_base + (uint32_t)b * kTT, pk);
           l += ps;
         }
         // value rows past the sequence in this tile: zero them before PV
