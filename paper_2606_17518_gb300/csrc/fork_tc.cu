@@ -215,19 +215,55 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t dv0 = smem_desc_sw128(sV(0), L::kRowsTile, 1024);
       constexpr uint64_t kStageDesc = L::kStage >> 4;
       constexpr uint32_t idesc_pv = idesc_bf16(128, D, true);
-      int t = 0;
+      // Ready-first issue: PV_v goes out as soon as its P is ready; S_u goes
+      // out when its K tile has landed, its score buffer is free (PV_{u-2}
+      // issued, so in-order execution has consumed P_{u-2}) and, for an item's
+      // first tile, its Q is in shared memory.  s_*: the next S to issue,
+      // v_*: the next PV to issue (item cursor, tile within item, global tile).
+      int s_ii = it_begin, s_j = 0, s_u = 0, v_ii = it_begin, v_j = 0, v_u = 0;
+      TcItem s_it = s_ii < it_end ? p.items[p.cta_items[s_ii]] : TcItem{};
+      TcItem v_it = s_it;
+      int s_nt = view<TT>(p, s_it).ntiles, v_nt = s_nt;
+      bool q_ok = false;
       bool ok = true;
-      for (int ii = it_begin; ok && ii < it_end; ++ii) {
-        const TcItem it = p.items[p.cta_items[ii]];
-        const ItemView v = view<TT>(p, it);
-        if (!(ok = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status))) break;
-        tc_fence_after();
-        for (int j = 0; j <= v.ntiles; ++j) {
-          if (j < v.ntiles) {  // S_u = Q K_u^T -> S[u%2]
-            const int u = t + j, s = u % ST, b = u & 1;
-            if (!(ok = mbar_wait(full(s), (u / ST) & 1, abort_flag, p.status))) break;
+      unsigned long long t0 = 0;
+      while (ok && v_ii < it_end) {
+        bool did = false;
+        if (v_u < s_u && mbar_try_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
+          tc_fence_after();
+          const int b = v_u & 1, s = v_u % ST;
+          const int np = (tile_tokens<TT>(v_it, v_j) + kPB - 1) / kPB;
+          const uint64_t dv = dv0 + (uint64_t)s * kStageDesc;
+          const uint32_t o_tmem = tmem + kTmemO + (uint32_t)(v_j & 1) * 128u;
+          const uint32_t p_tmem = tmem + (uint32_t)b * TT;
+          const uint32_t acc0 = v_j >= 2 ? 1u : 0u;
+          if (np == kPagesPerTile) {
+#pragma unroll
+            for (int kk = 0; kk < kPagesPerTile; ++kk)  // one page (16 tokens) per k-step
+              mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
+                          idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
+          } else {
+            for (int kk = 0; kk < np; ++kk)
+              mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
+                          idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
+          }
+          mma_commit(o_full(b));
+          mma_commit(empty(s));
+          ++v_u;
+          if (++v_j == v_nt) {
+            v_j = 0;
+            if (++v_ii < it_end) {
+              v_it = p.items[p.cta_items[v_ii]];
+              v_nt = view<TT>(p, v_it).ntiles;
+            }
+          }
+          did = true;
+        } else if (s_ii < it_end && s_u - v_u < 2) {
+          if (!q_ok && mbar_try_wait(q_ready, (s_ii - it_begin) & 1)) q_ok = true;
+          if (q_ok && mbar_try_wait(full(s_u % ST), (s_u / ST) & 1)) {
             tc_fence_after();
-            const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
+            const int b = s_u & 1, s = s_u % ST;
+            const int np = (tile_tokens<TT>(s_it, s_j) + kPB - 1) / kPB;
             const uint32_t idesc = idesc_bf16(128, np * kPB, false);
             const uint64_t dk = dk0 + (uint64_t)s * kStageDesc;
             const uint32_t d_s = tmem + (uint32_t)b * TT;
@@ -238,31 +274,29 @@ __global__ void __launch_bounds__(kThreads, 1)
               mma_bf16(d_s, dq + qo, dk + ko, idesc, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
-          }
-          if (j >= 1) {  // O[u%2] += P_u V_u (P_u in TMEM over S_u)
-            const int jj = j - 1, u = t + jj, b = u & 1, s = u % ST;
-            if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
-            tc_fence_after();
-            const int np = (tile_tokens<TT>(it, jj) + kPB - 1) / kPB;
-            const uint64_t dv = dv0 + (uint64_t)s * kStageDesc;
-            const uint32_t o_tmem = tmem + kTmemO + (uint32_t)(jj & 1) * 128u;
-            const uint32_t p_tmem = tmem + (uint32_t)b * TT;
-            const uint32_t acc0 = jj >= 2 ? 1u : 0u;
-            if (np == kPagesPerTile) {
-#pragma unroll
-              for (int kk = 0; kk < kPagesPerTile; ++kk)  // one page (16 tokens) per k-step
-                mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
-                            idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
-            } else {
-              for (int kk = 0; kk < np; ++kk)
-                mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
-                            idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
+            ++s_u;
+            if (++s_j == s_nt) {
+              s_j = 0;
+              q_ok = false;
+              if (++s_ii < it_end) {
+                s_it = p.items[p.cta_items[s_ii]];
+                s_nt = view<TT>(p, s_it).ntiles;
+              }
             }
-            mma_commit(o_full(b));
-            mma_commit(empty(s));
+            did = true;
           }
         }
-        t += v.ntiles;
+        if (did) {
+          t0 = 0;
+        } else if (t0 == 0) {
+          t0 = globaltimer();
+        } else if (*abort_flag) {
+          ok = false;
+        } else if (globaltimer() - t0 > kWaitLimitNs) {
+          atomicOr(p.status, kStatusTimeout);
+          *abort_flag = 1;
+          ok = false;
+        }
       }
       // every MMA issued by this thread has finished before TMEM is released
       mma_commit(mma_done);

@@ -163,19 +163,42 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint64_t kStageDesc = kStage >> 4;
       constexpr uint32_t idesc_s = idesc_bf16(128, kTT, false);
       constexpr uint32_t idesc_pv = idesc_bf16(128, kDvHalf, true);
-      int t = 0;
+      // Ready-first issue: PV_v goes out as soon as its P is ready; S_u goes
+      // out when its K tile has landed, its score buffer is free (PV_{u-2}
+      // issued, so in-order execution has consumed P_{u-2}) and, for an item's
+      // first tile, its Q is in shared memory.  s_*: the next S to issue,
+      // v_*: the next PV to issue (item cursor, tile within item, global tile).
+      int s_ii = it_begin, s_j = 0, s_u = 0, v_ii = it_begin, v_j = 0, v_u = 0;
+      TcItem s_it = s_ii < it_end ? p.items[p.cta_items[s_ii]] : TcItem{};
+      TcItem v_it = s_it;
+      bool q_ok = false;  // Q of the item at s_ii is known to be loaded
       bool ok = true;
-      for (int ii = it_begin; ok && ii < it_end; ++ii) {
-        const TcItem it = p.items[p.cta_items[ii]];
-        const int ntiles = ntiles_of(it);
-        const uint64_t vpanel = (uint64_t)((it.dv0 / 64) * kKPanel) >> 4;
-        if (!(ok = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status))) break;
-        tc_fence_after();
-        for (int j = 0; j <= ntiles; ++j) {
-          if (j < ntiles) {
-            const int u = t + j, s = u % kST, b = u & 1;
-            if (!(ok = mbar_wait(full(s), (u / kST) & 1, abort_flag, p.status))) break;
+      unsigned long long t0 = 0;
+      while (ok && v_ii < it_end) {
+        bool did = false;
+        if (v_u < s_u && mbar_try_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
+          tc_fence_after();
+          const int b = v_u & 1, s = v_u % kST;
+          const uint64_t vpanel = (uint64_t)((v_it.dv0 / 64) * kKPanel) >> 4;
+          const uint64_t dv = dvb0 + (uint64_t)s * kStageDesc + vpanel;
+#pragma unroll
+          for (int kk = 0; kk < kTT / 16; ++kk)
+            mma_bf16_ts(tmem + kTmemO, tmem + (uint32_t)b * kTT + kk * 8u,
+                        dv + (uint64_t)((kk * 2048u) >> 4), idesc_pv,
+                        (v_j > 0 || kk > 0) ? 1u : 0u);
+          mma_commit(o_full(b));
+          mma_commit(empty(s));
+          ++v_u;
+          if (++v_j == ntiles_of(v_it)) {
+            v_j = 0;
+            if (++v_ii < it_end) v_it = p.items[p.cta_items[v_ii]];
+          }
+          did = true;
+        } else if (s_ii < it_end && s_u - v_u < 2) {
+          if (!q_ok && mbar_try_wait(q_ready, (s_ii - it_begin) & 1)) q_ok = true;
+          if (q_ok && mbar_try_wait(full(s_u % kST), (s_u / kST) & 1)) {
             tc_fence_after();
+            const int b = s_u & 1, s = s_u % kST;
             const uint64_t dk = dk0 + (uint64_t)s * kStageDesc;
             const uint32_t d_s = tmem + (uint32_t)b * kTT;
 #pragma unroll
@@ -185,22 +208,26 @@ __global__ void __launch_bounds__(kThreads, 1)
               mma_bf16(d_s, dq + qo, dk + ko, idesc_s, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
-          }
-          if (j >= 1) {
-            const int u = t + j - 1, b = u & 1, s = u % kST;
-            if (!(ok = mbar_wait(p_full(b), (u >> 1) & 1, abort_flag, p.status))) break;
-            tc_fence_after();
-            const uint64_t dv = dvb0 + (uint64_t)s * kStageDesc + vpanel;
-#pragma unroll
-            for (int kk = 0; kk < kTT / 16; ++kk)
-              mma_bf16_ts(tmem + kTmemO, tmem + (uint32_t)b * kTT + kk * 8u,
-                          dv + (uint64_t)((kk * 2048u) >> 4), idesc_pv,
-                          (j > 1 || kk > 0) ? 1u : 0u);
-            mma_commit(o_full(b));
-            mma_commit(empty(s));
+            ++s_u;
+            if (++s_j == ntiles_of(s_it)) {
+              s_j = 0;
+              q_ok = false;
+              if (++s_ii < it_end) s_it = p.items[p.cta_items[s_ii]];
+            }
+            did = true;
           }
         }
-        t += ntiles;
+        if (did) {
+          t0 = 0;
+        } else if (t0 == 0) {
+          t0 = globaltimer();
+        } else if (*abort_flag) {
+          ok = false;
+        } else if (globaltimer() - t0 > kWaitLimitNs) {
+          atomicOr(p.status, kStatusTimeout);
+          *abort_flag = 1;
+          ok = false;
+        }
       }
       mma_commit(mma_done);
       mbar_wait_drain(mma_done, 0, p.status);
