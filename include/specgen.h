@@ -84,11 +84,15 @@ typedef struct {
 
 /* Host copies of the lengths: planning reads them, so no device->host copy is
  * needed.  The device block tables must hold at least ceil(len/page_size)
- * pages for every sequence. */
+ * pages for every sequence.  The two block-table offset arrays are optional
+ * host copies of args->prefix_bt_offsets / suffix_bt_offsets; when given (both
+ * non-NULL) the kernels skip one dependent device load per work item. */
 typedef struct {
   const int32_t* prefix_lens;   /* host [num_traces], >= 0 */
   const int32_t* fork_offsets;  /* host [num_traces + 1], non-decreasing, [0]=0, [T]=F */
   const int32_t* suffix_lens;   /* host [total_forks], >= 0 */
+  const int32_t* prefix_bt_offsets;  /* host [num_traces + 1] or NULL */
+  const int32_t* suffix_bt_offsets;  /* host [total_forks + 1] or NULL */
 } specgen_host_lens;
 
 /* Result of planning: work counts and workspace offsets.  Treat as opaque;

@@ -54,7 +54,8 @@ class ForkAttnArgs(C.Structure):
 
 class HostLens(C.Structure):
     _fields_ = [("prefix_lens", C.c_void_p), ("fork_offsets", C.c_void_p),
-                ("suffix_lens", C.c_void_p)]
+                ("suffix_lens", C.c_void_p), ("prefix_bt_offsets", C.c_void_p),
+                ("suffix_bt_offsets", C.c_void_p)]
 
 
 class Plan(C.Structure):
@@ -129,11 +130,12 @@ def _ptr(t) -> int | None:
     return t.data_ptr()
 
 
-def make_host_lens(prefix_lens, fork_offsets, suffix_lens):
+def make_host_lens(prefix_lens, fork_offsets, suffix_lens, prefix_bt_offsets=None,
+                   suffix_bt_offsets=None):
     """HostLens over int32 numpy arrays (kept alive by the returned tuple)."""
-    arrs = tuple(np.ascontiguousarray(a, dtype=np.int32) for a in
-                 (prefix_lens, fork_offsets, suffix_lens))
-    return HostLens(*(a.ctypes.data for a in arrs)), arrs
+    arrs = tuple(None if a is None else np.ascontiguousarray(a, dtype=np.int32) for a in
+                 (prefix_lens, fork_offsets, suffix_lens, prefix_bt_offsets, suffix_bt_offsets))
+    return HostLens(*(None if a is None else a.ctypes.data for a in arrs)), arrs
 
 
 def make_args(*, num_traces, total_forks, hq, hkv, head_dim_qk, head_dim_v, page_size,

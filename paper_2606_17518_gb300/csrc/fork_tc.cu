@@ -77,8 +77,9 @@ struct ItemView {
 template <int TT>
 __device__ __forceinline__ ItemView view(const TcParams& p, const TcItem& it) {
   ItemView v;
-  v.table = it.table_kind == 0 ? p.prefix_bt + p.prefix_bt_off[it.seq]
-                               : p.suffix_bt + p.suffix_bt_off[it.seq];
+  const int32_t* bt = it.table_kind == 0 ? p.prefix_bt : p.suffix_bt;
+  v.table = bt + (it.table_off >= 0 ? it.table_off
+                                    : (it.table_kind == 0 ? p.prefix_bt_off : p.suffix_bt_off)[it.seq]);
   v.ntiles = (it.tok_end - it.tok_begin + TT - 1) / TT;
   v.page0 = it.tok_begin / kPB;
   v.M = it.nforks * p.G;
@@ -164,7 +165,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int t = 0;  // tiles issued so far (across items)
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[p.cta_items[ii]];
+      const TcItem it = p.items[ii];
       const ItemView v = view<TT>(p, it);
       const int npages = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
       int cur = lane < npages ? v.table[v.page0 + lane] : 0;
@@ -221,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // first tile, its Q is in shared memory.  s_*: the next S to issue,
       // v_*: the next PV to issue (item cursor, tile within item, global tile).
       int s_ii = it_begin, s_j = 0, s_u = 0, v_ii = it_begin, v_j = 0, v_u = 0;
-      TcItem s_it = s_ii < it_end ? p.items[p.cta_items[s_ii]] : TcItem{};
+      TcItem s_it = s_ii < it_end ? p.items[s_ii] : TcItem{};
       TcItem v_it = s_it;
       int s_nt = view<TT>(p, s_it).ntiles, v_nt = s_nt;
       bool q_ok = false;
@@ -253,7 +254,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (++v_j == v_nt) {
             v_j = 0;
             if (++v_ii < it_end) {
-              v_it = p.items[p.cta_items[v_ii]];
+              v_it = p.items[v_ii];
               v_nt = view<TT>(p, v_it).ntiles;
             }
           }
@@ -279,7 +280,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               s_j = 0;
               q_ok = false;
               if (++s_ii < it_end) {
-                s_it = p.items[p.cta_items[s_ii]];
+                s_it = p.items[s_ii];
                 s_nt = view<TT>(p, s_it).ntiles;
               }
             }
@@ -319,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
 
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[p.cta_items[ii]];
+      const TcItem it = p.items[ii];
       const ItemView v = view<TT>(p, it);
       const bool warp_live = q4 * 32 < v.M;  // some real row in this warp
       const bool row_ok = row < v.M;

@@ -15,8 +15,7 @@ struct TcParams {
   const int32_t* suffix_bt;
   const int32_t* suffix_bt_off;
   const TcItem* items;
-  const int32_t* cta_items;    // item indices, grouped per CTA
-  const int32_t* cta_offsets;  // [grid + 1] into cta_items
+  const int32_t* cta_offsets;  // [grid + 1]: CTA c takes items [cta_offsets[c], cta_offsets[c+1])
   const int32_t* part_base;    // [forks] first partial slot of each fork
   float* part_o;               // [slots][hq][dv]
   float* part_lse;             // [slots][hq]

@@ -82,8 +82,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
   auto table_of = [&](const TcItem& it) {
-    return it.table_kind == 0 ? p.prefix_bt + p.prefix_bt_off[it.seq]
-                              : p.suffix_bt + p.suffix_bt_off[it.seq];
+    const int32_t* bt = it.table_kind == 0 ? p.prefix_bt : p.suffix_bt;
+    return bt + (it.table_off >= 0 ? it.table_off
+                                   : (it.table_kind == 0 ? p.prefix_bt_off : p.suffix_bt_off)[it.seq]);
   };
   auto ntiles_of = [&](const TcItem& it) { return (it.tok_end - it.tok_begin + kTT - 1) / kTT; };
   auto tile_tokens = [&](const TcItem& it, int j) {
@@ -120,7 +121,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int t = 0;
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[p.cta_items[ii]];
+      const TcItem it = p.items[ii];
       const int32_t* table = table_of(it);
       const int ntiles = ntiles_of(it);
       const int page0 = it.tok_begin / kPage;
@@ -169,7 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // first tile, its Q is in shared memory.  s_*: the next S to issue,
       // v_*: the next PV to issue (item cursor, tile within item, global tile).
       int s_ii = it_begin, s_j = 0, s_u = 0, v_ii = it_begin, v_j = 0, v_u = 0;
-      TcItem s_it = s_ii < it_end ? p.items[p.cta_items[s_ii]] : TcItem{};
+      TcItem s_it = s_ii < it_end ? p.items[s_ii] : TcItem{};
       TcItem v_it = s_it;
       bool q_ok = false;  // Q of the item at s_ii is known to be loaded
       bool ok = true;
@@ -191,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++v_u;
           if (++v_j == ntiles_of(v_it)) {
             v_j = 0;
-            if (++v_ii < it_end) v_it = p.items[p.cta_items[v_ii]];
+            if (++v_ii < it_end) v_it = p.items[v_ii];
           }
           did = true;
         } else if (s_ii < it_end && s_u - v_u < 2) {
@@ -212,7 +213,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (++s_j == ntiles_of(s_it)) {
               s_j = 0;
               q_ok = false;
-              if (++s_ii < it_end) s_it = p.items[p.cta_items[s_ii]];
+              if (++s_ii < it_end) s_it = p.items[s_ii];
             }
             did = true;
           }
@@ -244,7 +245,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int t = 0, oc = 0;  // tiles done; next o_full phase (tile index) to consume
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[p.cta_items[ii]];
+      const TcItem it = p.items[ii];
       const int32_t* table = table_of(it);
       const int ntiles = ntiles_of(it);
       const int page0 = it.tok_begin / kPage;

@@ -15,8 +15,7 @@ struct MlaParams {
   const int32_t* suffix_bt;
   const int32_t* suffix_bt_off;
   const TcItem* items;         // dv0 selects the value half (0 or 256)
-  const int32_t* cta_items;
-  const int32_t* cta_offsets;
+  const int32_t* cta_offsets;  // [grid + 1]: CTA c takes items [cta_offsets[c], cta_offsets[c+1])
   const int32_t* part_base;
   float* part_o;               // [slots][128][512]
   float* part_lse;             // [slots][128]

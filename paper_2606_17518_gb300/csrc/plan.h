@@ -43,6 +43,8 @@ struct TcItem {
   int32_t tok_end;
   int32_t part;
   int32_t dv0;         // first value column this item produces (latent KV: 0 or 256)
+  int32_t table_off;   // index of the sequence's first page in its block table, or -1
+                       // (then the kernel reads it from the device offset array)
 };
 
 // Plan header at the start of the plan region.

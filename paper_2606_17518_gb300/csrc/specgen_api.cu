@@ -128,6 +128,28 @@ void assign_lpt(const std::vector<long long>& cost, int n_cta, std::vector<int32
   }
 }
 
+// Assign tensor-core items to CTAs (longest first), store them in CTA order so
+// that CTA c walks items [cta_offsets[c], cta_offsets[c+1]), and resolve each
+// item's block-table start on the host when the host table offsets are given.
+void finish_tc_plan(HostPlan* hp, const std::vector<long long>& cost, int n_sm,
+                    const specgen_host_lens* lens) {
+  const int n_cta = (int)std::min<size_t>((size_t)n_sm, hp->tc.size());
+  std::vector<int32_t> order;
+  assign_lpt(cost, n_cta, &order, &hp->cta_offsets);
+  std::vector<TcItem> sorted;
+  sorted.reserve(hp->tc.size());
+  const bool host_off = lens->prefix_bt_offsets && lens->suffix_bt_offsets;
+  for (int32_t i : order) {
+    TcItem it = hp->tc[i];
+    it.table_off = host_off ? (it.table_kind == 0 ? lens->prefix_bt_offsets[it.seq]
+                                                  : lens->suffix_bt_offsets[it.seq])
+                            : -1;
+    sorted.push_back(it);
+  }
+  hp->tc.swap(sorted);
+  hp->cta_items.clear();
+}
+
 void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   const int n_sm = device_sm_count();
   const int32_t* fo = lens->fork_offsets;
@@ -156,7 +178,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
     long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
     chunk = std::max<long long>(fork_tc_tile_tokens(), (chunk + pg - 1) / pg * pg);
     std::vector<long long> cost;
-    const long long item_overhead = 64;  // token-equivalents per item (Q load, output write)
+    const long long item_overhead = 128;  // token-equivalents per item (Q load, output write)
     for (int t = 0; t < s.T; ++t) {
       const int P = lens->prefix_lens[t];
       const int np = (int)((P + chunk - 1) / chunk);
@@ -199,8 +221,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
             cost.push_back(it.tok_end - it.tok_begin + item_overhead);
           }
     }
-    const int n_cta = (int)std::min<size_t>((size_t)n_sm, hp->tc.size());
-    assign_lpt(cost, n_cta, &hp->cta_items, &hp->cta_offsets);
+    finish_tc_plan(hp, cost, n_sm, lens);
     hp->total_slots = slot;
     return;
   }
@@ -216,7 +237,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
     long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
     chunk = std::max<long long>(4 * tt, (chunk + tt - 1) / tt * tt);
     std::vector<long long> cost;
-    const long long item_overhead = 64;
+    const long long item_overhead = 128;
     for (int t = 0; t < s.T; ++t) {
       const int P = lens->prefix_lens[t];
       const int np = (int)((P + chunk - 1) / chunk);
@@ -246,8 +267,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
           }
       }
     }
-    const int n_cta = (int)std::min<size_t>((size_t)n_sm, hp->tc.size());
-    assign_lpt(cost, n_cta, &hp->cta_items, &hp->cta_offsets);
+    finish_tc_plan(hp, cost, n_sm, lens);
     hp->total_slots = slot;
     return;
   }
@@ -495,7 +515,6 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     tp.suffix_bt = args->suffix_block_table;
     tp.suffix_bt_off = args->suffix_bt_offsets;
     tp.items = reinterpret_cast<const TcItem*>(pl + plan->offsets[1]);
-    tp.cta_items = reinterpret_cast<const int32_t*>(pl + plan->offsets[2]);
     tp.cta_offsets = reinterpret_cast<const int32_t*>(pl + plan->offsets[3]);
     tp.part_base = reinterpret_cast<const int32_t*>(pl + plan->offsets[4]);
     tp.part_o = part_o;
@@ -516,7 +535,6 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
       mp.suffix_bt = tp.suffix_bt;
       mp.suffix_bt_off = tp.suffix_bt_off;
       mp.items = tp.items;
-      mp.cta_items = tp.cta_items;
       mp.cta_offsets = tp.cta_offsets;
       mp.part_base = tp.part_base;
       mp.part_o = part_o;

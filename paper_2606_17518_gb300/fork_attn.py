@@ -45,7 +45,8 @@ class ForkDecode:
         self.out = torch.empty((F, hq, dv), dtype=torch.bfloat16, device=device)
         self.lse = torch.empty((F, hq), dtype=torch.float32, device=device)
         self.lens, self._lens_keep = _lib.make_host_lens(
-            w["prefix_lens"], w["fork_offsets"], w["suffix_lens"])
+            w["prefix_lens"], w["fork_offsets"], w["suffix_lens"], w["prefix_bt_offsets"],
+            w["suffix_bt_offsets"])
         self.ws_bytes = _lib.specgen_fork_attn_workspace_size(self.args(with_ws=False), self.lens)
         if self.ws_bytes == 0:
             raise _lib.SpecgenError(_lib.SPECGEN_ERR_SHAPE, "specgen_fork_attn_workspace_size")

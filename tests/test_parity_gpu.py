@@ -192,3 +192,19 @@ def test_lse_merge_standalone(dtype):
     _lib.specgen_lse_merge(d_oa, d_la, d_ob, d_lb, d_oa, d_la, rows, dv, dtype)
     torch.cuda.synchronize()
     assert torch.equal(d_oa, d_o) and torch.equal(d_la, d_l)
+
+
+def test_without_host_table_offsets():
+    """The host copies of the block-table offsets are optional (device lookup)."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    for name in ["fork_p8k_f8", "mla_p16k_f8"]:
+        w = wl.make_workload(name)
+        fd = ForkDecode(w)
+        lens, keep = _lib.make_host_lens(w["prefix_lens"], w["fork_offsets"], w["suffix_lens"])
+        _lib.specgen_fork_attn_decode(fd.args(), lens)
+        torch.cuda.synchronize()
+        o, lse = fd.results()
+        fd.decode()
+        o2, l2 = fd.results()
+        assert np.array_equal(o, o2) and np.array_equal(lse, l2)
