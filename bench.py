@@ -42,6 +42,9 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--kv-layout", choices=["auto", "rows", "tiled"], default="auto",
+                    help="K/V pool layout: token-major rows or 8x8 tiles (auto: tiled where the "
+                         "tensor-core path supports it)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
     return ap.parse_args()
@@ -212,7 +215,7 @@ def kernel_source_sha(name: str) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2606_17518_gb300", "csrc")
     for fn in sorted(os.listdir(csrc)):
-        if fn.startswith(name) or fn in ("common.cuh", "plan.h"):
+        if fn.startswith(name) or fn in ("common.cuh", "plan.h", "tc_common.cuh"):
             with open(os.path.join(csrc, fn), "rb") as fh:
                 h.update(fh.read())
     return h.hexdigest()[:16]
@@ -267,7 +270,11 @@ def run_ours():
         f" {replicas} replicas")
     stream = torch.cuda.Stream(dev)
     sp = stream.cuda_stream
-    reps = [ForkDecode(w, device=dev) for _ in range(replicas)]
+    tiled_ok = (w["v_pages"] is not None and w["page_size"] == 16 and w["dqk"] == w["dv"]
+                and w["dqk"] in (64, 128) and w["hq"] // w["hkv"] <= 128)
+    layout = ARGS.kv_layout if ARGS.kv_layout != "auto" else ("tiled" if tiled_ok else "rows")
+    kv_layout = _lib.KV_TILED if layout == "tiled" else _lib.KV_ROWS
+    reps = [ForkDecode(w, device=dev, kv_layout=kv_layout) for _ in range(replicas)]
     with torch.cuda.stream(stream):
         for r in reps:
             r.plan(sp)
@@ -377,7 +384,22 @@ def run_ours():
     else:
         dom_bytes = nbytes["total"]
     achieved = dom_bytes / (kernel_ms[dom] * 1e-3) / 1e9 if kernel_ms else None
-    traffic = recorded_traffic(kernel_names[dom], ARGS.workload)
+    traffic = recorded_traffic(kernel_names[dom], f"{ARGS.workload}:{layout}")
+    if dom_name == "mla_tc":
+        # latent attention is a dense contraction (the 128 heads of a fork share
+        # every latent key): bound by the bf16 tensor pipe, timed inside a long
+        # loop of steps, so against the sustained bf16 peak
+        tflops = flops["total"] / (kernel_ms[dom] * 1e-3) / 1e12
+        roofline = {"bound": "tensor", "kernel": dom_name, "achieved": tflops, "peak": tf_sus,
+                    "unit": "TFLOP/s", "frac": tflops / tf_sus, "traffic": traffic,
+                    "peak_source": peak_src + " (bf16, sustained)",
+                    "algorithmic_flops_per_launch": flops["total"],
+                    "hbm_achieved_gbs": achieved}
+    else:
+        roofline = {"bound": "hbm", "kernel": dom_name, "achieved": achieved, "peak": hbm,
+                    "unit": "GB/s", "frac": achieved / hbm if achieved else None,
+                    "traffic": traffic, "peak_source": peak_src,
+                    "algorithmic_bytes_per_launch": dom_bytes}
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
@@ -387,7 +409,7 @@ def run_ours():
             "workload": ARGS.workload, "traces": w["num_traces"], "forks": F,
             "prefix_tokens": int(np.sum(w["prefix_lens"])),
             "suffix_tokens": int(np.sum(w["suffix_lens"])), "hq": w["hq"], "hkv": w["hkv"],
-            "head_dim": [w["dqk"], w["dv"]], "page_size": w["page_size"],
+            "head_dim": [w["dqk"], w["dv"]], "page_size": w["page_size"], "kv_layout": layout,
             "unique_bytes": nbytes["total"], "flops": flops["total"],
             "l2": f"inputs rotate over {replicas} resident replicas (>= 3x L2)",
             "timing": f"CUDA graphs of {per_graph} steps; per-kernel times from the last "
@@ -398,11 +420,7 @@ def run_ours():
         "kernels": {n: {"ms_per_launch": t, "share": t / max(1e-12, sum(kernel_ms))}
                     for n, t in zip(kernel_names, kernel_ms)},
         "achieved_gbs_whole_step": nbytes["total"] / (ms_per_step * 1e-3) / 1e9,
-        "roofline": {"bound": "hbm", "kernel": kernel_names[dom] if kernel_names else None,
-                     "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm if achieved else None, "traffic": traffic,
-                     "peak_source": peak_src,
-                     "algorithmic_bytes_per_launch": dom_bytes},
+        "roofline": roofline,
         "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
         "e2e": e2e,
     }

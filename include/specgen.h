@@ -19,8 +19,9 @@
  * rounding.
  *
  * Paged KV layout (caller-owned device memory, never freed by the library):
- *     k_pages  bf16 [num_pages][hkv][page_size][head_dim_qk]
- *     v_pages  bf16 [num_pages][hkv][page_size][head_dim_v]
+ *     k_pages  bf16 [num_pages][hkv][page_size x head_dim_qk block]
+ *     v_pages  bf16 [num_pages][hkv][page_size x head_dim_v block]
+ *              (block element order: args->kv_layout, see SPECGEN_KV_*)
  *              or NULL: latent KV, value row = first head_dim_v columns of the
  *              key row (MLA-style absorbed attention, hkv = 1 typically).
  *     Token j of a sequence lives in page table[j / page_size] at slot
@@ -80,7 +81,22 @@ typedef struct {
   float* lse;                   /* fp32 [total_forks][hq] natural-log LSE (written) */
   void* workspace;              /* >= specgen_fork_attn_workspace_size bytes, 256-B aligned */
   size_t workspace_bytes;
+  int kv_layout;                /* SPECGEN_KV_ROWS or SPECGEN_KV_TILED (see below) */
 } specgen_fork_attn_args;
+
+/* Layout of one (page, kv head) block of page_size x head_dim values in the
+ * separate K and V pools:
+ *   SPECGEN_KV_ROWS   token-major rows: element (t, d) at t * head_dim + d.
+ *   SPECGEN_KV_TILED  8 x 8 tiles: element (t, d) at
+ *                     ((t/8) * (head_dim/8) + d/8) * 64 + (t%8) * 8 + d%8,
+ *                     so the block is exactly the tensor cores' operand layout
+ *                     and moves with one bulk copy.  Requires the tensor-core
+ *                     path (separate V pool, head_dim 64 or 128, page_size 16).
+ * The latent pool (v_pages == NULL) is always token-major (kv_layout must be
+ * SPECGEN_KV_ROWS there).  Any other value: SPECGEN_ERR_SHAPE; TILED on a
+ * shape outside the tensor-core path: SPECGEN_ERR_UNSUPPORTED. */
+#define SPECGEN_KV_ROWS 0
+#define SPECGEN_KV_TILED 1
 
 /* Host copies of the lengths: planning reads them, so no device->host copy is
  * needed.  The device block tables must hold at least ceil(len/page_size)

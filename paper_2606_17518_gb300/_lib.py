@@ -48,8 +48,12 @@ class ForkAttnArgs(C.Structure):
         ("prefix_block_table", C.c_void_p), ("prefix_bt_offsets", C.c_void_p),
         ("suffix_block_table", C.c_void_p), ("suffix_bt_offsets", C.c_void_p),
         ("out", C.c_void_p), ("lse", C.c_void_p),
-        ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t),
+        ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("kv_layout", C.c_int),
     ]
+
+
+KV_ROWS = 0
+KV_TILED = 1
 
 
 class HostLens(C.Structure):
@@ -141,13 +145,13 @@ def make_host_lens(prefix_lens, fork_offsets, suffix_lens, prefix_bt_offsets=Non
 def make_args(*, num_traces, total_forks, hq, hkv, head_dim_qk, head_dim_v, page_size,
               num_pages, scale, q, k_pages, v_pages, prefix_block_table, prefix_bt_offsets,
               suffix_block_table, suffix_bt_offsets, out, lse, workspace=None,
-              workspace_bytes=0) -> ForkAttnArgs:
+              workspace_bytes=0, kv_layout=KV_ROWS) -> ForkAttnArgs:
     return ForkAttnArgs(
         int(num_traces), int(total_forks), int(hq), int(hkv), int(head_dim_qk),
         int(head_dim_v), int(page_size), int(num_pages), float(scale),
         _ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(prefix_block_table),
         _ptr(prefix_bt_offsets), _ptr(suffix_block_table), _ptr(suffix_bt_offsets),
-        _ptr(out), _ptr(lse), _ptr(workspace), int(workspace_bytes))
+        _ptr(out), _ptr(lse), _ptr(workspace), int(workspace_bytes), int(kv_layout))
 
 
 def specgen_fork_attn_workspace_size(args: ForkAttnArgs, lens: HostLens) -> int:

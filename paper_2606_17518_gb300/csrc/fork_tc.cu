@@ -18,6 +18,14 @@
 //                    is rescaled only when a row's max grows by more than
 //                    2^8 (lazy rescaling), otherwise P may exceed 1.
 // S is double-buffered in TMEM so S_{t+1} runs while tile t is in softmax.
+//
+// Two KV pool layouts.  Rows: every (page, head) block is 16 token rows of D
+// contiguous elements; the TMA engine gathers it with 64-column boxes into
+// 128B-swizzled panels.  Tiled: every block is stored as the tensor cores'
+// 8-token x 8-element core matrices, ((t/8)*(D/8) + d/8)*64 + (t%8)*8 + d%8,
+// so one contiguous bulk copy (D*32 bytes) lands it in the layout the MMA
+// reads directly (no swizzle): K is then K-major with 128-byte steps along d
+// and D*16-byte steps per 8 tokens, V is MN-major with the same two strides.
 // Warps whose 32 rows are all padding skip the softmax work.  Tokens past the
 // item, past the sequence or on an invalid page are masked to -inf, and value
 // rows past the sequence inside its last page are zeroed in shared memory
@@ -25,6 +33,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
+#include <string.h>
 
 #include "common.cuh"
 #include "fork_tc.h"
@@ -92,7 +101,7 @@ __device__ __forceinline__ int tile_tokens(const TcItem& it, int j) {
   return n < TT ? n : TT;
 }
 
-template <int D, int TT, int ST>
+template <int D, int TT, int ST, bool TL>
 __global__ void __launch_bounds__(kThreads, 1)
     fork_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tmk,
                    const __grid_constant__ CUtensorMap tmv) {
@@ -157,7 +166,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // The whole warp fetches page ids 32 at a time (one coalesced load, one
     // batch ahead).  Lane 0 waits for a free stage; then lanes 0..2*D/64-1
     // each issue one box of every page (K and V, one 64-column panel each).
-    constexpr int kIssuers = 2 * L::kPanels;
+    constexpr int kIssuers = TL ? 2 * kPagesPerTile : 2 * L::kPanels;
     const bool issuer = lane < kIssuers;
     const bool is_v = lane >= L::kPanels;
     const int pn = is_v ? lane - L::kPanels : lane;
@@ -180,6 +189,38 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int pg = 0; pg < kPagesPerTile; ++pg)
             pages[pg] = __shfl_sync(0xffffffffu, cur, tp + pg);
           const int s = t % ST;
+          if constexpr (TL) {
+            // one bulk copy per (page, K or V); an invalid page is reported and
+            // its value block zeroed here instead (its scores are masked)
+            constexpr uint32_t kBlk = kPB * D * 2u;
+            uint32_t bad = 0;
+#pragma unroll
+            for (int pg = 0; pg < kPagesPerTile; ++pg)
+              if (pg < np && (pages[pg] < 0 || pages[pg] >= p.num_pages)) bad |= 1u << pg;
+            if (lane == 0) ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            if (bad) {
+              for (int pg = 0; pg < np; ++pg)
+                if ((bad >> pg) & 1u)
+                  for (uint32_t x = lane * 16u; x < kBlk; x += 32u * 16u)
+                    st_shared_v4(sV(s) + pg * kBlk + x, 0u, 0u, 0u, 0u);
+              fence_proxy_async_smem();
+              __syncwarp();
+              if (lane == 0) atomicOr(p.status, kStatusIndex);
+            }
+            if (lane == 0)
+              mbar_arrive_expect_tx(full(s), (uint32_t)(np - __popc(bad)) * 2u * kBlk);
+            __syncwarp();
+            const int pg = lane % kPagesPerTile;
+            if (issuer && pg < np && !((bad >> pg) & 1u)) {
+              const bool v_side = lane >= kPagesPerTile;
+              const __nv_bfloat16* src = (v_side ? p.v_pages : p.k_pages) +
+                                         ((size_t)pages[pg] * p.hkv + it.kv_head) * (kPB * D);
+              bulk_load((v_side ? sV(s) : sK(s)) + pg * kBlk, src, kBlk, full(s));
+            }
+            continue;
+          }
           if (lane == 0) {
             ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
             if (ok) mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
@@ -212,8 +253,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       // descriptors are built once; every MMA only adds a constant offset
       // (in 16-byte units) to the start-address field
       const uint64_t dq = smem_desc_sw128(sQ, 16, 1024);
-      const uint64_t dk0 = smem_desc_sw128(sK(0), 16, 1024);
-      const uint64_t dv0 = smem_desc_sw128(sV(0), L::kRowsTile, 1024);
+      // tiled: K-major K (LBO = next 8 columns, SBO = next 8 tokens); MN-major V
+      // (LBO = next 8 tokens, SBO = next 8 columns)
+      const uint64_t dk0 = TL ? smem_desc_interleave(sK(0), 128, D * 16)
+                              : smem_desc_sw128(sK(0), 16, 1024);
+      const uint64_t dv0 = TL ? smem_desc_interleave(sV(0), D * 16, 128)
+                              : smem_desc_sw128(sV(0), L::kRowsTile, 1024);
+      // byte step of V per page (one 16-token k-step) and of K per 16 columns
+      constexpr uint32_t kVPage = TL ? kPB * D * 2u : kPB * 128u;
       constexpr uint64_t kStageDesc = L::kStage >> 4;
       constexpr uint32_t idesc_pv = idesc_bf16(128, D, true);
       // Ready-first issue: PV_v goes out as soon as its P is ready; S_u goes
@@ -241,11 +288,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (np == kPagesPerTile) {
 #pragma unroll
             for (int kk = 0; kk < kPagesPerTile; ++kk)  // one page (16 tokens) per k-step
-              mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
+              mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kVPage) >> 4),
                           idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
           } else {
             for (int kk = 0; kk < np; ++kk)
-              mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kPB * 128u) >> 4),
+              mma_bf16_ts(o_tmem, p_tmem + kk * 8u, dv + (uint64_t)((kk * kVPage) >> 4),
                           idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
           }
           mma_commit(o_full(b));
@@ -271,7 +318,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint64_t qo = ((kk >> 2) * L::kQPanel + (kk & 3) * 32u) >> 4;
-              const uint64_t ko = ((kk >> 2) * L::kRowsTile + (kk & 3) * 32u) >> 4;
+              const uint64_t ko =
+                  (TL ? kk * 256u : (kk >> 2) * L::kRowsTile + (kk & 3) * 32u) >> 4;
               mma_bf16(d_s, dq + qo, dk + ko, idesc, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
@@ -457,12 +505,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // value rows past the sequence inside its last page: zero them before PV
         if (j == v.ntiles - 1 && (nt % kPB) != 0) {
           const int pg = np - 1, first = nt % kPB;
-          const int units = (kPB - first) * L::kPanels * 8;
+          const int units = (kPB - first) * L::kPanels * 8;  // 16-byte pieces
           for (int x = gtid; x < units; x += 128) {
             const int rr = first + x / (L::kPanels * 8);
-            const int rem = x % (L::kPanels * 8);
-            st_shared_v4(sV(u % ST) + (rem >> 3) * L::kRowsTile + (pg * kPB + rr) * 128u +
-                             ((rem & 7) << 4), 0u, 0u, 0u, 0u);
+            const int rem = x % (L::kPanels * 8);  // 8-column chunk of the row
+            const int tt = pg * kPB + rr;
+            const uint32_t off = TL ? ((tt >> 3) * (D / 8) + rem) * 128u + (tt & 7) * 16u
+                                    : (rem >> 3) * L::kRowsTile + tt * 128u + ((rem & 7) << 4);
+            st_shared_v4(sV(u % ST) + off, 0u, 0u, 0u, 0u);
           }
           fence_proxy_async_smem();
         }
@@ -572,14 +622,14 @@ bool make_pool_map(CUtensorMap* map, const void* pool, int D, int page, int hkv,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D, int TT, int ST>
+template <int D, int TT, int ST, bool TL>
 cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap& mv, int grid,
                      cudaStream_t stream) {
   constexpr int smem = (int)Smem<D, TT, ST>::kBytes;
   static_assert(smem <= 232448, "fork_tc kernel shared memory exceeds 227 KB");
   static_assert(ST <= kMaxStages && (TT == 64 || TT == 128), "unsupported pipeline shape");
   static_assert(kTmemO + 128u * kWG <= kTmemCols && 2 * TT <= (int)kTmemO, "TMEM layout");
-  auto kern = fork_tc_kernel<D, TT, ST>;
+  auto kern = fork_tc_kernel<D, TT, ST, TL>;
   static thread_local int configured = -1;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -606,14 +656,24 @@ int fork_tc_tile_tokens() { return kTile; }
 int fork_tc_page_size() { return kPB; }
 
 cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
-                           int dqk, cudaStream_t stream) {
+                           int dqk, bool tiled, cudaStream_t stream) {
   if (grid == 0) return cudaSuccess;
   CUtensorMap mk, mv;
+  if (tiled) {
+    // bulk copies read the pools directly; the tensor maps stay unused
+    memset(&mk, 0, sizeof(mk));
+    memset(&mv, 0, sizeof(mv));
+    if (reinterpret_cast<uintptr_t>(k_pages) % 16 || reinterpret_cast<uintptr_t>(v_pages) % 16)
+      return cudaErrorInvalidValue;
+    if (dqk == 128) return launch_d<128, kTile, 3, true>(p, mk, mv, grid, stream);
+    if (dqk == 64) return launch_d<64, kTile, 4, true>(p, mk, mv, grid, stream);
+    return cudaErrorInvalidValue;
+  }
   if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
       !make_pool_map(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
     return cudaErrorInvalidValue;
-  if (dqk == 128) return launch_d<128, kTile, 3>(p, mk, mv, grid, stream);
-  if (dqk == 64) return launch_d<64, kTile, 4>(p, mk, mv, grid, stream);
+  if (dqk == 128) return launch_d<128, kTile, 3, false>(p, mk, mv, grid, stream);
+  if (dqk == 64) return launch_d<64, kTile, 4, false>(p, mk, mv, grid, stream);
   return cudaErrorInvalidValue;
 }
 

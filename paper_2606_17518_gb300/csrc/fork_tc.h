@@ -10,6 +10,8 @@ namespace specgen {
 
 struct TcParams {
   const __nv_bfloat16* q;
+  const __nv_bfloat16* k_pages;  // used directly with the tiled layout (bulk copies)
+  const __nv_bfloat16* v_pages;
   const int32_t* prefix_bt;
   const int32_t* prefix_bt_off;
   const int32_t* suffix_bt;
@@ -28,6 +30,6 @@ bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G);
 int fork_tc_tile_tokens();
 int fork_tc_page_size();
 cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
-                           int dqk, cudaStream_t stream);
+                           int dqk, bool tiled, cudaStream_t stream);
 
 }  // namespace specgen

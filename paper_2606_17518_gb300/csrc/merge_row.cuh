@@ -1,9 +1,9 @@
 // Combining a row's partial attentions, latency-tolerant form (device helper).
 //
 // A row owns n partials (O_i normalised by its own sum, LSE_i).  They are
-// combined online in batches of 8: the batch's 8 LSE words and 8 float4 output
-// slices are loaded together (independent loads, one memory round trip per
-// batch), the running maximum moves to the batch maximum and the accumulated
+// combined online in batches of kMergeBatch: the batch's LSE words and float4
+// output slices are loaded together (independent loads, one memory round trip
+// per batch), the running maximum moves to the batch maximum and the accumulated
 // sum is rescaled, exactly as in an online softmax:
 //     m' = max(m, max_b LSE_i),  acc' = acc e^{m-m'} + sum_b e^{LSE_i-m'} O_i,
 //     w' = w e^{m-m'} + sum_b e^{LSE_i-m'};   O = acc / w,  LSE = m + ln w.
@@ -12,6 +12,8 @@
 #include "common.cuh"
 
 namespace specgen {
+
+constexpr int kMergeBatch = 16;
 
 struct RowMerge {
   float4 acc;
@@ -26,18 +28,18 @@ __device__ __forceinline__ RowMerge merge_row(const float* lse_p, size_t lse_str
   r.acc = make_float4(0.f, 0.f, 0.f, 0.f);
   r.w = 0.f;
   r.m = -INFINITY;
-  for (int i0 = 0; i0 < n; i0 += 8) {
-    float li[8];
-    float4 v[8];
+  for (int i0 = 0; i0 < n; i0 += kMergeBatch) {
+    float li[kMergeBatch];
+    float4 v[kMergeBatch];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
+    for (int e = 0; e < kMergeBatch; ++e) {
       const bool in = i0 + e < n;
       li[e] = in ? __ldcg(lse_p + (size_t)(i0 + e) * lse_stride) : -INFINITY;
       v[e] = in ? __ldcg(o_p + (size_t)(i0 + e) * o_stride) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
     float mb = r.m;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) mb = fmaxf(mb, li[e]);
+    for (int e = 0; e < kMergeBatch; ++e) mb = fmaxf(mb, li[e]);
     if (mb == -INFINITY) continue;  // nothing yet
     const float sc = r.m == -INFINITY ? 0.f : fast_exp2((r.m - mb) * kLog2e);
     r.acc.x *= sc;
@@ -47,7 +49,7 @@ __device__ __forceinline__ RowMerge merge_row(const float* lse_p, size_t lse_str
     r.w *= sc;
     r.m = mb;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
+    for (int e = 0; e < kMergeBatch; ++e) {
       if (li[e] == -INFINITY) continue;
       const float we = fast_exp2((li[e] - mb) * kLog2e);
       r.w += we;

@@ -65,6 +65,10 @@ specgen_status check_shape(const specgen_fork_attn_args* a, const specgen_host_l
     return SPECGEN_ERR_UNSUPPORTED;
   if (a->page_size > 1024 || (a->page_size & (a->page_size - 1)) != 0)
     return SPECGEN_ERR_UNSUPPORTED;
+  if (a->kv_layout != SPECGEN_KV_ROWS && a->kv_layout != SPECGEN_KV_TILED) return SPECGEN_ERR_SHAPE;
+  if (a->kv_layout == SPECGEN_KV_TILED &&
+      !fork_tc_supported(a->head_dim_qk, a->head_dim_v, latent, a->page_size, a->hq / a->hkv))
+    return SPECGEN_ERR_UNSUPPORTED;
   const int32_t* fo = lens->fork_offsets;
   if (fo[0] != 0 || fo[a->num_traces] != a->total_forks) return SPECGEN_ERR_SHAPE;
   for (int t = 0; t < a->num_traces; ++t) {
@@ -409,7 +413,7 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   plan->n_split_items = h.n_split;
   plan->n_rows = s.F * s.hq;
   plan->total_slots = t_plan.total_slots;
-  plan->flags = s.latent ? 1 : 0;
+  plan->flags = (s.latent ? 1 : 0) | (args->kv_layout == SPECGEN_KV_TILED ? 2 : 0);
   plan->plan_bytes = (int64_t)L.plan_bytes;
   plan->ws_plan_off = (int64_t)L.ws_plan;
   plan->ws_part_o_off = (int64_t)L.ws_part_o;
@@ -481,6 +485,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   if (st != SPECGEN_OK) return st;
   if ((int64_t)args->workspace_bytes < plan->ws_end) return SPECGEN_ERR_WORKSPACE;
   if ((args->v_pages == nullptr) != (plan->flags & 1)) return SPECGEN_ERR_SHAPE;
+  if ((args->kv_layout == SPECGEN_KV_TILED) != ((plan->flags & 2) != 0)) return SPECGEN_ERR_SHAPE;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   unsigned char* ws = static_cast<unsigned char*>(args->workspace);
   unsigned char* pl = ws + plan->ws_plan_off;
@@ -545,8 +550,10 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
       mp.scale_log2 = tp.scale_log2;
       e = launch_mla_tc(mp, args->k_pages, plan->n_tc_ctas, stream);
     } else {
+      tp.k_pages = static_cast<const __nv_bfloat16*>(args->k_pages);
+      tp.v_pages = static_cast<const __nv_bfloat16*>(args->v_pages);
       e = launch_fork_tc(tp, args->k_pages, args->v_pages, plan->n_tc_ctas, args->head_dim_qk,
-                         stream);
+                         args->kv_layout == SPECGEN_KV_TILED, stream);
     }
     if (e != cudaSuccess) return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;

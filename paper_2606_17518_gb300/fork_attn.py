@@ -29,14 +29,18 @@ def _i32(a, device):
 class ForkDecode:
     """One workload resident on the GPU plus its output and workspace buffers."""
 
-    def __init__(self, w: dict, device="cuda", upload_kv: bool = True):
+    def __init__(self, w: dict, device="cuda", upload_kv: bool = True,
+                 kv_layout: int = _lib.KV_ROWS):
         import torch
+        from . import workloads
         self.w = w
         self.device = torch.device(device)
         self.latent = w["v_pages"] is None
+        self.kv_layout = kv_layout
+        lay = (lambda a: workloads.tile_kv_pool(a)) if kv_layout == _lib.KV_TILED else (lambda a: a)
         self.q = _bf16(w["q"], device)
-        self.k_pages = _bf16(w["k_pages"], device) if upload_kv else None
-        self.v_pages = (None if self.latent else _bf16(w["v_pages"], device)) if upload_kv else None
+        self.k_pages = _bf16(lay(w["k_pages"]), device) if upload_kv else None
+        self.v_pages = (None if self.latent else _bf16(lay(w["v_pages"]), device)) if upload_kv else None
         self.prefix_table = _i32(w["prefix_table"], device)
         self.prefix_off = _i32(w["prefix_bt_offsets"], device)
         self.suffix_table = _i32(w["suffix_table"], device)
@@ -63,7 +67,7 @@ class ForkDecode:
             prefix_bt_offsets=self.prefix_off, suffix_block_table=self.suffix_table,
             suffix_bt_offsets=self.suffix_off, out=self.out, lse=self.lse,
             workspace=self.workspace if with_ws else None,
-            workspace_bytes=self.ws_bytes if with_ws else 0)
+            workspace_bytes=self.ws_bytes if with_ws else 0, kv_layout=self.kv_layout)
         kw.update(override)
         return _lib.make_args(**kw)
 

@@ -207,3 +207,15 @@ def shard_traces(w: dict, rank: int, world: int) -> dict:
         global_forks=np.array(forks, dtype=np.int64),
     )
     return out
+
+
+def tile_kv_pool(pool: np.ndarray) -> np.ndarray:
+    """Re-lay a [pages][hkv][B][D] pool into 8 x 8 tiles (the SPECGEN_KV_TILED order).
+
+    Element (t, d) of a (page, head) block moves to
+    ((t/8) * (D/8) + d/8) * 64 + (t%8) * 8 + d%8 -- a pure permutation of the
+    block, no arithmetic.
+    """
+    P, H, B, D = pool.shape
+    t = pool.reshape(P, H, B // 8, 8, D // 8, 8)           # [.., tg, t8, dc, d8]
+    return np.ascontiguousarray(t.transpose(0, 1, 2, 4, 3, 5)).reshape(P, H, B, D)

@@ -128,6 +128,36 @@ def test_shape_errors(w):
     assert _lib.specgen_fork_attn_workspace_size(_fake_args(w, hq=7), lens) == 0
 
 
+def test_kv_layout_checks(w):
+    lens, keep = _lens(w)
+    S = _lib
+    assert _plan_status(_fake_args(w, kv_layout=2), lens) == S.SPECGEN_ERR_SHAPE
+    assert _plan_status(_fake_args(w, kv_layout=-1), lens) == S.SPECGEN_ERR_SHAPE
+    # the tiled layout exists only on the tensor-core shapes (page 16, head dim 64/128)
+    assert _plan_status(_fake_args(w, kv_layout=S.KV_TILED, page_size=64), lens) == \
+        S.SPECGEN_ERR_UNSUPPORTED
+    assert _plan_status(_fake_args(w, kv_layout=S.KV_TILED, head_dim_qk=256, head_dim_v=256),
+                        lens) == S.SPECGEN_ERR_UNSUPPORTED
+    wm = wl.make_workload(wl.WorkloadSpec(
+        name="m", num_traces=1, prefix_len=(64, 64), forks=(1, 1), suffix_len=(0, 0), hq=128,
+        hkv=1, dqk=576, dv=512, page_size=64, separate_v=False, seed=1))
+    lm, km = _lens(wm)
+    assert _plan_status(_fake_args(wm, kv_layout=S.KV_TILED), lm) == S.SPECGEN_ERR_UNSUPPORTED
+    assert _lib.specgen_fork_attn_workspace_size(_fake_args(w, kv_layout=S.KV_TILED), lens) > 0
+
+
+def test_tile_kv_pool_mapping():
+    """The tiled pool puts (t, d) of every (page, head) block at
+    ((t/8)*(D/8) + d/8)*64 + (t%8)*8 + d%8 and keeps the block in place."""
+    rng = np.random.default_rng(3)
+    pool = rng.integers(0, 1 << 15, (3, 2, 16, 64)).astype(np.uint16)
+    tiled = wl.tile_kv_pool(pool).reshape(3, 2, -1)
+    for t in range(16):
+        for d in range(64):
+            assert np.array_equal(tiled[:, :, ((t // 8) * 8 + d // 8) * 64 + (t % 8) * 8 + d % 8],
+                                  pool[:, :, t, d])
+
+
 def test_null_and_workspace_errors(w):
     lens, keep = _lens(w)
     S = _lib

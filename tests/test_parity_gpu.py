@@ -25,9 +25,9 @@ def built():
     __graft_entry__.build()
 
 
-def _gpu(w):
+def _gpu(w, kv_layout=_lib.KV_ROWS):
     from paper_2606_17518_gb300.fork_attn import ForkDecode
-    fd = ForkDecode(w)
+    fd = ForkDecode(w, kv_layout=kv_layout)
     fd.decode()
     o, lse = fd.results()
     assert fd.status() == _lib.SPECGEN_OK
@@ -91,6 +91,53 @@ def test_fuzz_small_shapes(case):
     o, lse, _ = _gpu(w)
     o_ref, lse_ref = oracle.fork_attn_decode(w)
     _compare(o, lse, o_ref, lse_ref, f"fuzz{case}")
+
+
+@pytest.mark.parametrize("name", ["tiny_p512_f4", "fork_p8k_f8"])
+def test_tiled_layout_workload_full(name):
+    """K/V pools in the 8x8-tiled layout (one bulk copy per page and head)."""
+    w = wl.make_workload(name)
+    o, lse, _ = _gpu(w, _lib.KV_TILED)
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, name + "/tiled")
+
+
+def test_tiled_layout_sampled_long():
+    w = wl.make_workload("long_p32k_f16")
+    o, lse, _ = _gpu(w, _lib.KV_TILED)
+    rng = np.random.default_rng(321)
+    F, hq = w["total_forks"], w["hq"]
+    rows = [(F - 1, h) for h in range(hq)]
+    rows += [(int(f), int(h)) for f, h in zip(rng.integers(0, F, 64), rng.integers(0, hq, 64))]
+    o_ref, lse_ref = oracle.fork_attn_decode_rows(w, rows)
+    idx_f = np.array([r[0] for r in rows])
+    idx_h = np.array([r[1] for r in rows])
+    _compare(o[idx_f, idx_h], lse[idx_f, idx_h], o_ref, lse_ref, "long/tiled")
+
+
+@pytest.mark.parametrize("case", [0, 2, 4, 6, 8, 10])
+def test_tiled_layout_fuzz(case):
+    """The page-16 fuzz shapes (ragged tails, empty sequences, G 1..16) in the tiled layout."""
+    rng = np.random.default_rng(1000 + case)
+    dqk = [64, 128][(case // 2) % 2]
+    G = [1, 4, 8, 16][case % 4]
+    hkv = [1, 2, 3][case % 3]
+    w = wl.make_workload(_fuzz_spec(rng, 16, dqk, G, hkv))
+    o, lse, _ = _gpu(w, _lib.KV_TILED)
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, f"tiled fuzz{case}")
+
+
+def test_tiled_invalid_page_id_is_reported_not_read():
+    w = dict(wl.make_workload("tiny_p512_f4"))
+    w["prefix_table"] = w["prefix_table"].copy()
+    w["prefix_table"][5] = w["num_pages"] + 3
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    fd = ForkDecode(w, kv_layout=_lib.KV_TILED)
+    fd.decode()
+    o, lse = fd.results()
+    assert fd.status() == _lib.SPECGEN_ERR_INDEX
+    assert np.all(np.isfinite(o))
 
 
 def test_empty_prefix_and_suffix_edges():
