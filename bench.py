@@ -284,10 +284,11 @@ def run_ours():
 
     # Timed steps replay CUDA graphs.  Each graph holds `per_graph` consecutive
     # steps (one library call each, on rotating replicas) so that host launch
-    # overhead never starves the GPU; inside every step the library records
-    # event marks between its kernels (external record nodes), so after the
-    # timed region each graph's marks hold the per-kernel times of its last
-    # replay.  K is covered exactly: full graphs plus one remainder graph.
+    # overhead never starves the GPU.  K is covered exactly: full graphs plus
+    # one remainder graph.  Per-kernel times come from separate graphs of the
+    # profiled call (event marks between its kernels, as external record
+    # nodes), replayed after the timed region, so the marks never sit between
+    # the kernels of a timed step.
     n_marks = 4
     K, W = ARGS.steps, ARGS.warmup
     per_graph = max(1, min(16, K))
@@ -302,7 +303,20 @@ def run_ours():
         assert st == 0, _lib.status_string(st)
     torch.cuda.synchronize(dev)
 
-    def make_graph(first_step, n_steps):
+    run_plain = lib.specgen_fork_attn_run
+
+    def make_graph(first_step, n_steps, profiled=False):
+        if not profiled:
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                for k in range(n_steps):
+                    r = (first_step + k) % replicas
+                    st = run_plain(arg_refs[r], plan_refs[r], sp_c)
+                    if st != 0:
+                        break
+            if st != 0:
+                raise RuntimeError(_lib.status_string(st))
+            return graph, None
         evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_marks)]
                for _ in range(n_steps)]
         with torch.cuda.stream(stream):
@@ -343,12 +357,18 @@ def run_ours():
     torch.cuda.synchronize(dev)
     barrier()
     clk = clocks.stop()
-    launches = n_l.value
     total_ms = start.elapsed_time(end)
-    sampled_graphs = full_graphs + ([rem_graph] if rem_graph else [])
-    sampled = sum(len(evs) for _, evs in sampled_graphs)
+    # per-kernel times: profiled graphs over the same rotation of replicas
+    prof_graphs = [make_graph(g * per_graph, per_graph, profiled=True)
+                   for g in range(max(1, min(8, K // per_graph)))]
+    for _ in range(2):
+        for graph, _ in prof_graphs:
+            graph.replay()
+    torch.cuda.synchronize(dev)
+    launches = n_l.value
+    sampled = sum(len(evs) for _, evs in prof_graphs)
     per_kernel = [0.0] * launches
-    for _, evs in sampled_graphs:
+    for _, evs in prof_graphs:
         for row in evs:
             for k in range(launches):
                 per_kernel[k] += row[k].elapsed_time(row[k + 1])
@@ -412,8 +432,9 @@ def run_ours():
             "head_dim": [w["dqk"], w["dv"]], "page_size": w["page_size"], "kv_layout": layout,
             "unique_bytes": nbytes["total"], "flops": flops["total"],
             "l2": f"inputs rotate over {replicas} resident replicas (>= 3x L2)",
-            "timing": f"CUDA graphs of {per_graph} steps; per-kernel times from the last "
-                      f"replay of each graph ({n_slots} timed steps)",
+            "timing": f"CUDA graphs of {per_graph} steps; per-kernel times from event marks "
+                      f"in separate profiled graphs ({n_slots} steps, replayed after the timed "
+                      f"region)",
             "parallelism": f"replicas x{world}",
         },
         "gpu_launches": K * launches,

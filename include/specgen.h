@@ -121,7 +121,7 @@ typedef struct {
   int32_t n_rows;               /* total_forks * hq */
   int32_t total_slots;          /* partial (O, LSE) slots */
   int32_t flags;
-  int32_t reserved0;
+  int32_t n_part_groups;        /* head groups with their own partial count per fork */
   int64_t plan_bytes;           /* plan bytes copied into the workspace */
   int64_t ws_plan_off, ws_part_o_off, ws_part_lse_off, ws_end;
   int64_t offsets[8];           /* internal offsets inside the plan region */

@@ -66,7 +66,7 @@ class Plan(C.Structure):
     _fields_ = [
         ("valid", C.c_int32), ("n_tc_items", C.c_int32), ("n_tc_ctas", C.c_int32),
         ("n_split_items", C.c_int32), ("n_rows", C.c_int32), ("total_slots", C.c_int32),
-        ("flags", C.c_int32), ("reserved0", C.c_int32),
+        ("flags", C.c_int32), ("n_part_groups", C.c_int32),
         ("plan_bytes", C.c_int64), ("ws_plan_off", C.c_int64), ("ws_part_o_off", C.c_int64),
         ("ws_part_lse_off", C.c_int64), ("ws_end", C.c_int64), ("offsets", C.c_int64 * 8),
     ]

@@ -52,24 +52,29 @@ constexpr int kThreads = 64 + 128 * kWG;     // warp 0 TMA, warp 1 MMA, 4 warps 
 constexpr uint32_t kTmemCols = 512;          // S[0] [0,TT) S[1] [TT,2TT) O[0] [256,..) O[1] [384,..)
 constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleLog2 = 8.0f;         // lazy-rescale threshold (factor 256)
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 4;
 constexpr int kTile = 128;                   // tokens per pipeline tile (8 pages)
 
-// Shared memory of one CTA: Q (128 rows x D) and a ring of `ST` (K, V) stages of
-// TT tokens.  Every operand tile is made of 64-column panels (128-byte rows,
-// 128B-swizzled), 1024-byte aligned.  P lives in tensor memory.
-template <int D, int TT, int ST>
+// Shared memory of one CTA: Q (128 rows x D, non-swizzled 8x8 core matrices:
+// LBO 128 B along d, SBO D*16 B per 8 rows), a ring of `ST` (K, V) stages of
+// TT tokens (rows layout: 64-column panels of 128-byte rows, 128B-swizzled;
+// tiled layout: the pool's own core-matrix tiles), barriers, the per-stage
+// valid-page masks, the second group's (m, l) and the CTA's first items.
+constexpr int kItemCache = 16;
+
+template <int D, int TT, int ST, bool TL>
 struct Smem {
   static constexpr int kPanels = D / 64;
-  static constexpr uint32_t kQPanel = 128 * 128u;         // 128 rows x 128 B
-  static constexpr uint32_t kQ = kPanels * kQPanel;
+  static constexpr uint32_t kQ = 128u * D * 2u;
   static constexpr uint32_t kRowsTile = TT * 128u;        // one 64-column panel of TT rows
-  static constexpr uint32_t kKV = kPanels * kRowsTile;    // one K or V tile
+  static constexpr uint32_t kKV = kPanels * kRowsTile;    // one K or V tile (TT x D bf16)
   static constexpr uint32_t kStage = 2 * kKV;
   static constexpr uint32_t kOffKV = kQ;
   static constexpr uint32_t kOffBar = kOffKV + ST * kStage;
   static constexpr uint32_t kOffML = kOffBar + 256;        // 128 x (m, l) of the second group
-  static constexpr uint32_t kBytes = kOffML + 128 * 8 + 1024;
+  static constexpr uint32_t kOffItems = kOffML + 128 * 8;
+  static constexpr uint32_t kAlign = TL ? 128u : 1024u;    // 128B-swizzled tiles: 1024-B aligned
+  static constexpr uint32_t kBytes = kOffItems + kItemCache * (uint32_t)sizeof(TcItem) + kAlign;
 };
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
@@ -101,42 +106,76 @@ __device__ __forceinline__ int tile_tokens(const TcItem& it, int j) {
   return n < TT ? n : TT;
 }
 
+// Item k of this CTA: the first kItemCache come from shared memory.
+__device__ __forceinline__ TcItem get_item(const TcItem* cache, const TcParams& p, int it_begin,
+                                           int k) {
+  return k < kItemCache ? cache[k] : p.items[it_begin + k];
+}
+
+// Page ids pb + lane of an item (lane-strided batch of 32); 0 past the item.
+__device__ __forceinline__ int page_batch(const TcParams& p, const TcItem& it, int pb, int lane) {
+  const int npages = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
+  if (pb + lane >= npages) return 0;
+  const int32_t* bt = it.table_kind == 0 ? p.prefix_bt : p.suffix_bt;
+  const int off = it.table_off >= 0
+                      ? it.table_off
+                      : (it.table_kind == 0 ? p.prefix_bt_off : p.suffix_bt_off)[it.seq];
+  return bt[off + it.tok_begin / kPB + pb + lane];
+}
+
 template <int D, int TT, int ST, bool TL>
 __global__ void __launch_bounds__(kThreads, 1)
     fork_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tmk,
                    const __grid_constant__ CUtensorMap tmv) {
-  using L = Smem<D, TT, ST>;
+  using L = Smem<D, TT, ST, TL>;
   constexpr int kPagesPerTile = TT / kPB;
   static_assert(32 % kPagesPerTile == 0, "a batch of 32 page ids holds whole tiles");
   extern __shared__ unsigned char smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
-  const uint32_t base = (raw + 1023u) & ~1023u;  // 128B-swizzled tiles: 1024-B aligned
+  const uint32_t base = (raw + L::kAlign - 1u) & ~(L::kAlign - 1u);
   unsigned char* gbase = smem_raw + (base - raw);
   const uint32_t sQ = base;
   const uint32_t bar0 = base + L::kOffBar;
   // barrier block: full[ST] empty[ST] s_full[2] p_full[2] o_full[2] q_ready mma_done
+  // ml_ready q_free merge_done ml_back, then the TMEM address, the abort flag
+  // and the per-stage valid-page masks
   auto full = [&](int s) { return bar0 + 8u * s; };
   auto empty = [&](int s) { return bar0 + 8u * (kMaxStages + s); };
   auto s_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + b); };
   auto p_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 2 + b); };
   auto o_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 4 + b); };
-  const uint32_t q_ready = bar0 + 8u * (2 * kMaxStages + 6);
+  const uint32_t q_ready = bar0 + 8u * (2 * kMaxStages + 6);     // Q of the next item stored
   const uint32_t mma_done = bar0 + 8u * (2 * kMaxStages + 7);
-  const uint32_t ml_ready = bar0 + 8u * (2 * kMaxStages + 8);  // group 1's (m, l) written
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 9));
-  volatile int* abort_flag =
-      reinterpret_cast<volatile int*>(gbase + L::kOffBar + 8 * (2 * kMaxStages + 9) + 4);
+  const uint32_t ml_ready = bar0 + 8u * (2 * kMaxStages + 8);    // group 1's (m, l) written
+  const uint32_t q_free = bar0 + 8u * (2 * kMaxStages + 9);      // an item's last S finished
+  const uint32_t merge_done = bar0 + 8u * (2 * kMaxStages + 10); // group 1 read its O halves
+  const uint32_t ml_back = bar0 + 8u * (2 * kMaxStages + 11);    // group 0's weights written
+  constexpr int kMisc = 8 * (2 * kMaxStages + 12);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + kMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + L::kOffBar + kMisc + 4);
+  volatile uint32_t* smask = reinterpret_cast<volatile uint32_t*>(gbase + L::kOffBar + kMisc + 8);
+  static_assert(kMisc + 8 + 4 * kMaxStages <= 256, "barrier block");
   float2* ml1 = reinterpret_cast<float2*>(gbase + L::kOffML);  // second group's (m, l) per row
+  TcItem* items = reinterpret_cast<TcItem*>(gbase + L::kOffItems);
   auto sK = [&](int s) { return base + L::kOffKV + s * L::kStage; };
   auto sV = [&](int s) { return base + L::kOffKV + s * L::kStage + L::kKV; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
+  const int n_items = it_end - it_begin;
   // let the merge grid (a programmatic dependent) get launched early; it waits
   // for this grid's completion before it reads anything
   if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
-  if (threadIdx.x == 0) {
+  if (warp == 0) {
+    // the CTA's first items, one per lane (40-byte records)
+    constexpr int kWords = sizeof(TcItem) / 4;
+    const int nw = (n_items < kItemCache ? n_items : kItemCache) * kWords;
+    const int32_t* src = reinterpret_cast<const int32_t*>(p.items + it_begin);
+    int32_t* dst = reinterpret_cast<int32_t*>(items);
+    for (int x = lane; x < nw; x += 32) dst[x] = src[x];
+  }
+  if (threadIdx.x == 32) {
     for (int i = 0; i < ST; ++i) {
       mbar_init(full(i), 1);
       mbar_init(empty(i), 1);
@@ -149,6 +188,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_ready, 128);
     mbar_init(mma_done, 1);
     mbar_init(ml_ready, 128);
+    mbar_init(q_free, 1);
+    mbar_init(merge_done, 128);
+    mbar_init(ml_back, 128);
     *abort_flag = 0;
     mbar_init_fence();
   }
@@ -162,10 +204,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+    // ------------------------------------------------------------ producer
     // The whole warp fetches page ids 32 at a time (one coalesced load, one
-    // batch ahead).  Lane 0 waits for a free stage; then lanes 0..2*D/64-1
-    // each issue one box of every page (K and V, one 64-column panel each).
+    // batch ahead, and the next item's first batch one item ahead).  Lane 0
+    // waits for a free stage and publishes the tile's valid-page mask; then
+    // the issuing lanes copy K and V of every page (rows layout: one TMA box per
+    // 64-column panel; tiled layout: one bulk copy per page).
     constexpr int kIssuers = TL ? 2 * kPagesPerTile : 2 * L::kPanels;
     const bool issuer = lane < kIssuers;
     const bool is_v = lane >= L::kPanels;
@@ -173,33 +217,38 @@ __global__ void __launch_bounds__(kThreads, 1)
     const void* tmap = is_v ? static_cast<const void*>(&tmv) : static_cast<const void*>(&tmk);
     int t = 0;  // tiles issued so far (across items)
     bool ok = true;
-    for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[ii];
-      const ItemView v = view<TT>(p, it);
+    int first_next = n_items > 0 ? page_batch(p, get_item(items, p, it_begin, 0), 0, lane) : 0;
+    for (int k = 0; ok && k < n_items; ++k) {
+      const TcItem it = get_item(items, p, it_begin, k);
       const int npages = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
-      int cur = lane < npages ? v.table[v.page0 + lane] : 0;
+      int cur = first_next;
+      first_next = k + 1 < n_items ? page_batch(p, get_item(items, p, it_begin, k + 1), 0, lane) : 0;
       for (int pb = 0; ok && pb < npages; pb += 32) {
-        const int nxt = pb + 32 + lane < npages ? v.table[v.page0 + pb + 32 + lane] : 0;
+        const int nxt = page_batch(p, it, pb + 32, lane);
         const int batch_pages = npages - pb < 32 ? npages - pb : 32;
         for (int tp = 0; tp < batch_pages; tp += kPagesPerTile, ++t) {
           const int j = (pb + tp) / kPagesPerTile;  // tile index within the item
           const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
           int pages[kPagesPerTile];
+          uint32_t valid = 0;
 #pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg)
+          for (int pg = 0; pg < kPagesPerTile; ++pg) {
             pages[pg] = __shfl_sync(0xffffffffu, cur, tp + pg);
+            if (pg < np && pages[pg] >= 0 && pages[pg] < p.num_pages) valid |= 1u << pg;
+          }
+          const uint32_t bad = ((1u << np) - 1u) & ~valid;
           const int s = t % ST;
+          if (lane == 0) {
+            ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
+            if (ok) smask[s] = valid;
+            if (bad) atomicOr(p.status, kStatusIndex);
+          }
+          ok = __shfl_sync(0xffffffffu, ok, 0);
+          if (!ok) break;
           if constexpr (TL) {
-            // one bulk copy per (page, K or V); an invalid page is reported and
-            // its value block zeroed here instead (its scores are masked)
+            // one bulk copy per (page, K or V); an invalid page's value block is
+            // zeroed here instead (its scores are masked)
             constexpr uint32_t kBlk = kPB * D * 2u;
-            uint32_t bad = 0;
-#pragma unroll
-            for (int pg = 0; pg < kPagesPerTile; ++pg)
-              if (pg < np && (pages[pg] < 0 || pages[pg] >= p.num_pages)) bad |= 1u << pg;
-            if (lane == 0) ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) break;
             if (bad) {
               for (int pg = 0; pg < np; ++pg)
                 if ((bad >> pg) & 1u)
@@ -207,38 +256,31 @@ __global__ void __launch_bounds__(kThreads, 1)
                     st_shared_v4(sV(s) + pg * kBlk + x, 0u, 0u, 0u, 0u);
               fence_proxy_async_smem();
               __syncwarp();
-              if (lane == 0) atomicOr(p.status, kStatusIndex);
             }
-            if (lane == 0)
-              mbar_arrive_expect_tx(full(s), (uint32_t)(np - __popc(bad)) * 2u * kBlk);
+            if (lane == 0) mbar_arrive_expect_tx(full(s), (uint32_t)__popc(valid) * 2u * kBlk);
             __syncwarp();
             const int pg = lane % kPagesPerTile;
-            if (issuer && pg < np && !((bad >> pg) & 1u)) {
+            if (issuer && ((valid >> pg) & 1u)) {
               const bool v_side = lane >= kPagesPerTile;
               const __nv_bfloat16* src = (v_side ? p.v_pages : p.k_pages) +
                                          ((size_t)pages[pg] * p.hkv + it.kv_head) * (kPB * D);
               bulk_load((v_side ? sV(s) : sK(s)) + pg * kBlk, src, kBlk, full(s));
             }
-            continue;
-          }
-          if (lane == 0) {
-            ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
-            if (ok) mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
-          }
-          ok = __shfl_sync(0xffffffffu, ok, 0);
-          if (!ok) break;
-          if (issuer) {
-            const uint32_t dst = (is_v ? sV(s) : sK(s)) + pn * L::kRowsTile;
+          } else {
+            // TMA zero-fills out-of-range pages, so every box counts
+            if (lane == 0)
+              mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
+            __syncwarp();
+            if (issuer) {
+              const uint32_t dst = (is_v ? sV(s) : sK(s)) + pn * L::kRowsTile;
 #pragma unroll
-            for (int pg = 0; pg < kPagesPerTile; ++pg) {
-              if (pg >= np) break;
-              tma_load_4d(dst + pg * (kPB * 128u), tmap, pn * 64, 0, it.kv_head, pages[pg], full(s));
+              for (int pg = 0; pg < kPagesPerTile; ++pg) {
+                if (pg >= np) break;
+                tma_load_4d(dst + pg * (kPB * 128u), tmap, pn * 64, 0, it.kv_head, pages[pg],
+                            full(s));
+              }
             }
           }
-          if (lane == 0)
-            for (int pg = 0; pg < np; ++pg)
-              if (pages[pg] < 0 || pages[pg] >= p.num_pages)
-                atomicOr(p.status, kStatusIndex);  // TMA zero-fills out-of-range pages
         }
         cur = nxt;
       }
@@ -252,32 +294,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       // descriptors are built once; every MMA only adds a constant offset
       // (in 16-byte units) to the start-address field
-      const uint64_t dq = smem_desc_sw128(sQ, 16, 1024);
+      const uint64_t dq = smem_desc_interleave(sQ, 128, D * 16);
       // tiled: K-major K (LBO = next 8 columns, SBO = next 8 tokens); MN-major V
       // (LBO = next 8 tokens, SBO = next 8 columns)
       const uint64_t dk0 = TL ? smem_desc_interleave(sK(0), 128, D * 16)
                               : smem_desc_sw128(sK(0), 16, 1024);
       const uint64_t dv0 = TL ? smem_desc_interleave(sV(0), D * 16, 128)
                               : smem_desc_sw128(sV(0), L::kRowsTile, 1024);
-      // byte step of V per page (one 16-token k-step) and of K per 16 columns
+      // byte step of V per page (one 16-token k-step)
       constexpr uint32_t kVPage = TL ? kPB * D * 2u : kPB * 128u;
       constexpr uint64_t kStageDesc = L::kStage >> 4;
       constexpr uint32_t idesc_pv = idesc_bf16(128, D, true);
       // Ready-first issue: PV_v goes out as soon as its P is ready; S_u goes
       // out when its K tile has landed, its score buffer is free (PV_{u-2}
       // issued, so in-order execution has consumed P_{u-2}) and, for an item's
-      // first tile, its Q is in shared memory.  s_*: the next S to issue,
-      // v_*: the next PV to issue (item cursor, tile within item, global tile).
-      int s_ii = it_begin, s_j = 0, s_u = 0, v_ii = it_begin, v_j = 0, v_u = 0;
-      TcItem s_it = s_ii < it_end ? p.items[s_ii] : TcItem{};
+      // first tile, its Q is in shared memory.  After an item's last S, q_free
+      // tells the Q loader that the buffer may be overwritten.  s_*: the next
+      // S to issue, v_*: the next PV (item index, tile within item, global tile).
+      int s_k = 0, s_j = 0, s_u = 0, v_k = 0, v_j = 0, v_u = 0;
+      TcItem s_it = n_items > 0 ? get_item(items, p, it_begin, 0) : TcItem{};
       TcItem v_it = s_it;
       int s_nt = view<TT>(p, s_it).ntiles, v_nt = s_nt;
       bool q_ok = false;
       bool ok = true;
       unsigned long long t0 = 0;
-      while (ok && v_ii < it_end) {
+      while (ok && v_k < n_items) {
         bool did = false;
-        if (v_u < s_u && mbar_try_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
+        if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
           tc_fence_after();
           const int b = v_u & 1, s = v_u % ST;
           const int np = (tile_tokens<TT>(v_it, v_j) + kPB - 1) / kPB;
@@ -300,15 +343,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++v_u;
           if (++v_j == v_nt) {
             v_j = 0;
-            if (++v_ii < it_end) {
-              v_it = p.items[v_ii];
+            if (++v_k < n_items) {
+              v_it = get_item(items, p, it_begin, v_k);
               v_nt = view<TT>(p, v_it).ntiles;
             }
           }
           did = true;
-        } else if (s_ii < it_end && s_u - v_u < 2) {
-          if (!q_ok && mbar_try_wait(q_ready, (s_ii - it_begin) & 1)) q_ok = true;
-          if (q_ok && mbar_try_wait(full(s_u % ST), (s_u / ST) & 1)) {
+        } else if (s_k < n_items && s_u - v_u < 2) {
+          if (!q_ok && mbar_test_wait(q_ready, s_k & 1)) q_ok = true;
+          if (q_ok && mbar_test_wait(full(s_u % ST), (s_u / ST) & 1)) {
             tc_fence_after();
             const int b = s_u & 1, s = s_u % ST;
             const int np = (tile_tokens<TT>(s_it, s_j) + kPB - 1) / kPB;
@@ -317,18 +360,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t d_s = tmem + (uint32_t)b * TT;
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
-              const uint64_t qo = ((kk >> 2) * L::kQPanel + (kk & 3) * 32u) >> 4;
               const uint64_t ko =
                   (TL ? kk * 256u : (kk >> 2) * L::kRowsTile + (kk & 3) * 32u) >> 4;
-              mma_bf16(d_s, dq + qo, dk + ko, idesc, kk > 0 ? 1u : 0u);
+              mma_bf16(d_s, dq + (uint64_t)((kk * 256u) >> 4), dk + ko, idesc, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
             ++s_u;
             if (++s_j == s_nt) {
+              mma_commit(q_free);
               s_j = 0;
               q_ok = false;
-              if (++s_ii < it_end) {
-                s_it = p.items[s_ii];
+              if (++s_k < n_items) {
+                s_it = get_item(items, p, it_begin, s_k);
                 s_nt = view<TT>(p, s_it).ntiles;
               }
             }
@@ -354,8 +397,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ------------------------------------------------------------ softmax groups
     // Group g (warps 2+4g .. 5+4g) takes the tiles j = g, g+2, ... of every item
-    // with its own running max/sum and its own TMEM output O[g]; group 0 merges
-    // the two halves at the end of the item.
+    // with its own running max/sum and its own TMEM output O[g].  Group 1 also
+    // stages Q: it loads the next item's rows into registers after its last
+    // tile and stores them once the MMA reports the current item's last S
+    // finished.  At the end of every item the groups combine their halves,
+    // each writing half of the value columns.
     const int grp = (warp - 2) >> 2;
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
@@ -366,51 +412,48 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float sl2 = p.scale_log2;
     int t = 0;
     bool ok = true;
+    uint4 qr[D / 8];  // group 1: the next item's Q row (zero for padding rows)
+    // (re)defines qr on every path, so it is never live across a tile loop
+    auto load_q = [&](bool want, const TcItem& it) {
+      const bool rok = want && row < it.nforks * p.G;
+      const int fl = row / p.G, gi = row % p.G;
+      const uint4* src = reinterpret_cast<const uint4*>(
+          p.q + ((size_t)(it.fork0 + (rok ? fl : 0)) * p.hq + (rok ? it.kv_head * p.G + gi : 0)) *
+                    D);
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c) qr[c] = rok ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+    };
+    load_q(grp == 1 && n_items > 0, get_item(items, p, it_begin, 0));
+    auto store_q = [&]() {
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c)
+        st_shared_v4(sQ + ((row >> 3) * (D / 8) + c) * 128u + (row & 7) * 16u, qr[c].x, qr[c].y,
+                     qr[c].z, qr[c].w);
+      fence_proxy_async_smem();
+      mbar_arrive(q_ready);
+    };
 
-    for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[ii];
-      const ItemView v = view<TT>(p, it);
-      const bool warp_live = q4 * 32 < v.M;  // some real row in this warp
-      const bool row_ok = row < v.M;
+    for (int k = 0; ok && k < n_items; ++k) {
+      const TcItem it = get_item(items, p, it_begin, k);
+      const int ntiles = (it.tok_end - it.tok_begin + TT - 1) / TT;
+      const int M = it.nforks * p.G;
+      const bool warp_live = q4 * 32 < M;  // some real row in this warp
+      const bool row_ok = row < M;
       const int fl = row / p.G, gi = row % p.G;
       const int head = it.kv_head * p.G + gi;
+      // this row's partial slot base, fetched now and used at the item's end
+      const int pbase = p.part_base[it.fork0 + (row_ok ? fl : 0)];
 
-      if (grp == 0) {
-        // Q row -> shared memory, 128B-swizzled K-major panels; padding rows are zero
-        const uint4* src = reinterpret_cast<const uint4*>(
-            p.q + ((size_t)(it.fork0 + (row_ok ? fl : 0)) * p.hq + (row_ok ? head : 0)) * D);
-        if (warp_live) {
-#pragma unroll
-          for (int c = 0; c < D / 8; ++c) {
-            const uint4 q = row_ok ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
-            st_shared_v4(sQ + (c >> 3) * L::kQPanel + row * 128u + (((c & 7) ^ (row & 7)) << 4),
-                         q.x, q.y, q.z, q.w);
-          }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        mbar_arrive(q_ready);
-      } else {
-        // group 1 starts an item only after group 0 has finished merging the
-        // previous one (group 0 arrives on q_ready after that merge)
-        const bool w = mbar_wait(q_ready, (ii - it_begin) & 1, abort_flag, p.status);
-        if (__any_sync(0xffffffffu, !w)) {
-          ok = false;
-          break;
-        }
-      }
+      // group 1 stores Q of the first item here, of every later item at the end
+      // of the previous one (as soon as that item's last S has finished)
+      if (grp == 1 && k == 0) store_q();
 
       float m = -INFINITY, l = 0.f;  // this group's running max (log2 units) and sum
-      // page ids: 32 per coalesced warp load (lane i holds page pb + i), one batch ahead
-      const int npages_item = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
-      auto load_batch = [&](int pb) {
-        return pb + lane < npages_item ? v.table[v.page0 + pb + lane] : 0;
-      };
-      int cur_batch = 0;
-      int cur_pages = load_batch(0), nxt_pages = load_batch(32);
-      for (int j = grp; j < v.ntiles; j += 2) {
-        const int u = t + j, b = u & 1;
-        const bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
+      for (int j = grp; j < ntiles; j += 2) {
+        const int u = t + j, b = u & 1, s = u % ST;
+        bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
+        // the tile's valid-page mask (published before its copies were counted)
+        w = w && mbar_wait(full(s), (u / ST) & 1, abort_flag, p.status);
         if (__any_sync(0xffffffffu, !w)) {
           ok = false;
           break;
@@ -421,21 +464,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (j >= 2) mbar_wait(o_full(b), ((u - 2) >> 1) & 1, abort_flag, p.status);
         const int nt = tile_tokens<TT>(it, j);
         const int np = (nt + kPB - 1) / kPB;
-        const int batch = (j * kPagesPerTile) >> 5;
-        while (cur_batch < batch) {  // at most one step per visited tile
-          cur_pages = nxt_pages;
-          ++cur_batch;
-          nxt_pages = load_batch(cur_batch * 32 + 32);
-        }
-        const int tp0 = (j * kPagesPerTile) & 31;
         if (warp_live) {
-          uint32_t pv = 0;  // valid pages of this tile
-#pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg) {
-            const int page = __shfl_sync(0xffffffffu, cur_pages, (tp0 + pg) & 31);
-            if (pg < np && page >= 0 && page < p.num_pages) pv |= 1u << pg;
-          }
-          float s[TT];
+          const uint32_t pv = smask[s];  // valid pages of this tile
+          float sc[TT];
           {
             uint32_t r[TT / 32][32];
             const uint32_t sa = s_base + (uint32_t)b * TT;
@@ -445,21 +476,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int c = 0; c < TT / 32; ++c)
 #pragma unroll
-              for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[c][i]);
+              for (int i = 0; i < 32; ++i) sc[c * 32 + i] = __uint_as_float(r[c][i]);
           }
           const bool full_tile = nt == TT && pv == (1u << kPagesPerTile) - 1u;
           if (!full_tile) {
 #pragma unroll
             for (int i = 0; i < TT; ++i)
-              if (!(i < nt && ((pv >> (i / kPB)) & 1u))) s[i] = -INFINITY;
+              if (!(i < nt && ((pv >> (i / kPB)) & 1u))) sc[i] = -INFINITY;
           }
-          float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+          float mx0 = sc[0], mx1 = sc[1], mx2 = sc[2], mx3 = sc[3];
 #pragma unroll
           for (int i = 4; i < TT; i += 4) {
-            mx0 = fmaxf(mx0, s[i]);
-            mx1 = fmaxf(mx1, s[i + 1]);
-            mx2 = fmaxf(mx2, s[i + 2]);
-            mx3 = fmaxf(mx3, s[i + 3]);
+            mx0 = fmaxf(mx0, sc[i]);
+            mx1 = fmaxf(mx1, sc[i + 1]);
+            mx2 = fmaxf(mx2, sc[i + 2]);
+            mx3 = fmaxf(mx3, sc[i + 3]);
           }
           const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;  // scale > 0
           bool rescale = false;
@@ -478,8 +509,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t pk[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              const float p0 = fast_exp2(fmaf(s[c * 64 + 2 * i], sl2, -sub));
-              const float p1 = fast_exp2(fmaf(s[c * 64 + 2 * i + 1], sl2, -sub));
+              const float p0 = fast_exp2(fmaf(sc[c * 64 + 2 * i], sl2, -sub));
+              const float p1 = fast_exp2(fmaf(sc[c * 64 + 2 * i + 1], sl2, -sub));
               ps0 += p0;
               ps1 += p1;
               pk[i] = pack_bf16x2(p0, p1);
@@ -503,7 +534,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_wait_st();
         }
         // value rows past the sequence inside its last page: zero them before PV
-        if (j == v.ntiles - 1 && (nt % kPB) != 0) {
+        if (j == ntiles - 1 && (nt % kPB) != 0) {
           const int pg = np - 1, first = nt % kPB;
           const int units = (kPB - first) * L::kPanels * 8;  // 16-byte pieces
           for (int x = gtid; x < units; x += 128) {
@@ -512,7 +543,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int tt = pg * kPB + rr;
             const uint32_t off = TL ? ((tt >> 3) * (D / 8) + rem) * 128u + (tt & 7) * 16u
                                     : (rem >> 3) * L::kRowsTile + tt * 128u + ((rem & 7) << 4);
-            st_shared_v4(sV(u % ST) + off, 0u, 0u, 0u, 0u);
+            st_shared_v4(sV(s) + off, 0u, 0u, 0u, 0u);
           }
           fence_proxy_async_smem();
         }
@@ -520,62 +551,94 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(p_full(b));
       }
       if (!ok) break;
-      // ---- end of item: wait for this group's last PV, then merge the groups
-      const int last = grp + ((v.ntiles - 1 - grp) >> 1) * 2;  // this group's last tile (if any)
-      const bool has = grp < v.ntiles;
+      // ---- end of item: both groups wait for their last PV, exchange (m, l)
+      // through ml1 in two steps (group 1's (m, l) to group 0, the two final
+      // weights back), and each writes half of the value columns
+      const int last = grp + ((ntiles - 1 - grp) >> 1) * 2;  // this group's last tile (if any)
+      const bool has = grp < ntiles;
+      load_q(grp == 1 && k + 1 < n_items, get_item(items, p, it_begin, k + 1 < n_items ? k + 1 : k));
       if (has) {
         const int u = t + last, b = u & 1;
         const bool w = mbar_wait(o_full(b), (u >> 1) & 1, abort_flag, p.status);
         if (__any_sync(0xffffffffu, !w)) ok = false;
         tc_fence_after();
       }
+      float a0 = 0.f, a1 = 0.f;  // O = a0 O[0] + a1 O[1] (weights already divided by the sum)
       if (grp == 1) {
         ml1[row] = make_float2(has ? m : -INFINITY, has ? l : 0.f);
-        tc_fence_before();
+        tc_fence_before();  // O[1] complete before group 0 reads it
         mbar_arrive(ml_ready);
-      } else {
-        const bool w = mbar_wait(ml_ready, (ii - it_begin) & 1, abort_flag, p.status);
+        if (k + 1 < n_items) {
+          // the next item's Q, once this item's last S has finished with the buffer
+          const bool wq = mbar_wait(q_free, k & 1, abort_flag, p.status);
+          if (__any_sync(0xffffffffu, !wq)) ok = false;
+          if (ok) store_q();
+        }
+        const bool w = mbar_wait(ml_back, k & 1, abort_flag, p.status);
         if (__any_sync(0xffffffffu, !w)) ok = false;
         tc_fence_after();
-        if (ok && warp_live) {
-          const float2 o1 = ml1[row];
-          const float mm = fmaxf(m, o1.x);
-          const float w0 = m == -INFINITY ? 0.f : fast_exp2(m - mm);
-          const float w1 = o1.x == -INFINITY ? 0.f : fast_exp2(o1.x - mm);
-          const float lsum = l * w0 + o1.y * w1;
-          const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
-          const int fork = it.fork0 + (row_ok ? fl : 0);
-          const size_t prow_out = (size_t)(p.part_base[fork] + it.part) * p.hq + head;
-          float4* dst = reinterpret_cast<float4*>(p.part_o + prow_out * p.dv);
-          const uint32_t o0 = tmem + lane_addr + kTmemO, o1a = o0 + 128u;
+        const float2 wg = ml1[row];
+        a0 = wg.x;
+        a1 = wg.y;
+      } else {
+        const bool w = mbar_wait(ml_ready, k & 1, abort_flag, p.status);
+        if (__any_sync(0xffffffffu, !w)) ok = false;
+        tc_fence_after();
+        const float2 o1 = ml1[row];
+        const float mm = fmaxf(m, o1.x);
+        const float w0 = m == -INFINITY ? 0.f : fast_exp2(m - mm);
+        const float w1 = o1.x == -INFINITY ? 0.f : fast_exp2(o1.x - mm);
+        const float lsum = l * w0 + o1.y * w1;
+        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+        a0 = w0 * inv;
+        a1 = w1 * inv;
+        ml1[row] = make_float2(a0, a1);
+        tc_fence_before();  // O[0] complete before group 1 reads it
+        mbar_arrive(ml_back);
+        if (ok && row_ok)
+          p.part_lse[(size_t)(pbase + it.part) * p.hq + head] =
+              mm == -INFINITY ? -INFINITY : (mm + log2f(lsum)) * kLn2;
+      }
+      if (ok && warp_live) {
+        // one 32-column chunk of O[0] and O[1] per TMEM round trip (group 1
+        // holds the next item's Q row in registers meanwhile)
+        const uint32_t o0 = tmem + lane_addr + kTmemO + (uint32_t)grp * (D / 2), o1 = o0 + 128u;
+        float4* dst = reinterpret_cast<float4*>(p.part_o) +
+                      part_o_f4((size_t)pbase + it.part, head, grp * (D / 8), p.hq, p.dv);
 #pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t r0[32], r1[32];
-            tmem_ld32(o0 + c * 32u, r0);
-            tmem_ld32(o1a + c * 32u, r1);
-            tmem_wait_ld();
-            if (row_ok) {
+        for (int c = 0; c < D / 64; ++c) {
+          uint32_t r0[32], r1[32];
+          tmem_ld32(o0 + c * 32u, r0);
+          tmem_ld32(o1 + c * 32u, r1);
+          tmem_wait_ld();
+          if (row_ok) {
 #pragma unroll
-              for (int i = 0; i < 32; i += 4) {
-                float x[4];
+            for (int i = 0; i < 32; i += 4) {
+              float x[4];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                  // an unused output buffer (weight 0) may hold anything: never multiply it
-                  const float a0 = w0 == 0.f ? 0.f : __uint_as_float(r0[i + e]) * w0;
-                  const float a1 = w1 == 0.f ? 0.f : __uint_as_float(r1[i + e]) * w1;
-                  x[e] = (a0 + a1) * inv;
-                }
-                dst[c * 8 + i / 4] = make_float4(x[0], x[1], x[2], x[3]);
+              for (int e = 0; e < 4; ++e) {
+                // an unused output buffer (weight 0) may hold anything: never multiply it
+                const float v0 = a0 == 0.f ? 0.f : __uint_as_float(r0[i + e]) * a0;
+                const float v1 = a1 == 0.f ? 0.f : __uint_as_float(r1[i + e]) * a1;
+                x[e] = v0 + v1;
               }
+              dst[(size_t)(c * 8 + i / 4) * p.hq] = make_float4(x[0], x[1], x[2], x[3]);
             }
           }
-          if (row_ok)
-            p.part_lse[prow_out] = mm == -INFINITY ? -INFINITY : (mm + log2f(lsum)) * kLn2;
         }
-        tc_fence_before();
+      }
+      tc_fence_before();
+      if (grp == 1) {
+        mbar_arrive(merge_done);
+      } else {
+        // group 1 has read its half of O[0] before the next item's first PV
+        // (issued after this group's next p_full) overwrites it
+        const bool w = mbar_wait(merge_done, k & 1, abort_flag, p.status);
+        if (__any_sync(0xffffffffu, !w)) ok = false;
+        tc_fence_after();
       }
       if (__any_sync(0xffffffffu, !ok)) ok = false;
-      t += v.ntiles;
+      t += ntiles;
     }
   }
 
@@ -625,7 +688,7 @@ bool make_pool_map(CUtensorMap* map, const void* pool, int D, int page, int hkv,
 template <int D, int TT, int ST, bool TL>
 cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap& mv, int grid,
                      cudaStream_t stream) {
-  constexpr int smem = (int)Smem<D, TT, ST>::kBytes;
+  constexpr int smem = (int)Smem<D, TT, ST, TL>::kBytes;
   static_assert(smem <= 232448, "fork_tc kernel shared memory exceeds 227 KB");
   static_assert(ST <= kMaxStages && (TT == 64 || TT == 128), "unsupported pipeline shape");
   static_assert(kTmemO + 128u * kWG <= kTmemCols && 2 * TT <= (int)kTmemO, "TMEM layout");

@@ -19,7 +19,7 @@ struct TcParams {
   const TcItem* items;
   const int32_t* cta_offsets;  // [grid + 1]: CTA c takes items [cta_offsets[c], cta_offsets[c+1])
   const int32_t* part_base;    // [forks] first partial slot of each fork
-  float* part_o;               // [slots][hq][dv]
+  float* part_o;               // head-interleaved partials (part_o_f4)
   float* part_lse;             // [slots][hq]
   uint32_t* status;
   int hq, hkv, G, dv, num_pages;

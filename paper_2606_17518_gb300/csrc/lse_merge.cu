@@ -13,6 +13,7 @@
 #include "common.cuh"
 #include "lse_merge.h"
 #include "merge_row.cuh"
+#include "plan.h"
 
 namespace specgen {
 
@@ -31,10 +32,10 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// One thread per (row, 4-column slice): every thread reads the LSE of all of its
-// row's parts (the 32 threads of a row read the same words) and the parts'
-// float4 slices, all loads independent, so a row costs about two memory round
-// trips.  With programmatic dependent launch the grid starts while the kernel
+// One thread per (fork, 4-column slice, head), heads fastest: a warp reads
+// consecutive heads' LSE words and float4 slices of each part (contiguous in
+// the head-interleaved partial layout), all loads independent, so a row costs
+// about two memory round trips.  With programmatic dependent launch the grid starts while the kernel
 // producing the partials is still running and waits for it here.
 constexpr int kMergeThreads = 128;  // small blocks can sit beside a running tensor-core CTA
 
@@ -42,14 +43,16 @@ __global__ void __launch_bounds__(kMergeThreads) merge_parts_kernel(const MergeP
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
   const int c4n = p.dv / 4;
   const int gid = blockIdx.x * kMergeThreads + threadIdx.x;
-  const int row = gid / c4n, c4 = gid % c4n;
-  if (row >= p.n_rows) return;
-  const int f = row / p.hq, h = row % p.hq;
-  const int base = p.part_base[f], n = p.n_parts[f];
+  if (gid >= p.n_rows * c4n) return;
+  const int h = gid % p.hq, rest = gid / p.hq;
+  const int c4 = rest % c4n, f = rest / c4n;
+  const int row = f * p.hq + h;
+  const int base = p.part_base[f];
+  const int n = p.n_parts[f * p.n_groups + h / (p.hq / p.n_groups)];
   const RowMerge mr = merge_row(
       p.part_lse + (size_t)base * p.hq + h, (size_t)p.hq,
-      reinterpret_cast<const float4*>(p.part_o + ((size_t)base * p.hq + h) * p.dv) + c4,
-      (size_t)p.hq * p.dv / 4, n);
+      reinterpret_cast<const float4*>(p.part_o) + part_o_f4(base, h, c4, p.hq, p.dv),
+      (size_t)c4n * p.hq, n);
   store_merged(mr, p.out + (size_t)row * p.dv, c4, p.lse + row, c4 == 0);
 }
 

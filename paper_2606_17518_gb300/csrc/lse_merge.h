@@ -7,13 +7,13 @@
 namespace specgen {
 
 struct MergeParams {
-  const float* part_o;       // [slots][hq][dv]
+  const float* part_o;       // head-interleaved partials (part_o_f4)
   const float* part_lse;     // [slots][hq]
   const int32_t* part_base;  // [forks]
-  const int32_t* n_parts;    // [forks]
+  const int32_t* n_parts;    // [forks][n_groups]: slots used by each group of hq/n_groups heads
   __nv_bfloat16* out;        // [forks][hq][dv]
   float* lse;                // [forks][hq]
-  int n_rows, hq, dv;
+  int n_rows, hq, dv, n_groups;
 };
 
 // after_dependent: launch as a programmatic dependent of the previous kernel on

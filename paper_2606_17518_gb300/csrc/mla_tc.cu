@@ -177,7 +177,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       unsigned long long t0 = 0;
       while (ok && v_ii < it_end) {
         bool did = false;
-        if (v_u < s_u && mbar_try_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
+        if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
           tc_fence_after();
           const int b = v_u & 1, s = v_u % kST;
           const uint64_t vpanel = (uint64_t)((v_it.dv0 / 64) * kKPanel) >> 4;
@@ -196,8 +196,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           did = true;
         } else if (s_ii < it_end && s_u - v_u < 2) {
-          if (!q_ok && mbar_try_wait(q_ready, (s_ii - it_begin) & 1)) q_ok = true;
-          if (q_ok && mbar_try_wait(full(s_u % kST), (s_u / kST) & 1)) {
+          if (!q_ok && mbar_test_wait(q_ready, (s_ii - it_begin) & 1)) q_ok = true;
+          if (q_ok && mbar_test_wait(full(s_u % kST), (s_u / kST) & 1)) {
             tc_fence_after();
             const int b = s_u & 1, s = s_u % kST;
             const uint64_t dk = dk0 + (uint64_t)s * kStageDesc;
@@ -246,6 +246,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
       const TcItem it = p.items[ii];
+      // this fork's partial slot base, fetched now and used at the item's end
+      const int pbase = p.part_base[it.fork0];
       const int32_t* table = table_of(it);
       const int ntiles = ntiles_of(it);
       const int page0 = it.tok_begin / kPage;
@@ -370,8 +372,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-        const size_t prow = (size_t)(p.part_base[it.fork0] + it.part) * p.hq + row;
-        float4* dst = reinterpret_cast<float4*>(p.part_o + prow * kDv + it.dv0);
+        const size_t prow = (size_t)(pbase + it.part) * p.hq + row;
+        float4* dst = reinterpret_cast<float4*>(p.part_o) +
+                      part_o_f4((size_t)pbase + it.part, row, it.dv0 / 4, p.hq, kDv);
         const float inv = l > 0.f ? 1.f / l : 0.f;
         for (int c = 0; c < kDvHalf / 32; ++c) {
           uint32_t r[32];
@@ -379,7 +382,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_wait_ld();
 #pragma unroll
           for (int i = 0; i < 32; i += 4)
-            dst[c * 8 + i / 4] =
+            dst[(size_t)(c * 8 + i / 4) * p.hq] =
                 make_float4(__uint_as_float(r[i]) * inv, __uint_as_float(r[i + 1]) * inv,
                             __uint_as_float(r[i + 2]) * inv, __uint_as_float(r[i + 3]) * inv);
         }

@@ -17,7 +17,7 @@ struct MlaParams {
   const TcItem* items;         // dv0 selects the value half (0 or 256)
   const int32_t* cta_offsets;  // [grid + 1]: CTA c takes items [cta_offsets[c], cta_offsets[c+1])
   const int32_t* part_base;
-  float* part_o;               // [slots][128][512]
+  float* part_o;               // head-interleaved partials (part_o_f4), hq = 128, dv = 512
   float* part_lse;             // [slots][128]
   uint32_t* status;
   int hq, num_pages;

@@ -6,9 +6,21 @@
 // row owns `n_parts` consecutive partial slots starting at `part_base`; the
 // merge kernel combines them by log-sum-exp.
 #pragma once
+#include <stddef.h>
 #include <stdint.h>
 
 namespace specgen {
+
+// Partial outputs in the workspace, "head-interleaved": element (slot, head h,
+// value column c) of part_o sits at ((slot * dv/4 + c/4) * hq + h) * 4 + c%4, so
+// threads that hold consecutive heads store (and the merge loads) consecutive
+// 16-byte pieces.  part_lse is [slot][hq].  Index of the float4 (slot, h, c4):
+#ifdef __CUDACC__
+__host__ __device__
+#endif
+inline size_t part_o_f4(size_t slot, int h, int c4, int hq, int dv) {
+  return (slot * (size_t)(dv / 4) + (size_t)c4) * (size_t)hq + (size_t)h;
+}
 
 constexpr uint32_t kStatusIndex = 1u;    // a page id outside [0, num_pages) was seen
 constexpr uint32_t kStatusTimeout = 2u;  // a device wait hit its iteration limit
@@ -26,7 +38,7 @@ struct SplitItem {
   int32_t dv0;
   int32_t tok_begin;
   int32_t tok_end;
-  int32_t slot;        // partial slot: part_o[slot][h][dv], part_lse[slot][h]
+  int32_t slot;        // partial slot of rows h0.. (part_o_f4 layout), part_lse[slot][h]
 };
 
 // Tensor-core item (shared prefix or one fork's suffix): the query rows of

@@ -102,7 +102,9 @@ struct HostPlan {
   std::vector<SplitItem> split;
   std::vector<TcItem> tc;
   std::vector<int32_t> cta_items, cta_offsets;
-  std::vector<int32_t> part_base, n_parts;
+  std::vector<int32_t> part_base;
+  std::vector<int32_t> n_parts;  // [forks][n_groups]: partial slots used by each head group
+  int n_groups = 1;
   int total_slots = 0;
 };
 
@@ -154,6 +156,187 @@ void finish_tc_plan(HostPlan* hp, const std::vector<long long>& cost, int n_sm,
   hp->cta_items.clear();
 }
 
+// Budget packing of the tensor-core work.  A unit is one kv head of either a
+// fork's suffix (cut only when it alone exceeds the budget) or a group of forks'
+// shared prefix (cut freely at page boundaries).  Under a per-CTA budget T, in
+// token-equivalents with kItemCost per item, one pass deals the suffix pieces
+// (longest first) over the CTAs in snake order, then visits the CTAs from the
+// least loaded up and fills each one's spare budget with prefix chunks.  The
+// plan takes the smallest budget for which the prefix fits.
+constexpr long long kItemCost = 384;  // fixed cost of an item (Q staging, merge, pipeline refill)
+constexpr int kMinChunk = 128;        // smallest prefix chunk carved into a CTA's spare budget
+
+struct TcUnit {
+  int kind, seq, g, fork0, nforks, len;
+};
+
+struct TcPlacement {
+  int cta;
+  TcItem item;
+};
+
+// One packing pass under budget T.  `load` and `order` are caller-owned
+// scratch; `out` (when given) receives the items with their CTAs.
+bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int n_cta,
+             long long T, int page, std::vector<long long>* load, std::vector<int>* order,
+             std::vector<TcPlacement>* out) {
+  load->assign(n_cta, 0);
+  if (out) out->clear();
+  const long long lmax = (T - kItemCost) / page * page;
+  if (lmax < page) return false;
+  auto place = [&](int cta, const TcUnit& u, int b, int e, int part) {
+    (*load)[cta] += (e - b) + kItemCost;
+    if (!out) return;
+    TcPlacement pl;
+    pl.cta = cta;
+    TcItem& it = pl.item;
+    it.table_kind = u.kind;
+    it.seq = u.seq;
+    it.kv_head = u.g;
+    it.fork0 = u.fork0;
+    it.nforks = u.nforks;
+    it.tok_begin = b;
+    it.tok_end = e;
+    it.part = part;
+    it.dv0 = 0;
+    it.table_off = -1;
+    out->push_back(pl);
+  };
+  long long k_dealt = 0;  // suffix pieces dealt so far (snake order over the CTAs)
+  for (const TcUnit& u : sfx) {
+    const long long k = (u.len + lmax - 1) / lmax;
+    const int piece = (int)(((u.len + k - 1) / k + page - 1) / page * page);
+    for (int c = 0, pos = 0; pos < u.len; ++c, pos += piece, ++k_dealt) {
+      const long long round = k_dealt / n_cta, i = k_dealt % n_cta;
+      place((int)(round & 1 ? n_cta - 1 - i : i), u, pos, std::min(u.len, pos + piece), c);
+    }
+  }
+  order->resize(n_cta);
+  for (int c = 0; c < n_cta; ++c) (*order)[c] = c;
+  std::sort(order->begin(), order->end(),
+            [&](int x, int y) { return (*load)[x] < (*load)[y] || ((*load)[x] == (*load)[y] && x < y); });
+  size_t ui = 0;
+  int pos = 0, part = 0;
+  for (int oc = 0; oc < n_cta && ui < pfx.size(); ++oc) {
+    const int cta = (*order)[oc];
+    while (ui < pfx.size()) {
+      const TcUnit& u = pfx[ui];
+      const int rem = u.len - pos;
+      const long long spare = (T - (*load)[cta] - kItemCost) / page * page;
+      if (spare < std::min(kMinChunk, rem)) break;  // this CTA is full
+      long long len = std::min<long long>(rem, spare);
+      if (rem - len < kMinChunk / 2) len = rem;  // leave no sliver behind
+      place(cta, u, pos, pos + (int)len, part);
+      pos += (int)len;
+      ++part;
+      if (pos == u.len) {
+        ++ui;
+        pos = 0;
+        part = 0;
+      }
+    }
+  }
+  return ui == pfx.size();
+}
+
+void build_tc_plan(const Shape& s, const specgen_host_lens* lens, int n_sm, HostPlan* hp) {
+  const int32_t* fo = lens->fork_offsets;
+  const int page = fork_tc_page_size();
+  const int forks_per_item = std::max(1, 128 / s.G);
+  std::vector<TcUnit> sfx, pfx;
+  long long total = 0;
+  for (int t = 0; t < s.T; ++t) {
+    for (int g = 0; g < s.hkv; ++g) {
+      if (lens->prefix_lens[t] > 0)
+        for (int f0 = fo[t]; f0 < fo[t + 1]; f0 += forks_per_item)
+          pfx.push_back(TcUnit{0, t, g, f0, std::min(forks_per_item, fo[t + 1] - f0),
+                               lens->prefix_lens[t]});
+      for (int f = fo[t]; f < fo[t + 1]; ++f)
+        if (lens->suffix_lens[f] > 0) sfx.push_back(TcUnit{1, f, g, f, 1, lens->suffix_lens[f]});
+    }
+  }
+  for (const TcUnit& u : sfx) total += u.len;
+  for (const TcUnit& u : pfx) total += u.len;
+  auto longer = [](const TcUnit& a, const TcUnit& b) { return a.len > b.len; };
+  std::stable_sort(sfx.begin(), sfx.end(), longer);
+  std::stable_sort(pfx.begin(), pfx.end(), longer);
+  std::vector<TcPlacement> placed;
+  const int n_units = (int)(sfx.size() + pfx.size());
+  const int n_cta = std::max(1, n_sm);
+  if (n_units > 0) {
+    // Budget search.  Start from the average load with one item per suffix
+    // unit and about one prefix chunk per CTA, step up by 1/32 until the
+    // packing fits, then bisect the last step (a few linear passes in all).
+    std::vector<long long> load;
+    std::vector<int> order;
+    const long long n_items = (long long)sfx.size() + std::max<long long>((long long)pfx.size(), n_cta);
+    long long lo = std::max<long long>(kItemCost + page, (total + kItemCost * n_items) / n_cta);
+    long long hi = lo;
+    while (!pack_tc(sfx, pfx, n_cta, hi, page, &load, &order, nullptr)) {
+      lo = hi;
+      hi += std::max<long long>(page, hi / 32);
+    }
+    while (hi - lo > std::max<long long>(page, hi / 256)) {
+      const long long mid = (lo + hi) / 2;
+      if (pack_tc(sfx, pfx, n_cta, mid, page, &load, &order, nullptr))
+        hi = mid;
+      else
+        lo = mid;
+    }
+    pack_tc(sfx, pfx, n_cta, hi, page, &load, &order, &placed);
+  }
+  // partial slots: per (fork, head group) the prefix chunks come first, then
+  // the suffix pieces; a fork owns as many slots as its busiest head group
+  hp->n_groups = s.hkv;
+  hp->n_parts.assign((size_t)s.F * s.hkv, 0);
+  std::vector<int32_t> n_pre((size_t)s.F * s.hkv, 0), n_suf((size_t)s.F * s.hkv, 0);
+  for (const TcPlacement& pl : placed) {
+    const TcItem& it = pl.item;
+    for (int f = it.fork0; f < it.fork0 + it.nforks; ++f) {
+      int32_t& n = (it.table_kind == 0 ? n_pre : n_suf)[(size_t)f * s.hkv + it.kv_head];
+      n = std::max(n, it.part + 1);
+    }
+  }
+  int slot = 0;
+  for (int f = 0; f < s.F; ++f) {
+    int most = 0;
+    for (int g = 0; g < s.hkv; ++g) {
+      const size_t i = (size_t)f * s.hkv + g;
+      hp->n_parts[i] = n_pre[i] + n_suf[i];
+      most = std::max(most, hp->n_parts[i]);
+    }
+    hp->part_base[f] = slot;
+    slot += most;
+  }
+  hp->total_slots = slot;
+  // items in CTA order (empty CTAs dropped), suffix parts after the prefix ones,
+  // block-table starts resolved on the host when the host offsets are given
+  const bool host_off = lens->prefix_bt_offsets && lens->suffix_bt_offsets;
+  hp->tc.clear();
+  hp->cta_offsets.assign(1, 0);
+  std::vector<int> per_cta(n_cta + 1, 0);  // counting sort of the placements by CTA
+  for (const TcPlacement& pl : placed) ++per_cta[pl.cta + 1];
+  for (int c = 0; c < n_cta; ++c) per_cta[c + 1] += per_cta[c];
+  std::vector<TcItem> by_cta(placed.size());
+  {
+    std::vector<int> next(per_cta.begin(), per_cta.end() - 1);
+    for (const TcPlacement& pl : placed) by_cta[next[pl.cta]++] = pl.item;
+  }
+  for (int c = 0; c < n_cta; ++c) {
+    if (per_cta[c + 1] == per_cta[c]) continue;  // empty CTAs are dropped
+    for (int i = per_cta[c]; i < per_cta[c + 1]; ++i) {
+      TcItem it = by_cta[i];
+      if (it.table_kind == 1) it.part += n_pre[(size_t)it.fork0 * s.hkv + it.kv_head];
+      it.table_off = host_off ? (it.table_kind == 0 ? lens->prefix_bt_offsets[it.seq]
+                                                    : lens->suffix_bt_offsets[it.seq])
+                              : -1;
+      hp->tc.push_back(it);
+    }
+    hp->cta_offsets.push_back((int32_t)hp->tc.size());
+  }
+  hp->cta_items.clear();
+}
+
 void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   const int n_sm = device_sm_count();
   const int32_t* fo = lens->fork_offsets;
@@ -164,69 +347,11 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   hp->cta_offsets.assign(1, 0);
   hp->part_base.assign(s.F, 0);
   hp->n_parts.assign(s.F, 0);
+  hp->n_groups = 1;
   int slot = 0;
 
   if (tc) {
-    // Tensor-core path: the prefix of each trace is cut into chunks whose query
-    // rows are all forks of the trace (up to 128 rows per item); every suffix is
-    // cut into chunks of the same length.  The chunk length spreads the total
-    // token work over one persistent CTA per SM.
-    const int pg = fork_tc_page_size();
-    const int forks_per_item = std::max(1, 128 / s.G);
-    long long work = 0;
-    for (int t = 0; t < s.T; ++t) {
-      const int nf = fo[t + 1] - fo[t];
-      work += (long long)lens->prefix_lens[t] * s.hkv * ((nf + forks_per_item - 1) / forks_per_item);
-      for (int f = fo[t]; f < fo[t + 1]; ++f) work += (long long)lens->suffix_lens[f] * s.hkv;
-    }
-    long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
-    chunk = std::max<long long>(fork_tc_tile_tokens(), (chunk + pg - 1) / pg * pg);
-    std::vector<long long> cost;
-    const long long item_overhead = 128;  // token-equivalents per item (Q load, output write)
-    for (int t = 0; t < s.T; ++t) {
-      const int P = lens->prefix_lens[t];
-      const int np = (int)((P + chunk - 1) / chunk);
-      for (int f = fo[t]; f < fo[t + 1]; ++f) {
-        const int S = lens->suffix_lens[f];
-        const int ns = (int)((S + chunk - 1) / chunk);
-        hp->part_base[f] = slot;
-        hp->n_parts[f] = np + ns;
-        slot += np + ns;
-        for (int g = 0; g < s.hkv; ++g)
-          for (int c = 0; c < ns; ++c) {
-            TcItem it;
-            it.table_kind = 1;
-            it.seq = f;
-            it.kv_head = g;
-            it.fork0 = f;
-            it.nforks = 1;
-            it.tok_begin = (int)(c * chunk);
-            it.tok_end = (int)std::min<long long>(S, (c + 1) * chunk);
-            it.part = np + c;
-            it.dv0 = 0;
-            hp->tc.push_back(it);
-            cost.push_back(it.tok_end - it.tok_begin + item_overhead);
-          }
-      }
-      for (int g = 0; g < s.hkv; ++g)
-        for (int f0 = fo[t]; f0 < fo[t + 1]; f0 += forks_per_item)
-          for (int c = 0; c < np; ++c) {
-            TcItem it;
-            it.table_kind = 0;
-            it.seq = t;
-            it.kv_head = g;
-            it.fork0 = f0;
-            it.nforks = std::min(forks_per_item, fo[t + 1] - f0);
-            it.tok_begin = (int)(c * chunk);
-            it.tok_end = (int)std::min<long long>(P, (c + 1) * chunk);
-            it.part = c;
-            it.dv0 = 0;
-            hp->tc.push_back(it);
-            cost.push_back(it.tok_end - it.tok_begin + item_overhead);
-          }
-    }
-    finish_tc_plan(hp, cost, n_sm, lens);
-    hp->total_slots = slot;
+    build_tc_plan(s, lens, n_sm, hp);
     return;
   }
 
@@ -338,7 +463,7 @@ Layout layout_of(const Shape& s, const HostPlan& hp) {
   L.cta_offsets_off = align_up(L.cta_items_off + hp.cta_items.size() * 4, 16);
   L.part_base_off = align_up(L.cta_offsets_off + hp.cta_offsets.size() * 4, 16);
   L.n_parts_off = align_up(L.part_base_off + (size_t)s.F * 4, 16);
-  L.plan_bytes = L.n_parts_off + (size_t)s.F * 4;
+  L.plan_bytes = L.n_parts_off + hp.n_parts.size() * 4;
   L.ws_plan = kHeaderBytes;
   L.ws_part_o = align_up(L.ws_plan + L.plan_bytes, kAlign);
   L.ws_part_lse =
@@ -398,7 +523,7 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   put(L.cta_items_off, t_plan.cta_items.data(), t_plan.cta_items.size() * 4);
   put(L.cta_offsets_off, t_plan.cta_offsets.data(), t_plan.cta_offsets.size() * 4);
   put(L.part_base_off, t_plan.part_base.data(), (size_t)s.F * 4);
-  put(L.n_parts_off, t_plan.n_parts.data(), (size_t)s.F * 4);
+  put(L.n_parts_off, t_plan.n_parts.data(), t_plan.n_parts.size() * 4);
 
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   unsigned char* ws = static_cast<unsigned char*>(args->workspace);
@@ -413,6 +538,7 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   plan->n_split_items = h.n_split;
   plan->n_rows = s.F * s.hq;
   plan->total_slots = t_plan.total_slots;
+  plan->n_part_groups = t_plan.n_groups;
   plan->flags = (s.latent ? 1 : 0) | (args->kv_layout == SPECGEN_KV_TILED ? 2 : 0);
   plan->plan_bytes = (int64_t)L.plan_bytes;
   plan->ws_plan_off = (int64_t)L.ws_plan;
@@ -574,6 +700,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     mp.out = static_cast<__nv_bfloat16*>(args->out);
     mp.lse = args->lse;
     mp.n_rows = plan->n_rows;
+    mp.n_groups = plan->n_part_groups;
     mp.hq = args->hq;
     mp.dv = args->head_dim_v;
     if (launch_merge_parts(mp, stream, plan->n_tc_ctas > 0 && plan->n_split_items == 0) !=

@@ -276,7 +276,9 @@ __global__ void __launch_bounds__(kThreads, 2) split_decode_kernel(const SplitPa
       }
     }
     const size_t row = (size_t)it.slot * p.hq + it.h0 + r;
-    p.part_o[row * p.dv + it.dv0 + col] = mm == -INFINITY ? 0.f : acc / lsum;
+    const int cc = it.dv0 + col;
+    p.part_o[part_o_f4(it.slot, it.h0 + r, cc / 4, p.hq, p.dv) * 4 + cc % 4] =
+        mm == -INFINITY ? 0.f : acc / lsum;
     if (col == 0 && it.dv0 == 0)
       p.part_lse[row] = mm == -INFINITY ? -INFINITY : (mm + log2f(lsum)) * kLn2;
   }

@@ -17,7 +17,7 @@ struct SplitParams {
   const int32_t* suffix_bt;
   const int32_t* suffix_bt_off;
   const SplitItem* items;
-  float* part_o;    // [slots][hq][dv]
+  float* part_o;    // head-interleaved partials (part_o_f4)
   float* part_lse;  // [slots][hq]
   uint32_t* status;
   int hq, hkv, dqk, dv, page_size, num_pages;
