@@ -12,9 +12,11 @@ in [64, 512], Hq=64, Hkv=8, head dim 128, page 16, shuffled pages.
 Timing: W untimed warm-up steps, then K steps between CUDA events on the
 launching stream, bracketed by a barrier and a device synchronise.  Inputs
 rotate over enough resident replicas that every step's KV is evicted from L2
-before it is read again (the union of replicas is >= 3x L2).  The dominant
-kernel's time comes from events the library records between its launches
-(specgen_fork_attn_run_profiled) during the same timed steps.
+before it is read again (the union of replicas is >= 3x L2).  Steps replay
+CUDA graphs of 16 library calls.  Each kernel's average launch time comes from
+graphs of its stage alone (specgen_fork_attn_run_partials / _run_merge) run
+back to back over the same replicas after the timed region, timed with events
+on the same stream.
 
 With N > 1 (torchrun) every rank runs its own replica of the workload: fork
 decode shards by independent traces with no exchange, so scaling is weak and
@@ -285,16 +287,12 @@ def run_ours():
     # Timed steps replay CUDA graphs.  Each graph holds `per_graph` consecutive
     # steps (one library call each, on rotating replicas) so that host launch
     # overhead never starves the GPU.  K is covered exactly: full graphs plus
-    # one remainder graph.  Per-kernel times come from separate graphs of the
-    # profiled call (event marks between its kernels, as external record
-    # nodes), replayed after the timed region, so the marks never sit between
-    # the kernels of a timed step.
-    n_marks = 4
+    # one remainder graph.  Per-kernel times come from graphs of one stage
+    # alone (specgen_fork_attn_run_partials / _run_merge, back to back on the
+    # same stream and replicas), timed with events after the timed region.
     K, W = ARGS.steps, ARGS.warmup
     per_graph = max(1, min(16, K))
     lib = _lib.load()
-    n_l = C.c_int(0)
-    run_prof = lib.specgen_fork_attn_run_profiled
     arg_refs = [C.byref(a) for a in args]
     plan_refs = [C.byref(p) for p in plans]
     sp_c = C.c_void_p(sp)
@@ -303,38 +301,17 @@ def run_ours():
         assert st == 0, _lib.status_string(st)
     torch.cuda.synchronize(dev)
 
-    run_plain = lib.specgen_fork_attn_run
-
-    def make_graph(first_step, n_steps, profiled=False):
-        if not profiled:
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph, stream=stream):
-                for k in range(n_steps):
-                    r = (first_step + k) % replicas
-                    st = run_plain(arg_refs[r], plan_refs[r], sp_c)
-                    if st != 0:
-                        break
-            if st != 0:
-                raise RuntimeError(_lib.status_string(st))
-            return graph, None
-        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_marks)]
-               for _ in range(n_steps)]
-        with torch.cuda.stream(stream):
-            for row in evs:
-                for e in row:
-                    e.record(stream)  # create the CUDA events before the capture
-        torch.cuda.synchronize(dev)
-        handles = [(C.c_void_p * n_marks)(*[e.cuda_event for e in row]) for row in evs]
+    def make_graph(first_step, n_steps, call=lib.specgen_fork_attn_run):
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=stream):
             for k in range(n_steps):
                 r = (first_step + k) % replicas
-                st = run_prof(arg_refs[r], plan_refs[r], sp_c, handles[k], n_marks, C.byref(n_l))
+                st = call(arg_refs[r], plan_refs[r], sp_c)
                 if st != 0:
                     break
         if st != 0:
             raise RuntimeError(_lib.status_string(st))
-        return graph, evs
+        return graph, None
 
     n_full, rem = divmod(K, per_graph)
     n_distinct = max(1, min(n_full, 8))
@@ -358,22 +335,34 @@ def run_ours():
     barrier()
     clk = clocks.stop()
     total_ms = start.elapsed_time(end)
-    # per-kernel times: profiled graphs over the same rotation of replicas
-    prof_graphs = [make_graph(g * per_graph, per_graph, profiled=True)
-                   for g in range(max(1, min(8, K // per_graph)))]
-    for _ in range(2):
-        for graph, _ in prof_graphs:
-            graph.replay()
-    torch.cuda.synchronize(dev)
-    launches = n_l.value
-    sampled = sum(len(evs) for _, evs in prof_graphs)
-    per_kernel = [0.0] * launches
-    for _, evs in prof_graphs:
-        for row in evs:
-            for k in range(launches):
-                per_kernel[k] += row[k].elapsed_time(row[k + 1])
-    per_kernel = [x * K / sampled for x in per_kernel]  # scale the sample to K steps
-    n_slots = sampled
+    # per-kernel times: each stage alone, back to back, over the same replicas
+    def stage_ms(call):
+        g_list = [make_graph(g * per_graph, per_graph, call)[0]
+                  for g in range(max(1, min(8, K // per_graph)))]
+        for g in g_list:
+            g.replay()
+        torch.cuda.synchronize(dev)
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_rep = max(1, min(64, (K + per_graph * len(g_list) - 1) // (per_graph * len(g_list))))
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+            for _ in range(n_rep):
+                for g in g_list:
+                    g.replay()
+            t1.record(stream)
+        torch.cuda.synchronize(dev)
+        return t0.elapsed_time(t1) / (n_rep * len(g_list) * per_graph)
+
+    tc_name = "mla_tc" if w["v_pages"] is None else "fork_tc"
+    kernel_names = ([tc_name] if plans[0].n_tc_items > 0 else []) + \
+        (["split_decode"] if plans[0].n_split_items > 0 else [])
+    partials_ms = stage_ms(lib.specgen_fork_attn_run_partials)
+    merge_ms = stage_ms(lib.specgen_fork_attn_run_merge)
+    # one launch per partial kernel kind (a plan uses one of them) plus the merge
+    kernel_ms = [partials_ms / max(1, len(kernel_names))] * len(kernel_names) + [merge_ms]
+    kernel_names = kernel_names + ["lse_merge"]
+    launches = len(kernel_names)
+    n_slots = per_graph * max(1, min(8, K // per_graph))
     status = reps[0].status(sp)
     if status != 0:
         raise RuntimeError(f"workspace status {_lib.status_string(status)}")
@@ -389,11 +378,6 @@ def run_ours():
     # ---- end to end through the public API: host buffers, copies in the timed region
     e2e = measure_e2e(w, reps, stream, dev, K=min(K, 500), W=min(W, 5))
 
-    tc_name = "mla_tc" if w["v_pages"] is None else "fork_tc"
-    kernel_names = ([tc_name] if plans[0].n_tc_items > 0 else []) + \
-        (["split_decode"] if plans[0].n_split_items > 0 else []) + ["lse_merge"]
-    kernel_names = kernel_names[:launches]
-    kernel_ms = [t / K for t in per_kernel]
     dom = int(np.argmax(kernel_ms)) if kernel_ms else 0
     hbm, tf_burst, tf_sus, peak_src = measured_peaks()
     # algorithmic bytes of the dominant launch: what that kernel must read/write once
@@ -432,9 +416,9 @@ def run_ours():
             "head_dim": [w["dqk"], w["dv"]], "page_size": w["page_size"], "kv_layout": layout,
             "unique_bytes": nbytes["total"], "flops": flops["total"],
             "l2": f"inputs rotate over {replicas} resident replicas (>= 3x L2)",
-            "timing": f"CUDA graphs of {per_graph} steps; per-kernel times from event marks "
-                      f"in separate profiled graphs ({n_slots} steps, replayed after the timed "
-                      f"region)",
+            "timing": f"CUDA graphs of {per_graph} steps; per-kernel times from graphs of "
+                      f"one stage alone ({n_slots} distinct steps, replayed back to back after "
+                      f"the timed region)",
             "parallelism": f"replicas x{world}",
         },
         "gpu_launches": K * launches,

@@ -146,6 +146,21 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
 specgen_status specgen_fork_attn_run(const specgen_fork_attn_args* args,
                                      const specgen_plan* plan, void* cuda_stream);
 
+/* The two stages of specgen_fork_attn_run, for callers that schedule them
+ * apart (or time each kernel alone).  _partials launches the attention kernels
+ * (tensor-core and/or split-K), which write every work item's partial (O
+ * normalised by its own softmax sum, LSE) into the workspace; _merge launches
+ * the log-sum-exp merge that combines each (fork, head) row's partials into
+ * out / lse (exact merge of attention over disjoint key sets, the prefix and
+ * suffix stages above).  _partials then _merge on one stream equals one
+ * specgen_fork_attn_run.  (No separate counterpart in the paper: a scheduling
+ * and timing convenience.)  Same arguments, checks and status codes as
+ * specgen_fork_attn_run. */
+specgen_status specgen_fork_attn_run_partials(const specgen_fork_attn_args* args,
+                                              const specgen_plan* plan, void* cuda_stream);
+specgen_status specgen_fork_attn_run_merge(const specgen_fork_attn_args* args,
+                                           const specgen_plan* plan, void* cuda_stream);
+
 /* specgen_fork_attn_run with timing marks for per-kernel measurement: records
  * events[0] on `cuda_stream` before the first kernel and events[i] after the
  * i-th kernel (i = 1 .. n_events-1; extra launches get no mark).  `events`

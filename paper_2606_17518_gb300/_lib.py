@@ -30,6 +30,8 @@ EXPORTED = [
     "specgen_fork_attn_plan",
     "specgen_fork_attn_run",
     "specgen_fork_attn_run_profiled",
+    "specgen_fork_attn_run_partials",
+    "specgen_fork_attn_run_merge",
     "specgen_fork_attn_decode",
     "specgen_fork_attn_decode_static",
     "specgen_lse_merge",
@@ -97,6 +99,9 @@ def load() -> C.CDLL:
     lib.specgen_fork_attn_plan.argtypes = [P(ForkAttnArgs), P(HostLens), P(Plan), C.c_void_p]
     lib.specgen_fork_attn_run.restype = C.c_int
     lib.specgen_fork_attn_run.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
+    for stage in ("specgen_fork_attn_run_partials", "specgen_fork_attn_run_merge"):
+        getattr(lib, stage).restype = C.c_int
+        getattr(lib, stage).argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
     lib.specgen_fork_attn_run_profiled.restype = C.c_int
     lib.specgen_fork_attn_run_profiled.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p,
                                                    C.c_void_p, C.c_int, P(C.c_int)]
@@ -168,6 +173,17 @@ def specgen_fork_attn_plan(args: ForkAttnArgs, lens: HostLens, stream: int = 0) 
 def specgen_fork_attn_run(args: ForkAttnArgs, plan: Plan, stream: int = 0) -> None:
     _check(load().specgen_fork_attn_run(C.byref(args), C.byref(plan), C.c_void_p(stream)),
            "specgen_fork_attn_run")
+
+
+def specgen_fork_attn_run_partials(args: ForkAttnArgs, plan: Plan, stream: int = 0) -> None:
+    _check(load().specgen_fork_attn_run_partials(C.byref(args), C.byref(plan),
+                                                 C.c_void_p(stream)),
+           "specgen_fork_attn_run_partials")
+
+
+def specgen_fork_attn_run_merge(args: ForkAttnArgs, plan: Plan, stream: int = 0) -> None:
+    _check(load().specgen_fork_attn_run_merge(C.byref(args), C.byref(plan), C.c_void_p(stream)),
+           "specgen_fork_attn_run_merge")
 
 
 def specgen_fork_attn_run_profiled(args: ForkAttnArgs, plan: Plan, stream: int, events,

@@ -576,8 +576,9 @@ struct Marks {
   }
 };
 
+// stages: bit 0 the partial-attention kernels, bit 1 the merge.
 specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* plan,
-                        void* cuda_stream, Marks& marks);
+                        void* cuda_stream, Marks& marks, int stages = 3);
 
 }  // namespace
 
@@ -587,6 +588,18 @@ specgen_status specgen_fork_attn_run(const specgen_fork_attn_args* args, const s
                                      void* cuda_stream) {
   Marks marks{nullptr, 0};
   return run_impl(args, plan, cuda_stream, marks);
+}
+
+specgen_status specgen_fork_attn_run_partials(const specgen_fork_attn_args* args,
+                                              const specgen_plan* plan, void* cuda_stream) {
+  Marks marks{nullptr, 0};
+  return run_impl(args, plan, cuda_stream, marks, 1);
+}
+
+specgen_status specgen_fork_attn_run_merge(const specgen_fork_attn_args* args,
+                                           const specgen_plan* plan, void* cuda_stream) {
+  Marks marks{nullptr, 0};
+  return run_impl(args, plan, cuda_stream, marks, 2);
 }
 
 specgen_status specgen_fork_attn_run_profiled(const specgen_fork_attn_args* args,
@@ -604,7 +617,7 @@ specgen_status specgen_fork_attn_run_profiled(const specgen_fork_attn_args* args
 namespace {
 
 specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* plan,
-                        void* cuda_stream, Marks& marks) {
+                        void* cuda_stream, Marks& marks, int stages) {
   if (!args || !plan) return SPECGEN_ERR_NULL;
   if (!plan->valid) return SPECGEN_ERR_SHAPE;
   specgen_status st = check_pointers(args);
@@ -638,7 +651,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   sp.num_pages = args->num_pages;
   sp.scale_log2 = args->scale * 1.4426950408889634f;
   if (!marks.mark(stream, 0)) return SPECGEN_ERR_CUDA;
-  if (plan->n_tc_ctas > 0) {
+  if ((stages & 1) && plan->n_tc_ctas > 0) {
     TcParams tp;
     tp.q = sp.q;
     tp.prefix_bt = args->prefix_block_table;
@@ -684,14 +697,14 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     if (e != cudaSuccess) return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
   }
-  if (plan->n_split_items > 0) {
+  if ((stages & 1) && plan->n_split_items > 0) {
     if (launch_split_decode(sp, plan->n_split_items, args->v_pages == nullptr, stream) !=
         cudaSuccess)
       return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
   }
 
-  {  // merge pass: combine every row's partials
+  if (stages & 2) {  // merge pass: combine every row's partials
     MergeParams mp;
     mp.part_o = part_o;
     mp.part_lse = part_lse;

@@ -255,3 +255,22 @@ def test_without_host_table_offsets():
         fd.decode()
         o2, l2 = fd.results()
         assert np.array_equal(o, o2) and np.array_equal(lse, l2)
+
+
+@pytest.mark.parametrize("name", ["fork_p8k_f8", "mla_p16k_f8"])
+def test_stages_equal_one_run(name):
+    """run_partials then run_merge on one stream gives the bits of one run."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload(name)
+    fd = ForkDecode(w)
+    fd.plan()
+    fd.run()
+    o1, l1 = fd.results()
+    fd.out.zero_()
+    fd.lse.zero_()
+    _lib.specgen_fork_attn_run_partials(fd.args(), fd.plan_info)
+    _lib.specgen_fork_attn_run_merge(fd.args(), fd.plan_info)
+    torch.cuda.synchronize()
+    o2, l2 = fd.results()
+    assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
