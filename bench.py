@@ -44,9 +44,9 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--kv-layout", choices=["auto", "rows", "tiled"], default="auto",
-                    help="K/V pool layout: token-major rows or 8x8 tiles (auto: tiled where the "
-                         "tensor-core path supports it)")
+    ap.add_argument("--kv-layout", choices=["rows", "tiled"], default="rows",
+                    help="K/V pool layout: token-major rows (default) or 8x8 core-matrix tiles "
+                         "(tensor-core shapes only)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
     return ap.parse_args()
@@ -272,9 +272,7 @@ def run_ours():
         f" {replicas} replicas")
     stream = torch.cuda.Stream(dev)
     sp = stream.cuda_stream
-    tiled_ok = (w["v_pages"] is not None and w["page_size"] == 16 and w["dqk"] == w["dv"]
-                and w["dqk"] in (64, 128) and w["hq"] // w["hkv"] <= 128)
-    layout = ARGS.kv_layout if ARGS.kv_layout != "auto" else ("tiled" if tiled_ok else "rows")
+    layout = ARGS.kv_layout if w["v_pages"] is not None else "rows"
     kv_layout = _lib.KV_TILED if layout == "tiled" else _lib.KV_ROWS
     reps = [ForkDecode(w, device=dev, kv_layout=kv_layout) for _ in range(replicas)]
     with torch.cuda.stream(stream):
