@@ -9,10 +9,13 @@
 //
 // Tensor memory cannot hold a 128 x 512 fp32 output next to the scores, so an
 // item produces one half of the value columns (dv0 = 0 or 256); the score tile
-// is computed for each half.  Per 32-token tile t (half a page):
-//   warp 0 (TMA)   nine boxes of 32 rows x 64 columns (128B swizzle) -> 2-stage ring
-//   warp 1 (MMA)   S_t = Q K_t^T (36 k-steps, N = 32), then
-//                  O += P_t V_t[:, dv0:dv0+256] (A = P in TMEM, N = 256)
+// is computed for each half.  Q (128 x 576 bf16, 144 KB) does not fit in
+// shared memory next to two 64-token K tiles (72 KB each), so its first 256
+// columns live in tensor memory (the A operand of the first 16 k-steps) and
+// the other 320 in shared memory.  Per 64-token tile t (one page):
+//   warp 0 (TMA)   nine boxes of 64 rows x 64 columns (128B swizzle) -> 2-stage ring
+//   warp 1 (MMA)   S_t = Q K_t^T (36 k-steps, N = 64; A from TMEM, then shared
+//                  memory), then O += P_t V_t[:, dv0:dv0+256] (A = P in TMEM, N = 256)
 //   warps 2-5      one thread per head: the tile's scores, masked, online
 //                  softmax in log2 units with lazy rescaling, P back to TMEM
 //                  as bf16 pairs.
@@ -37,17 +40,19 @@ constexpr int kDqk = 576;
 constexpr int kDv = 512;
 constexpr int kDvHalf = 256;
 constexpr int kPage = 64;
-constexpr int kTT = 32;                      // tokens per tile (half a page)
+constexpr int kTT = 64;                      // tokens per tile (one page)
 constexpr int kST = 2;                       // pipeline stages
 constexpr int kPanels = kDqk / 64;           // 9 column panels of 64
 constexpr int kSteps = kDqk / 16;            // 36 k-steps of 16 for the scores
 constexpr int kThreads = 192;                // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
-constexpr uint32_t kTmemCols = 512;          // S[0] [0,32) S[1] [32,64) O [256,512)
+constexpr uint32_t kTmemCols = 512;          // S[0] [0,64) S[1] [64,128) Q [128,256) O [256,512)
+constexpr uint32_t kTmemQ = 128;
 constexpr uint32_t kTmemO = 256;
+constexpr int kQTmemPanels = 4;              // Q columns [0, 256) in TMEM: k-steps 0..15
 constexpr float kRescaleLog2 = 8.0f;
 constexpr uint32_t kQPanel = 128 * 128u;     // 128 rows x 128 B
-constexpr uint32_t kKPanel = kTT * 128u;     // 32 rows x 128 B
-constexpr uint32_t kOffKV = kPanels * kQPanel;
+constexpr uint32_t kKPanel = kTT * 128u;     // 64 rows x 128 B
+constexpr uint32_t kOffKV = (kPanels - kQTmemPanels) * kQPanel;  // Q panels 4..8
 constexpr uint32_t kStage = kPanels * kKPanel;
 constexpr uint32_t kOffBar = kOffKV + kST * kStage;
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
@@ -116,8 +121,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
-    // A tile is half a page; page ids are fetched 32 at a time (64 tiles) by
-    // the warp, one batch ahead.  Lanes 0..8 each issue one 64-column box.
+    // A tile is one page; page ids are fetched 32 at a time by the warp, one
+    // batch ahead.  Lanes 0..8 each issue one 64-column box.
     int t = 0;
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
@@ -158,7 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       // descriptors are built once; every MMA adds a constant offset to them
-      const uint64_t dq = smem_desc_sw128(sQ, 16, 1024);
+      const uint64_t dq = smem_desc_sw128(sQ, 16, 1024);  // Q panels 4..8 from panel 0 here
       const uint64_t dk0 = smem_desc_sw128(sK(0), 16, 1024);
       const uint64_t dvb0 = smem_desc_sw128(sK(0), kKPanel, 1024);
       constexpr uint64_t kStageDesc = kStage >> 4;
@@ -183,7 +188,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t vpanel = (uint64_t)((v_it.dv0 / 64) * kKPanel) >> 4;
           const uint64_t dv = dvb0 + (uint64_t)s * kStageDesc + vpanel;
 #pragma unroll
-          for (int kk = 0; kk < kTT / 16; ++kk)
+          for (int kk = 0; kk < kTT / 16; ++kk)  // 16 tokens (16 rows x 128 B) a step
             mma_bf16_ts(tmem + kTmemO, tmem + (uint32_t)b * kTT + kk * 8u,
                         dv + (uint64_t)((kk * 2048u) >> 4), idesc_pv,
                         (v_j > 0 || kk > 0) ? 1u : 0u);
@@ -203,10 +208,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t dk = dk0 + (uint64_t)s * kStageDesc;
             const uint32_t d_s = tmem + (uint32_t)b * kTT;
 #pragma unroll
-            for (int kk = 0; kk < kSteps; ++kk) {
-              const uint64_t qo = ((kk >> 2) * kQPanel + (kk & 3) * 32u) >> 4;
+            for (int kk = 0; kk < kQTmemPanels * 4; ++kk) {  // A = Q from TMEM, 8 columns a step
               const uint64_t ko = ((kk >> 2) * kKPanel + (kk & 3) * 32u) >> 4;
-              mma_bf16(d_s, dq + qo, dk + ko, idesc_s, kk > 0 ? 1u : 0u);
+              mma_bf16_ts(d_s, tmem + kTmemQ + kk * 8u, dk + ko, idesc_s, kk > 0 ? 1u : 0u);
+            }
+#pragma unroll
+            for (int kk = kQTmemPanels * 4; kk < kSteps; ++kk) {  // A = Q from shared memory
+              const uint64_t qo = (((kk >> 2) - kQTmemPanels) * kQPanel + (kk & 3) * 32u) >> 4;
+              const uint64_t ko = ((kk >> 2) * kKPanel + (kk & 3) * 32u) >> 4;
+              mma_bf16(d_s, dq + qo, dk + ko, idesc_s, 1u);
             }
             mma_commit(s_full(b));
             ++s_u;
@@ -252,14 +262,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int ntiles = ntiles_of(it);
       const int page0 = it.tok_begin / kPage;
 
-      {  // Q row of this head -> shared memory, nine 128B-swizzled panels
+      {  // Q row of this head: columns [0, 256) -> TMEM (this thread's lane),
+         // the rest -> shared memory as five 128B-swizzled panels
         const uint4* src = reinterpret_cast<const uint4*>(p.q + ((size_t)it.fork0 * 128 + row) * kDqk);
-#pragma unroll 8
-        for (int c = 0; c < kDqk / 8; ++c) {
-          const uint4 q = __ldg(src + c);
-          st_shared_v4(sQ + (c >> 3) * kQPanel + row * 128u + (((c & 7) ^ (row & 7)) << 4), q.x,
-                       q.y, q.z, q.w);
+#pragma unroll
+        for (int c4 = 0; c4 < kQTmemPanels * 8; c4 += 8) {  // 8 x 16 B = 32 TMEM columns
+          uint32_t v[32];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const uint4 q = __ldg(src + c4 + e);
+            v[4 * e] = q.x;
+            v[4 * e + 1] = q.y;
+            v[4 * e + 2] = q.z;
+            v[4 * e + 3] = q.w;
+          }
+          tmem_st32(s_base + kTmemQ + (uint32_t)(c4 * 4), v);
         }
+#pragma unroll 8
+        for (int c = kQTmemPanels * 8; c < kDqk / 8; ++c) {
+          const uint4 q = __ldg(src + c);
+          st_shared_v4(sQ + ((c >> 3) - kQTmemPanels) * kQPanel + row * 128u +
+                           (((c & 7) ^ (row & 7)) << 4),
+                       q.x, q.y, q.z, q.w);
+        }
+        tmem_wait_st();
         fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(q_ready);
@@ -284,24 +310,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool page_ok = page >= 0 && page < p.num_pages;
         float s[kTT];
         {
-          uint32_t r[32];
-          tmem_ld32(s_base + (uint32_t)b * kTT, r);
+          uint32_t r[kTT / 32][32];
+#pragma unroll
+          for (int c = 0; c < kTT / 32; ++c) tmem_ld32(s_base + (uint32_t)b * kTT + c * 32u, r[c]);
           tmem_wait_ld();
 #pragma unroll
-          for (int i = 0; i < kTT; ++i) s[i] = __uint_as_float(r[i]);
+          for (int c = 0; c < kTT / 32; ++c)
+#pragma unroll
+            for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[c][i]);
         }
         if (nt < kTT || !page_ok) {
 #pragma unroll
           for (int i = 0; i < kTT; ++i)
             if (!(i < nt && page_ok)) s[i] = -INFINITY;
         }
-        float mx0 = s[0], mx1 = s[1];
+        float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
 #pragma unroll
-        for (int i = 2; i < kTT; i += 2) {
+        for (int i = 4; i < kTT; i += 4) {
           mx0 = fmaxf(mx0, s[i]);
           mx1 = fmaxf(mx1, s[i + 1]);
+          mx2 = fmaxf(mx2, s[i + 2]);
+          mx3 = fmaxf(mx3, s[i + 3]);
         }
-        const float m_tile = fmaxf(mx0, mx1) * sl2;
+        const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
         bool rescale = false;
         float alpha = 1.f;
         if (m_tile > m + kRescaleLog2 || (m == -INFINITY && m_tile != -INFINITY)) {
@@ -312,17 +343,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const float sub = m == -INFINITY ? 0.f : m;
         {
-          uint32_t pk[16];
-          float ps = 0.f;
+          uint32_t pk[kTT / 2];
+          float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
+          for (int i = 0; i < kTT / 2; ++i) {
             const float p0 = fast_exp2(fmaf(s[2 * i], sl2, -sub));
             const float p1 = fast_exp2(fmaf(s[2 * i + 1], sl2, -sub));
-            ps += p0 + p1;
+            ps0 += p0;
+            ps1 += p1;
             pk[i] = pack_bf16x2(p0, p1);
           }
-          tmem_st16(s_base + (uint32_t)b * kTT, pk);
-          l += ps;
+          tmem_st32(s_base + (uint32_t)b * kTT, pk);
+          l += ps0 + ps1;
         }
         // value rows past the sequence in this tile: zero them before PV
         if (nt < kTT) {
@@ -434,7 +466,7 @@ cudaError_t launch_mla_tc(const MlaParams& p, const void* k_pages, int grid, cud
   EncodeTiledFn enc = encode_fn();
   if (!enc || !k_pages || p.num_pages < 1) return cudaErrorInvalidValue;
   // latent pool [num_pages][1][64][576] as a 4-D tensor (576, 64, 1, pages);
-  // one box = 64 columns x 32 rows (half a page)
+  // one box = 64 columns x 64 rows (one page)
   CUtensorMap mk;
   const cuuint64_t dims[4] = {(cuuint64_t)kDqk, (cuuint64_t)kPage, 1, (cuuint64_t)p.num_pages};
   const cuuint64_t strides[3] = {(cuuint64_t)kDqk * 2, (cuuint64_t)kPage * kDqk * 2,
