@@ -4,7 +4,8 @@ TEST INFRASTRUCTURE ONLY.  Nothing in the product path may import, call or
 link anything under ``oracle/``; only the test suite, the package smoke check
 and the benchmark's CPU-baseline leg use it.  It shares no code with the CUDA
 path: it computes the plain definition of softmax attention in float64 from
-the bf16 bit patterns the GPU path also reads.
+the bf16 bit patterns the GPU path also reads, and the plain row copies of a
+decode step's append into paged suffixes (``paging.py``).
 
 Every function here is pinned by ``tests/test_oracle_pins.py`` (closed forms,
 brute force, library cross-checks and invariants); no function carries the
@@ -21,3 +22,4 @@ from .attention import (  # noqa: F401
     fork_attn_decode_rows,
     fork_attn_split_merge,
 )
+from .paging import append_kv  # noqa: F401

@@ -1,0 +1,59 @@
+"""Plain reference for appending one decode step's K/V to paged suffixes (test infrastructure only).
+
+What is computed and where it comes from
+----------------------------------------
+After a fork event every fork decodes its own continuation while the reasoning
+prefix stays shared (Algorithm 1, "Fork K spec. generations"; Section 4.2):
+each decode step adds one key/value row per fork to that fork's private
+suffix.  In the paged layout (token j of a sequence at page ``table[j // B]``,
+slot ``j % B``), the new token of fork f with S_f tokens already in its suffix
+goes to slot ``S_f % B`` of page ``table[S_f // B]``; when ``S_f % B == 0`` that
+page does not exist yet and the fork takes the next id of a free list, in fork
+order, and records it in its block table.
+
+Readings where the paper is silent (listed in the design notes): the free list
+is consumed in increasing fork order; a fork's block table has a fixed capacity
+(its CSR range) and an append past it is an error; the latent pool (no value
+pool) stores only the key row.
+
+Deliberately plain: one fork at a time, numpy copies of whole rows.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+
+def append_kv(k_pages, v_pages, suffix_table, suffix_bt_offsets, suffix_lens, k_new, v_new,
+              free_pages, page_size):
+    """Return (k_pages, v_pages, suffix_table, pages_taken) after one append.
+
+    k_pages / v_pages: [num_pages, Hkv, B, width] bf16 bits (v_pages may be None);
+    suffix_table / suffix_bt_offsets: CSR block tables (capacity per fork);
+    suffix_lens[f]: tokens already in fork f's suffix; k_new / v_new:
+    [F, Hkv, width] rows to append; free_pages: ids to take, in order.
+    The inputs are not modified.
+    """
+    k = np.array(k_pages, copy=True)
+    v = None if v_pages is None else np.array(v_pages, copy=True)
+    table = np.array(suffix_table, copy=True)
+    offs = np.asarray(suffix_bt_offsets)
+    taken = 0
+    for f in range(len(suffix_lens)):
+        n = int(suffix_lens[f])
+        page_index, slot = divmod(n, page_size)
+        start, cap = int(offs[f]), int(offs[f + 1] - offs[f])
+        if page_index >= cap:
+            raise ValueError(f"fork {f}: block table full ({cap} pages)")
+        if slot == 0:
+            if taken >= len(free_pages):
+                raise ValueError("free list exhausted")
+            page = int(free_pages[taken])
+            taken += 1
+            table[start + page_index] = page
+        else:
+            page = int(table[start + page_index])
+        k[page, :, slot, :] = k_new[f]
+        if v is not None:
+            v[page, :, slot, :] = v_new[f]
+    return k, v, table, taken

@@ -219,3 +219,43 @@ def tile_kv_pool(pool: np.ndarray) -> np.ndarray:
     P, H, B, D = pool.shape
     t = pool.reshape(P, H, B // 8, 8, D // 8, 8)           # [.., tg, t8, dc, d8]
     return np.ascontiguousarray(t.transpose(0, 1, 2, 4, 3, 5)).reshape(P, H, B, D)
+
+
+def make_decode_state(w: dict, steps: int, seed: int = 12345) -> dict:
+    """A workload prepared for `steps` decode steps that append to the suffixes.
+
+    Adds spare pages to the pools (NaN-filled, ids appended at the end of the
+    pool and handed out through a shuffled free list), widens every fork's
+    suffix block table to hold ``suffix_lens + steps`` tokens (unallocated
+    entries are -1), and draws the new key/value rows of every step
+    (``k_new``: [steps, F, Hkv, dqk], ``v_new``: [steps, F, Hkv, dv] or None).
+    Inputs only: no arithmetic of the method.  Returns a new dict.
+    """
+    B, F = w["page_size"], w["total_forks"]
+    rng = np.random.default_rng(seed)
+    lens = w["suffix_lens"].astype(np.int64)
+    used = -(-lens // B)
+    cap = -(-(lens + steps) // B)
+    spare = int((cap - used).sum())
+    n_old = w["num_pages"]
+    offs = np.concatenate([[0], np.cumsum(cap)]).astype(np.int32)
+    table = np.full(int(cap.sum()), -1, dtype=np.int32)
+    old_offs = w["suffix_bt_offsets"]
+    for f in range(F):
+        table[offs[f]: offs[f] + used[f]] = w["suffix_table"][old_offs[f]: old_offs[f + 1]]
+    free = (n_old + rng.permutation(spare)).astype(np.int32)
+
+    def grow(pool):
+        if pool is None:
+            return None
+        extra = np.full((spare,) + pool.shape[1:], BF16_QNAN, dtype=np.uint16)
+        return np.concatenate([pool, extra], axis=0)
+
+    out = dict(w)
+    out.update(
+        k_pages=grow(w["k_pages"]), v_pages=grow(w["v_pages"]), num_pages=n_old + spare,
+        suffix_table=table, suffix_bt_offsets=offs, free_pages=free, steps=steps,
+        k_new=bf16_normal(rng, (steps, F, w["hkv"], w["dqk"])),
+        v_new=(bf16_normal(rng, (steps, F, w["hkv"], w["dv"])) if w["v_pages"] is not None
+               else None))
+    return out

@@ -359,3 +359,100 @@ def test_rows_entry_matches_full():
     for i, (f, h) in enumerate(rows):
         np.testing.assert_allclose(ro[i], o[f, h], rtol=0, atol=1e-14)
         np.testing.assert_allclose(rl[i], lse[f, h], rtol=0, atol=1e-14)
+
+
+# ----------------------------------------------------------------- decode-step append
+
+def _read_fixture(name):
+    vals = {}
+    for line in open(os.path.join(GOLDEN, name)):
+        line = line.strip()
+        if line and not line.startswith("#"):
+            key, *rest = line.split()
+            vals[key] = rest
+    return vals
+
+
+def test_append_golden_fixture():
+    g = _read_fixture("append_small.txt")
+    B = int(g["page_size"][0])
+    lens = np.array([int(x) for x in g["lens"]], dtype=np.int32)
+    offs = np.array([int(x) for x in g["offsets"]], dtype=np.int32)
+    table = np.array([int(x) for x in g["table_before"]], dtype=np.int32)
+    free = np.array([int(x) for x in g["free"]], dtype=np.int32)
+    rows = [float(x) for x in g["new_row_values"]]
+    pool = np.full((8, 1, B, 2), 0x7FC0, dtype=np.uint16)   # NaN everywhere
+    k_new = wl.round_to_bf16_bits(np.array([[[r, r]] for r in rows], dtype=np.float32))
+    k, v, t, taken = oracle.append_kv(pool, None, table, offs, lens, k_new, None, free, B)
+    assert v is None
+    assert t.tolist() == [int(x) for x in g["table_after"]]
+    assert taken == int(g["taken"][0])
+    written = [tuple(int(y) for y in w.split(":")) for w in g["written"]]
+    for (page, head, slot), r in zip(written, rows):
+        assert oracle.bf16_bits_to_f64(k[page, head, slot]).tolist() == [r, r]
+    mask = np.ones(k.shape[:3], dtype=bool)
+    for page, head, slot in written:
+        mask[page, head, slot] = False
+    assert np.array_equal(k[mask], pool[mask])          # nothing else touched
+    assert table.tolist() == [int(x) for x in g["table_before"]]   # inputs not modified
+
+
+def _python_sequence(pool, table, offs, f, n, B, head):
+    """Pure-Python gather of the first n rows of fork f's paged sequence."""
+    out = []
+    for j in range(n):
+        page = int(table[int(offs[f]) + j // B])
+        out.append([int(x) for x in pool[page, head, j % B]])
+    return out
+
+
+@pytest.mark.parametrize("B", [1, 2, 16])
+def test_append_grows_every_sequence_by_its_row(B):
+    """Appending n steps one at a time gives, for every fork and head, the old
+    sequence followed by the n new rows in order (pure-Python gather), with the
+    free list consumed exactly when a fork crosses a page boundary."""
+    rng = np.random.default_rng(B)
+    F, H, W, steps = 5, 2, 3, 2 * B + 3
+    lens0 = rng.integers(0, 3 * B, F).astype(np.int32)
+    cap = -(-(lens0 + steps) // B)
+    offs = np.concatenate([[0], np.cumsum(cap)]).astype(np.int32)
+    used = -(-lens0 // B)
+    n_pages = int(cap.sum()) + 4
+    perm = rng.permutation(n_pages).astype(np.int32)
+    table = np.full(int(cap.sum()), -1, dtype=np.int32)
+    nxt = 0
+    for f in range(F):
+        table[offs[f]: offs[f] + used[f]] = perm[nxt: nxt + used[f]]
+        nxt += int(used[f])
+    free = perm[nxt:].copy()
+    pool_k = rng.integers(0, 1 << 15, (n_pages, H, B, W)).astype(np.uint16)
+    pool_v = rng.integers(0, 1 << 15, (n_pages, H, B, W)).astype(np.uint16)
+    before = {f: [_python_sequence(pool_k, table, offs, f, int(lens0[f]), B, h) for h in range(H)]
+              for f in range(F)}
+    news = rng.integers(0, 1 << 15, (steps, F, H, 2, W)).astype(np.uint16)
+    k, v, t, lens, fi = pool_k, pool_v, table, lens0.copy(), 0
+    for s in range(steps):
+        k, v, t, taken = oracle.append_kv(k, v, t, offs, lens, news[s, :, :, 0], news[s, :, :, 1],
+                                          free[fi:], B)
+        assert taken == int(np.sum(lens % B == 0))
+        fi += taken
+        lens = lens + 1
+    for f in range(F):
+        for h in range(H):
+            seq_k = _python_sequence(k, t, offs, f, int(lens[f]), B, h)
+            seq_v = _python_sequence(v, t, offs, f, int(lens[f]), B, h)
+            assert seq_k[: lens0[f]] == before[f][h]
+            assert seq_k[lens0[f]:] == [[int(x) for x in news[s, f, h, 0]] for s in range(steps)]
+            assert seq_v[lens0[f]:] == [[int(x) for x in news[s, f, h, 1]] for s in range(steps)]
+    assert fi == int(np.sum(cap - used))  # every fork filled its capacity exactly
+
+
+def test_append_rejects_full_table_and_empty_free_list():
+    pool = np.zeros((4, 1, 2, 2), dtype=np.uint16)
+    row = np.zeros((1, 1, 2), dtype=np.uint16)
+    with pytest.raises(ValueError):   # length 2 needs a second page; capacity is 1
+        oracle.append_kv(pool, None, np.array([0], np.int32), np.array([0, 1], np.int32),
+                         np.array([2], np.int32), row, None, np.array([3], np.int32), 2)
+    with pytest.raises(ValueError):   # new page needed, free list empty
+        oracle.append_kv(pool, None, np.array([-1], np.int32), np.array([0, 1], np.int32),
+                         np.array([0], np.int32), row, None, np.array([], np.int32), 2)
