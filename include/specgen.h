@@ -210,6 +210,47 @@ specgen_status specgen_lse_merge(const void* out_a, const float* lse_a,
                                  void* out, float* lse, int rows, int dv,
                                  int dtype, void* cuda_stream);
 
+/* ---- Decode-step append --------------------------------------------------
+ * After a fork event every fork decodes its own continuation while the prefix
+ * stays shared (Algorithm 1, "Fork K spec. generations"; Section 4.2), so each
+ * decode step adds one key/value row per fork to the fork's private suffix,
+ * before that step's attention reads it.  Fork f with n = suffix_lens[f]
+ * tokens already in its suffix writes its rows to slot n % page_size of page
+ * suffix_block_table[suffix_bt_offsets[f] + n / page_size]; when
+ * n % page_size == 0 that page is new: the fork takes free_pages[j], where j
+ * counts the forks before f that also start a page in this call (fork order),
+ * and the id is written into the fork's block table.  All inputs are device
+ * memory and nothing is planned on the host, so the call can be captured in a
+ * CUDA graph; the caller then adds 1 to every suffix length (host and device
+ * copies) and drops the j ids taken from the front of its free list.
+ * A fork whose block table has no room (n / page_size >= its CSR capacity),
+ * whose free-list entry does not exist, or whose page id is outside
+ * [0, num_pages) writes nothing and ORs SPECGEN_ERR_INDEX's bit (1) into
+ * *status (when status is not NULL; a fork-attention workspace's first word
+ * serves, read back with specgen_workspace_status).  Rows are copied bit for
+ * bit.  (An extension of the decode path; the paper shows no kernel for it.) */
+typedef struct {
+  int total_forks, hkv, head_dim_qk, head_dim_v, page_size, num_pages;
+  int kv_layout;                    /* layout of the pools: SPECGEN_KV_ROWS / _TILED */
+  const void* k_new;                /* bf16 [total_forks][hkv][head_dim_qk], 16-B aligned */
+  const void* v_new;                /* bf16 [total_forks][hkv][head_dim_v]; NULL iff v_pages is */
+  void* k_pages;                    /* pools as in specgen_fork_attn_args (written), 16-B aligned */
+  void* v_pages;                    /* NULL: latent pool, only the key row is stored */
+  int32_t* suffix_block_table;      /* CSR with spare capacity per fork; new ids written */
+  const int32_t* suffix_bt_offsets; /* [total_forks + 1] */
+  const int32_t* suffix_lens;       /* [total_forks] tokens already in each suffix */
+  const int32_t* free_pages;        /* [num_free] page ids handed out in fork order */
+  int num_free;
+  uint32_t* status;                 /* device status word, or NULL */
+} specgen_append_args;
+
+/* Head dims must be multiples of 8 (rows move in 16-byte pieces); page_size a power of
+ * two <= 1024; the tiled layout needs page_size % 8 == 0 and a value pool.
+ * Returns SPECGEN_OK after launching (asynchronous on cuda_stream),
+ * SPECGEN_ERR_NULL / _SHAPE / _UNSUPPORTED on bad arguments (nothing
+ * launched), SPECGEN_ERR_CUDA if the launch fails. */
+specgen_status specgen_append_kv(const specgen_append_args* args, void* cuda_stream);
+
 /* Read the workspace status word written by the kernels (synchronises
  * `cuda_stream`).  Returns SPECGEN_OK, SPECGEN_ERR_INDEX or SPECGEN_ERR_TIMEOUT. */
 specgen_status specgen_workspace_status(const void* workspace, void* cuda_stream);

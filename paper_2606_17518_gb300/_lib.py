@@ -35,6 +35,7 @@ EXPORTED = [
     "specgen_fork_attn_decode",
     "specgen_fork_attn_decode_static",
     "specgen_lse_merge",
+    "specgen_append_kv",
     "specgen_workspace_status",
     "specgen_status_string",
     "specgen_version",
@@ -56,6 +57,18 @@ class ForkAttnArgs(C.Structure):
 
 KV_ROWS = 0
 KV_TILED = 1
+
+
+class AppendArgs(C.Structure):
+    _fields_ = [
+        ("total_forks", C.c_int), ("hkv", C.c_int), ("head_dim_qk", C.c_int),
+        ("head_dim_v", C.c_int), ("page_size", C.c_int), ("num_pages", C.c_int),
+        ("kv_layout", C.c_int),
+        ("k_new", C.c_void_p), ("v_new", C.c_void_p), ("k_pages", C.c_void_p),
+        ("v_pages", C.c_void_p), ("suffix_block_table", C.c_void_p),
+        ("suffix_bt_offsets", C.c_void_p), ("suffix_lens", C.c_void_p),
+        ("free_pages", C.c_void_p), ("num_free", C.c_int), ("status", C.c_void_p),
+    ]
 
 
 class HostLens(C.Structure):
@@ -99,6 +112,8 @@ def load() -> C.CDLL:
     lib.specgen_fork_attn_plan.argtypes = [P(ForkAttnArgs), P(HostLens), P(Plan), C.c_void_p]
     lib.specgen_fork_attn_run.restype = C.c_int
     lib.specgen_fork_attn_run.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
+    lib.specgen_append_kv.restype = C.c_int
+    lib.specgen_append_kv.argtypes = [P(AppendArgs), C.c_void_p]
     for stage in ("specgen_fork_attn_run_partials", "specgen_fork_attn_run_merge"):
         getattr(lib, stage).restype = C.c_int
         getattr(lib, stage).argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
@@ -131,9 +146,11 @@ def _check(status: int, what: str):
 
 
 def _ptr(t) -> int | None:
-    """Data pointer of a torch tensor / numpy array, or None."""
+    """Data pointer of a torch tensor / numpy array (or a raw address), or None."""
     if t is None:
         return None
+    if isinstance(t, int):
+        return t
     if isinstance(t, np.ndarray):
         return t.ctypes.data
     return t.data_ptr()
@@ -157,6 +174,21 @@ def make_args(*, num_traces, total_forks, hq, hkv, head_dim_qk, head_dim_v, page
         _ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(prefix_block_table),
         _ptr(prefix_bt_offsets), _ptr(suffix_block_table), _ptr(suffix_bt_offsets),
         _ptr(out), _ptr(lse), _ptr(workspace), int(workspace_bytes), int(kv_layout))
+
+
+def make_append_args(*, total_forks, hkv, head_dim_qk, head_dim_v, page_size, num_pages,
+                     k_new, v_new, k_pages, v_pages, suffix_block_table, suffix_bt_offsets,
+                     suffix_lens, free_pages, num_free, status=None,
+                     kv_layout=KV_ROWS) -> AppendArgs:
+    return AppendArgs(
+        int(total_forks), int(hkv), int(head_dim_qk), int(head_dim_v), int(page_size),
+        int(num_pages), int(kv_layout), _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages),
+        _ptr(suffix_block_table), _ptr(suffix_bt_offsets), _ptr(suffix_lens), _ptr(free_pages),
+        int(num_free), _ptr(status))
+
+
+def specgen_append_kv(args: AppendArgs, stream: int = 0) -> None:
+    _check(load().specgen_append_kv(C.byref(args), C.c_void_p(stream)), "specgen_append_kv")
 
 
 def specgen_fork_attn_workspace_size(args: ForkAttnArgs, lens: HostLens) -> int:

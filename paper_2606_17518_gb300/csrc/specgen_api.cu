@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "../../include/specgen.h"
+#include "append_kv.h"
 #include "lse_merge.h"
 #include "plan.h"
 #include "fork_tc.h"
@@ -734,6 +735,49 @@ specgen_status specgen_fork_attn_decode(const specgen_fork_attn_args* args,
   specgen_status st = specgen_fork_attn_plan(args, lens, &plan, cuda_stream);
   if (st != SPECGEN_OK) return st;
   return specgen_fork_attn_run(args, &plan, cuda_stream);
+}
+
+specgen_status specgen_append_kv(const specgen_append_args* a, void* cuda_stream) {
+  if (!a) return SPECGEN_ERR_NULL;
+  if (a->total_forks < 0 || a->hkv < 1 || a->page_size < 1 || a->num_pages < 0 || a->num_free < 0)
+    return SPECGEN_ERR_SHAPE;
+  if (a->head_dim_qk < 8 || a->head_dim_qk % 8 != 0) return SPECGEN_ERR_UNSUPPORTED;
+  const bool latent = a->v_pages == nullptr;
+  if (latent != (a->v_new == nullptr)) return SPECGEN_ERR_SHAPE;
+  if (!latent && (a->head_dim_v < 8 || a->head_dim_v % 8 != 0)) return SPECGEN_ERR_UNSUPPORTED;
+  if (a->page_size > 1024 || (a->page_size & (a->page_size - 1)) != 0)
+    return SPECGEN_ERR_UNSUPPORTED;
+  if (a->kv_layout != SPECGEN_KV_ROWS && a->kv_layout != SPECGEN_KV_TILED) return SPECGEN_ERR_SHAPE;
+  if (a->kv_layout == SPECGEN_KV_TILED && (latent || a->page_size % 8 != 0))
+    return SPECGEN_ERR_UNSUPPORTED;
+  if (a->total_forks == 0) return SPECGEN_OK;
+  if (!a->k_new || !a->k_pages || !a->suffix_block_table || !a->suffix_bt_offsets ||
+      !a->suffix_lens || (a->num_free > 0 && !a->free_pages))
+    return SPECGEN_ERR_NULL;
+  const void* rows[4] = {a->k_new, a->v_new, a->k_pages, a->v_pages};
+  for (const void* r : rows)
+    if (reinterpret_cast<uintptr_t>(r) % 16 != 0) return SPECGEN_ERR_SHAPE;
+  AppendParams p;
+  p.k_new = static_cast<const __nv_bfloat16*>(a->k_new);
+  p.v_new = static_cast<const __nv_bfloat16*>(a->v_new);
+  p.k_pages = static_cast<__nv_bfloat16*>(a->k_pages);
+  p.v_pages = static_cast<__nv_bfloat16*>(a->v_pages);
+  p.table = a->suffix_block_table;
+  p.offs = a->suffix_bt_offsets;
+  p.lens = a->suffix_lens;
+  p.free_pages = a->free_pages;
+  p.status = a->status;
+  p.F = a->total_forks;
+  p.hkv = a->hkv;
+  p.dqk = a->head_dim_qk;
+  p.dv = latent ? 0 : a->head_dim_v;
+  p.B = a->page_size;
+  p.num_pages = a->num_pages;
+  p.num_free = a->num_free;
+  p.tiled = a->kv_layout == SPECGEN_KV_TILED;
+  if (launch_append_kv(p, static_cast<cudaStream_t>(cuda_stream)) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
 }
 
 specgen_status specgen_lse_merge(const void* out_a, const float* lse_a, const void* out_b,

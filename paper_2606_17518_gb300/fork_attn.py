@@ -3,7 +3,8 @@
 ``ForkDecode`` owns the device copies of one workload (PyTorch is used only
 to allocate device memory and provide streams), builds the C-ABI argument
 structs and calls ``specgen_fork_attn_plan`` / ``specgen_fork_attn_run`` /
-``specgen_fork_attn_decode``.  It does no arithmetic of its own.
+``specgen_fork_attn_decode`` and, for multi-step decode, ``specgen_append_kv``.
+It does no arithmetic of its own.
 """
 
 from __future__ import annotations
@@ -33,7 +34,7 @@ class ForkDecode:
                  kv_layout: int = _lib.KV_ROWS):
         import torch
         from . import workloads
-        self.w = w
+        self.w = dict(w)  # lengths change under multi-step decode; the caller's dict does not
         self.device = torch.device(device)
         self.latent = w["v_pages"] is None
         self.kv_layout = kv_layout
@@ -45,17 +46,46 @@ class ForkDecode:
         self.prefix_off = _i32(w["prefix_bt_offsets"], device)
         self.suffix_table = _i32(w["suffix_table"], device)
         self.suffix_off = _i32(w["suffix_bt_offsets"], device)
+        self.suffix_lens_dev = _i32(w["suffix_lens"], device)  # read by specgen_append_kv
         F, hq, dv = w["total_forks"], w["hq"], w["dv"]
         self.out = torch.empty((F, hq, dv), dtype=torch.bfloat16, device=device)
         self.lse = torch.empty((F, hq), dtype=torch.float32, device=device)
+        self.workspace = None
+        self.ws_bytes = 0
+        self.set_suffix_lens(w["suffix_lens"])
+
+    def set_suffix_lens(self, suffix_lens):
+        """Host suffix lengths for the next plan (the device copy is updated too);
+        the workspace grows if the new lengths need more."""
+        import torch
+        w = self.w
+        w["suffix_lens"] = np.ascontiguousarray(suffix_lens, dtype=np.int32)
         self.lens, self._lens_keep = _lib.make_host_lens(
             w["prefix_lens"], w["fork_offsets"], w["suffix_lens"], w["prefix_bt_offsets"],
             w["suffix_bt_offsets"])
-        self.ws_bytes = _lib.specgen_fork_attn_workspace_size(self.args(with_ws=False), self.lens)
-        if self.ws_bytes == 0:
+        need = _lib.specgen_fork_attn_workspace_size(self.args(with_ws=False), self.lens)
+        if need == 0:
             raise _lib.SpecgenError(_lib.SPECGEN_ERR_SHAPE, "specgen_fork_attn_workspace_size")
-        self.workspace = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        if need > self.ws_bytes:
+            self.ws_bytes = need
+            self.workspace = torch.zeros(need, dtype=torch.uint8, device=self.device)
+        if self.suffix_lens_dev is not None and w["total_forks"] > 0:
+            self.suffix_lens_dev.copy_(torch.from_numpy(w["suffix_lens"]))
         self.plan_info = None
+
+    def append_kv(self, k_new, v_new, free_pages, num_free: int, stream: int = 0):
+        """One decode step's K/V rows (device bf16 [F][Hkv][D]) into the suffixes,
+        taking pages from ``free_pages`` (device int32); status bits go to the
+        workspace status word.  The caller then advances the lengths."""
+        w = self.w
+        args = _lib.make_append_args(
+            total_forks=w["total_forks"], hkv=w["hkv"], head_dim_qk=w["dqk"],
+            head_dim_v=w["dv"], page_size=w["page_size"], num_pages=w["num_pages"],
+            k_new=k_new, v_new=v_new, k_pages=self.k_pages, v_pages=self.v_pages,
+            suffix_block_table=self.suffix_table, suffix_bt_offsets=self.suffix_off,
+            suffix_lens=self.suffix_lens_dev, free_pages=free_pages, num_free=num_free,
+            status=self.workspace, kv_layout=self.kv_layout)
+        _lib.specgen_append_kv(args, stream)
 
     def args(self, with_ws: bool = True, **override) -> _lib.ForkAttnArgs:
         w = self.w

@@ -198,3 +198,25 @@ def test_product_path_has_no_oracle_import():
                 src = open(os.path.join(dirpath, fn)).read()
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", src, re.M), fn
                 assert "oracle/" not in src, fn
+
+
+def test_append_host_checks():
+    S = _lib
+    lib = _lib.load()
+    fake = 0x10000
+    base = dict(total_forks=4, hkv=2, head_dim_qk=64, head_dim_v=64, page_size=16, num_pages=10,
+                k_new=fake, v_new=fake, k_pages=fake, v_pages=fake, suffix_block_table=fake,
+                suffix_bt_offsets=fake, suffix_lens=fake, free_pages=fake, num_free=3)
+    st = lambda **kw: lib.specgen_append_kv(C.byref(_lib.make_append_args(**{**base, **kw})), None)
+    assert lib.specgen_append_kv(None, None) == S.SPECGEN_ERR_NULL
+    assert st(total_forks=0) == S.SPECGEN_OK                    # nothing to do, nothing launched
+    assert st(total_forks=-1) == S.SPECGEN_ERR_SHAPE
+    assert st(hkv=0) == S.SPECGEN_ERR_SHAPE
+    assert st(head_dim_qk=60) == S.SPECGEN_ERR_UNSUPPORTED      # rows move in 16-byte pieces
+    assert st(page_size=12) == S.SPECGEN_ERR_UNSUPPORTED
+    assert st(v_new=None) == S.SPECGEN_ERR_SHAPE                # value rows without a value pool
+    assert st(kv_layout=7) == S.SPECGEN_ERR_SHAPE
+    assert st(kv_layout=S.KV_TILED, v_pages=None, v_new=None) == S.SPECGEN_ERR_UNSUPPORTED
+    assert st(suffix_lens=None) == S.SPECGEN_ERR_NULL
+    assert st(free_pages=None) == S.SPECGEN_ERR_NULL
+    assert st(k_new=fake + 8) == S.SPECGEN_ERR_SHAPE            # not 16-byte aligned
