@@ -44,6 +44,10 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--op", choices=["attend", "decode_step"], default="attend",
+                    help="attend: one fork-decode attention call per step (the headline); "
+                         "decode_step: append one K/V row per fork, then attend over the grown "
+                         "suffixes, planning every step on the host")
     ap.add_argument("--kv-layout", choices=["rows", "tiled"], default="rows",
                     help="K/V pool layout: token-major rows (default) or 8x8 core-matrix tiles "
                          "(tensor-core shapes only)")
@@ -489,11 +493,148 @@ def measure_e2e(w, reps, stream, dev, K, W):
             "d2h_bytes_per_step": bo, "steps": K}
 
 
+def run_decode_steps():
+    """--op decode_step: K serving steps of append + attention with growing suffixes.
+
+    Every step copies the step's Q and new K/V rows from pinned host memory,
+    appends the rows (specgen_append_kv, pages taken from a device free list),
+    plans the attention on the host for the new lengths, runs it, and copies
+    O and LSE back to pinned memory.  The whole loop is timed with CUDA events
+    on the stream; each kernel's share comes from events around its launch.
+    """
+    import torch
+
+    import __graft_entry__
+    from paper_2606_17518_gb300 import _lib, workloads as wl
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+
+    rank, local_rank, world = dist_env()
+    __graft_entry__.build()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    K, W = ARGS.steps, ARGS.warmup
+    w = wl.make_workload(ARGS.workload)
+    st = wl.make_decode_state(w, K + W)
+    layout = ARGS.kv_layout if w["v_pages"] is not None else "rows"
+    fd = ForkDecode(st, device=dev, kv_layout=_lib.KV_TILED if layout == "tiled" else _lib.KV_ROWS)
+    stream = torch.cuda.Stream(dev)
+    sp = stream.cuda_stream
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).pin_memory()
+    h_q = pin(st["q"])
+    h_k = pin(st["k_new"])
+    h_v = None if st["v_new"] is None else pin(st["v_new"])
+    d_k = torch.empty(h_k.shape[1:], dtype=torch.int16, device=dev)
+    d_v = None if h_v is None else torch.empty(h_v.shape[1:], dtype=torch.int16, device=dev)
+    h_o = torch.empty(fd.out.shape, dtype=fd.out.dtype).pin_memory()
+    h_l = torch.empty(fd.lse.shape, dtype=fd.lse.dtype).pin_memory()
+    free = torch.from_numpy(st["free_pages"]).to(dev)
+    n_free = len(st["free_pages"])
+    lens = st["suffix_lens"].astype(np.int32).copy()
+    used = 0
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    marks = [(ev(), ev(), ev()) for _ in range(K)]
+
+    def step(s, m=None):
+        nonlocal lens, used
+        with torch.cuda.stream(stream):
+            fd.q.view(torch.int16).copy_(h_q, non_blocking=True)
+            d_k.copy_(h_k[s], non_blocking=True)
+            if d_v is not None:
+                d_v.copy_(h_v[s], non_blocking=True)
+            if m:
+                m[0].record(stream)
+            fd.append_kv(d_k.view(torch.bfloat16),
+                         None if d_v is None else d_v.view(torch.bfloat16), free[used:],
+                         n_free - used, sp)
+            if m:
+                m[1].record(stream)
+            used += int(np.sum(lens % st["page_size"] == 0))
+            lens = lens + 1
+            fd.suffix_lens_dev.add_(1)
+            fd.set_suffix_lens(lens, update_device=False)
+            fd.plan(sp)
+            fd.run(sp)
+            if m:
+                m[2].record(stream)
+            h_o.copy_(fd.out, non_blocking=True)
+            h_l.copy_(fd.lse, non_blocking=True)
+
+    for s in range(W):
+        step(s)
+    torch.cuda.synchronize(dev)
+    start, end = ev(), ev()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    with torch.cuda.stream(stream):
+        start.record(stream)
+    for i in range(K):
+        step(W + i, marks[i])
+    with torch.cuda.stream(stream):
+        end.record(stream)
+    torch.cuda.synchronize(dev)
+    clk = clocks.stop()
+    status = fd.status(sp)
+    if status != 0:
+        raise RuntimeError(f"workspace status {_lib.status_string(status)}")
+    total_ms = start.elapsed_time(end)
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    F = w["total_forks"]
+    ms_per_step = total_ms / K
+    app_ms = sum(m[0].elapsed_time(m[1]) for m in marks) / K
+    att_ms = sum(m[1].elapsed_time(m[2]) for m in marks) / K
+    w_mid = dict(st, suffix_lens=st["suffix_lens"] + W + K // 2)
+    nbytes = wl.algorithmic_bytes(w_mid)
+    att_bytes = nbytes["prefix"] + nbytes["suffix"] + nbytes["q"]
+    hbm, _, _, peak_src = measured_peaks()
+    achieved = att_bytes / (att_ms * 1e-3) / 1e9
+    attn = "mla_tc" if w["v_pages"] is None else "fork_tc"
+    row_bytes = F * w["hkv"] * (w["dqk"] + (w["dv"] if w["v_pages"] is not None else 0)) * 2
+    line = {
+        "metric": "fork-decode step tokens/s (append + attention, growing suffixes)",
+        "value": world * F / (ms_per_step * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": ARGS.workload, "op": "decode_step", "forks": F,
+                   "suffix_growth": K + W, "kv_layout": layout,
+                   "timing": "host-driven steps (plan every step) between CUDA events; "
+                             "per-kernel times from events around each launch",
+                   "l2": "inputs of one workload (KV stays resident, as in serving)"},
+        "gpu_launches": K * 3,  # append, attention, merge
+        "kernels": {"append_kv": {"ms_per_launch": app_ms,
+                                  "bytes_per_launch": 2 * row_bytes},
+                    attn + "+lse_merge": {"ms_per_launch": att_ms}},
+        "roofline": {"bound": "hbm", "kernel": attn + "+lse_merge", "achieved": achieved,
+                     "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                     "peak_source": peak_src, "algorithmic_bytes_per_launch": att_bytes},
+        "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+        "e2e": {"value": world * F / (ms_per_step * 1e-3), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(h_q.numel() * 2 + row_bytes),
+                "d2h_bytes_per_step": int(h_o.numel() * 2 + h_l.numel() * 4),
+                "note": "the step itself includes the copies"},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def main():
     if os.environ.get("SPECGEN_ORACLE_CHILD"):
         return
     if ARGS.impl == "reference":
         run_reference()
+    elif ARGS.op == "decode_step":
+        run_decode_steps()
     else:
         run_ours()
 

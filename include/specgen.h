@@ -82,6 +82,11 @@ typedef struct {
   void* workspace;              /* >= specgen_fork_attn_workspace_size bytes, 256-B aligned */
   size_t workspace_bytes;
   int kv_layout;                /* SPECGEN_KV_ROWS or SPECGEN_KV_TILED (see below) */
+  const int32_t* suffix_lens;   /* optional device [total_forks]: the suffix lengths to use,
+                                   each <= the host length the plan was made for; NULL =
+                                   the planned lengths.  Lets one plan serve several decode
+                                   steps (plan for the lengths a few steps ahead, advance
+                                   this array on the device after each append). */
 } specgen_fork_attn_args;
 
 /* Layout of one (page, kv head) block of page_size x head_dim values in the

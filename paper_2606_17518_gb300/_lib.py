@@ -52,6 +52,7 @@ class ForkAttnArgs(C.Structure):
         ("suffix_block_table", C.c_void_p), ("suffix_bt_offsets", C.c_void_p),
         ("out", C.c_void_p), ("lse", C.c_void_p),
         ("workspace", C.c_void_p), ("workspace_bytes", C.c_size_t), ("kv_layout", C.c_int),
+        ("suffix_lens", C.c_void_p),
     ]
 
 
@@ -167,13 +168,14 @@ def make_host_lens(prefix_lens, fork_offsets, suffix_lens, prefix_bt_offsets=Non
 def make_args(*, num_traces, total_forks, hq, hkv, head_dim_qk, head_dim_v, page_size,
               num_pages, scale, q, k_pages, v_pages, prefix_block_table, prefix_bt_offsets,
               suffix_block_table, suffix_bt_offsets, out, lse, workspace=None,
-              workspace_bytes=0, kv_layout=KV_ROWS) -> ForkAttnArgs:
+              workspace_bytes=0, kv_layout=KV_ROWS, suffix_lens=None) -> ForkAttnArgs:
     return ForkAttnArgs(
         int(num_traces), int(total_forks), int(hq), int(hkv), int(head_dim_qk),
         int(head_dim_v), int(page_size), int(num_pages), float(scale),
         _ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(prefix_block_table),
         _ptr(prefix_bt_offsets), _ptr(suffix_block_table), _ptr(suffix_bt_offsets),
-        _ptr(out), _ptr(lse), _ptr(workspace), int(workspace_bytes), int(kv_layout))
+        _ptr(out), _ptr(lse), _ptr(workspace), int(workspace_bytes), int(kv_layout),
+        _ptr(suffix_lens))
 
 
 def make_append_args(*, total_forks, hkv, head_dim_qk, head_dim_v, page_size, num_pages,

@@ -106,10 +106,11 @@ __device__ __forceinline__ int tile_tokens(const TcItem& it, int j) {
   return n < TT ? n : TT;
 }
 
-// Item k of this CTA: the first kItemCache come from shared memory.
+// Item k of this CTA: the first kItemCache come from shared memory (already
+// cut to the current suffix lengths), the rest are read and cut here.
 __device__ __forceinline__ TcItem get_item(const TcItem* cache, const TcParams& p, int it_begin,
                                            int k) {
-  return k < kItemCache ? cache[k] : p.items[it_begin + k];
+  return k < kItemCache ? cache[k] : clamp_item(p.items[it_begin + k], p.suffix_lens);
 }
 
 // Page ids pb + lane of an item (lane-strided batch of 32); 0 past the item.
@@ -174,6 +175,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int32_t* src = reinterpret_cast<const int32_t*>(p.items + it_begin);
     int32_t* dst = reinterpret_cast<int32_t*>(items);
     for (int x = lane; x < nw; x += 32) dst[x] = src[x];
+    __syncwarp();
+    for (int k = lane; k < nw / kWords; k += 32) items[k] = clamp_item(items[k], p.suffix_lens);
   }
   if (threadIdx.x == 32) {
     for (int i = 0; i < ST; ++i) {
@@ -318,9 +321,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool q_ok = false;
       bool ok = true;
       unsigned long long t0 = 0;
-      while (ok && v_k < n_items) {
+      // items cut to nothing by the current suffix lengths have no tiles: the
+      // PV cursor steps over them, the S cursor still takes their Q phase and
+      // releases the Q buffer (q_free) so the item sequence stays in step
+      while (v_k < n_items && v_nt == 0 && ++v_k < n_items) {
+        v_it = get_item(items, p, it_begin, v_k);
+        v_nt = view<TT>(p, v_it).ntiles;
+      }
+      while (ok && (v_k < n_items || s_k < n_items)) {
         bool did = false;
-        if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
+        if (s_k < n_items && s_nt == 0 && mbar_test_wait(q_ready, s_k & 1)) {
+          mma_commit(q_free);  // an empty item: its Q phase taken, the buffer released
+          q_ok = false;
+          if (++s_k < n_items) {
+            s_it = get_item(items, p, it_begin, s_k);
+            s_nt = view<TT>(p, s_it).ntiles;
+          }
+          did = true;
+        } else if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
           tc_fence_after();
           const int b = v_u & 1, s = v_u % ST;
           const int np = (tile_tokens<TT>(v_it, v_j) + kPB - 1) / kPB;
@@ -343,13 +361,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++v_u;
           if (++v_j == v_nt) {
             v_j = 0;
-            if (++v_k < n_items) {
-              v_it = get_item(items, p, it_begin, v_k);
-              v_nt = view<TT>(p, v_it).ntiles;
-            }
+            do {
+              if (++v_k < n_items) {
+                v_it = get_item(items, p, it_begin, v_k);
+                v_nt = view<TT>(p, v_it).ntiles;
+              }
+            } while (v_k < n_items && v_nt == 0);
           }
           did = true;
-        } else if (s_k < n_items && s_u - v_u < 2) {
+        } else if (s_k < n_items && s_nt > 0 && s_u - v_u < 2) {
           if (!q_ok && mbar_test_wait(q_ready, s_k & 1)) q_ok = true;
           if (q_ok && mbar_test_wait(full(s_u % ST), (s_u / ST) & 1)) {
             tc_fence_after();

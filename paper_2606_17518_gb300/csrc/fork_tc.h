@@ -22,6 +22,7 @@ struct TcParams {
   float* part_o;               // head-interleaved partials (part_o_f4)
   float* part_lse;             // [slots][hq]
   uint32_t* status;
+  const int32_t* suffix_lens;  // device lengths that clamp suffix items, or nullptr
   int hq, hkv, G, dv, num_pages;
   float scale_log2;            // softmax scale * log2(e), > 0
 };

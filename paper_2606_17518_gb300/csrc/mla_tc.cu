@@ -126,11 +126,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     int t = 0;
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[ii];
+      const TcItem it = clamp_item(p.items[ii], p.suffix_lens);
       const int32_t* table = table_of(it);
       const int ntiles = ntiles_of(it);
       const int page0 = it.tok_begin / kPage;
-      const int npages = (it.tok_end - 1) / kPage - page0 + 1;
+      const int npages = ntiles;  // one page per tile
       int cur = lane < npages ? table[page0 + lane] : 0;
       int nxt = 32 + lane < npages ? table[page0 + 32 + lane] : 0;
       int batch = 0;
@@ -175,14 +175,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       // first tile, its Q is in shared memory.  s_*: the next S to issue,
       // v_*: the next PV to issue (item cursor, tile within item, global tile).
       int s_ii = it_begin, s_j = 0, s_u = 0, v_ii = it_begin, v_j = 0, v_u = 0;
-      TcItem s_it = s_ii < it_end ? p.items[s_ii] : TcItem{};
+      TcItem s_it = s_ii < it_end ? clamp_item(p.items[s_ii], p.suffix_lens) : TcItem{};
       TcItem v_it = s_it;
       bool q_ok = false;  // Q of the item at s_ii is known to be loaded
       bool ok = true;
       unsigned long long t0 = 0;
-      while (ok && v_ii < it_end) {
+      // items cut to nothing by the current suffix lengths: the PV cursor steps
+      // over them, the S cursor still takes their Q phase
+      while (v_ii < it_end && ntiles_of(v_it) == 0 && ++v_ii < it_end)
+        v_it = clamp_item(p.items[v_ii], p.suffix_lens);
+      while (ok && (v_ii < it_end || s_ii < it_end)) {
         bool did = false;
-        if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
+        if (s_ii < it_end && ntiles_of(s_it) == 0 &&
+            mbar_test_wait(q_ready, (s_ii - it_begin) & 1)) {
+          q_ok = false;
+          if (++s_ii < it_end) s_it = clamp_item(p.items[s_ii], p.suffix_lens);
+          did = true;
+        } else if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
           tc_fence_after();
           const int b = v_u & 1, s = v_u % kST;
           const uint64_t vpanel = (uint64_t)((v_it.dv0 / 64) * kKPanel) >> 4;
@@ -197,10 +206,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++v_u;
           if (++v_j == ntiles_of(v_it)) {
             v_j = 0;
-            if (++v_ii < it_end) v_it = p.items[v_ii];
+            do {
+              if (++v_ii < it_end) v_it = clamp_item(p.items[v_ii], p.suffix_lens);
+            } while (v_ii < it_end && ntiles_of(v_it) == 0);
           }
           did = true;
-        } else if (s_ii < it_end && s_u - v_u < 2) {
+        } else if (s_ii < it_end && ntiles_of(s_it) > 0 && s_u - v_u < 2) {
           if (!q_ok && mbar_test_wait(q_ready, (s_ii - it_begin) & 1)) q_ok = true;
           if (q_ok && mbar_test_wait(full(s_u % kST), (s_u / kST) & 1)) {
             tc_fence_after();
@@ -223,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (++s_j == ntiles_of(s_it)) {
               s_j = 0;
               q_ok = false;
-              if (++s_ii < it_end) s_it = p.items[s_ii];
+              if (++s_ii < it_end) s_it = clamp_item(p.items[s_ii], p.suffix_lens);
             }
             did = true;
           }
@@ -255,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int t = 0, oc = 0;  // tiles done; next o_full phase (tile index) to consume
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
-      const TcItem it = p.items[ii];
+      const TcItem it = clamp_item(p.items[ii], p.suffix_lens);
       // this fork's partial slot base, fetched now and used at the item's end
       const int pbase = p.part_base[it.fork0];
       const int32_t* table = table_of(it);

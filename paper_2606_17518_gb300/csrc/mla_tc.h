@@ -20,6 +20,7 @@ struct MlaParams {
   float* part_o;               // head-interleaved partials (part_o_f4), hq = 128, dv = 512
   float* part_lse;             // [slots][128]
   uint32_t* status;
+  const int32_t* suffix_lens;  // device lengths that clamp suffix items, or nullptr
   int hq, num_pages;
   float scale_log2;
 };

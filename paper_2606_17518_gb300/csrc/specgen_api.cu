@@ -651,6 +651,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   sp.page_size = args->page_size;
   sp.num_pages = args->num_pages;
   sp.scale_log2 = args->scale * 1.4426950408889634f;
+  sp.suffix_lens = args->suffix_lens;
   if (!marks.mark(stream, 0)) return SPECGEN_ERR_CUDA;
   if ((stages & 1) && plan->n_tc_ctas > 0) {
     TcParams tp;
@@ -671,6 +672,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     tp.dv = args->head_dim_v;
     tp.num_pages = args->num_pages;
     tp.scale_log2 = sp.scale_log2;
+    tp.suffix_lens = args->suffix_lens;
     cudaError_t e;
     if (args->v_pages == nullptr) {
       MlaParams mp;
@@ -688,6 +690,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
       mp.hq = args->hq;
       mp.num_pages = args->num_pages;
       mp.scale_log2 = tp.scale_log2;
+      mp.suffix_lens = args->suffix_lens;
       e = launch_mla_tc(mp, args->k_pages, plan->n_tc_ctas, stream);
     } else {
       tp.k_pages = static_cast<const __nv_bfloat16*>(args->k_pages);

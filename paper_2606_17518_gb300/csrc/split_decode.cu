@@ -61,7 +61,11 @@ __global__ void __launch_bounds__(kThreads, 2) split_decode_kernel(const SplitPa
   unsigned char* s_q = smem + STAGES * S::kStage;              // kQ
   uint8_t* s_ok = reinterpret_cast<uint8_t*>(s_q + S::kQ);     // STAGES * kTile
 
-  const SplitItem it = p.items[blockIdx.x];
+  SplitItem it = p.items[blockIdx.x];
+  if (p.suffix_lens != nullptr && it.table_kind == 1) {  // one plan, several decode steps
+    const int n = p.suffix_lens[it.seq];
+    it.tok_end = n < it.tok_begin ? it.tok_begin : (n < it.tok_end ? n : it.tok_end);
+  }
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int B = p.page_size;
   const int32_t* table = it.table_kind == 0 ? p.prefix_bt + p.prefix_bt_off[it.seq]

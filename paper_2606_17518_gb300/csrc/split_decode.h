@@ -20,6 +20,7 @@ struct SplitParams {
   float* part_o;    // head-interleaved partials (part_o_f4)
   float* part_lse;  // [slots][hq]
   uint32_t* status;
+  const int32_t* suffix_lens;  // device lengths that clamp suffix items, or nullptr
   int hq, hkv, dqk, dv, page_size, num_pages;
   float scale_log2;  // softmax scale * log2(e)
 };

@@ -115,6 +115,17 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
       : "memory");
 }
 
+// A suffix item's token range cut to its fork's current suffix length when a
+// device length array is given (one plan serving several decode steps); the
+// range may become empty.
+__device__ __forceinline__ TcItem clamp_item(TcItem it, const int32_t* suffix_lens) {
+  if (suffix_lens != nullptr && it.table_kind == 1) {
+    const int n = suffix_lens[it.seq];
+    it.tok_end = n < it.tok_begin ? it.tok_begin : (n < it.tok_end ? n : it.tok_end);
+  }
+  return it;
+}
+
 // ---------------------------------------------------------------- tcgen05
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(

@@ -52,11 +52,15 @@ class ForkDecode:
         self.lse = torch.empty((F, hq), dtype=torch.float32, device=device)
         self.workspace = None
         self.ws_bytes = 0
+        # when True the kernels cut suffix items to suffix_lens_dev (a plan made
+        # for longer host lengths then serves several decode steps)
+        self.use_device_lens = False
         self.set_suffix_lens(w["suffix_lens"])
 
-    def set_suffix_lens(self, suffix_lens):
-        """Host suffix lengths for the next plan (the device copy is updated too);
-        the workspace grows if the new lengths need more."""
+    def set_suffix_lens(self, suffix_lens, update_device: bool = True):
+        """Host suffix lengths for the next plan (the device copy is updated too,
+        unless the caller advanced it on the device itself); the workspace grows
+        if the new lengths need more."""
         import torch
         w = self.w
         w["suffix_lens"] = np.ascontiguousarray(suffix_lens, dtype=np.int32)
@@ -69,7 +73,7 @@ class ForkDecode:
         if need > self.ws_bytes:
             self.ws_bytes = need
             self.workspace = torch.zeros(need, dtype=torch.uint8, device=self.device)
-        if self.suffix_lens_dev is not None and w["total_forks"] > 0:
+        if update_device and self.suffix_lens_dev is not None and w["total_forks"] > 0:
             self.suffix_lens_dev.copy_(torch.from_numpy(w["suffix_lens"]))
         self.plan_info = None
 
@@ -97,7 +101,8 @@ class ForkDecode:
             prefix_bt_offsets=self.prefix_off, suffix_block_table=self.suffix_table,
             suffix_bt_offsets=self.suffix_off, out=self.out, lse=self.lse,
             workspace=self.workspace if with_ws else None,
-            workspace_bytes=self.ws_bytes if with_ws else 0, kv_layout=self.kv_layout)
+            workspace_bytes=self.ws_bytes if with_ws else 0, kv_layout=self.kv_layout,
+            suffix_lens=self.suffix_lens_dev if self.use_device_lens else None)
         kw.update(override)
         return _lib.make_args(**kw)
 

@@ -122,3 +122,98 @@ def test_append_reports_exhausted_free_list_and_full_table():
     fd2.set_suffix_lens(np.full(4, 32, np.int32))   # exactly 2 pages each: no room for a third
     fd2.append_kv(k_new, v_new, free, 4)
     assert fd2.status() == _lib.SPECGEN_ERR_INDEX
+
+
+def _fuzz_page64(seed):
+    return wl.WorkloadSpec(name="split64", num_traces=2, prefix_len=(100, 300), forks=(2, 3),
+                           suffix_len=(1, 70), hq=8, hkv=2, dqk=128, dv=128, page_size=64,
+                           seed=seed)
+
+
+@pytest.mark.parametrize("name", ["tiny_p512_f4", "fork_p8k_f8", "mla_p16k_f8", "split64"])
+@pytest.mark.parametrize("ahead", [0, 7, 40])
+def test_plan_ahead_cut_to_device_lengths(name, ahead):
+    """A plan made for suffixes `ahead` tokens longer, run with the actual
+    lengths in the device array: the oracle's result at the actual lengths.
+    Slots past the actual lengths hold NaN, so any read there would show; with
+    ahead = 40 whole suffix items are cut to nothing."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    base = wl.make_workload(_fuzz_page64(3) if name == "split64" else name)
+    st = wl.make_decode_state(base, ahead)
+    fd = ForkDecode(st)
+    fd.use_device_lens = True
+    lens = st["suffix_lens"].copy()
+    fd.set_suffix_lens(lens + ahead, update_device=False)   # plan for the longer lengths
+    fd.suffix_lens_dev.copy_(torch.from_numpy(lens))         # run with the actual ones
+    fd.decode()
+    o, lse = fd.results()
+    assert fd.status() == _lib.SPECGEN_OK
+    o_ref, lse_ref = oracle.fork_attn_decode(dict(st, suffix_lens=lens))
+    assert np.all(np.isfinite(o))
+    assert float(np.max(np.abs(o - o_ref))) <= TOL_O
+    fin = np.isfinite(lse_ref)
+    assert np.array_equal(np.isfinite(lse), fin)
+    assert float(np.max(np.abs(lse[fin] - lse_ref[fin]))) <= TOL_LSE
+
+
+@pytest.mark.parametrize("name", ["fork_p8k_f8", "mla_p16k_f8"])
+def test_one_plan_many_decode_steps_in_a_graph(name):
+    """One plan for 12 steps ahead; 12 steps of (append, advance the device
+    lengths, attention) captured in one CUDA graph; the last step's output and
+    the pools match the oracle."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    steps = 12
+    st = wl.make_decode_state(wl.make_workload(name), steps)
+    fd = ForkDecode(st)
+    fd.use_device_lens = True
+    lens0 = st["suffix_lens"].copy()
+    fd.set_suffix_lens(lens0 + steps, update_device=False)
+    fd.suffix_lens_dev.copy_(torch.from_numpy(lens0))
+    stream = torch.cuda.Stream()
+    sp = stream.cuda_stream
+    fd.plan(sp)
+    torch.cuda.synchronize()
+    free = torch.from_numpy(st["free_pages"]).cuda()
+    k_new = torch.from_numpy(st["k_new"].view(np.int16)).cuda().view(torch.bfloat16)
+    v_new = (None if st["v_new"] is None else
+             torch.from_numpy(st["v_new"].view(np.int16)).cuda().view(torch.bfloat16))
+    # pages each step takes: known on the host from the lengths
+    offs, lens = [], lens0.copy()
+    used = 0
+    for s in range(steps):
+        offs.append(used)
+        used += int(np.sum(lens % st["page_size"] == 0))
+        lens = lens + 1
+    fd.run(sp)                      # first launches configure the kernels outside the capture
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for s in range(steps):
+            fd.append_kv(k_new[s], None if v_new is None else v_new[s], free[offs[s]:],
+                         len(st["free_pages"]) - offs[s], sp)
+            fd.suffix_lens_dev.add_(1)
+            fd.run(sp)
+    graph.replay()
+    torch.cuda.synchronize()
+    o, lse = fd.results()
+    assert fd.status() == _lib.SPECGEN_OK
+    ref_k, ref_v, ref_t, lens = st["k_pages"], st["v_pages"], st["suffix_table"], lens0.copy()
+    used = 0
+    for s in range(steps):
+        ref_k, ref_v, ref_t, taken = oracle.append_kv(
+            ref_k, ref_v, ref_t, st["suffix_bt_offsets"], lens, st["k_new"][s],
+            None if st["v_new"] is None else st["v_new"][s], st["free_pages"][used:],
+            st["page_size"])
+        used += taken
+        lens = lens + 1
+    k, v, t = _pools(fd, st)
+    assert np.array_equal(t, ref_t) and np.array_equal(k, ref_k)
+    if ref_v is not None:
+        assert np.array_equal(v, ref_v)
+    o_ref, lse_ref = oracle.fork_attn_decode(
+        dict(st, k_pages=ref_k, v_pages=ref_v, suffix_table=ref_t, suffix_lens=lens))
+    assert float(np.max(np.abs(o - o_ref))) <= TOL_O
+    fin = np.isfinite(lse_ref)
+    assert float(np.max(np.abs(lse[fin] - lse_ref[fin]))) <= TOL_LSE
