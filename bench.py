@@ -496,12 +496,18 @@ def measure_e2e(w, reps, stream, dev, K, W):
 def run_decode_steps():
     """--op decode_step: K serving steps of append + attention with growing suffixes.
 
-    Every step copies the step's Q and new K/V rows from pinned host memory,
-    appends the rows (specgen_append_kv, pages taken from a device free list),
-    plans the attention on the host for the new lengths, runs it, and copies
-    O and LSE back to pinned memory.  The whole loop is timed with CUDA events
-    on the stream; each kernel's share comes from events around its launch.
+    One plan is made for the lengths after the last step; the kernels cut the
+    suffix items to the current lengths in a device array, which every step
+    advances after its append.  Each step (copy of the step's Q and new K/V
+    rows from pinned host memory, specgen_append_kv with pages from a device
+    free list, length advance, attention, copy of O and LSE back to pinned
+    memory) is captured in CUDA graphs of 16 steps; the K timed steps replay
+    them between CUDA events on the stream.  Per-kernel times: graphs of the
+    attention stages alone at the final lengths, and a graph of appends into a
+    second copy of the state.
     """
+    import ctypes as C
+
     import torch
 
     import __graft_entry__
@@ -517,13 +523,36 @@ def run_decode_steps():
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    K, W = ARGS.steps, ARGS.warmup
+    per_graph = 16
+    K = ARGS.steps
+    W = -(-max(3, ARGS.warmup) // per_graph) * per_graph  # whole graphs of warm-up steps
+    n = K + W
     w = wl.make_workload(ARGS.workload)
-    st = wl.make_decode_state(w, K + W)
     layout = ARGS.kv_layout if w["v_pages"] is not None else "rows"
-    fd = ForkDecode(st, device=dev, kv_layout=_lib.KV_TILED if layout == "tiled" else _lib.KV_ROWS)
+    kvl = _lib.KV_TILED if layout == "tiled" else _lib.KV_ROWS
     stream = torch.cuda.Stream(dev)
     sp = stream.cuda_stream
+    B = w["page_size"]
+
+    def prepare(steps):
+        st = wl.make_decode_state(w, steps)
+        fd = ForkDecode(st, device=dev, kv_layout=kvl)
+        fd.use_device_lens = True
+        lens0 = st["suffix_lens"].astype(np.int32).copy()
+        fd.set_suffix_lens(lens0 + steps, update_device=False)
+        fd.suffix_lens_dev.copy_(torch.from_numpy(lens0))
+        with torch.cuda.stream(stream):
+            fd.plan(sp)
+        offs, lens, used = [], lens0.copy(), 0
+        for _ in range(steps):
+            offs.append(used)
+            used += int(np.sum(lens % B == 0))
+            lens = lens + 1
+        free = torch.from_numpy(st["free_pages"]).to(dev)
+        return st, fd, offs, free
+
+    st, fd, offs, free = prepare(n)
+    n_free = len(st["free_pages"])
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).pin_memory()
     h_q = pin(st["q"])
     h_k = pin(st["k_new"])
@@ -532,49 +561,42 @@ def run_decode_steps():
     d_v = None if h_v is None else torch.empty(h_v.shape[1:], dtype=torch.int16, device=dev)
     h_o = torch.empty(fd.out.shape, dtype=fd.out.dtype).pin_memory()
     h_l = torch.empty(fd.lse.shape, dtype=fd.lse.dtype).pin_memory()
-    free = torch.from_numpy(st["free_pages"]).to(dev)
-    n_free = len(st["free_pages"])
-    lens = st["suffix_lens"].astype(np.int32).copy()
-    used = 0
-    ev = lambda: torch.cuda.Event(enable_timing=True)
-    marks = [(ev(), ev(), ev()) for _ in range(K)]
-
-    def step(s, m=None):
-        nonlocal lens, used
-        with torch.cuda.stream(stream):
-            fd.q.view(torch.int16).copy_(h_q, non_blocking=True)
-            d_k.copy_(h_k[s], non_blocking=True)
-            if d_v is not None:
-                d_v.copy_(h_v[s], non_blocking=True)
-            if m:
-                m[0].record(stream)
-            fd.append_kv(d_k.view(torch.bfloat16),
-                         None if d_v is None else d_v.view(torch.bfloat16), free[used:],
-                         n_free - used, sp)
-            if m:
-                m[1].record(stream)
-            used += int(np.sum(lens % st["page_size"] == 0))
-            lens = lens + 1
-            fd.suffix_lens_dev.add_(1)
-            fd.set_suffix_lens(lens, update_device=False)
-            fd.plan(sp)
-            fd.run(sp)
-            if m:
-                m[2].record(stream)
-            h_o.copy_(fd.out, non_blocking=True)
-            h_l.copy_(fd.lse, non_blocking=True)
-
-    for s in range(W):
-        step(s)
+    with torch.cuda.stream(stream):
+        fd.run(sp)  # first launches configure the kernels outside any capture
     torch.cuda.synchronize(dev)
+
+    def step(s):
+        fd.q.view(torch.int16).copy_(h_q, non_blocking=True)
+        d_k.copy_(h_k[s], non_blocking=True)
+        if d_v is not None:
+            d_v.copy_(h_v[s], non_blocking=True)
+        fd.append_kv(d_k.view(torch.bfloat16), None if d_v is None else d_v.view(torch.bfloat16),
+                     free[offs[s]:], n_free - offs[s], sp)
+        fd.suffix_lens_dev.add_(1)
+        fd.run(sp)
+        h_o.copy_(fd.out, non_blocking=True)
+        h_l.copy_(fd.lse, non_blocking=True)
+
+    graphs = []
+    for g0 in range(0, n, per_graph):
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for s in range(g0, min(n, g0 + per_graph)):
+                step(s)
+        graphs.append((g0, graph))
+    warm = [g for g in graphs if g[0] < W]
+    timed = [g for g in graphs if g[0] >= W]
+    for _, g in warm:
+        g.replay()
+    torch.cuda.synchronize(dev)
+    ev = lambda: torch.cuda.Event(enable_timing=True)
     start, end = ev(), ev()
     clocks = ClockSampler(local_rank)
     clocks.start()
     with torch.cuda.stream(stream):
         start.record(stream)
-    for i in range(K):
-        step(W + i, marks[i])
-    with torch.cuda.stream(stream):
+        for _, g in timed:
+            g.replay()
         end.record(stream)
     torch.cuda.synchronize(dev)
     clk = clocks.stop()
@@ -589,37 +611,75 @@ def run_decode_steps():
         total_ms = float(t.item())
     F = w["total_forks"]
     ms_per_step = total_ms / K
-    app_ms = sum(m[0].elapsed_time(m[1]) for m in marks) / K
-    att_ms = sum(m[1].elapsed_time(m[2]) for m in marks) / K
-    w_mid = dict(st, suffix_lens=st["suffix_lens"] + W + K // 2)
-    nbytes = wl.algorithmic_bytes(w_mid)
+
+    def graph_ms(fn, reps=16):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(reps):
+                fn(i)
+        g.replay()
+        torch.cuda.synchronize(dev)
+        a, b = ev(), ev()
+        with torch.cuda.stream(stream):
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        return a.elapsed_time(b) / reps
+
+    # attention stages alone at the final lengths
+    args, plan = fd.args(), fd.plan_info
+    lib = _lib.load()
+    part_ms = graph_ms(lambda i: lib.specgen_fork_attn_run_partials(C.byref(args), C.byref(plan),
+                                                                     C.c_void_p(sp)))
+    merge_ms = graph_ms(lambda i: lib.specgen_fork_attn_run_merge(C.byref(args), C.byref(plan),
+                                                                   C.c_void_p(sp)))
+    # appends alone, into a second copy of the state (16 steps of room, replayed once more)
+    st_a, fd_a, offs_a, free_a = prepare(2 * per_graph)
+    kn = torch.from_numpy(st_a["k_new"].view(np.int16)).to(dev).view(torch.bfloat16)
+    vn = (None if st_a["v_new"] is None else
+          torch.from_numpy(st_a["v_new"].view(np.int16)).to(dev).view(torch.bfloat16))
+    nf_a = len(st_a["free_pages"])
+    app_ms = graph_ms(lambda i: fd_a.append_kv(kn[i], None if vn is None else vn[i],
+                                               free_a[offs_a[i]:], nf_a - offs_a[i], sp))
+    w_end = dict(st, suffix_lens=st["suffix_lens"] + n)
+    nbytes = wl.algorithmic_bytes(w_end)
     att_bytes = nbytes["prefix"] + nbytes["suffix"] + nbytes["q"]
-    hbm, _, _, peak_src = measured_peaks()
-    achieved = att_bytes / (att_ms * 1e-3) / 1e9
+    hbm, _, tf_sus, peak_src = measured_peaks()
+    achieved = att_bytes / (part_ms * 1e-3) / 1e9
     attn = "mla_tc" if w["v_pages"] is None else "fork_tc"
+    if attn == "mla_tc":  # dense contraction: against the sustained bf16 tensor peak
+        tflops = wl.algorithmic_flops(w_end)["total"] / (part_ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "kernel": attn, "achieved": tflops, "peak": tf_sus,
+                "unit": "TFLOP/s", "frac": tflops / tf_sus, "traffic": None,
+                "peak_source": peak_src + " (bf16, sustained)",
+                "algorithmic_flops_per_launch": wl.algorithmic_flops(w_end)["total"]}
+    else:
+        roof = {"bound": "hbm", "kernel": attn, "achieved": achieved, "peak": hbm,
+                "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                "peak_source": peak_src, "algorithmic_bytes_per_launch": att_bytes}
     row_bytes = F * w["hkv"] * (w["dqk"] + (w["dv"] if w["v_pages"] is not None else 0)) * 2
+    kern = {"append_kv": app_ms, attn: part_ms, "lse_merge": merge_ms}
     line = {
         "metric": "fork-decode step tokens/s (append + attention, growing suffixes)",
         "value": world * F / (ms_per_step * 1e-3), "unit": "tokens/s", "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": ARGS.workload, "op": "decode_step", "forks": F,
-                   "suffix_growth": K + W, "kv_layout": layout,
-                   "timing": "host-driven steps (plan every step) between CUDA events; "
-                             "per-kernel times from events around each launch",
-                   "l2": "inputs of one workload (KV stays resident, as in serving)"},
+                   "suffix_growth": n, "kv_layout": layout,
+                   "timing": "one plan for all steps (device suffix lengths); CUDA graphs of "
+                             "16 steps incl. per-step H2D/D2H copies; per-kernel times from "
+                             "graphs of each kernel alone",
+                   "l2": "one resident state (KV stays resident across steps, as in serving)"},
         "gpu_launches": K * 3,  # append, attention, merge
-        "kernels": {"append_kv": {"ms_per_launch": app_ms,
-                                  "bytes_per_launch": 2 * row_bytes},
-                    attn + "+lse_merge": {"ms_per_launch": att_ms}},
-        "roofline": {"bound": "hbm", "kernel": attn + "+lse_merge", "achieved": achieved,
-                     "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
-                     "peak_source": peak_src, "algorithmic_bytes_per_launch": att_bytes},
+        "kernels": {k: {"ms_per_launch": v, "share": v / sum(kern.values())}
+                    for k, v in kern.items()},
+        "roofline": roof,
         "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
         "e2e": {"value": world * F / (ms_per_step * 1e-3), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(h_q.numel() * 2 + row_bytes),
                 "d2h_bytes_per_step": int(h_o.numel() * 2 + h_l.numel() * 4),
-                "note": "the step itself includes the copies"},
+                "note": "every timed step includes its own host copies"},
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
