@@ -22,4 +22,4 @@ from .attention import (  # noqa: F401
     fork_attn_decode_rows,
     fork_attn_split_merge,
 )
-from .paging import append_kv  # noqa: F401
+from .paging import append_kv, pack_pages, unpack_pages  # noqa: F401

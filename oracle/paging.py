@@ -1,4 +1,6 @@
-"""Plain reference for appending one decode step's K/V to paged suffixes (test infrastructure only).
+"""Plain references for the paged-KV bookkeeping around fork decode (test infrastructure only):
+appending one decode step's K/V to paged suffixes, and packing / unpacking a
+sequence's pages for the remote prefix cache.
 
 What is computed and where it comes from
 ----------------------------------------
@@ -57,3 +59,34 @@ def append_kv(k_pages, v_pages, suffix_table, suffix_bt_offsets, suffix_lens, k_
         if v is not None:
             v[page, :, slot, :] = v_new[f]
     return k, v, table, taken
+
+
+def pack_pages(k_pages, v_pages, table):
+    """Contiguous copy of the pages ``table[0..n)`` of a paged sequence.
+
+    The remote prefix cache (Section 6.2.3) moves a suspended trace's prefix KV
+    off the GPU and back; its device side gathers the sequence's pages into one
+    buffer and scatters them back under a new block table.  Layout of the
+    buffer: the K blocks of the n pages in table order ([n, Hkv, B, Dk] bf16
+    bits), then the V blocks ([n, Hkv, B, Dv]) when there is a value pool.
+    Returns a flat uint16 array.
+    """
+    t = np.asarray(table, dtype=np.int64)
+    parts = [np.asarray(k_pages)[t].reshape(-1)]
+    if v_pages is not None:
+        parts.append(np.asarray(v_pages)[t].reshape(-1))
+    return np.concatenate(parts) if parts else np.zeros(0, np.uint16)
+
+
+def unpack_pages(k_pages, v_pages, table, packed):
+    """Pools with page ``table[i]`` overwritten by page i of ``packed`` (the
+    layout of pack_pages); the inputs are not modified.  Returns (k, v)."""
+    k = np.array(k_pages, copy=True)
+    v = None if v_pages is None else np.array(v_pages, copy=True)
+    t = np.asarray(table, dtype=np.int64)
+    n = len(t)
+    nk = n * int(np.prod(k.shape[1:]))
+    k[t] = np.asarray(packed[:nk]).reshape((n,) + k.shape[1:])
+    if v is not None:
+        v[t] = np.asarray(packed[nk: nk + n * int(np.prod(v.shape[1:]))]).reshape((n,) + v.shape[1:])
+    return k, v

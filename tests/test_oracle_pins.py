@@ -456,3 +456,40 @@ def test_append_rejects_full_table_and_empty_free_list():
     with pytest.raises(ValueError):   # new page needed, free list empty
         oracle.append_kv(pool, None, np.array([-1], np.int32), np.array([0, 1], np.int32),
                          np.array([0], np.int32), row, None, np.array([], np.int32), 2)
+
+
+# ----------------------------------------------------------------- prefix page pack / unpack
+
+def test_pack_pages_hand_example():
+    """Two pages (ids 2 then 0) of a 3-page pool, B = 2, one head, width 1:
+    the buffer is K of page 2, K of page 0, V of page 2, V of page 0."""
+    k = np.arange(6, dtype=np.uint16).reshape(3, 1, 2, 1)          # page p holds 2p, 2p+1
+    v = (100 + np.arange(6, dtype=np.uint16)).reshape(3, 1, 2, 1)
+    buf = oracle.pack_pages(k, v, [2, 0])
+    assert buf.tolist() == [4, 5, 0, 1, 104, 105, 100, 101]
+    assert oracle.pack_pages(k, None, [1]).tolist() == [2, 3]
+
+
+@pytest.mark.parametrize("latent", [False, True])
+def test_pack_then_unpack_moves_a_sequence(latent):
+    """Packing a sequence and unpacking it under a new table gives, by a
+    pure-Python gather, the same logical rows at the new pages; pages outside
+    the new table keep their contents."""
+    rng = np.random.default_rng(5)
+    P, H, B, W = 12, 2, 4, 3
+    k = rng.integers(0, 1 << 15, (P, H, B, W)).astype(np.uint16)
+    v = None if latent else rng.integers(0, 1 << 15, (P, H, B, W + 1)).astype(np.uint16)
+    perm = rng.permutation(P)
+    old, new = perm[:5], perm[5:10]
+    buf = oracle.pack_pages(k, v, old)
+    k2, v2 = oracle.unpack_pages(k, v, new, buf)
+    n = len(old) * B
+    for h in range(H):
+        assert _python_sequence(k2, new, [0], 0, n, B, h) == _python_sequence(k, old, [0], 0, n, B, h)
+        if v is not None:
+            assert (_python_sequence(v2, new, [0], 0, n, B, h)
+                    == _python_sequence(v, old, [0], 0, n, B, h))
+    rest = np.setdiff1d(np.arange(P), new)
+    assert np.array_equal(k2[rest], k[rest])
+    if v is not None:
+        assert np.array_equal(v2[rest], v[rest])
