@@ -44,10 +44,11 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--op", choices=["attend", "decode_step"], default="attend",
+    ap.add_argument("--op", choices=["attend", "decode_step", "pack"], default="attend",
                     help="attend: one fork-decode attention call per step (the headline); "
                          "decode_step: append one K/V row per fork, then attend over the grown "
-                         "suffixes, planning every step on the host")
+                         "suffixes, one plan for all steps; pack: move every trace's prefix "
+                         "pages into one buffer and back (remote prefix cache)")
     ap.add_argument("--kv-layout", choices=["rows", "tiled"], default="rows",
                     help="K/V pool layout: token-major rows (default) or 8x8 core-matrix tiles "
                          "(tensor-core shapes only)")
@@ -688,6 +689,122 @@ def run_decode_steps():
         dist.destroy_process_group()
 
 
+def run_pack():
+    """--op pack: every trace's prefix pages packed into one buffer and unpacked
+    back under the same table (a round trip of the remote prefix cache's device
+    side), on rotating replicas (>= 3x L2), CUDA graphs of 16 steps."""
+    import ctypes as C
+
+    import torch
+
+    import __graft_entry__
+    from paper_2606_17518_gb300 import _lib, workloads as wl
+
+    rank, local_rank, world = dist_env()
+    __graft_entry__.build()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    K, W = ARGS.steps, max(3, ARGS.warmup)
+    w = wl.make_workload(ARGS.workload)
+    stream = torch.cuda.Stream(dev)
+    sp = stream.cuda_stream
+    table = torch.from_numpy(w["prefix_table"]).to(dev)
+    n = len(w["prefix_table"])
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev)
+    probe = _lib.make_pool_desc(hkv=w["hkv"], head_dim_qk=w["dqk"], head_dim_v=w["dv"],
+                                page_size=w["page_size"], num_pages=w["num_pages"],
+                                k_pages=0x100, v_pages=None if w["v_pages"] is None else 0x100)
+    nbytes = _lib.specgen_packed_bytes(probe, n)
+    props = torch.cuda.get_device_properties(dev)
+    l2 = int(getattr(props, "L2_cache_size", 126 * 2 ** 20))
+    replicas = max(1, math.ceil(3 * l2 / (2 * nbytes)))
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    reps = []
+    for _ in range(replicas):
+        k = to_dev(w["k_pages"])
+        v = None if w["v_pages"] is None else to_dev(w["v_pages"])
+        buf = torch.empty(nbytes // 2, dtype=torch.int16, device=dev)
+        desc = _lib.make_pool_desc(hkv=w["hkv"], head_dim_qk=w["dqk"], head_dim_v=w["dv"],
+                                   page_size=w["page_size"], num_pages=w["num_pages"],
+                                   k_pages=k, v_pages=v, status=status)
+        reps.append((k, v, buf, desc))
+    lib = _lib.load()
+    tab = C.c_void_p(table.data_ptr())
+    pack = lambda r: lib.specgen_pack_pages(C.byref(reps[r][3]), tab, n,
+                                            C.c_void_p(reps[r][2].data_ptr()), C.c_void_p(sp))
+    unpack = lambda r: lib.specgen_unpack_pages(C.byref(reps[r][3]), tab, n,
+                                                C.c_void_p(reps[r][2].data_ptr()), C.c_void_p(sp))
+    per_graph = 16
+
+    def graph_of(fns):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(per_graph):
+                for fn in fns:
+                    st = fn(i % replicas)
+                    if st != 0:
+                        raise RuntimeError(_lib.status_string(st))
+        return g
+
+    with torch.cuda.stream(stream):
+        pack(0)
+        unpack(0)
+    torch.cuda.synchronize(dev)
+    g_step, g_pack, g_unpack = graph_of([pack, unpack]), graph_of([pack]), graph_of([unpack])
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+
+    def timed(g, steps):
+        reps_n = max(1, -(-steps // per_graph))
+        a, b = ev(), ev()
+        with torch.cuda.stream(stream):
+            a.record(stream)
+            for _ in range(reps_n):
+                g.replay()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        return a.elapsed_time(b) / (reps_n * per_graph)
+
+    timed(g_step, W)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    ms_per_step = timed(g_step, K)
+    clk = clocks.stop()
+    pack_ms, unpack_ms = timed(g_pack, K), timed(g_unpack, K)
+    if int(status.item()) != 0:
+        raise RuntimeError("pack/unpack reported a bad page id")
+    hbm, _, _, peak_src = measured_peaks()
+    tokens = int(np.sum(w["prefix_lens"]))
+    achieved = 2 * nbytes / (pack_ms * 1e-3) / 1e9
+    line = {
+        "metric": "prefix KV pack+unpack tokens/s", "value": world * tokens / (ms_per_step * 1e-3),
+        "unit": "tokens/s", "n_gpus": world, "steps": per_graph * max(1, -(-K // per_graph)),
+        "warmup": W, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": ARGS.workload, "op": "pack", "pages": n, "prefix_tokens": tokens,
+                   "packed_bytes": nbytes,
+                   "l2": f"rotating over {replicas} replicas (>= 3x L2)",
+                   "timing": "CUDA graphs of 16 steps; per-kernel times from graphs of "
+                             "each direction alone"},
+        "gpu_launches": 2 * per_graph * max(1, -(-K // per_graph)),
+        "kernels": {"pack_pages": {"ms_per_launch": pack_ms},
+                    "unpack_pages": {"ms_per_launch": unpack_ms}},
+        "roofline": {"bound": "hbm", "kernel": "pack_pages", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                     "peak_source": peak_src, "algorithmic_bytes_per_launch": 2 * nbytes},
+        "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def main():
     if os.environ.get("SPECGEN_ORACLE_CHILD"):
         return
@@ -695,6 +812,8 @@ def main():
         run_reference()
     elif ARGS.op == "decode_step":
         run_decode_steps()
+    elif ARGS.op == "pack":
+        run_pack()
     else:
         run_ours()
 

@@ -256,6 +256,34 @@ typedef struct {
  * launched), SPECGEN_ERR_CUDA if the launch fails. */
 specgen_status specgen_append_kv(const specgen_append_args* args, void* cuda_stream);
 
+/* ---- Prefix page pack / unpack ----------------------------------------------
+ * The remote prefix cache (Section 6.2.3) moves a suspended trace's prefix KV
+ * off the GPU and back.  On the device that is a gather of the sequence's pages
+ * into one contiguous buffer and a scatter back under a new block table:
+ *   specgen_pack_pages    packed = K[table[0]] .. K[table[n-1]] V[table[0]] .. V[table[n-1]]
+ *   specgen_unpack_pages  page table[i] of each pool <- page i of packed
+ * where a page block is hkv x page_size x head_dim bf16 in the pool's own block
+ * layout (bytes are copied as they are: rows and tiled pools both work; the
+ * latent pool has no V section).  Pools hold num_pages blocks.  A page id
+ * outside [0, num_pages) is skipped and ORs SPECGEN_ERR_INDEX's bit (1) into
+ * *status (when status is not NULL).  table, packed and the pools are device
+ * memory (16-byte aligned); asynchronous on cuda_stream, capturable.
+ * (An extension for the remote prefix cache; the paper shows no kernel for it.) */
+typedef struct {
+  int hkv, head_dim_qk, head_dim_v, page_size, num_pages;
+  void* k_pages;                    /* bf16 [num_pages][hkv][page_size][head_dim_qk] */
+  void* v_pages;                    /* bf16 [num_pages][hkv][page_size][head_dim_v] or NULL */
+  uint32_t* status;                 /* device status word, or NULL */
+} specgen_pool_desc;
+
+/* Bytes of the packed buffer for n_pages pages (0 on invalid input; a page
+ * block must be a multiple of 16 bytes). */
+size_t specgen_packed_bytes(const specgen_pool_desc* pool, int n_pages);
+specgen_status specgen_pack_pages(const specgen_pool_desc* pool, const int32_t* table,
+                                  int n_pages, void* packed, void* cuda_stream);
+specgen_status specgen_unpack_pages(const specgen_pool_desc* pool, const int32_t* table,
+                                    int n_pages, const void* packed, void* cuda_stream);
+
 /* Read the workspace status word written by the kernels (synchronises
  * `cuda_stream`).  Returns SPECGEN_OK, SPECGEN_ERR_INDEX or SPECGEN_ERR_TIMEOUT. */
 specgen_status specgen_workspace_status(const void* workspace, void* cuda_stream);

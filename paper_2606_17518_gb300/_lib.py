@@ -36,6 +36,9 @@ EXPORTED = [
     "specgen_fork_attn_decode_static",
     "specgen_lse_merge",
     "specgen_append_kv",
+    "specgen_packed_bytes",
+    "specgen_pack_pages",
+    "specgen_unpack_pages",
     "specgen_workspace_status",
     "specgen_status_string",
     "specgen_version",
@@ -69,6 +72,14 @@ class AppendArgs(C.Structure):
         ("v_pages", C.c_void_p), ("suffix_block_table", C.c_void_p),
         ("suffix_bt_offsets", C.c_void_p), ("suffix_lens", C.c_void_p),
         ("free_pages", C.c_void_p), ("num_free", C.c_int), ("status", C.c_void_p),
+    ]
+
+
+class PoolDesc(C.Structure):
+    _fields_ = [
+        ("hkv", C.c_int), ("head_dim_qk", C.c_int), ("head_dim_v", C.c_int),
+        ("page_size", C.c_int), ("num_pages", C.c_int), ("k_pages", C.c_void_p),
+        ("v_pages", C.c_void_p), ("status", C.c_void_p),
     ]
 
 
@@ -115,6 +126,11 @@ def load() -> C.CDLL:
     lib.specgen_fork_attn_run.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
     lib.specgen_append_kv.restype = C.c_int
     lib.specgen_append_kv.argtypes = [P(AppendArgs), C.c_void_p]
+    lib.specgen_packed_bytes.restype = C.c_size_t
+    lib.specgen_packed_bytes.argtypes = [P(PoolDesc), C.c_int]
+    for name in ("specgen_pack_pages", "specgen_unpack_pages"):
+        getattr(lib, name).restype = C.c_int
+        getattr(lib, name).argtypes = [P(PoolDesc), C.c_void_p, C.c_int, C.c_void_p, C.c_void_p]
     for stage in ("specgen_fork_attn_run_partials", "specgen_fork_attn_run_merge"):
         getattr(lib, stage).restype = C.c_int
         getattr(lib, stage).argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
@@ -191,6 +207,26 @@ def make_append_args(*, total_forks, hkv, head_dim_qk, head_dim_v, page_size, nu
 
 def specgen_append_kv(args: AppendArgs, stream: int = 0) -> None:
     _check(load().specgen_append_kv(C.byref(args), C.c_void_p(stream)), "specgen_append_kv")
+
+
+def make_pool_desc(*, hkv, head_dim_qk, head_dim_v, page_size, num_pages, k_pages, v_pages,
+                   status=None) -> PoolDesc:
+    return PoolDesc(int(hkv), int(head_dim_qk), int(head_dim_v), int(page_size),
+                    int(num_pages), _ptr(k_pages), _ptr(v_pages), _ptr(status))
+
+
+def specgen_packed_bytes(pool: PoolDesc, n_pages: int) -> int:
+    return int(load().specgen_packed_bytes(C.byref(pool), int(n_pages)))
+
+
+def specgen_pack_pages(pool: PoolDesc, table, n_pages: int, packed, stream: int = 0) -> None:
+    _check(load().specgen_pack_pages(C.byref(pool), _ptr(table), int(n_pages), _ptr(packed),
+                                     C.c_void_p(stream)), "specgen_pack_pages")
+
+
+def specgen_unpack_pages(pool: PoolDesc, table, n_pages: int, packed, stream: int = 0) -> None:
+    _check(load().specgen_unpack_pages(C.byref(pool), _ptr(table), int(n_pages), _ptr(packed),
+                                       C.c_void_p(stream)), "specgen_unpack_pages")
 
 
 def specgen_fork_attn_workspace_size(args: ForkAttnArgs, lens: HostLens) -> int:

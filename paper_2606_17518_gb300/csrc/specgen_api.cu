@@ -15,6 +15,7 @@
 
 #include "../../include/specgen.h"
 #include "append_kv.h"
+#include "pack_pages.h"
 #include "lse_merge.h"
 #include "plan.h"
 #include "fork_tc.h"
@@ -781,6 +782,68 @@ specgen_status specgen_append_kv(const specgen_append_args* a, void* cuda_stream
   if (launch_append_kv(p, static_cast<cudaStream_t>(cuda_stream)) != cudaSuccess)
     return SPECGEN_ERR_CUDA;
   return SPECGEN_OK;
+}
+
+namespace {
+
+// Checks a pool description; fills the 16-byte words per page of each pool.
+specgen_status check_pool(const specgen_pool_desc* d, size_t* k16, size_t* v16) {
+  if (!d) return SPECGEN_ERR_NULL;
+  if (d->hkv < 1 || d->page_size < 1 || d->num_pages < 0 || d->head_dim_qk < 1)
+    return SPECGEN_ERR_SHAPE;
+  if (d->v_pages && d->head_dim_v < 1) return SPECGEN_ERR_SHAPE;
+  const size_t kb = (size_t)d->hkv * d->page_size * d->head_dim_qk * 2;
+  const size_t vb = d->v_pages ? (size_t)d->hkv * d->page_size * d->head_dim_v * 2 : 0;
+  if (kb % 16 != 0 || vb % 16 != 0) return SPECGEN_ERR_UNSUPPORTED;
+  *k16 = kb / 16;
+  *v16 = vb / 16;
+  return SPECGEN_OK;
+}
+
+specgen_status pack_impl(const specgen_pool_desc* d, const int32_t* table, int n_pages,
+                         void* packed, bool unpack, void* cuda_stream) {
+  size_t k16 = 0, v16 = 0;
+  specgen_status st = check_pool(d, &k16, &v16);
+  if (st != SPECGEN_OK) return st;
+  if (n_pages < 0) return SPECGEN_ERR_SHAPE;
+  if (n_pages == 0) return SPECGEN_OK;
+  if (!table || !packed || !d->k_pages) return SPECGEN_ERR_NULL;
+  const void* ptrs[3] = {packed, d->k_pages, d->v_pages};
+  for (const void* q : ptrs)
+    if (reinterpret_cast<uintptr_t>(q) % 16 != 0) return SPECGEN_ERR_SHAPE;
+  PackParams p;
+  p.k_pages = static_cast<uint4*>(d->k_pages);
+  p.v_pages = static_cast<uint4*>(d->v_pages);
+  p.packed = static_cast<uint4*>(packed);
+  p.table = table;
+  p.status = d->status;
+  p.k_block16 = k16;
+  p.v_block16 = v16;
+  p.n_pages = n_pages;
+  p.num_pages = d->num_pages;
+  p.unpack = unpack;
+  if (launch_pack_pages(p, device_sm_count(), static_cast<cudaStream_t>(cuda_stream)) !=
+      cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
+}
+
+}  // namespace
+
+size_t specgen_packed_bytes(const specgen_pool_desc* pool, int n_pages) {
+  size_t k16 = 0, v16 = 0;
+  if (n_pages < 0 || check_pool(pool, &k16, &v16) != SPECGEN_OK) return 0;
+  return (size_t)n_pages * (k16 + v16) * 16;
+}
+
+specgen_status specgen_pack_pages(const specgen_pool_desc* pool, const int32_t* table,
+                                  int n_pages, void* packed, void* cuda_stream) {
+  return pack_impl(pool, table, n_pages, packed, false, cuda_stream);
+}
+
+specgen_status specgen_unpack_pages(const specgen_pool_desc* pool, const int32_t* table,
+                                    int n_pages, const void* packed, void* cuda_stream) {
+  return pack_impl(pool, table, n_pages, const_cast<void*>(packed), true, cuda_stream);
 }
 
 specgen_status specgen_lse_merge(const void* out_a, const float* lse_a, const void* out_b,

@@ -220,3 +220,25 @@ def test_append_host_checks():
     assert st(suffix_lens=None) == S.SPECGEN_ERR_NULL
     assert st(free_pages=None) == S.SPECGEN_ERR_NULL
     assert st(k_new=fake + 8) == S.SPECGEN_ERR_SHAPE            # not 16-byte aligned
+
+
+def test_pack_host_checks():
+    S = _lib
+    lib = _lib.load()
+    fake = 0x10000
+    base = dict(hkv=8, head_dim_qk=128, head_dim_v=128, page_size=16, num_pages=100,
+                k_pages=fake, v_pages=fake)
+    d = lambda **kw: _lib.make_pool_desc(**{**base, **kw})
+    assert _lib.specgen_packed_bytes(d(), 3) == 3 * 2 * 8 * 16 * 128 * 2
+    assert _lib.specgen_packed_bytes(d(v_pages=None), 3) == 3 * 8 * 16 * 128 * 2
+    assert _lib.specgen_packed_bytes(d(hkv=1, page_size=1, head_dim_qk=3, v_pages=None), 1) == 0
+    assert _lib.specgen_packed_bytes(d(hkv=0), 1) == 0
+    pk = lambda desc, n, table=fake, packed=fake: lib.specgen_pack_pages(
+        C.byref(desc), table, n, packed, None)
+    assert pk(d(), 0) == S.SPECGEN_OK                           # nothing to copy
+    assert pk(d(), -1) == S.SPECGEN_ERR_SHAPE
+    assert pk(d(), 2, table=None) == S.SPECGEN_ERR_NULL
+    assert pk(d(), 2, packed=None) == S.SPECGEN_ERR_NULL
+    assert pk(d(), 2, packed=fake + 4) == S.SPECGEN_ERR_SHAPE    # not 16-byte aligned
+    assert pk(d(hkv=1, page_size=1, head_dim_qk=4, v_pages=None), 2) == S.SPECGEN_ERR_UNSUPPORTED
+    assert lib.specgen_pack_pages(None, fake, 1, fake, None) == S.SPECGEN_ERR_NULL
