@@ -21,5 +21,6 @@ from .attention import (  # noqa: F401
     fork_attn_decode,
     fork_attn_decode_rows,
     fork_attn_split_merge,
+    fork_prefill,
 )
 from .paging import append_kv, pack_pages, unpack_pages  # noqa: F401

@@ -219,3 +219,41 @@ def fork_attn_split_merge(w: dict) -> tuple[np.ndarray, np.ndarray]:
             o_s, l_s = attention_rows(q, ks, vs, w["scale"])
             o[f, heads], lse[f, heads] = lse_merge(o_p, l_p, o_s, l_s)
     return o, lse
+
+
+def fork_prefill(w: dict, chunk_lens, q_rows) -> tuple[np.ndarray, np.ndarray]:
+    """Causal prefill of every fork's newest suffix tokens (Algorithm 1: the
+    fork's prompt follows the shared prefix and is processed before it decodes).
+
+    ``w`` is a fork-decode workload whose suffix lengths already count the
+    chunk; fork f's chunk is its last ``chunk_lens[f]`` suffix tokens.  Query
+    row r = (f, j), fork by fork and j < chunk_lens[f] (``q_rows`` [R, hq, dqk]
+    bf16 bits), attends to the trace's prefix and the fork's suffix tokens
+    0 .. S_f - chunk_lens[f] + j: its own token and everything before it.
+    Returns O [R, hq, dv] and LSE [R, hq] (float64).
+    """
+    _check(w)
+    hq, g_size, dv = w["hq"], w["hq"] // w["hkv"], w["dv"]
+    chunk_lens = np.asarray(chunk_lens)
+    n_rows = int(chunk_lens.sum())
+    out_o = np.zeros((n_rows, hq, dv))
+    out_lse = np.zeros((n_rows, hq))
+    fo = w["fork_offsets"]
+    trace_of = np.searchsorted(fo, np.arange(w["total_forks"]), side="right") - 1
+    r = 0
+    for f in range(w["total_forks"]):
+        t = int(trace_of[f])
+        pt = w["prefix_table"][w["prefix_bt_offsets"][t]:w["prefix_bt_offsets"][t + 1]]
+        st = w["suffix_table"][w["suffix_bt_offsets"][f]:w["suffix_bt_offsets"][f + 1]]
+        before = int(w["suffix_lens"][f]) - int(chunk_lens[f])
+        for j in range(int(chunk_lens[f])):
+            for g in range(w["hkv"]):
+                k, v = _fork_kv(w["k_pages"], w.get("v_pages"), dv, w["page_size"], pt,
+                                int(w["prefix_lens"][t]), st, before + j + 1, g)
+                heads = list(range(g * g_size, (g + 1) * g_size))
+                q = bf16_bits_to_f64(np.asarray(q_rows)[r, heads, :])
+                o, lse = attention_rows(q, k, v, w["scale"])
+                out_o[r, heads] = o
+                out_lse[r, heads] = lse
+            r += 1
+    return out_o, out_lse

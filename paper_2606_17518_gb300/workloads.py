@@ -259,3 +259,17 @@ def make_decode_state(w: dict, steps: int, seed: int = 12345) -> dict:
         v_new=(bf16_normal(rng, (steps, F, w["hkv"], w["dv"])) if w["v_pages"] is not None
                else None))
     return out
+
+
+def make_prefill(w: dict, chunk: int, seed: int = 777) -> dict:
+    """Prefill inputs over a workload: fork f's chunk is its last
+    min(chunk, S_f) suffix tokens (their K/V are already in the pools) and each
+    chunk token gets its own query row (``q_rows`` [R, hq, dqk], fork by fork).
+    Inputs only.  Returns a new dict with ``chunk_lens``, ``q_rows``, ``rows``."""
+    rng = np.random.default_rng(seed)
+    chunk_lens = np.minimum(w["suffix_lens"], chunk).astype(np.int32)
+    rows = int(chunk_lens.sum())
+    out = dict(w)
+    out.update(chunk_lens=chunk_lens, rows=rows,
+               q_rows=bf16_normal(rng, (rows, w["hq"], w["dqk"])))
+    return out

@@ -493,3 +493,40 @@ def test_pack_then_unpack_moves_a_sequence(latent):
     assert np.array_equal(k2[rest], k[rest])
     if v is not None:
         assert np.array_equal(v2[rest], v[rest])
+
+
+# ----------------------------------------------------------------- fork prefill
+
+def test_prefill_with_one_token_chunks_is_decode():
+    """A chunk of one token per fork is the decode of that fork's last token."""
+    w = wl.make_workload(_tiny(seed=3))
+    pf = wl.make_prefill(w, 1)
+    o, lse = oracle.fork_prefill(w, pf["chunk_lens"], pf["q_rows"])
+    has = pf["chunk_lens"] > 0
+    w_dec = dict(w, q=np.zeros_like(w["q"]))
+    w_dec["q"][has] = pf["q_rows"]
+    o_d, lse_d = oracle.fork_attn_decode(w_dec)
+    assert np.allclose(o, o_d[has], rtol=0, atol=1e-14)
+    assert np.allclose(lse, lse_d[has], rtol=0, atol=1e-14)
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_prefill_is_causal_brute_force(seed):
+    """Row (f, j) equals the pure-Python brute force over the prefix and the
+    fork's first S_f - c_f + j + 1 suffix tokens, with the row's own query."""
+    w = wl.make_workload(_tiny(seed=seed))
+    pf = wl.make_prefill(w, 5)
+    o, lse = oracle.fork_prefill(w, pf["chunk_lens"], pf["q_rows"])
+    r = 0
+    for f in range(w["total_forks"]):
+        c = int(pf["chunk_lens"][f])
+        for j in range(c):
+            lens = w["suffix_lens"].copy()
+            lens[f] = w["suffix_lens"][f] - c + j + 1
+            q = w["q"].copy()
+            q[f] = pf["q_rows"][r]
+            ob, lb = _brute(dict(w, suffix_lens=lens, q=q))
+            assert np.allclose(o[r], ob[f], rtol=0, atol=1e-12)
+            assert np.allclose(lse[r], lb[f], rtol=0, atol=1e-12)
+            r += 1
+    assert r == pf["rows"]
