@@ -44,11 +44,14 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--op", choices=["attend", "decode_step", "pack"], default="attend",
+    ap.add_argument("--op", choices=["attend", "decode_step", "pack", "prefill"],
+                    default="attend",
                     help="attend: one fork-decode attention call per step (the headline); "
                          "decode_step: append one K/V row per fork, then attend over the grown "
                          "suffixes, one plan for all steps; pack: move every trace's prefix "
-                         "pages into one buffer and back (remote prefix cache)")
+                         "pages into one buffer and back (remote prefix cache); prefill: "
+                         "causal prefill of a --chunk-token prompt chunk per fork")
+    ap.add_argument("--chunk", type=int, default=64, help="prefill chunk tokens per fork")
     ap.add_argument("--kv-layout", choices=["rows", "tiled"], default="rows",
                     help="K/V pool layout: token-major rows (default) or 8x8 core-matrix tiles "
                          "(tensor-core shapes only)")
@@ -805,6 +808,117 @@ def run_pack():
         dist.destroy_process_group()
 
 
+def run_prefill():
+    """--op prefill: every fork prefills its last --chunk suffix tokens (one query
+    row per token, causal), plan made once, CUDA graphs of 16 runs on rotating
+    replicas (>= 3x L2).  Value: prefilled tokens per second."""
+    import ctypes as C
+
+    import torch
+
+    import __graft_entry__
+    from paper_2606_17518_gb300 import _lib, workloads as wl
+    from paper_2606_17518_gb300.fork_attn import ForkPrefill
+
+    rank, local_rank, world = dist_env()
+    __graft_entry__.build()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    K, W = ARGS.steps, max(3, ARGS.warmup)
+    pf = wl.make_prefill(wl.make_workload(ARGS.workload), ARGS.chunk)
+    nbytes = wl.algorithmic_bytes(pf)["total"]
+    props = torch.cuda.get_device_properties(dev)
+    l2 = int(getattr(props, "L2_cache_size", 126 * 2 ** 20))
+    replicas = max(1, math.ceil(3 * l2 / nbytes))
+    stream = torch.cuda.Stream(dev)
+    sp = stream.cuda_stream
+    reps = [ForkPrefill(pf, device=dev) for _ in range(replicas)]
+    with torch.cuda.stream(stream):
+        for r in reps:
+            r.plan(sp)
+            r.run(sp)
+    torch.cuda.synchronize(dev)
+    lib = _lib.load()
+    args = [r.args() for r in reps]
+    plans = [r.plan_info for r in reps]
+    per_graph = 16
+
+    def graph_of(call):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(per_graph):
+                st = call(C.byref(args[i % replicas]), C.byref(plans[i % replicas]),
+                          C.c_void_p(sp))
+                if st != 0:
+                    raise RuntimeError(_lib.status_string(st))
+        return g
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+
+    def timed(g, steps):
+        n_rep = max(1, -(-steps // per_graph))
+        a, b = ev(), ev()
+        with torch.cuda.stream(stream):
+            a.record(stream)
+            for _ in range(n_rep):
+                g.replay()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        return a.elapsed_time(b) / (n_rep * per_graph)
+
+    g_run = graph_of(lib.specgen_fork_attn_run)
+    timed(g_run, W)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    ms_per_step = timed(g_run, K)
+    clk = clocks.stop()
+    part_ms = timed(graph_of(lib.specgen_fork_attn_run_partials), K)
+    merge_ms = timed(graph_of(lib.specgen_fork_attn_run_merge), K)
+    if reps[0].status(sp) != 0:
+        raise RuntimeError("prefill reported an error")
+    rows = pf["rows"]
+    # algorithmic flops: every query row against its own key count
+    fo = pf["fork_offsets"]
+    keys = 0
+    for t in range(pf["num_traces"]):
+        for f in range(fo[t], fo[t + 1]):
+            c = int(pf["chunk_lens"][f])
+            before = int(pf["suffix_lens"][f]) - c
+            keys += c * int(pf["prefix_lens"][t]) + sum(before + j + 1 for j in range(c))
+    flops = 2 * keys * pf["hq"] * (pf["dqk"] + pf["dv"])
+    _, _, tf_sus, peak_src = measured_peaks()
+    attn = "mla_tc" if pf["v_pages"] is None else "fork_tc"
+    tflops = flops / (part_ms * 1e-3) / 1e12
+    line = {
+        "metric": "fork prefill tokens/s", "value": world * rows / (ms_per_step * 1e-3),
+        "unit": "tokens/s", "n_gpus": world, "steps": per_graph * max(1, -(-K // per_graph)),
+        "warmup": W, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": ARGS.workload, "op": "prefill", "chunk": ARGS.chunk,
+                   "query_rows": rows, "flops": flops, "unique_bytes": nbytes,
+                   "l2": f"rotating over {replicas} replicas (>= 3x L2)",
+                   "timing": "CUDA graphs of 16 runs; per-kernel times from graphs of each "
+                             "stage alone"},
+        "gpu_launches": 2 * per_graph * max(1, -(-K // per_graph)),
+        "kernels": {attn: {"ms_per_launch": part_ms}, "lse_merge": {"ms_per_launch": merge_ms}},
+        "roofline": {"bound": "tensor", "kernel": attn, "achieved": tflops, "peak": tf_sus,
+                     "unit": "TFLOP/s", "frac": tflops / tf_sus, "traffic": None,
+                     "peak_source": peak_src + " (bf16, sustained)",
+                     "algorithmic_flops_per_launch": flops},
+        "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def main():
     if os.environ.get("SPECGEN_ORACLE_CHILD"):
         return
@@ -814,6 +928,8 @@ def main():
         run_decode_steps()
     elif ARGS.op == "pack":
         run_pack()
+    elif ARGS.op == "prefill":
+        run_prefill()
     else:
         run_ours()
 

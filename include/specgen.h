@@ -215,6 +215,36 @@ specgen_status specgen_lse_merge(const void* out_a, const float* lse_a,
                                  void* out, float* lse, int rows, int dv,
                                  int dtype, void* cuda_stream);
 
+/* ---- Fork prefill ---------------------------------------------------------
+ * Before a fork decodes, its new prompt tokens (the iteration prompt after the
+ * shared reasoning prefix, Algorithm 1 and Section 6.1.1) are prefilled: fork f
+ * appends chunk_lens[f] tokens after its suffix_lens[f] existing suffix tokens
+ * (their K/V rows already written into its suffix pages, e.g. by the caller's
+ * projection), and query j of the chunk attends to the trace's prefix, the
+ * fork's existing suffix and, causally, chunk tokens 0..j: exactly a decode
+ * query whose suffix length is suffix_lens[f] + j + 1.  The call plans one row
+ * block per chunk token (fork by fork, trace by trace), so the prefix stage
+ * still reads each prefix page once for up to 128 / (hq / hkv) query rows.
+ * args: as for decode except total_forks = sum of chunk_lens (query rows):
+ * q, out, lse are [rows][hq][...] in that order, while the block tables and
+ * suffix_bt_offsets stay per fork (fork_offsets[num_traces] forks);
+ * args->suffix_lens must be NULL.  Run the plan with specgen_fork_attn_run
+ * (or _partials / _merge); same status codes as the decode entry points. */
+typedef struct {
+  const int32_t* prefix_lens;       /* host [num_traces] */
+  const int32_t* fork_offsets;      /* host [num_traces + 1] over forks */
+  const int32_t* suffix_lens;       /* host [forks]: suffix tokens before the chunk */
+  const int32_t* chunk_lens;        /* host [forks]: new tokens of each fork (>= 0) */
+  const int32_t* prefix_bt_offsets; /* host [num_traces + 1] or NULL */
+  const int32_t* suffix_bt_offsets; /* host [forks + 1] or NULL */
+} specgen_prefill_lens;
+
+size_t specgen_fork_prefill_workspace_size(const specgen_fork_attn_args* args,
+                                           const specgen_prefill_lens* lens);
+specgen_status specgen_fork_prefill_plan(const specgen_fork_attn_args* args,
+                                         const specgen_prefill_lens* lens, specgen_plan* plan,
+                                         void* cuda_stream);
+
 /* ---- Decode-step append --------------------------------------------------
  * After a fork event every fork decodes its own continuation while the prefix
  * stays shared (Algorithm 1, "Fork K spec. generations"; Section 4.2), so each

@@ -32,6 +32,8 @@ EXPORTED = [
     "specgen_fork_attn_run_profiled",
     "specgen_fork_attn_run_partials",
     "specgen_fork_attn_run_merge",
+    "specgen_fork_prefill_workspace_size",
+    "specgen_fork_prefill_plan",
     "specgen_fork_attn_decode",
     "specgen_fork_attn_decode_static",
     "specgen_lse_merge",
@@ -89,6 +91,12 @@ class HostLens(C.Structure):
                 ("suffix_bt_offsets", C.c_void_p)]
 
 
+class PrefillLens(C.Structure):
+    _fields_ = [("prefix_lens", C.c_void_p), ("fork_offsets", C.c_void_p),
+                ("suffix_lens", C.c_void_p), ("chunk_lens", C.c_void_p),
+                ("prefix_bt_offsets", C.c_void_p), ("suffix_bt_offsets", C.c_void_p)]
+
+
 class Plan(C.Structure):
     _fields_ = [
         ("valid", C.c_int32), ("n_tc_items", C.c_int32), ("n_tc_ctas", C.c_int32),
@@ -124,6 +132,11 @@ def load() -> C.CDLL:
     lib.specgen_fork_attn_plan.argtypes = [P(ForkAttnArgs), P(HostLens), P(Plan), C.c_void_p]
     lib.specgen_fork_attn_run.restype = C.c_int
     lib.specgen_fork_attn_run.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
+    lib.specgen_fork_prefill_workspace_size.restype = C.c_size_t
+    lib.specgen_fork_prefill_workspace_size.argtypes = [P(ForkAttnArgs), P(PrefillLens)]
+    lib.specgen_fork_prefill_plan.restype = C.c_int
+    lib.specgen_fork_prefill_plan.argtypes = [P(ForkAttnArgs), P(PrefillLens), P(Plan),
+                                              C.c_void_p]
     lib.specgen_append_kv.restype = C.c_int
     lib.specgen_append_kv.argtypes = [P(AppendArgs), C.c_void_p]
     lib.specgen_packed_bytes.restype = C.c_size_t
@@ -227,6 +240,28 @@ def specgen_pack_pages(pool: PoolDesc, table, n_pages: int, packed, stream: int 
 def specgen_unpack_pages(pool: PoolDesc, table, n_pages: int, packed, stream: int = 0) -> None:
     _check(load().specgen_unpack_pages(C.byref(pool), _ptr(table), int(n_pages), _ptr(packed),
                                        C.c_void_p(stream)), "specgen_unpack_pages")
+
+
+def make_prefill_lens(prefix_lens, fork_offsets, suffix_lens, chunk_lens,
+                      prefix_bt_offsets=None, suffix_bt_offsets=None):
+    """PrefillLens over host int32 copies; returns (struct, keepalive)."""
+    keep = [np.ascontiguousarray(a, dtype=np.int32)
+            for a in (prefix_lens, fork_offsets, suffix_lens, chunk_lens)]
+    opt = [None if a is None else np.ascontiguousarray(a, dtype=np.int32)
+           for a in (prefix_bt_offsets, suffix_bt_offsets)]
+    ptrs = [a.ctypes.data for a in keep] + [None if a is None else a.ctypes.data for a in opt]
+    return PrefillLens(*ptrs), keep + opt
+
+
+def specgen_fork_prefill_workspace_size(args: ForkAttnArgs, lens: PrefillLens) -> int:
+    return int(load().specgen_fork_prefill_workspace_size(C.byref(args), C.byref(lens)))
+
+
+def specgen_fork_prefill_plan(args: ForkAttnArgs, lens: PrefillLens, stream: int = 0) -> Plan:
+    plan = Plan()
+    _check(load().specgen_fork_prefill_plan(C.byref(args), C.byref(lens), C.byref(plan),
+                                            C.c_void_p(stream)), "specgen_fork_prefill_plan")
+    return plan
 
 
 def specgen_fork_attn_workspace_size(args: ForkAttnArgs, lens: HostLens) -> int:

@@ -52,10 +52,9 @@ struct Shape {
   bool latent;
 };
 
-specgen_status check_shape(const specgen_fork_attn_args* a, const specgen_host_lens* lens,
-                           Shape* s) {
-  if (!a || !lens || !lens->prefix_lens || !lens->fork_offsets || !lens->suffix_lens)
-    return SPECGEN_ERR_NULL;
+// Checks of the scalar arguments shared by decode and prefill; fills s (F = the
+// query rows, args->total_forks).
+specgen_status check_common(const specgen_fork_attn_args* a, Shape* s) {
   if (a->num_traces < 1 || a->total_forks < 1 || a->hq < 1 || a->hkv < 1 || a->page_size < 1 ||
       a->num_pages < 0 || a->head_dim_qk < 1 || a->head_dim_v < 1)
     return SPECGEN_ERR_SHAPE;
@@ -71,13 +70,6 @@ specgen_status check_shape(const specgen_fork_attn_args* a, const specgen_host_l
   if (a->kv_layout == SPECGEN_KV_TILED &&
       !fork_tc_supported(a->head_dim_qk, a->head_dim_v, latent, a->page_size, a->hq / a->hkv))
     return SPECGEN_ERR_UNSUPPORTED;
-  const int32_t* fo = lens->fork_offsets;
-  if (fo[0] != 0 || fo[a->num_traces] != a->total_forks) return SPECGEN_ERR_SHAPE;
-  for (int t = 0; t < a->num_traces; ++t) {
-    if (fo[t + 1] < fo[t] || lens->prefix_lens[t] < 0) return SPECGEN_ERR_SHAPE;
-  }
-  for (int f = 0; f < a->total_forks; ++f)
-    if (lens->suffix_lens[f] < 0) return SPECGEN_ERR_SHAPE;
   s->T = a->num_traces;
   s->F = a->total_forks;
   s->hq = a->hq;
@@ -88,6 +80,46 @@ specgen_status check_shape(const specgen_fork_attn_args* a, const specgen_host_l
   s->B = a->page_size;
   s->num_pages = a->num_pages;
   s->latent = latent;
+  return SPECGEN_OK;
+}
+
+specgen_status check_shape(const specgen_fork_attn_args* a, const specgen_host_lens* lens,
+                           Shape* s) {
+  if (!a || !lens || !lens->prefix_lens || !lens->fork_offsets || !lens->suffix_lens)
+    return SPECGEN_ERR_NULL;
+  const specgen_status st = check_common(a, s);
+  if (st != SPECGEN_OK) return st;
+  const int32_t* fo = lens->fork_offsets;
+  if (fo[0] != 0 || fo[a->num_traces] != a->total_forks) return SPECGEN_ERR_SHAPE;
+  for (int t = 0; t < a->num_traces; ++t) {
+    if (fo[t + 1] < fo[t] || lens->prefix_lens[t] < 0) return SPECGEN_ERR_SHAPE;
+  }
+  for (int f = 0; f < a->total_forks; ++f)
+    if (lens->suffix_lens[f] < 0) return SPECGEN_ERR_SHAPE;
+  return SPECGEN_OK;
+}
+
+// Prefill: args->total_forks counts query rows (the sum of the chunk lengths);
+// the forks themselves are lens->fork_offsets[num_traces].
+specgen_status check_prefill(const specgen_fork_attn_args* a, const specgen_prefill_lens* lens,
+                             Shape* s) {
+  if (!a || !lens || !lens->prefix_lens || !lens->fork_offsets || !lens->suffix_lens ||
+      !lens->chunk_lens)
+    return SPECGEN_ERR_NULL;
+  const specgen_status st = check_common(a, s);
+  if (st != SPECGEN_OK) return st;
+  if (a->suffix_lens != nullptr) return SPECGEN_ERR_SHAPE;  // device lengths: decode only
+  const int32_t* fo = lens->fork_offsets;
+  if (fo[0] != 0) return SPECGEN_ERR_SHAPE;
+  for (int t = 0; t < a->num_traces; ++t)
+    if (fo[t + 1] < fo[t] || lens->prefix_lens[t] < 0) return SPECGEN_ERR_SHAPE;
+  long long rows = 0;
+  for (int f = 0; f < fo[a->num_traces]; ++f) {
+    if (lens->suffix_lens[f] < 0 || lens->chunk_lens[f] < 0) return SPECGEN_ERR_SHAPE;
+    if ((long long)lens->suffix_lens[f] + lens->chunk_lens[f] > INT32_MAX) return SPECGEN_ERR_SHAPE;
+    rows += lens->chunk_lens[f];
+  }
+  if (rows != a->total_forks) return SPECGEN_ERR_SHAPE;
   return SPECGEN_OK;
 }
 
@@ -109,6 +141,53 @@ struct HostPlan {
   int n_groups = 1;
   int total_slots = 0;
 };
+
+// The query rows a plan serves, trace by trace.  Decode: one row per fork.
+// Prefill: one row per new token of every fork; row j of fork f attends to the
+// fork's first S_f + j + 1 suffix tokens (its earlier tokens and, causally, the
+// chunk up to itself).  A row reads the suffix table of fork `seq`.
+struct Rows {
+  const int32_t* prefix_lens = nullptr;        // host [T]
+  std::vector<int32_t> trace_off;              // [T + 1]
+  std::vector<int32_t> seq;                    // [R]
+  std::vector<int32_t> len;                    // [R]
+  const int32_t* prefix_bt_offsets = nullptr;  // optional host copies of the table offsets
+  const int32_t* suffix_bt_offsets = nullptr;
+};
+
+Rows rows_for_decode(const specgen_host_lens* lens, int T, int F) {
+  Rows r;
+  r.prefix_lens = lens->prefix_lens;
+  r.trace_off.assign(lens->fork_offsets, lens->fork_offsets + T + 1);
+  r.seq.resize(F);
+  r.len.assign(lens->suffix_lens, lens->suffix_lens + F);
+  for (int f = 0; f < F; ++f) r.seq[f] = f;
+  if (lens->prefix_bt_offsets && lens->suffix_bt_offsets) {
+    r.prefix_bt_offsets = lens->prefix_bt_offsets;
+    r.suffix_bt_offsets = lens->suffix_bt_offsets;
+  }
+  return r;
+}
+
+Rows rows_for_prefill(const specgen_prefill_lens* lens, int T) {
+  Rows r;
+  r.prefix_lens = lens->prefix_lens;
+  const int32_t* fo = lens->fork_offsets;
+  r.trace_off.assign(1, 0);
+  for (int t = 0; t < T; ++t) {
+    for (int f = fo[t]; f < fo[t + 1]; ++f)
+      for (int j = 0; j < lens->chunk_lens[f]; ++j) {
+        r.seq.push_back(f);
+        r.len.push_back(lens->suffix_lens[f] + j + 1);  // causal within the chunk
+      }
+    r.trace_off.push_back((int32_t)r.seq.size());
+  }
+  if (lens->prefix_bt_offsets && lens->suffix_bt_offsets) {
+    r.prefix_bt_offsets = lens->prefix_bt_offsets;
+    r.suffix_bt_offsets = lens->suffix_bt_offsets;
+  }
+  return r;
+}
 
 // Longest-processing-time-first assignment of items to `n_cta` persistent CTAs:
 // items in decreasing cost, each to the currently least-loaded CTA.
@@ -140,17 +219,17 @@ void assign_lpt(const std::vector<long long>& cost, int n_cta, std::vector<int32
 // that CTA c walks items [cta_offsets[c], cta_offsets[c+1]), and resolve each
 // item's block-table start on the host when the host table offsets are given.
 void finish_tc_plan(HostPlan* hp, const std::vector<long long>& cost, int n_sm,
-                    const specgen_host_lens* lens) {
+                    const Rows& rows) {
   const int n_cta = (int)std::min<size_t>((size_t)n_sm, hp->tc.size());
   std::vector<int32_t> order;
   assign_lpt(cost, n_cta, &order, &hp->cta_offsets);
   std::vector<TcItem> sorted;
   sorted.reserve(hp->tc.size());
-  const bool host_off = lens->prefix_bt_offsets && lens->suffix_bt_offsets;
+  const bool host_off = rows.prefix_bt_offsets && rows.suffix_bt_offsets;
   for (int32_t i : order) {
     TcItem it = hp->tc[i];
-    it.table_off = host_off ? (it.table_kind == 0 ? lens->prefix_bt_offsets[it.seq]
-                                                  : lens->suffix_bt_offsets[it.seq])
+    it.table_off = host_off ? (it.table_kind == 0 ? rows.prefix_bt_offsets[it.seq]
+                                                  : rows.suffix_bt_offsets[it.seq])
                             : -1;
     sorted.push_back(it);
   }
@@ -241,20 +320,20 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
   return ui == pfx.size();
 }
 
-void build_tc_plan(const Shape& s, const specgen_host_lens* lens, int n_sm, HostPlan* hp) {
-  const int32_t* fo = lens->fork_offsets;
+void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
+  const int32_t* fo = rows.trace_off.data();
   const int page = fork_tc_page_size();
   const int forks_per_item = std::max(1, 128 / s.G);
   std::vector<TcUnit> sfx, pfx;
   long long total = 0;
   for (int t = 0; t < s.T; ++t) {
     for (int g = 0; g < s.hkv; ++g) {
-      if (lens->prefix_lens[t] > 0)
+      if (rows.prefix_lens[t] > 0)
         for (int f0 = fo[t]; f0 < fo[t + 1]; f0 += forks_per_item)
           pfx.push_back(TcUnit{0, t, g, f0, std::min(forks_per_item, fo[t + 1] - f0),
-                               lens->prefix_lens[t]});
+                               rows.prefix_lens[t]});
       for (int f = fo[t]; f < fo[t + 1]; ++f)
-        if (lens->suffix_lens[f] > 0) sfx.push_back(TcUnit{1, f, g, f, 1, lens->suffix_lens[f]});
+        if (rows.len[f] > 0) sfx.push_back(TcUnit{1, rows.seq[f], g, f, 1, rows.len[f]});
     }
   }
   for (const TcUnit& u : sfx) total += u.len;
@@ -313,7 +392,7 @@ void build_tc_plan(const Shape& s, const specgen_host_lens* lens, int n_sm, Host
   hp->total_slots = slot;
   // items in CTA order (empty CTAs dropped), suffix parts after the prefix ones,
   // block-table starts resolved on the host when the host offsets are given
-  const bool host_off = lens->prefix_bt_offsets && lens->suffix_bt_offsets;
+  const bool host_off = rows.prefix_bt_offsets && rows.suffix_bt_offsets;
   hp->tc.clear();
   hp->cta_offsets.assign(1, 0);
   std::vector<int> per_cta(n_cta + 1, 0);  // counting sort of the placements by CTA
@@ -329,8 +408,8 @@ void build_tc_plan(const Shape& s, const specgen_host_lens* lens, int n_sm, Host
     for (int i = per_cta[c]; i < per_cta[c + 1]; ++i) {
       TcItem it = by_cta[i];
       if (it.table_kind == 1) it.part += n_pre[(size_t)it.fork0 * s.hkv + it.kv_head];
-      it.table_off = host_off ? (it.table_kind == 0 ? lens->prefix_bt_offsets[it.seq]
-                                                    : lens->suffix_bt_offsets[it.seq])
+      it.table_off = host_off ? (it.table_kind == 0 ? rows.prefix_bt_offsets[it.seq]
+                                                    : rows.suffix_bt_offsets[it.seq])
                               : -1;
       hp->tc.push_back(it);
     }
@@ -339,9 +418,9 @@ void build_tc_plan(const Shape& s, const specgen_host_lens* lens, int n_sm, Host
   hp->cta_items.clear();
 }
 
-void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
+void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
   const int n_sm = device_sm_count();
-  const int32_t* fo = lens->fork_offsets;
+  const int32_t* fo = rows.trace_off.data();
   const bool tc = fork_tc_supported(s.dqk, s.dv, s.latent, s.B, s.G);
   hp->split.clear();
   hp->tc.clear();
@@ -353,7 +432,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   int slot = 0;
 
   if (tc) {
-    build_tc_plan(s, lens, n_sm, hp);
+    build_tc_plan(s, rows, n_sm, hp);
     return;
   }
 
@@ -364,16 +443,16 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
     long long work = 0;
     for (int t = 0; t < s.T; ++t)
       for (int f = fo[t]; f < fo[t + 1]; ++f)
-        work += 2LL * ((long long)lens->prefix_lens[t] + lens->suffix_lens[f]);
+        work += 2LL * ((long long)rows.prefix_lens[t] + rows.len[f]);
     long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
     chunk = std::max<long long>(4 * tt, (chunk + tt - 1) / tt * tt);
     std::vector<long long> cost;
     const long long item_overhead = 128;
     for (int t = 0; t < s.T; ++t) {
-      const int P = lens->prefix_lens[t];
+      const int P = rows.prefix_lens[t];
       const int np = (int)((P + chunk - 1) / chunk);
       for (int f = fo[t]; f < fo[t + 1]; ++f) {
-        const int S = lens->suffix_lens[f];
+        const int S = rows.len[f];
         const int ns = (int)((S + chunk - 1) / chunk);
         hp->part_base[f] = slot;
         hp->n_parts[f] = np + ns;
@@ -385,7 +464,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
             const int len = pre ? P : S;
             TcItem it;
             it.table_kind = pre ? 0 : 1;
-            it.seq = pre ? t : f;
+            it.seq = pre ? t : rows.seq[f];
             it.kv_head = 0;
             it.fork0 = f;
             it.nforks = 1;
@@ -398,7 +477,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
           }
       }
     }
-    finish_tc_plan(hp, cost, n_sm, lens);
+    finish_tc_plan(hp, cost, n_sm, rows);
     hp->total_slots = slot;
     return;
   }
@@ -412,16 +491,16 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
   long long split_tokens = 0;
   for (int t = 0; t < s.T; ++t)
     for (int f = fo[t]; f < fo[t + 1]; ++f)
-      split_tokens += (long long)lens->prefix_lens[t] + lens->suffix_lens[f];
+      split_tokens += (long long)rows.prefix_lens[t] + rows.len[f];
   const long long target_items = (long long)n_sm * 4;
   long long chunk = (split_tokens * units + target_items - 1) / std::max(1LL, target_items);
   chunk = std::max<long long>(kTileTokens, (chunk + kTileTokens - 1) / kTileTokens * kTileTokens);
   chunk = std::min<long long>(chunk, 1 << 20);
   for (int t = 0; t < s.T; ++t) {
-    const int P = lens->prefix_lens[t];
+    const int P = rows.prefix_lens[t];
     const int np = (int)((P + chunk - 1) / chunk);
     for (int f = fo[t]; f < fo[t + 1]; ++f) {
-      const int S = lens->suffix_lens[f];
+      const int S = rows.len[f];
       const int ns = (int)((S + chunk - 1) / chunk);
       hp->part_base[f] = slot;
       hp->n_parts[f] = np + ns;
@@ -439,7 +518,7 @@ void build_plan(const Shape& s, const specgen_host_lens* lens, HostPlan* hp) {
               const int cc = pre ? c : c - np;
               const int len = pre ? P : S;
               it.table_kind = pre ? 0 : 1;
-              it.seq = pre ? t : f;
+              it.seq = pre ? t : rows.seq[f];
               it.tok_begin = (int)(cc * chunk);
               it.tok_end = (int)std::min<long long>(len, (cc + 1) * chunk);
               it.slot = slot + c;
@@ -477,6 +556,9 @@ Layout layout_of(const Shape& s, const HostPlan& hp) {
 thread_local HostPlan t_plan;
 thread_local std::vector<unsigned char> t_plan_bytes;
 
+specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
+                         specgen_plan* plan, void* cuda_stream);
+
 }  // namespace
 
 extern "C" {
@@ -486,7 +568,7 @@ size_t specgen_fork_attn_workspace_size(const specgen_fork_attn_args* args,
   Shape s;
   if (check_shape(args, lens, &s) != SPECGEN_OK) return 0;
   HostPlan hp;
-  build_plan(s, lens, &hp);
+  build_plan(s, rows_for_decode(lens, s.T, s.F), &hp);
   return layout_of(s, hp).ws_end;
 }
 
@@ -498,8 +580,38 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   Shape s;
   specgen_status st = check_shape(args, lens, &s);
   if (st != SPECGEN_OK) return st;
+  return plan_impl(args, s, rows_for_decode(lens, s.T, s.F), plan, cuda_stream);
+}
+
+size_t specgen_fork_prefill_workspace_size(const specgen_fork_attn_args* args,
+                                           const specgen_prefill_lens* lens) {
+  Shape s;
+  if (check_prefill(args, lens, &s) != SPECGEN_OK) return 0;
+  HostPlan hp;
+  build_plan(s, rows_for_prefill(lens, s.T), &hp);
+  return layout_of(s, hp).ws_end;
+}
+
+specgen_status specgen_fork_prefill_plan(const specgen_fork_attn_args* args,
+                                         const specgen_prefill_lens* lens, specgen_plan* plan,
+                                         void* cuda_stream) {
+  if (!plan) return SPECGEN_ERR_NULL;
+  memset(plan, 0, sizeof(*plan));
+  Shape s;
+  specgen_status st = check_prefill(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
+  return plan_impl(args, s, rows_for_prefill(lens, s.T), plan, cuda_stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
+                         specgen_plan* plan, void* cuda_stream) {
+  specgen_status st;
   if ((st = check_pointers(args)) != SPECGEN_OK) return st;
-  build_plan(s, lens, &t_plan);
+  build_plan(s, rows, &t_plan);
   const Layout L = layout_of(s, t_plan);
   if (args->workspace_bytes < L.ws_end) return SPECGEN_ERR_WORKSPACE;
 
@@ -555,6 +667,10 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   plan->offsets[5] = (int64_t)L.n_parts_off;
   return SPECGEN_OK;
 }
+
+}  // namespace
+
+extern "C" {
 
 }  // extern "C"
 

@@ -127,3 +127,72 @@ class ForkDecode:
         torch.cuda.synchronize(self.device)
         return (self.out.float().cpu().numpy().astype(np.float64),
                 self.lse.cpu().numpy().astype(np.float64))
+
+
+class ForkPrefill:
+    """Causal prefill of every fork's newest suffix tokens (one query row per
+    chunk token) through ``specgen_fork_prefill_plan`` + ``specgen_fork_attn_run``.
+
+    ``w`` is a workload whose suffix lengths already count the chunk, plus
+    ``chunk_lens`` and ``q_rows`` (see ``workloads.make_prefill``).
+    """
+
+    def __init__(self, w: dict, device="cuda", kv_layout: int = _lib.KV_ROWS):
+        import torch
+        from . import workloads
+        self.w = w
+        self.device = torch.device(device)
+        self.kv_layout = kv_layout
+        lay = (lambda a: workloads.tile_kv_pool(a)) if kv_layout == _lib.KV_TILED else (lambda a: a)
+        self.latent = w["v_pages"] is None
+        self.q = _bf16(w["q_rows"], device)
+        self.k_pages = _bf16(lay(w["k_pages"]), device)
+        self.v_pages = None if self.latent else _bf16(lay(w["v_pages"]), device)
+        self.prefix_table = _i32(w["prefix_table"], device)
+        self.prefix_off = _i32(w["prefix_bt_offsets"], device)
+        self.suffix_table = _i32(w["suffix_table"], device)
+        self.suffix_off = _i32(w["suffix_bt_offsets"], device)
+        R, hq, dv = w["rows"], w["hq"], w["dv"]
+        self.out = torch.empty((R, hq, dv), dtype=torch.bfloat16, device=device)
+        self.lse = torch.empty((R, hq), dtype=torch.float32, device=device)
+        before = (w["suffix_lens"] - w["chunk_lens"]).astype(np.int32)
+        self.lens, self._keep = _lib.make_prefill_lens(
+            w["prefix_lens"], w["fork_offsets"], before, w["chunk_lens"],
+            w["prefix_bt_offsets"], w["suffix_bt_offsets"])
+        self.workspace, self.ws_bytes = None, 0
+        self.ws_bytes = _lib.specgen_fork_prefill_workspace_size(self.args(with_ws=False),
+                                                                 self.lens)
+        if self.ws_bytes == 0:
+            raise _lib.SpecgenError(_lib.SPECGEN_ERR_SHAPE, "specgen_fork_prefill_workspace_size")
+        self.workspace = torch.zeros(self.ws_bytes, dtype=torch.uint8, device=device)
+        self.plan_info = None
+
+    def args(self, with_ws: bool = True) -> _lib.ForkAttnArgs:
+        w = self.w
+        return _lib.make_args(
+            num_traces=w["num_traces"], total_forks=w["rows"], hq=w["hq"], hkv=w["hkv"],
+            head_dim_qk=w["dqk"], head_dim_v=w["dv"], page_size=w["page_size"],
+            num_pages=w["num_pages"], scale=w["scale"], q=self.q, k_pages=self.k_pages,
+            v_pages=self.v_pages, prefix_block_table=self.prefix_table,
+            prefix_bt_offsets=self.prefix_off, suffix_block_table=self.suffix_table,
+            suffix_bt_offsets=self.suffix_off, out=self.out, lse=self.lse,
+            workspace=self.workspace if with_ws else None,
+            workspace_bytes=self.ws_bytes if with_ws else 0, kv_layout=self.kv_layout)
+
+    def plan(self, stream: int = 0):
+        self.plan_info = _lib.specgen_fork_prefill_plan(self.args(), self.lens, stream)
+        return self.plan_info
+
+    def run(self, stream: int = 0):
+        if self.plan_info is None:
+            self.plan(stream)
+        _lib.specgen_fork_attn_run(self.args(), self.plan_info, stream)
+
+    def status(self, stream: int = 0) -> int:
+        return _lib.specgen_workspace_status(self.workspace, stream)
+
+    def results(self):
+        import torch
+        torch.cuda.synchronize(self.device)
+        return (self.out.float().cpu().numpy().astype(np.float64),
+                self.lse.cpu().numpy().astype(np.float64))
