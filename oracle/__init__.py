@@ -22,5 +22,6 @@ from .attention import (  # noqa: F401
     fork_attn_decode_rows,
     fork_attn_split_merge,
     fork_prefill,
+    fork_cascade_decode,
 )
 from .paging import append_kv, pack_pages, unpack_pages  # noqa: F401

@@ -257,3 +257,44 @@ def fork_prefill(w: dict, chunk_lens, q_rows) -> tuple[np.ndarray, np.ndarray]:
                 out_lse[r, heads] = lse
             r += 1
     return out_o, out_lse
+
+
+def fork_cascade_decode(w: dict) -> tuple[np.ndarray, np.ndarray]:
+    """Decode over a tree of shared prefix segments (repeated fork events at
+    growing prefixes, Algorithm 1: pi_1 is a prefix of pi_2 ...).
+
+    ``w`` is a fork-decode workload whose prefix tables are *segments*:
+    segment s has ``prefix_lens[s]`` tokens at pages ``prefix_table[
+    prefix_bt_offsets[s]:prefix_bt_offsets[s+1]]`` (its token 0 at slot 0 of its
+    first page) and serves the forks ``segment_rows[s][0] <= f < segment_rows[s][1]``.
+    Fork f attends to every segment that serves it and then to its own suffix;
+    the key set is a union, so the order of segments does not matter.
+    Returns O [F, hq, dv] and LSE [F, hq].
+    """
+    _check(w)
+    F, hq, dv, B = w["total_forks"], w["hq"], w["dv"], w["page_size"]
+    g_size = hq // w["hkv"]
+    seg_rows = np.asarray(w["segment_rows"]).reshape(-1, 2)
+    out_o = np.zeros((F, hq, dv))
+    out_lse = np.zeros((F, hq))
+    for f in range(F):
+        st = w["suffix_table"][w["suffix_bt_offsets"][f]:w["suffix_bt_offsets"][f + 1]]
+        for g in range(w["hkv"]):
+            ks, vs = [], []
+            for s in range(len(seg_rows)):
+                if seg_rows[s][0] <= f < seg_rows[s][1]:
+                    pt = w["prefix_table"][w["prefix_bt_offsets"][s]:w["prefix_bt_offsets"][s + 1]]
+                    k, v = _fork_kv(w["k_pages"], w.get("v_pages"), dv, B, pt,
+                                    int(w["prefix_lens"][s]), pt, 0, g)
+                    ks.append(k)
+                    vs.append(v)
+            k, v = _fork_kv(w["k_pages"], w.get("v_pages"), dv, B, st, 0, st,
+                            int(w["suffix_lens"][f]), g)
+            ks.append(k)
+            vs.append(v)
+            heads = list(range(g * g_size, (g + 1) * g_size))
+            q = bf16_bits_to_f64(w["q"][f, heads, :])
+            o, lse = attention_rows(q, np.concatenate(ks), np.concatenate(vs), w["scale"])
+            out_o[f, heads] = o
+            out_lse[f, heads] = lse
+    return out_o, out_lse

@@ -273,3 +273,69 @@ def make_prefill(w: dict, chunk: int, seed: int = 777) -> dict:
     out.update(chunk_lens=chunk_lens, rows=rows,
                q_rows=bf16_normal(rng, (rows, w["hq"], w["dqk"])))
     return out
+
+
+def make_cascade(fork_points, forks, suffix_len=(64, 512), hq=64, hkv=8, dqk=128, dv=128,
+                 page_size=16, separate_v=True, seed=9) -> dict:
+    """A reasoning trace forked repeatedly at growing, page-aligned points.
+
+    ``fork_points[i]`` is the prefix length of fork event i (increasing,
+    multiples of page_size) and ``forks[i]`` its number of forks.  Segment s
+    holds the trace's tokens [fork_points[s-1], fork_points[s]) (fork_points[-1]
+    read as 0) in its own pages and serves every fork of events >= s; forks are
+    listed deepest event first, so each segment serves a contiguous range of
+    forks (``segment_rows``, flattened [begin, end) pairs).  Suffixes, pools,
+    NaN fill and Q follow ``make_workload``.  Also returns ``flat``: the same
+    forks as an ordinary workload with one trace per event (prefix = the
+    concatenated pages of its segments) for comparisons.  Inputs only.
+    """
+    rng = np.random.default_rng(seed)
+    B = page_size
+    pts = [int(p) for p in fork_points]
+    if any(p % B or p <= 0 for p in pts) or any(b <= a for a, b in zip(pts, pts[1:])):
+        raise ValueError("fork points must be increasing positive multiples of page_size")
+    L = len(pts)
+    order = list(range(L - 1, -1, -1))                   # deepest event first
+    n_forks = [int(forks[i]) for i in order]
+    F = sum(n_forks)
+    suffix_lens = _uniform(rng, suffix_len, F)
+    s_pages = -(-suffix_lens // B)
+    n_trace = pts[-1] // B
+    num_pages = n_trace + int(s_pages.sum()) + 2
+    phys = rng.permutation(num_pages).astype(np.int32)
+    trace_pages = phys[:n_trace].copy()
+    suffix_bt_offsets = np.concatenate([[0], np.cumsum(s_pages)]).astype(np.int32)
+    suffix_table = phys[n_trace: n_trace + int(s_pages.sum())].copy()
+    sentinel_ids = phys[n_trace + int(s_pages.sum()):].copy()
+    bounds = [0] + pts
+    seg_lens = np.diff(bounds).astype(np.int32)
+    seg_bt_offsets = (np.array(bounds) // B).astype(np.int32)
+    seg_rows = []
+    for s in range(L):   # segment s serves events s..L-1, which come first in the fork order
+        seg_rows += [0, sum(int(forks[i]) for i in range(s, L))]
+    k_pages = bf16_normal(rng, (num_pages, hkv, B, dqk))
+    v_pages = bf16_normal(rng, (num_pages, hkv, B, dv)) if separate_v else None
+    q = bf16_normal(rng, (F, hq, dqk))
+    for pool in [k_pages] + ([v_pages] if v_pages is not None else []):
+        pool[sentinel_ids] = BF16_QNAN
+        for f, n in enumerate(suffix_lens):
+            used = int(n) % B
+            if used:
+                pool[suffix_table[suffix_bt_offsets[f + 1] - 1], :, used:, :] = BF16_QNAN
+    common = dict(q=q, k_pages=k_pages, v_pages=v_pages, suffix_table=suffix_table,
+                  suffix_bt_offsets=suffix_bt_offsets, suffix_lens=suffix_lens.astype(np.int32),
+                  total_forks=F, num_pages=num_pages, hq=hq, hkv=hkv, dqk=dqk, dv=dv,
+                  page_size=B, scale=1.0 / float(np.sqrt(dqk)), sentinel_ids=sentinel_ids)
+    cascade = dict(common, name="cascade", num_traces=L, prefix_table=trace_pages,
+                   prefix_bt_offsets=seg_bt_offsets, prefix_lens=seg_lens,
+                   fork_offsets=np.array([0, F], dtype=np.int32),
+                   segment_rows=np.array(seg_rows, dtype=np.int32))
+    flat_tables = [trace_pages[: pts[i] // B] for i in order]
+    flat = dict(common, name="cascade_flat", num_traces=L,
+                prefix_table=np.concatenate(flat_tables).astype(np.int32),
+                prefix_bt_offsets=np.concatenate(
+                    [[0], np.cumsum([len(t) for t in flat_tables])]).astype(np.int32),
+                prefix_lens=np.array([pts[i] for i in order], dtype=np.int32),
+                fork_offsets=np.concatenate([[0], np.cumsum(n_forks)]).astype(np.int32))
+    cascade["flat"] = flat
+    return cascade

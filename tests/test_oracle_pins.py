@@ -530,3 +530,28 @@ def test_prefill_is_causal_brute_force(seed):
             assert np.allclose(lse[r], lb[f], rtol=0, atol=1e-12)
             r += 1
     assert r == pf["rows"]
+
+
+# ----------------------------------------------------------------- nested-prefix cascade
+
+@pytest.mark.parametrize("points,forks", [((8,), (3,)), ((8, 20, 28), (2, 1, 3)),
+                                          ((4, 12), (1, 2))])
+def test_cascade_equals_flat_decode(points, forks):
+    """Forks that attend to a chain of shared segments get the decode result of
+    one flat prefix per fork event (the segments' pages concatenated)."""
+    w = wl.make_cascade(points, forks, suffix_len=(0, 9), hq=6, hkv=2, dqk=8, dv=4,
+                        page_size=4, seed=len(points))
+    o, lse = oracle.fork_cascade_decode(w)
+    o_f, lse_f = oracle.fork_attn_decode(w["flat"])
+    assert np.allclose(o, o_f, rtol=0, atol=1e-13)
+    assert np.allclose(lse[np.isfinite(lse)], lse_f[np.isfinite(lse_f)], rtol=0, atol=1e-13)
+    assert np.array_equal(np.isfinite(lse), np.isfinite(lse_f))
+
+
+def test_cascade_brute_force():
+    w = wl.make_cascade((8, 16), (2, 2), suffix_len=(1, 6), hq=4, hkv=2, dqk=8, dv=8,
+                        page_size=4, seed=1)
+    o, lse = oracle.fork_cascade_decode(w)
+    ob, lb = _brute(w["flat"])
+    assert np.allclose(o, ob, rtol=0, atol=1e-12)
+    assert np.allclose(lse, lb, rtol=0, atol=1e-12)
