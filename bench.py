@@ -44,13 +44,15 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--op", choices=["attend", "decode_step", "pack", "prefill"],
+    ap.add_argument("--op", choices=["attend", "decode_step", "pack", "prefill", "cascade"],
                     default="attend",
                     help="attend: one fork-decode attention call per step (the headline); "
                          "decode_step: append one K/V row per fork, then attend over the grown "
                          "suffixes, one plan for all steps; pack: move every trace's prefix "
                          "pages into one buffer and back (remote prefix cache); prefill: "
-                         "causal prefill of a --chunk-token prompt chunk per fork")
+                         "causal prefill of a --chunk-token prompt chunk per fork; cascade: "
+                         "decode over nested prefixes (fork events at 4096 and 8192 tokens, "
+                         "8 forks each), timed beside the same forks as flat traces")
     ap.add_argument("--chunk", type=int, default=64, help="prefill chunk tokens per fork")
     ap.add_argument("--kv-layout", choices=["rows", "tiled"], default="rows",
                     help="K/V pool layout: token-major rows (default) or 8x8 core-matrix tiles "
@@ -919,6 +921,122 @@ def run_prefill():
         dist.destroy_process_group()
 
 
+def run_cascade():
+    """--op cascade: decode over nested shared prefixes (a reasoning trace forked
+    at 4096 and at 8192 tokens, 8 forks each, GQA 64/8, head dim 128): the
+    shared segments are read once for every fork they serve.  The same forks
+    planned as flat traces (each fork event re-reading its whole prefix) are
+    timed beside it for comparison.  Plain CUDA graphs of 16 calls on rotating
+    replicas (>= 3x L2)."""
+    import ctypes as C
+
+    import torch
+
+    import __graft_entry__
+    from paper_2606_17518_gb300 import _lib, workloads as wl
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+
+    rank, local_rank, world = dist_env()
+    __graft_entry__.build()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    K, W = ARGS.steps, max(3, ARGS.warmup)
+    wc = wl.make_cascade((4096, 8192), (8, 8))
+    F = wc["total_forks"]
+    stream = torch.cuda.Stream(dev)
+    sp = stream.cuda_stream
+    props = torch.cuda.get_device_properties(dev)
+    l2 = int(getattr(props, "L2_cache_size", 126 * 2 ** 20))
+    per_graph = 16
+    lib = _lib.load()
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+
+    def measure(w, unique):
+        replicas = max(1, math.ceil(3 * l2 / unique))
+        reps = [ForkDecode(w, device=dev) for _ in range(replicas)]
+        with torch.cuda.stream(stream):
+            for r in reps:
+                r.plan(sp)
+                r.run(sp)
+        torch.cuda.synchronize(dev)
+        args = [r.args() for r in reps]
+        plans = [r.plan_info for r in reps]
+
+        def graph_of(call):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for i in range(per_graph):
+                    st = call(C.byref(args[i % replicas]), C.byref(plans[i % replicas]),
+                              C.c_void_p(sp))
+                    if st != 0:
+                        raise RuntimeError(_lib.status_string(st))
+            return g
+
+        def timed(g, steps):
+            n_rep = max(1, -(-steps // per_graph))
+            a, b = ev(), ev()
+            with torch.cuda.stream(stream):
+                a.record(stream)
+                for _ in range(n_rep):
+                    g.replay()
+                b.record(stream)
+            torch.cuda.synchronize(dev)
+            return a.elapsed_time(b) / (n_rep * per_graph)
+
+        g = graph_of(lib.specgen_fork_attn_run)
+        timed(g, W)
+        clocks = ClockSampler(local_rank)
+        clocks.start()
+        step = timed(g, K)
+        clk = clocks.stop()
+        part = timed(graph_of(lib.specgen_fork_attn_run_partials), K)
+        merge = timed(graph_of(lib.specgen_fork_attn_run_merge), K)
+        if reps[0].status(sp) != 0:
+            raise RuntimeError("cascade decode reported an error")
+        return step, part, merge, clk
+
+    page_bytes = wc["hkv"] * wc["page_size"] * (wc["dqk"] + wc["dv"]) * 2
+    seg_bytes = int(np.sum(wc["prefix_lens"])) // wc["page_size"] * page_bytes
+    flat_bytes = int(np.sum(wc["flat"]["prefix_lens"])) // wc["page_size"] * page_bytes
+    sfx_bytes = int(np.sum(-(-wc["suffix_lens"] // wc["page_size"]))) * page_bytes
+    q_bytes = wc["q"].size * 2
+    alg = seg_bytes + sfx_bytes + q_bytes
+    step, part, merge, clk = measure(wc, alg)
+    f_step, f_part, _, _ = measure(wc["flat"], flat_bytes + sfx_bytes + q_bytes)
+    hbm, _, _, peak_src = measured_peaks()
+    achieved = alg / (part * 1e-3) / 1e9
+    line = {
+        "metric": "fork-decode attention tokens/s (nested prefixes)",
+        "value": world * F / (step * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "steps": per_graph * max(1, -(-K // per_graph)), "warmup": W, "ms_per_step": step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": "cascade_p4k_p8k_f8x2", "op": "cascade",
+                   "fork_points": [4096, 8192], "forks": [8, 8],
+                   "algorithmic_bytes": alg, "flat_prefix_bytes": flat_bytes,
+                   "flat_ms_per_step": f_step, "flat_kernel_ms": f_part,
+                   "speedup_vs_flat": f_step / step,
+                   "timing": "CUDA graphs of 16 calls; per-kernel times from graphs of each "
+                             "stage alone"},
+        "gpu_launches": 2 * per_graph * max(1, -(-K // per_graph)),
+        "kernels": {"fork_tc": {"ms_per_launch": part}, "lse_merge": {"ms_per_launch": merge}},
+        "roofline": {"bound": "hbm", "kernel": "fork_tc", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                     "peak_source": peak_src, "algorithmic_bytes_per_launch": alg},
+        "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
 def main():
     if os.environ.get("SPECGEN_ORACLE_CHILD"):
         return
@@ -930,6 +1048,8 @@ def main():
         run_pack()
     elif ARGS.op == "prefill":
         run_prefill()
+    elif ARGS.op == "cascade":
+        run_cascade()
     else:
         run_ours()
 

@@ -245,6 +245,35 @@ specgen_status specgen_fork_prefill_plan(const specgen_fork_attn_args* args,
                                          const specgen_prefill_lens* lens, specgen_plan* plan,
                                          void* cuda_stream);
 
+/* ---- Nested-prefix cascade -------------------------------------------------
+ * Fork events taken repeatedly along one reasoning trace, at growing prefixes
+ * pi_1, pi_2, ... (Algorithm 1 triggers speculation again and again), give a
+ * tree of shared prefix segments.  Segment s holds segment_lens[s] tokens in
+ * prefix table s (args->prefix_block_table / prefix_bt_offsets are indexed by
+ * segment; token 0 sits at slot 0 of the segment's first page, so a fork point
+ * inside a page leaves that page's tail to each fork's own suffix) and serves
+ * the forks [segment_rows[2s], segment_rows[2s+1]).  Fork f attends to every
+ * segment that serves it, then to its own suffix.  The ranges must be laminar
+ * (any two nested or disjoint: number the forks depth-first); each segment's
+ * pages are then read once for up to 128 / (hq / hkv) forks, not once per fork
+ * event.  args: num_traces = num_segments, everything else as for decode
+ * (args->suffix_lens may cut suffixes).  Run the plan with
+ * specgen_fork_attn_run; same status codes as the decode entry points. */
+typedef struct {
+  int num_segments;
+  const int32_t* segment_lens;       /* host [num_segments], >= 0 */
+  const int32_t* segment_rows;       /* host [2 * num_segments]: [begin, end) of forks */
+  const int32_t* suffix_lens;        /* host [total_forks], >= 0 */
+  const int32_t* segment_bt_offsets; /* host [num_segments + 1] or NULL */
+  const int32_t* suffix_bt_offsets;  /* host [total_forks + 1] or NULL */
+} specgen_cascade_lens;
+
+size_t specgen_fork_cascade_workspace_size(const specgen_fork_attn_args* args,
+                                           const specgen_cascade_lens* lens);
+specgen_status specgen_fork_cascade_plan(const specgen_fork_attn_args* args,
+                                         const specgen_cascade_lens* lens, specgen_plan* plan,
+                                         void* cuda_stream);
+
 /* ---- Decode-step append --------------------------------------------------
  * After a fork event every fork decodes its own continuation while the prefix
  * stays shared (Algorithm 1, "Fork K spec. generations"; Section 4.2), so each

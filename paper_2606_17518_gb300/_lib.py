@@ -32,6 +32,8 @@ EXPORTED = [
     "specgen_fork_attn_run_profiled",
     "specgen_fork_attn_run_partials",
     "specgen_fork_attn_run_merge",
+    "specgen_fork_cascade_workspace_size",
+    "specgen_fork_cascade_plan",
     "specgen_fork_prefill_workspace_size",
     "specgen_fork_prefill_plan",
     "specgen_fork_attn_decode",
@@ -97,6 +99,12 @@ class PrefillLens(C.Structure):
                 ("prefix_bt_offsets", C.c_void_p), ("suffix_bt_offsets", C.c_void_p)]
 
 
+class CascadeLens(C.Structure):
+    _fields_ = [("num_segments", C.c_int), ("segment_lens", C.c_void_p),
+                ("segment_rows", C.c_void_p), ("suffix_lens", C.c_void_p),
+                ("segment_bt_offsets", C.c_void_p), ("suffix_bt_offsets", C.c_void_p)]
+
+
 class Plan(C.Structure):
     _fields_ = [
         ("valid", C.c_int32), ("n_tc_items", C.c_int32), ("n_tc_ctas", C.c_int32),
@@ -132,6 +140,11 @@ def load() -> C.CDLL:
     lib.specgen_fork_attn_plan.argtypes = [P(ForkAttnArgs), P(HostLens), P(Plan), C.c_void_p]
     lib.specgen_fork_attn_run.restype = C.c_int
     lib.specgen_fork_attn_run.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
+    lib.specgen_fork_cascade_workspace_size.restype = C.c_size_t
+    lib.specgen_fork_cascade_workspace_size.argtypes = [P(ForkAttnArgs), P(CascadeLens)]
+    lib.specgen_fork_cascade_plan.restype = C.c_int
+    lib.specgen_fork_cascade_plan.argtypes = [P(ForkAttnArgs), P(CascadeLens), P(Plan),
+                                              C.c_void_p]
     lib.specgen_fork_prefill_workspace_size.restype = C.c_size_t
     lib.specgen_fork_prefill_workspace_size.argtypes = [P(ForkAttnArgs), P(PrefillLens)]
     lib.specgen_fork_prefill_plan.restype = C.c_int
@@ -251,6 +264,29 @@ def make_prefill_lens(prefix_lens, fork_offsets, suffix_lens, chunk_lens,
            for a in (prefix_bt_offsets, suffix_bt_offsets)]
     ptrs = [a.ctypes.data for a in keep] + [None if a is None else a.ctypes.data for a in opt]
     return PrefillLens(*ptrs), keep + opt
+
+
+def make_cascade_lens(segment_lens, segment_rows, suffix_lens, segment_bt_offsets=None,
+                      suffix_bt_offsets=None):
+    """CascadeLens over host int32 copies; returns (struct, keepalive)."""
+    keep = [np.ascontiguousarray(a, dtype=np.int32)
+            for a in (segment_lens, segment_rows, suffix_lens)]
+    opt = [None if a is None else np.ascontiguousarray(a, dtype=np.int32)
+           for a in (segment_bt_offsets, suffix_bt_offsets)]
+    return CascadeLens(len(keep[0]), keep[0].ctypes.data, keep[1].ctypes.data,
+                       keep[2].ctypes.data, *[None if a is None else a.ctypes.data
+                                              for a in opt]), keep + opt
+
+
+def specgen_fork_cascade_workspace_size(args: ForkAttnArgs, lens: CascadeLens) -> int:
+    return int(load().specgen_fork_cascade_workspace_size(C.byref(args), C.byref(lens)))
+
+
+def specgen_fork_cascade_plan(args: ForkAttnArgs, lens: CascadeLens, stream: int = 0) -> Plan:
+    plan = Plan()
+    _check(load().specgen_fork_cascade_plan(C.byref(args), C.byref(lens), C.byref(plan),
+                                            C.c_void_p(stream)), "specgen_fork_cascade_plan")
+    return plan
 
 
 def specgen_fork_prefill_workspace_size(args: ForkAttnArgs, lens: PrefillLens) -> int:

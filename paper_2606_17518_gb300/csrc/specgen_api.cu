@@ -9,6 +9,8 @@
 #include <string.h>
 
 #include <algorithm>
+#include <map>
+#include <tuple>
 #include <queue>
 #include <utility>
 #include <vector>
@@ -142,23 +144,69 @@ struct HostPlan {
   int total_slots = 0;
 };
 
-// The query rows a plan serves, trace by trace.  Decode: one row per fork.
-// Prefill: one row per new token of every fork; row j of fork f attends to the
-// fork's first S_f + j + 1 suffix tokens (its earlier tokens and, causally, the
-// chunk up to itself).  A row reads the suffix table of fork `seq`.
+// A shared prefix segment: `len` tokens in prefix table `index` (its token 0 at
+// slot 0 of the table's first page), attended to by the query rows
+// [row_begin, row_end).  Decode and prefill have one segment per trace; a
+// cascade (repeated fork events at growing prefixes) has nested segments.
+struct Segment {
+  int len, row_begin, row_end;
+};
+
+// The query rows a plan serves.  Decode: one row per fork.  Prefill: one row per
+// new token of every fork; row j of fork f attends to the fork's first
+// S_f + j + 1 suffix tokens (its earlier tokens and, causally, the chunk up to
+// itself).  A row reads the suffix table of fork `seq`.
 struct Rows {
-  const int32_t* prefix_lens = nullptr;        // host [T]
-  std::vector<int32_t> trace_off;              // [T + 1]
+  std::vector<Segment> segs;
   std::vector<int32_t> seq;                    // [R]
   std::vector<int32_t> len;                    // [R]
   const int32_t* prefix_bt_offsets = nullptr;  // optional host copies of the table offsets
   const int32_t* suffix_bt_offsets = nullptr;
+  // Derived by order_segments: enclosing segments before enclosed ones, each
+  // segment's enclosing chain (outermost first) and its outermost segment.
+  std::vector<int> order, root;
+  std::vector<std::vector<int>> anc;
 };
+
+// Segment ranges must be laminar (any two nested or disjoint); checked by the
+// callers that accept nested segments.
+void order_segments(Rows* r) {
+  const int n = (int)r->segs.size();
+  r->order.resize(n);
+  for (int i = 0; i < n; ++i) r->order[i] = i;
+  std::stable_sort(r->order.begin(), r->order.end(), [&](int x, int y) {
+    const Segment &a = r->segs[x], &b = r->segs[y];
+    return a.row_begin < b.row_begin || (a.row_begin == b.row_begin && a.row_end > b.row_end);
+  });
+  r->root.assign(n, 0);
+  r->anc.assign(n, std::vector<int>());
+  std::vector<int> stack;
+  for (int s : r->order) {
+    const Segment& g = r->segs[s];
+    while (!stack.empty() && r->segs[stack.back()].row_end <= g.row_begin) stack.pop_back();
+    while (!stack.empty() && r->segs[stack.back()].row_end < g.row_end) stack.pop_back();
+    r->anc[s] = stack;
+    r->root[s] = stack.empty() ? s : stack.front();
+    stack.push_back(s);
+  }
+}
+
+bool laminar(const std::vector<Segment>& segs) {
+  for (size_t i = 0; i < segs.size(); ++i)
+    for (size_t j = i + 1; j < segs.size(); ++j) {
+      const Segment &a = segs[i], &b = segs[j];
+      const bool disjoint = a.row_end <= b.row_begin || b.row_end <= a.row_begin;
+      const bool nested = (a.row_begin <= b.row_begin && b.row_end <= a.row_end) ||
+                          (b.row_begin <= a.row_begin && a.row_end <= b.row_end);
+      if (!disjoint && !nested) return false;
+    }
+  return true;
+}
 
 Rows rows_for_decode(const specgen_host_lens* lens, int T, int F) {
   Rows r;
-  r.prefix_lens = lens->prefix_lens;
-  r.trace_off.assign(lens->fork_offsets, lens->fork_offsets + T + 1);
+  for (int t = 0; t < T; ++t)
+    r.segs.push_back(Segment{lens->prefix_lens[t], lens->fork_offsets[t], lens->fork_offsets[t + 1]});
   r.seq.resize(F);
   r.len.assign(lens->suffix_lens, lens->suffix_lens + F);
   for (int f = 0; f < F; ++f) r.seq[f] = f;
@@ -166,26 +214,63 @@ Rows rows_for_decode(const specgen_host_lens* lens, int T, int F) {
     r.prefix_bt_offsets = lens->prefix_bt_offsets;
     r.suffix_bt_offsets = lens->suffix_bt_offsets;
   }
+  order_segments(&r);
   return r;
 }
 
 Rows rows_for_prefill(const specgen_prefill_lens* lens, int T) {
   Rows r;
-  r.prefix_lens = lens->prefix_lens;
   const int32_t* fo = lens->fork_offsets;
-  r.trace_off.assign(1, 0);
   for (int t = 0; t < T; ++t) {
+    const int begin = (int)r.seq.size();
     for (int f = fo[t]; f < fo[t + 1]; ++f)
       for (int j = 0; j < lens->chunk_lens[f]; ++j) {
         r.seq.push_back(f);
         r.len.push_back(lens->suffix_lens[f] + j + 1);  // causal within the chunk
       }
-    r.trace_off.push_back((int32_t)r.seq.size());
+    r.segs.push_back(Segment{lens->prefix_lens[t], begin, (int)r.seq.size()});
   }
   if (lens->prefix_bt_offsets && lens->suffix_bt_offsets) {
     r.prefix_bt_offsets = lens->prefix_bt_offsets;
     r.suffix_bt_offsets = lens->suffix_bt_offsets;
   }
+  order_segments(&r);
+  return r;
+}
+
+specgen_status check_cascade(const specgen_fork_attn_args* a, const specgen_cascade_lens* lens,
+                             Shape* s) {
+  if (!a || !lens || !lens->segment_lens || !lens->segment_rows || !lens->suffix_lens)
+    return SPECGEN_ERR_NULL;
+  const specgen_status st = check_common(a, s);
+  if (st != SPECGEN_OK) return st;
+  if (lens->num_segments != a->num_traces) return SPECGEN_ERR_SHAPE;
+  std::vector<Segment> segs;
+  for (int i = 0; i < lens->num_segments; ++i) {
+    const Segment g{lens->segment_lens[i], lens->segment_rows[2 * i], lens->segment_rows[2 * i + 1]};
+    if (g.len < 0 || g.row_begin < 0 || g.row_end < g.row_begin || g.row_end > a->total_forks)
+      return SPECGEN_ERR_SHAPE;
+    segs.push_back(g);
+  }
+  if (!laminar(segs)) return SPECGEN_ERR_SHAPE;
+  for (int f = 0; f < a->total_forks; ++f)
+    if (lens->suffix_lens[f] < 0) return SPECGEN_ERR_SHAPE;
+  return SPECGEN_OK;
+}
+
+Rows rows_for_cascade(const specgen_cascade_lens* lens, int F) {
+  Rows r;
+  for (int s = 0; s < lens->num_segments; ++s)
+    r.segs.push_back(Segment{lens->segment_lens[s], lens->segment_rows[2 * s],
+                             lens->segment_rows[2 * s + 1]});
+  r.seq.resize(F);
+  r.len.assign(lens->suffix_lens, lens->suffix_lens + F);
+  for (int f = 0; f < F; ++f) r.seq[f] = f;
+  if (lens->segment_bt_offsets && lens->suffix_bt_offsets) {
+    r.prefix_bt_offsets = lens->segment_bt_offsets;
+    r.suffix_bt_offsets = lens->suffix_bt_offsets;
+  }
+  order_segments(&r);
   return r;
 }
 
@@ -321,21 +406,31 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
 }
 
 void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
-  const int32_t* fo = rows.trace_off.data();
   const int page = fork_tc_page_size();
   const int forks_per_item = std::max(1, 128 / s.G);
+  const int R = (int)rows.seq.size();
+  // Prefix units: the rows of a segment in groups of forks_per_item, on the grid
+  // of its outermost enclosing segment, so that every row of a group sees the
+  // same groups (and chunk counts) in the segments that enclose this one.
+  auto group_of = [&](int seg, int f) {
+    return (f - rows.segs[rows.root[seg]].row_begin) / forks_per_item;
+  };
   std::vector<TcUnit> sfx, pfx;
   long long total = 0;
-  for (int t = 0; t < s.T; ++t) {
-    for (int g = 0; g < s.hkv; ++g) {
-      if (rows.prefix_lens[t] > 0)
-        for (int f0 = fo[t]; f0 < fo[t + 1]; f0 += forks_per_item)
-          pfx.push_back(TcUnit{0, t, g, f0, std::min(forks_per_item, fo[t + 1] - f0),
-                               rows.prefix_lens[t]});
-      for (int f = fo[t]; f < fo[t + 1]; ++f)
-        if (rows.len[f] > 0) sfx.push_back(TcUnit{1, rows.seq[f], g, f, 1, rows.len[f]});
-    }
+  for (int sg = 0; sg < (int)rows.segs.size(); ++sg) {
+    const Segment& seg = rows.segs[sg];
+    if (seg.len <= 0) continue;
+    const int r0 = rows.segs[rows.root[sg]].row_begin;
+    for (int g = 0; g < s.hkv; ++g)
+      for (int f0 = seg.row_begin; f0 < seg.row_end;) {
+        const int f1 = std::min(seg.row_end, r0 + (group_of(sg, f0) + 1) * forks_per_item);
+        pfx.push_back(TcUnit{0, sg, g, f0, f1 - f0, seg.len});
+        f0 = f1;
+      }
   }
+  for (int g = 0; g < s.hkv; ++g)
+    for (int f = 0; f < R; ++f)
+      if (rows.len[f] > 0) sfx.push_back(TcUnit{1, rows.seq[f], g, f, 1, rows.len[f]});
   for (const TcUnit& u : sfx) total += u.len;
   for (const TcUnit& u : pfx) total += u.len;
   auto longer = [](const TcUnit& a, const TcUnit& b) { return a.len > b.len; };
@@ -366,17 +461,36 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     }
     pack_tc(sfx, pfx, n_cta, hi, page, &load, &order, &placed);
   }
-  // partial slots: per (fork, head group) the prefix chunks come first, then
-  // the suffix pieces; a fork owns as many slots as its busiest head group
+  // Partial slots: per (row, head group) the prefix chunks come first (segment
+  // by segment, enclosing segments first), then the suffix pieces; a row owns
+  // as many slots as its busiest head group.  A prefix chunk's part is the
+  // chunk index plus the chunks of the enclosing segments' same-row groups.
   hp->n_groups = s.hkv;
   hp->n_parts.assign((size_t)s.F * s.hkv, 0);
+  std::map<std::tuple<int, int, int>, int> chunks;  // (segment, head, group) -> chunk count
   std::vector<int32_t> n_pre((size_t)s.F * s.hkv, 0), n_suf((size_t)s.F * s.hkv, 0);
   for (const TcPlacement& pl : placed) {
     const TcItem& it = pl.item;
-    for (int f = it.fork0; f < it.fork0 + it.nforks; ++f) {
-      int32_t& n = (it.table_kind == 0 ? n_pre : n_suf)[(size_t)f * s.hkv + it.kv_head];
+    if (it.table_kind == 0) {
+      int& c = chunks[std::make_tuple(it.seq, it.kv_head, group_of(it.seq, it.fork0))];
+      c = std::max(c, it.part + 1);
+    } else {
+      int32_t& n = n_suf[(size_t)it.fork0 * s.hkv + it.kv_head];
       n = std::max(n, it.part + 1);
     }
+  }
+  auto base_of = [&](int seg, int g, int f) {  // chunks of the enclosing segments for row f
+    int b = 0;
+    for (int a : rows.anc[seg]) {
+      auto q = chunks.find(std::make_tuple(a, g, group_of(a, f)));
+      if (q != chunks.end()) b += q->second;
+    }
+    return b;
+  };
+  for (const TcUnit& u : pfx) {
+    auto q = chunks.find(std::make_tuple(u.seq, u.g, group_of(u.seq, u.fork0)));
+    const int c = q == chunks.end() ? 0 : q->second;
+    for (int f = u.fork0; f < u.fork0 + u.nforks; ++f) n_pre[(size_t)f * s.hkv + u.g] += c;
   }
   int slot = 0;
   for (int f = 0; f < s.F; ++f) {
@@ -407,7 +521,10 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     if (per_cta[c + 1] == per_cta[c]) continue;  // empty CTAs are dropped
     for (int i = per_cta[c]; i < per_cta[c + 1]; ++i) {
       TcItem it = by_cta[i];
-      if (it.table_kind == 1) it.part += n_pre[(size_t)it.fork0 * s.hkv + it.kv_head];
+      if (it.table_kind == 1)
+        it.part += n_pre[(size_t)it.fork0 * s.hkv + it.kv_head];
+      else
+        it.part += base_of(it.seq, it.kv_head, it.fork0);
       it.table_off = host_off ? (it.table_kind == 0 ? rows.prefix_bt_offsets[it.seq]
                                                     : rows.suffix_bt_offsets[it.seq])
                               : -1;
@@ -420,8 +537,8 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
 
 void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
   const int n_sm = device_sm_count();
-  const int32_t* fo = rows.trace_off.data();
   const bool tc = fork_tc_supported(s.dqk, s.dv, s.latent, s.B, s.G);
+  const int R = (int)rows.seq.size();
   hp->split.clear();
   hp->tc.clear();
   hp->cta_items.clear();
@@ -436,97 +553,106 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
     return;
   }
 
+  // The non-tensor-core planners give every row its own items: the segments
+  // that serve a row (enclosing ones first), then its suffix.
+  std::vector<std::vector<int>> serving(R);
+  for (int sg : rows.order)
+    if (rows.segs[sg].len > 0)
+      for (int f = rows.segs[sg].row_begin; f < rows.segs[sg].row_end; ++f) serving[f].push_back(sg);
+
   if (mla_tc_supported(s.dqk, s.dv, s.latent, s.B, s.hq, s.hkv)) {
-    // Latent-KV tensor-core path: one item = one fork's 128 heads x one value
-    // half x a chunk of its prefix or suffix; chunks are whole tiles.
+    // Latent-KV tensor-core path: one item = one row's 128 heads x one value
+    // half x a chunk of a prefix segment or of its suffix; chunks are whole tiles.
     const int tt = mla_tc_tile_tokens();
     long long work = 0;
-    for (int t = 0; t < s.T; ++t)
-      for (int f = fo[t]; f < fo[t + 1]; ++f)
-        work += 2LL * ((long long)rows.prefix_lens[t] + rows.len[f]);
+    for (int f = 0; f < R; ++f) {
+      long long keys = rows.len[f];
+      for (int sg : serving[f]) keys += rows.segs[sg].len;
+      work += 2LL * keys;
+    }
     long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
     chunk = std::max<long long>(4 * tt, (chunk + tt - 1) / tt * tt);
     std::vector<long long> cost;
     const long long item_overhead = 128;
-    for (int t = 0; t < s.T; ++t) {
-      const int P = rows.prefix_lens[t];
-      const int np = (int)((P + chunk - 1) / chunk);
-      for (int f = fo[t]; f < fo[t + 1]; ++f) {
-        const int S = rows.len[f];
-        const int ns = (int)((S + chunk - 1) / chunk);
-        hp->part_base[f] = slot;
-        hp->n_parts[f] = np + ns;
-        slot += np + ns;
-        for (int c = 0; c < np + ns; ++c)
-          for (int half = 0; half < 2; ++half) {
-            const bool pre = c < np;
-            const int cc = pre ? c : c - np;
-            const int len = pre ? P : S;
-            TcItem it;
-            it.table_kind = pre ? 0 : 1;
-            it.seq = pre ? t : rows.seq[f];
-            it.kv_head = 0;
-            it.fork0 = f;
-            it.nforks = 1;
-            it.tok_begin = (int)(cc * chunk);
-            it.tok_end = (int)std::min<long long>(len, (cc + 1) * chunk);
-            it.part = c;
-            it.dv0 = half * 256;
-            hp->tc.push_back(it);
-            cost.push_back(it.tok_end - it.tok_begin + item_overhead);
-          }
-      }
+    auto emit = [&](int kind, int seq, int f, int len, int part0) {
+      const int n = (int)((len + chunk - 1) / chunk);
+      for (int c = 0; c < n; ++c)
+        for (int half = 0; half < 2; ++half) {
+          TcItem it;
+          it.table_kind = kind;
+          it.seq = seq;
+          it.kv_head = 0;
+          it.fork0 = f;
+          it.nforks = 1;
+          it.tok_begin = (int)(c * chunk);
+          it.tok_end = (int)std::min<long long>(len, (c + 1) * chunk);
+          it.part = part0 + c;
+          it.dv0 = half * 256;
+          hp->tc.push_back(it);
+          cost.push_back(it.tok_end - it.tok_begin + item_overhead);
+        }
+      return n;
+    };
+    for (int f = 0; f < R; ++f) {
+      int parts = 0;
+      for (int sg : serving[f]) parts += emit(0, sg, f, rows.segs[sg].len, parts);
+      parts += emit(1, rows.seq[f], f, rows.len[f], parts);
+      hp->part_base[f] = slot;
+      hp->n_parts[f] = parts;
+      slot += parts;
     }
     finish_tc_plan(hp, cost, n_sm, rows);
     hp->total_slots = slot;
     return;
   }
 
-  // Split-K path (shapes the tensor-core kernels do not cover): every fork
-  // reads its trace's prefix and its own suffix in chunks of whole tiles.
+  // Split-K path (shapes the tensor-core kernels do not cover): every row reads
+  // its prefix segments and its own suffix in chunks of whole tiles.
   const int dvt = split_dv_tile(s.dqk, s.dv, s.latent);
   const int row_blocks = (s.G + kRowBlock - 1) / kRowBlock;
   const int dv_blocks = s.dv / dvt;
   const long long units = (long long)s.hkv * row_blocks * dv_blocks;
   long long split_tokens = 0;
-  for (int t = 0; t < s.T; ++t)
-    for (int f = fo[t]; f < fo[t + 1]; ++f)
-      split_tokens += (long long)rows.prefix_lens[t] + rows.len[f];
+  for (int f = 0; f < R; ++f) {
+    split_tokens += rows.len[f];
+    for (int sg : serving[f]) split_tokens += rows.segs[sg].len;
+  }
   const long long target_items = (long long)n_sm * 4;
   long long chunk = (split_tokens * units + target_items - 1) / std::max(1LL, target_items);
   chunk = std::max<long long>(kTileTokens, (chunk + kTileTokens - 1) / kTileTokens * kTileTokens);
   chunk = std::min<long long>(chunk, 1 << 20);
-  for (int t = 0; t < s.T; ++t) {
-    const int P = rows.prefix_lens[t];
-    const int np = (int)((P + chunk - 1) / chunk);
-    for (int f = fo[t]; f < fo[t + 1]; ++f) {
-      const int S = rows.len[f];
-      const int ns = (int)((S + chunk - 1) / chunk);
-      hp->part_base[f] = slot;
-      hp->n_parts[f] = np + ns;
-      for (int g = 0; g < s.hkv; ++g)
-        for (int rb = 0; rb < row_blocks; ++rb)
-          for (int db = 0; db < dv_blocks; ++db) {
-            SplitItem it;
-            it.fork = f;
-            it.kv_head = g;
-            it.h0 = g * s.G + rb * kRowBlock;
-            it.nrows = std::min(kRowBlock, s.G - rb * kRowBlock);
-            it.dv0 = db * dvt;
-            for (int c = 0; c < np + ns; ++c) {
-              const bool pre = c < np;
-              const int cc = pre ? c : c - np;
-              const int len = pre ? P : S;
-              it.table_kind = pre ? 0 : 1;
-              it.seq = pre ? t : rows.seq[f];
-              it.tok_begin = (int)(cc * chunk);
-              it.tok_end = (int)std::min<long long>(len, (cc + 1) * chunk);
-              it.slot = slot + c;
+  for (int f = 0; f < R; ++f) {
+    // (kind, table, length) of every key range of this row, in slot order
+    std::vector<std::tuple<int, int, int>> ranges;
+    for (int sg : serving[f]) ranges.push_back(std::make_tuple(0, sg, rows.segs[sg].len));
+    ranges.push_back(std::make_tuple(1, (int)rows.seq[f], (int)rows.len[f]));
+    int parts = 0;
+    for (auto& r : ranges) parts += (int)((std::get<2>(r) + chunk - 1) / chunk);
+    hp->part_base[f] = slot;
+    hp->n_parts[f] = parts;
+    for (int g = 0; g < s.hkv; ++g)
+      for (int rb = 0; rb < row_blocks; ++rb)
+        for (int db = 0; db < dv_blocks; ++db) {
+          SplitItem it;
+          it.fork = f;
+          it.kv_head = g;
+          it.h0 = g * s.G + rb * kRowBlock;
+          it.nrows = std::min(kRowBlock, s.G - rb * kRowBlock);
+          it.dv0 = db * dvt;
+          int part = 0;
+          for (auto& r : ranges) {
+            const int len = std::get<2>(r);
+            for (long long c = 0; c * chunk < len; ++c, ++part) {
+              it.table_kind = std::get<0>(r);
+              it.seq = std::get<1>(r);
+              it.tok_begin = (int)(c * chunk);
+              it.tok_end = (int)std::min<long long>(len, (c + 1) * chunk);
+              it.slot = slot + part;
               hp->split.push_back(it);
             }
           }
-      slot += np + ns;
-    }
+        }
+    slot += parts;
   }
   hp->total_slots = slot;
 }
@@ -581,6 +707,26 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   specgen_status st = check_shape(args, lens, &s);
   if (st != SPECGEN_OK) return st;
   return plan_impl(args, s, rows_for_decode(lens, s.T, s.F), plan, cuda_stream);
+}
+
+size_t specgen_fork_cascade_workspace_size(const specgen_fork_attn_args* args,
+                                           const specgen_cascade_lens* lens) {
+  Shape s;
+  if (check_cascade(args, lens, &s) != SPECGEN_OK) return 0;
+  HostPlan hp;
+  build_plan(s, rows_for_cascade(lens, s.F), &hp);
+  return layout_of(s, hp).ws_end;
+}
+
+specgen_status specgen_fork_cascade_plan(const specgen_fork_attn_args* args,
+                                         const specgen_cascade_lens* lens, specgen_plan* plan,
+                                         void* cuda_stream) {
+  if (!plan) return SPECGEN_ERR_NULL;
+  memset(plan, 0, sizeof(*plan));
+  Shape s;
+  specgen_status st = check_cascade(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
+  return plan_impl(args, s, rows_for_cascade(lens, s.F), plan, cuda_stream);
 }
 
 size_t specgen_fork_prefill_workspace_size(const specgen_fork_attn_args* args,

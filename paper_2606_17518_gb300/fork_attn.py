@@ -55,6 +55,7 @@ class ForkDecode:
         # when True the kernels cut suffix items to suffix_lens_dev (a plan made
         # for longer host lengths then serves several decode steps)
         self.use_device_lens = False
+        self.cascade = "segment_rows" in w
         self.set_suffix_lens(w["suffix_lens"])
 
     def set_suffix_lens(self, suffix_lens, update_device: bool = True):
@@ -64,10 +65,16 @@ class ForkDecode:
         import torch
         w = self.w
         w["suffix_lens"] = np.ascontiguousarray(suffix_lens, dtype=np.int32)
-        self.lens, self._lens_keep = _lib.make_host_lens(
-            w["prefix_lens"], w["fork_offsets"], w["suffix_lens"], w["prefix_bt_offsets"],
-            w["suffix_bt_offsets"])
-        need = _lib.specgen_fork_attn_workspace_size(self.args(with_ws=False), self.lens)
+        if self.cascade:   # prefix tables are nested segments serving ranges of forks
+            self.lens, self._lens_keep = _lib.make_cascade_lens(
+                w["prefix_lens"], w["segment_rows"], w["suffix_lens"], w["prefix_bt_offsets"],
+                w["suffix_bt_offsets"])
+            need = _lib.specgen_fork_cascade_workspace_size(self.args(with_ws=False), self.lens)
+        else:
+            self.lens, self._lens_keep = _lib.make_host_lens(
+                w["prefix_lens"], w["fork_offsets"], w["suffix_lens"], w["prefix_bt_offsets"],
+                w["suffix_bt_offsets"])
+            need = _lib.specgen_fork_attn_workspace_size(self.args(with_ws=False), self.lens)
         if need == 0:
             raise _lib.SpecgenError(_lib.SPECGEN_ERR_SHAPE, "specgen_fork_attn_workspace_size")
         if need > self.ws_bytes:
@@ -107,7 +114,8 @@ class ForkDecode:
         return _lib.make_args(**kw)
 
     def plan(self, stream: int = 0):
-        self.plan_info = _lib.specgen_fork_attn_plan(self.args(), self.lens, stream)
+        planner = _lib.specgen_fork_cascade_plan if self.cascade else _lib.specgen_fork_attn_plan
+        self.plan_info = planner(self.args(), self.lens, stream)
         return self.plan_info
 
     def run(self, stream: int = 0):
@@ -116,6 +124,10 @@ class ForkDecode:
         _lib.specgen_fork_attn_run(self.args(), self.plan_info, stream)
 
     def decode(self, stream: int = 0):
+        if self.cascade:
+            self.plan(stream)
+            self.run(stream)
+            return
         _lib.specgen_fork_attn_decode(self.args(), self.lens, stream)
 
     def status(self, stream: int = 0) -> int:
