@@ -7,25 +7,35 @@
 // private suffix (M = G rows).  Each item writes a partial (O / l, LSE) per row.
 //
 // Per 128-token tile t (8 pages of 16 tokens), with t counted across items:
-//   warp 0 (TMA)     K_t, V_t pages -> 2-stage shared-memory ring (two 64-column
-//                    boxes per page, 128B swizzle), byte-counted on full[t%2]
-//   warp 1 (MMA)     S_t = Q K_t^T -> TMEM S[t%2]   (M=128, N=16*pages, K=D)
-//                    O  += P_t V_t -> TMEM O         (M=128, N=D,  K=16*pages)
-//   warps 2-5        one thread per row (= TMEM lane): the 128 scores of the
-//                    tile in registers, masked where needed, running max kept
-//                    in log2 units; P_t = exp2(s*scale*log2e - m) to shared
-//                    memory as bf16 (128B-swizzled, K-major); the TMEM output
-//                    is rescaled only when a row's max grows by more than
-//                    2^8 (lazy rescaling), otherwise P may exceed 1.
+//   warp 0 (TMA)     K_t pages -> K ring, byte-counted on k_full[t%ST]
+//   warp 10 (TMA)    V_t pages -> V ring, byte-counted on v_full[t%ST]
+//   warp 1 (MMA)     S_t = Q K_t^T -> TMEM S[t%2]   (M=128, N=16*pages, K=D);
+//                    the K stage is released as soon as S_t has finished
+//                    O  += P_t V_t -> TMEM O         (M=128, N=D,  K=16*pages);
+//                    then the V stage is released
+//   warps 2-9        two groups of 4 warps on alternate tiles, one thread per
+//                    row (= TMEM lane): the 128 scores of the tile in
+//                    registers, masked where needed, running max kept in log2
+//                    units; P_t = exp2(s*scale*log2e - m) back to TMEM as bf16;
+//                    the TMEM output is rescaled only when a row's max grows
+//                    by more than 2^8 (lazy rescaling), otherwise P may exceed 1.
 // S is double-buffered in TMEM so S_{t+1} runs while tile t is in softmax.
+// Separate K and V rings keep more bytes in flight: a K stage is held only
+// until its score MMA is done, a V stage until its PV product is done.  Every
+// copy issue costs the issuing warp a roughly fixed time, so the copies are as
+// large as the layouts allow and all copies of a tile leave in one warp
+// instruction.
 //
 // Two KV pool layouts.  Rows: every (page, head) block is 16 token rows of D
-// contiguous elements; the TMA engine gathers it with 64-column boxes into
-// 128B-swizzled panels.  Tiled: every block is stored as the tensor cores'
-// 8-token x 8-element core matrices, ((t/8)*(D/8) + d/8)*64 + (t%8)*8 + d%8,
-// so one contiguous bulk copy (D*32 bytes) lands it in the layout the MMA
-// reads directly (no swizzle): K is then K-major with 128-byte steps along d
-// and D*16-byte steps per 8 tokens, V is MN-major with the same two strides.
+// contiguous elements.  K is gathered with one 64-column TMA box per panel and
+// page into 128B-swizzled panels of the whole tile (the score MMA needs every
+// panel's tokens at one stride); V with one box per page that holds all its
+// panels ([page][panel][16 rows], which the PV MMA reads page by page).
+// Tiled: every block is stored as the tensor cores' 8-token x 8-element core
+// matrices, ((t/8)*(D/8) + d/8)*64 + (t%8)*8 + d%8, so one contiguous bulk copy
+// (D*32 bytes) lands it in the layout the MMA reads directly (no swizzle): K is
+// then K-major with 128-byte steps along d and D*16-byte steps per 8 tokens, V
+// is MN-major with the same two strides.
 // Warps whose 32 rows are all padding skip the softmax work.  Tokens past the
 // item, past the sequence or on an invalid page are masked to -inf, and value
 // rows past the sequence inside its last page are zeroed in shared memory
@@ -48,7 +58,8 @@ using namespace tc;
 
 constexpr int kPB = 16;                      // page size (tokens)
 constexpr int kWG = 2;                       // softmax warpgroups (alternating tiles)
-constexpr int kThreads = 64 + 128 * kWG;     // warp 0 TMA, warp 1 MMA, 4 warps per softmax group
+constexpr int kVWarp = 2 + 4 * kWG;          // the V copy warp, after the softmax groups
+constexpr int kThreads = 32 * (kVWarp + 1);  // warp 0 K copies, warp 1 MMA, 4 warps per softmax group, V copies
 constexpr uint32_t kTmemCols = 512;          // S[0] [0,TT) S[1] [TT,2TT) O[0] [256,..) O[1] [384,..)
 constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleLog2 = 8.0f;         // lazy-rescale threshold (factor 256)
@@ -56,10 +67,11 @@ constexpr int kMaxStages = 4;
 constexpr int kTile = 128;                   // tokens per pipeline tile (8 pages)
 
 // Shared memory of one CTA: Q (128 rows x D, non-swizzled 8x8 core matrices:
-// LBO 128 B along d, SBO D*16 B per 8 rows), a ring of `ST` (K, V) stages of
-// TT tokens (rows layout: 64-column panels of 128-byte rows, 128B-swizzled;
-// tiled layout: the pool's own core-matrix tiles), barriers, the per-stage
-// valid-page masks, the second group's (m, l) and the CTA's first items.
+// LBO 128 B along d, SBO D*16 B per 8 rows), a ring of `ST` K stages and one of
+// `ST` V stages of TT tokens each (rows layout: 128B-swizzled 64-column panels,
+// K as [panel][TT rows], V as [page][panel][16 rows]; tiled layout: the pool's
+// own core-matrix blocks, page after page), barriers, the per-stage valid-page
+// masks, the second group's (m, l) and the CTA's first items.
 constexpr int kItemCache = 16;
 
 template <int D, int TT, int ST, bool TL>
@@ -68,9 +80,10 @@ struct Smem {
   static constexpr uint32_t kQ = 128u * D * 2u;
   static constexpr uint32_t kRowsTile = TT * 128u;        // one 64-column panel of TT rows
   static constexpr uint32_t kKV = kPanels * kRowsTile;    // one K or V tile (TT x D bf16)
-  static constexpr uint32_t kStage = 2 * kKV;
-  static constexpr uint32_t kOffKV = kQ;
-  static constexpr uint32_t kOffBar = kOffKV + ST * kStage;
+  static constexpr uint32_t kBlk = kPB * D * 2u;          // one (page, head) block
+  static constexpr uint32_t kOffK = kQ;
+  static constexpr uint32_t kOffV = kOffK + ST * kKV;
+  static constexpr uint32_t kOffBar = kOffV + ST * kKV;
   static constexpr uint32_t kOffML = kOffBar + 256;        // 128 x (m, l) of the second group
   static constexpr uint32_t kOffItems = kOffML + 128 * 8;
   static constexpr uint32_t kAlign = TL ? 128u : 1024u;    // 128B-swizzled tiles: 1024-B aligned
@@ -128,6 +141,8 @@ template <int D, int TT, int ST, bool TL>
 __global__ void __launch_bounds__(kThreads, 1)
     fork_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tmk,
                    const __grid_constant__ CUtensorMap tmv) {
+  // tmk: 4-D map, one 64-column panel of one (page, head) block per box;
+  // tmv: the same for D = 64, else a 5-D map whose box is a whole block.
   using L = Smem<D, TT, ST, TL>;
   constexpr int kPagesPerTile = TT / kPB;
   static_assert(32 % kPagesPerTile == 0, "a batch of 32 page ids holds whole tiles");
@@ -137,29 +152,35 @@ __global__ void __launch_bounds__(kThreads, 1)
   unsigned char* gbase = smem_raw + (base - raw);
   const uint32_t sQ = base;
   const uint32_t bar0 = base + L::kOffBar;
-  // barrier block: full[ST] empty[ST] s_full[2] p_full[2] o_full[2] q_ready mma_done
-  // ml_ready q_free merge_done ml_back, then the TMEM address, the abort flag
-  // and the per-stage valid-page masks
-  auto full = [&](int s) { return bar0 + 8u * s; };
-  auto empty = [&](int s) { return bar0 + 8u * (kMaxStages + s); };
-  auto s_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + b); };
-  auto p_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 2 + b); };
-  auto o_full = [&](int b) { return bar0 + 8u * (2 * kMaxStages + 4 + b); };
-  const uint32_t q_ready = bar0 + 8u * (2 * kMaxStages + 6);     // Q of the next item stored
-  const uint32_t mma_done = bar0 + 8u * (2 * kMaxStages + 7);
-  const uint32_t ml_ready = bar0 + 8u * (2 * kMaxStages + 8);    // group 1's (m, l) written
-  const uint32_t q_free = bar0 + 8u * (2 * kMaxStages + 9);      // an item's last S finished
-  const uint32_t merge_done = bar0 + 8u * (2 * kMaxStages + 10); // group 1 read its O halves
-  const uint32_t ml_back = bar0 + 8u * (2 * kMaxStages + 11);    // group 0's weights written
-  constexpr int kMisc = 8 * (2 * kMaxStages + 12);
+  // barrier block: k_full[4] k_empty[4] v_full[4] v_empty[4] s_full[2] p_full[2]
+  // o_full[2] q_ready mma_done ml_ready q_free merge_done ml_back, then the TMEM
+  // address, the abort flag, the per-stage valid-page masks (K copy warp -> MMA)
+  // and the per-score-buffer masks (MMA -> softmax)
+  auto k_full = [&](int s) { return bar0 + 8u * s; };
+  auto k_empty = [&](int s) { return bar0 + 8u * (kMaxStages + s); };
+  auto v_full = [&](int s) { return bar0 + 8u * (2 * kMaxStages + s); };
+  auto v_empty = [&](int s) { return bar0 + 8u * (3 * kMaxStages + s); };
+  constexpr int kB = 4 * kMaxStages;
+  auto s_full = [&](int b) { return bar0 + 8u * (kB + b); };
+  auto p_full = [&](int b) { return bar0 + 8u * (kB + 2 + b); };
+  auto o_full = [&](int b) { return bar0 + 8u * (kB + 4 + b); };
+  const uint32_t q_ready = bar0 + 8u * (kB + 6);     // Q of the next item stored
+  const uint32_t mma_done = bar0 + 8u * (kB + 7);
+  const uint32_t ml_ready = bar0 + 8u * (kB + 8);    // group 1's (m, l) written
+  const uint32_t q_free = bar0 + 8u * (kB + 9);      // an item's last S finished
+  const uint32_t merge_done = bar0 + 8u * (kB + 10); // group 1 read its O halves
+  const uint32_t ml_back = bar0 + 8u * (kB + 11);    // group 0's weights written
+  constexpr int kMisc = 8 * (kB + 12);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + L::kOffBar + kMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(gbase + L::kOffBar + kMisc + 4);
   volatile uint32_t* smask = reinterpret_cast<volatile uint32_t*>(gbase + L::kOffBar + kMisc + 8);
-  static_assert(kMisc + 8 + 4 * kMaxStages <= 256, "barrier block");
+  volatile uint32_t* smask_s =
+      reinterpret_cast<volatile uint32_t*>(gbase + L::kOffBar + kMisc + 8 + 4 * kMaxStages);
+  static_assert(kMisc + 8 + 4 * kMaxStages + 8 <= 256, "barrier block");
   float2* ml1 = reinterpret_cast<float2*>(gbase + L::kOffML);  // second group's (m, l) per row
   TcItem* items = reinterpret_cast<TcItem*>(gbase + L::kOffItems);
-  auto sK = [&](int s) { return base + L::kOffKV + s * L::kStage; };
-  auto sV = [&](int s) { return base + L::kOffKV + s * L::kStage + L::kKV; };
+  auto sK = [&](int s) { return base + L::kOffK + s * L::kKV; };
+  auto sV = [&](int s) { return base + L::kOffV + s * L::kKV; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
@@ -168,23 +189,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   // for this grid's completion before it reads anything
   if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
+  // the CTA's first items, one per lane (40-byte records): the plan is written
+  // by a host copy, never by a kernel, so it is read before the wait below
+  constexpr int kWords = sizeof(TcItem) / 4;
+  const int n_cached = n_items < kItemCache ? n_items : kItemCache;
   if (warp == 0) {
-    // the CTA's first items, one per lane (40-byte records)
-    constexpr int kWords = sizeof(TcItem) / 4;
-    const int nw = (n_items < kItemCache ? n_items : kItemCache) * kWords;
     const int32_t* src = reinterpret_cast<const int32_t*>(p.items + it_begin);
     int32_t* dst = reinterpret_cast<int32_t*>(items);
-    for (int x = lane; x < nw; x += 32) dst[x] = src[x];
-    __syncwarp();
-    for (int k = lane; k < nw / kWords; k += 32) items[k] = clamp_item(items[k], p.suffix_lens);
+    for (int x = lane; x < n_cached * kWords; x += 32) dst[x] = src[x];
   }
   if (threadIdx.x == 32) {
     for (int i = 0; i < ST; ++i) {
-      mbar_init(full(i), 1);
-      mbar_init(empty(i), 1);
+      mbar_init(k_full(i), 1);
+      mbar_init(k_empty(i), 1);
+      mbar_init(v_full(i), 1);
+      mbar_init(v_empty(i), 1);
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(s_full(i), 1);
+      // the score MMAs' commit, and the MMA thread once it has stored the tile's mask
+      mbar_init(s_full(i), 2);
       mbar_init(p_full(i), 128);
       mbar_init(o_full(i), 1);
     }
@@ -201,24 +224,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
   }
+  // Launched as a programmatic dependent, this grid may start while the previous
+  // kernel of the stream is still running: everything above touches only this
+  // CTA's own resources and the plan.  The inputs (device lengths, block tables,
+  // Q, K/V, possibly written by that kernel) and the partial buffers (possibly
+  // still read by it) are used only after this wait.
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  if (warp == 0) {
+    __syncwarp();
+    for (int k = lane; k < n_cached; k += 32) items[k] = clamp_item(items[k], p.suffix_lens);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer
-    // The whole warp fetches page ids 32 at a time (one coalesced load, one
-    // batch ahead, and the next item's first batch one item ahead).  Lane 0
-    // waits for a free stage and publishes the tile's valid-page mask; then
-    // the issuing lanes copy K and V of every page (rows layout: one TMA box per
-    // 64-column panel; tiled layout: one bulk copy per page).
-    constexpr int kIssuers = TL ? 2 * kPagesPerTile : 2 * L::kPanels;
-    const bool issuer = lane < kIssuers;
-    const bool is_v = lane >= L::kPanels;
-    const int pn = is_v ? lane - L::kPanels : lane;
-    const void* tmap = is_v ? static_cast<const void*>(&tmv) : static_cast<const void*>(&tmk);
-    int t = 0;  // tiles issued so far (across items)
+  if (warp == 0 || warp == kVWarp) {
+    // ------------------------------------------------------------ copy warps
+    // Warp 0 copies K tiles, warp kVWarp V tiles, each through its own ring.
+    // Both fetch page ids 32 at a time (one coalesced load, one batch ahead, and
+    // the next item's first batch one item ahead).  Lane 0 waits for a free
+    // stage (the K warp also publishes the tile's valid-page mask); then one
+    // lane per copy issues all copies of the tile in one instruction.
+    const bool is_v = warp == kVWarp;
+    const int pg = lane % kPagesPerTile;  // the page this lane copies
+    int t = 0;                            // tiles issued so far (across items)
     bool ok = true;
     int first_next = n_items > 0 ? page_batch(p, get_item(items, p, it_begin, 0), 0, lane) : 0;
     for (int k = 0; ok && k < n_items; ++k) {
@@ -232,56 +262,54 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int tp = 0; tp < batch_pages; tp += kPagesPerTile, ++t) {
           const int j = (pb + tp) / kPagesPerTile;  // tile index within the item
           const int np = (tile_tokens<TT>(it, j) + kPB - 1) / kPB;
-          int pages[kPagesPerTile];
-          uint32_t valid = 0;
-#pragma unroll
-          for (int pg = 0; pg < kPagesPerTile; ++pg) {
-            pages[pg] = __shfl_sync(0xffffffffu, cur, tp + pg);
-            if (pg < np && pages[pg] >= 0 && pages[pg] < p.num_pages) valid |= 1u << pg;
-          }
+          const int page = __shfl_sync(0xffffffffu, cur, tp + pg);
+          const bool page_ok = pg < np && page >= 0 && page < p.num_pages;
+          const uint32_t valid = __ballot_sync(0xffffffffu, page_ok && lane < kPagesPerTile);
           const uint32_t bad = ((1u << np) - 1u) & ~valid;
           const int s = t % ST;
+          const uint32_t fbar = is_v ? v_full(s) : k_full(s);
           if (lane == 0) {
-            ok = mbar_wait(empty(s), ((t / ST) & 1) ^ 1, abort_flag, p.status);
-            if (ok) smask[s] = valid;
-            if (bad) atomicOr(p.status, kStatusIndex);
+            ok = mbar_wait(is_v ? v_empty(s) : k_empty(s), ((t / ST) & 1) ^ 1, abort_flag,
+                           p.status);
+            if (ok && !is_v) smask[s] = valid;
+            if (bad && !is_v) atomicOr(p.status, kStatusIndex);
           }
           ok = __shfl_sync(0xffffffffu, ok, 0);
           if (!ok) break;
           if constexpr (TL) {
-            // one bulk copy per (page, K or V); an invalid page's value block is
-            // zeroed here instead (its scores are masked)
-            constexpr uint32_t kBlk = kPB * D * 2u;
-            if (bad) {
-              for (int pg = 0; pg < np; ++pg)
-                if ((bad >> pg) & 1u)
-                  for (uint32_t x = lane * 16u; x < kBlk; x += 32u * 16u)
-                    st_shared_v4(sV(s) + pg * kBlk + x, 0u, 0u, 0u, 0u);
+            // one bulk copy per page; an invalid page's value block is zeroed
+            // here instead (its scores are masked)
+            if (is_v && bad) {
+              for (int q = 0; q < np; ++q)
+                if ((bad >> q) & 1u)
+                  for (uint32_t x = lane * 16u; x < L::kBlk; x += 32u * 16u)
+                    st_shared_v4(sV(s) + q * L::kBlk + x, 0u, 0u, 0u, 0u);
               fence_proxy_async_smem();
               __syncwarp();
             }
-            if (lane == 0) mbar_arrive_expect_tx(full(s), (uint32_t)__popc(valid) * 2u * kBlk);
+            if (lane == 0) mbar_arrive_expect_tx(fbar, (uint32_t)__popc(valid) * L::kBlk);
             __syncwarp();
-            const int pg = lane % kPagesPerTile;
-            if (issuer && ((valid >> pg) & 1u)) {
-              const bool v_side = lane >= kPagesPerTile;
-              const __nv_bfloat16* src = (v_side ? p.v_pages : p.k_pages) +
-                                         ((size_t)pages[pg] * p.hkv + it.kv_head) * (kPB * D);
-              bulk_load((v_side ? sV(s) : sK(s)) + pg * kBlk, src, kBlk, full(s));
+            if (lane < kPagesPerTile && ((valid >> pg) & 1u)) {
+              const __nv_bfloat16* src = (is_v ? p.v_pages : p.k_pages) +
+                                         ((size_t)page * p.hkv + it.kv_head) * (kPB * D);
+              bulk_load((is_v ? sV(s) : sK(s)) + pg * L::kBlk, src, L::kBlk, fbar);
             }
           } else {
             // TMA zero-fills out-of-range pages, so every box counts
-            if (lane == 0)
-              mbar_arrive_expect_tx(full(s), (uint32_t)np * 2u * L::kPanels * (kPB * 128u));
+            if (lane == 0) mbar_arrive_expect_tx(fbar, (uint32_t)np * L::kBlk);
             __syncwarp();
-            if (issuer) {
-              const uint32_t dst = (is_v ? sV(s) : sK(s)) + pn * L::kRowsTile;
-#pragma unroll
-              for (int pg = 0; pg < kPagesPerTile; ++pg) {
-                if (pg >= np) break;
-                tma_load_4d(dst + pg * (kPB * 128u), tmap, pn * 64, 0, it.kv_head, pages[pg],
-                            full(s));
+            if (is_v) {
+              if (lane < kPagesPerTile && pg < np) {
+                if constexpr (L::kPanels > 1)
+                  tma_load_5d(sV(s) + pg * L::kBlk, &tmv, 0, 0, 0, it.kv_head, page, fbar);
+                else
+                  tma_load_4d(sV(s) + pg * L::kBlk, &tmv, 0, 0, it.kv_head, page, fbar);
               }
+            } else {
+              const int pn = lane / kPagesPerTile;  // this lane's 64-column panel
+              if (pn < L::kPanels && pg < np)
+                tma_load_4d(sK(s) + pn * L::kRowsTile + pg * (kPB * 128u), &tmk, pn * 64, 0,
+                            it.kv_head, page, fbar);
             }
           }
         }
@@ -291,7 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // never leave a copy in flight into this CTA's shared memory
     if (lane == 0)
       for (int u = t - ST < 0 ? 0 : t - ST; u < t; ++u)
-        mbar_wait_drain(full(u % ST), (u / ST) & 1, p.status);
+        mbar_wait_drain(is_v ? v_full(u % ST) : k_full(u % ST), (u / ST) & 1, p.status);
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -302,11 +330,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       // (LBO = next 8 tokens, SBO = next 8 columns)
       const uint64_t dk0 = TL ? smem_desc_interleave(sK(0), 128, D * 16)
                               : smem_desc_sw128(sK(0), 16, 1024);
+      // rows: V panels of one page are 16 rows x 128 B apart (LBO), 8-token
+      // groups 1024 B apart (SBO)
       const uint64_t dv0 = TL ? smem_desc_interleave(sV(0), D * 16, 128)
-                              : smem_desc_sw128(sV(0), L::kRowsTile, 1024);
-      // byte step of V per page (one 16-token k-step)
-      constexpr uint32_t kVPage = TL ? kPB * D * 2u : kPB * 128u;
-      constexpr uint64_t kStageDesc = L::kStage >> 4;
+                              : smem_desc_sw128(sV(0), kPB * 128u, 1024);
+      // byte step of V per page (one 16-token k-step): one block in both layouts
+      constexpr uint32_t kVPage = L::kBlk;
+      constexpr uint64_t kStageDesc = L::kKV >> 4;
       constexpr uint32_t idesc_pv = idesc_bf16(128, D, true);
       // Ready-first issue: PV_v goes out as soon as its P is ready; S_u goes
       // out when its K tile has landed, its score buffer is free (PV_{u-2}
@@ -338,7 +368,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             s_nt = view<TT>(p, s_it).ntiles;
           }
           did = true;
-        } else if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1)) {
+        } else if (v_u < s_u && mbar_test_wait(p_full(v_u & 1), (v_u >> 1) & 1) &&
+                   mbar_test_wait(v_full(v_u % ST), (v_u / ST) & 1)) {
           tc_fence_after();
           const int b = v_u & 1, s = v_u % ST;
           const int np = (tile_tokens<TT>(v_it, v_j) + kPB - 1) / kPB;
@@ -357,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                           idesc_pv, (acc0 | (kk > 0)) ? 1u : 0u);
           }
           mma_commit(o_full(b));
-          mma_commit(empty(s));
+          mma_commit(v_empty(s));
           ++v_u;
           if (++v_j == v_nt) {
             v_j = 0;
@@ -371,9 +402,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           did = true;
         } else if (s_k < n_items && s_nt > 0 && s_u - v_u < 2) {
           if (!q_ok && mbar_test_wait(q_ready, s_k & 1)) q_ok = true;
-          if (q_ok && mbar_test_wait(full(s_u % ST), (s_u / ST) & 1)) {
+          if (q_ok && mbar_test_wait(k_full(s_u % ST), (s_u / ST) & 1)) {
             tc_fence_after();
             const int b = s_u & 1, s = s_u % ST;
+            // the tile's page mask for the softmax (its previous reader, two
+            // tiles back, is done: PV_{u-2} has been issued)
+            smask_s[b] = smask[s];
+            mbar_arrive(s_full(b));
             const int np = (tile_tokens<TT>(s_it, s_j) + kPB - 1) / kPB;
             const uint32_t idesc = idesc_bf16(128, np * kPB, false);
             const uint64_t dk = dk0 + (uint64_t)s * kStageDesc;
@@ -385,6 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               mma_bf16(d_s, dq + (uint64_t)((kk * 256u) >> 4), dk + ko, idesc, kk > 0 ? 1u : 0u);
             }
             mma_commit(s_full(b));
+            mma_commit(k_empty(s));
             ++s_u;
             if (++s_j == s_nt) {
               mma_commit(q_free);
@@ -467,13 +503,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       // group 1 stores Q of the first item here, of every later item at the end
       // of the previous one (as soon as that item's last S has finished)
       if (grp == 1 && k == 0) store_q();
+      // and asks L2 for the next item's Q rows now, so that loading them at this
+      // item's end (on the path to the next item's first score MMA) hits L2
+      if (grp == 1 && k + 1 < n_items) {
+        const TcItem nx = get_item(items, p, it_begin, k + 1);
+        if (row < nx.nforks * p.G) {
+          const char* qrow = reinterpret_cast<const char*>(
+              p.q + ((size_t)(nx.fork0 + row / p.G) * p.hq + nx.kv_head * p.G + row % p.G) * D);
+#pragma unroll
+          for (int c = 0; c < D * 2; c += 128)
+            asm volatile("prefetch.global.L2 [%0];\n" ::"l"(qrow + c));
+        }
+      }
 
       float m = -INFINITY, l = 0.f;  // this group's running max (log2 units) and sum
       for (int j = grp; j < ntiles; j += 2) {
         const int u = t + j, b = u & 1, s = u % ST;
-        bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
-        // the tile's valid-page mask (published before its copies were counted)
-        w = w && mbar_wait(full(s), (u / ST) & 1, abort_flag, p.status);
+        const bool w = mbar_wait(s_full(b), (u >> 1) & 1, abort_flag, p.status);
         if (__any_sync(0xffffffffu, !w)) {
           ok = false;
           break;
@@ -485,7 +531,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nt = tile_tokens<TT>(it, j);
         const int np = (nt + kPB - 1) / kPB;
         if (warp_live) {
-          const uint32_t pv = smask[s];  // valid pages of this tile
+          const uint32_t pv = smask_s[b];  // valid pages of this tile
           float sc[TT];
           {
             uint32_t r[TT / 32][32];
@@ -554,7 +600,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_wait_st();
         }
         // value rows past the sequence inside its last page: zero them before PV
+        // (once the V tile has landed; its stage cannot be refilled before this
+        // group's p_full, so the phase is still the current one)
         if (j == ntiles - 1 && (nt % kPB) != 0) {
+          if (!mbar_wait(v_full(s), (u / ST) & 1, abort_flag, p.status)) ok = false;
           const int pg = np - 1, first = nt % kPB;
           const int units = (kPB - first) * L::kPanels * 8;  // 16-byte pieces
           for (int x = gtid; x < units; x += 128) {
@@ -562,7 +611,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int rem = x % (L::kPanels * 8);  // 8-column chunk of the row
             const int tt = pg * kPB + rr;
             const uint32_t off = TL ? ((tt >> 3) * (D / 8) + rem) * 128u + (tt & 7) * 16u
-                                    : (rem >> 3) * L::kRowsTile + tt * 128u + ((rem & 7) << 4);
+                                    : pg * L::kBlk + (rem >> 3) * (kPB * 128u) + rr * 128u +
+                                          ((rem & 7) << 4);
             st_shared_v4(sV(s) + off, 0u, 0u, 0u, 0u);
           }
           fence_proxy_async_smem();
@@ -705,6 +755,25 @@ bool make_pool_map(CUtensorMap* map, const void* pool, int D, int page, int hkv,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Value map of the rows layout: (64 columns, page rows, D/64 panels, hkv, pages)
+// with the panel stride (128 B) inside the row stride, so one box is one whole
+// (page, head) block, landing in shared memory as [panel][page rows], 128-byte
+// swizzled.  D = 64 has one panel: the key map serves.
+bool make_pool_map_v(CUtensorMap* map, const void* pool, int D, int page, int hkv, int num_pages) {
+  if (D == 64) return make_pool_map(map, pool, D, page, hkv, num_pages);
+  EncodeTiledFn enc = encode_fn();
+  if (!enc || !pool || num_pages < 1) return false;
+  const cuuint64_t dims[5] = {64, (cuuint64_t)page, (cuuint64_t)(D / 64), (cuuint64_t)hkv,
+                              (cuuint64_t)num_pages};
+  const cuuint64_t strides[4] = {(cuuint64_t)D * 2, 128, (cuuint64_t)page * D * 2,
+                                 (cuuint64_t)hkv * page * D * 2};
+  const cuuint32_t box[5] = {64, (cuuint32_t)page, (cuuint32_t)(D / 64), 1, 1};
+  const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(pool), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int D, int TT, int ST, bool TL>
 cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap& mv, int grid,
                      cudaStream_t stream) {
@@ -725,8 +794,19 @@ cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap
     if (e != cudaSuccess) return e;
     configured = dev;
   }
-  kern<<<grid, kThreads, smem, stream>>>(p, mk, mv);
-  return cudaGetLastError();
+  // programmatic dependent launch: the grid may start while the previous kernel
+  // of the stream finishes (the kernel waits for it before touching its inputs)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, p, mk, mv);
 }
 
 }  // namespace
@@ -753,7 +833,7 @@ cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v
     return cudaErrorInvalidValue;
   }
   if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
-      !make_pool_map(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
+      !make_pool_map_v(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
     return cudaErrorInvalidValue;
   if (dqk == 128) return launch_d<128, kTile, 3, false>(p, mk, mv, grid, stream);
   if (dqk == 64) return launch_d<64, kTile, 4, false>(p, mk, mv, grid, stream);

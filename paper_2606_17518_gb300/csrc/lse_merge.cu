@@ -40,6 +40,9 @@ __device__ __forceinline__ float warp_sum(float v) {
 constexpr int kMergeThreads = 128;  // small blocks can sit beside a running tensor-core CTA
 
 __global__ void __launch_bounds__(kMergeThreads) merge_parts_kernel(const MergeParams p) {
+  // the next kernel of the stream may get launched now (it waits for this grid
+  // before it uses anything this grid writes or reads)
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
   const int c4n = p.dv / 4;
   const int gid = blockIdx.x * kMergeThreads + threadIdx.x;
