@@ -72,7 +72,7 @@ constexpr int kTile = 128;                   // tokens per pipeline tile (8 page
 // K as [panel][TT rows], V as [page][panel][16 rows]; tiled layout: the pool's
 // own core-matrix blocks, page after page), barriers, the per-stage valid-page
 // masks, the second group's (m, l) and the CTA's first items.
-constexpr int kItemCache = 16;
+constexpr int kItemCache = 14;
 
 template <int D, int TT, int ST, bool TL>
 struct Smem {
@@ -84,7 +84,7 @@ struct Smem {
   static constexpr uint32_t kOffK = kQ;
   static constexpr uint32_t kOffV = kOffK + ST * kKV;
   static constexpr uint32_t kOffBar = kOffV + ST * kKV;
-  static constexpr uint32_t kOffML = kOffBar + 256;        // 128 x (m, l) of the second group
+  static constexpr uint32_t kOffML = kOffBar + 320;        // 128 x (m, l) of the second group
   static constexpr uint32_t kOffItems = kOffML + 128 * 8;
   static constexpr uint32_t kAlign = TL ? 128u : 1024u;    // 128B-swizzled tiles: 1024-B aligned
   static constexpr uint32_t kBytes = kOffItems + kItemCache * (uint32_t)sizeof(TcItem) + kAlign;
@@ -176,7 +176,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile uint32_t* smask = reinterpret_cast<volatile uint32_t*>(gbase + L::kOffBar + kMisc + 8);
   volatile uint32_t* smask_s =
       reinterpret_cast<volatile uint32_t*>(gbase + L::kOffBar + kMisc + 8 + 4 * kMaxStages);
-  static_assert(kMisc + 8 + 4 * kMaxStages + 8 <= 256, "barrier block");
+  // K tiles issued so far: the V copy warp never runs ahead of it, so that at
+  // the start the copies leave in the order the tiles are consumed
+  volatile int* k_issued =
+      reinterpret_cast<volatile int*>(gbase + L::kOffBar + kMisc + 16 + 4 * kMaxStages);
+  static_assert(kMisc + 20 + 4 * kMaxStages <= 320, "barrier block");
   float2* ml1 = reinterpret_cast<float2*>(gbase + L::kOffML);  // second group's (m, l) per row
   TcItem* items = reinterpret_cast<TcItem*>(gbase + L::kOffItems);
   auto sK = [&](int s) { return base + L::kOffK + s * L::kKV; };
@@ -218,6 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(merge_done, 128);
     mbar_init(ml_back, 128);
     *abort_flag = 0;
+    *k_issued = 0;
     mbar_init_fence();
   }
   if (warp == 1) {
@@ -273,6 +278,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                            p.status);
             if (ok && !is_v) smask[s] = valid;
             if (bad && !is_v) atomicOr(p.status, kStatusIndex);
+            if (ok && is_v && *k_issued <= t) {  // bounded wait for K_t to be issued
+              const unsigned long long w0 = globaltimer();
+              while (*k_issued <= t) {
+                if (*abort_flag) {
+                  ok = false;
+                  break;
+                }
+                if (globaltimer() - w0 > kWaitLimitNs) {
+                  atomicOr(p.status, kStatusTimeout);
+                  *abort_flag = 1;
+                  ok = false;
+                  break;
+                }
+              }
+            }
           }
           ok = __shfl_sync(0xffffffffu, ok, 0);
           if (!ok) break;
@@ -312,6 +332,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                             it.kv_head, page, fbar);
             }
           }
+          __syncwarp();
+          if (!is_v && lane == 0) *k_issued = t + 1;
         }
         cur = nxt;
       }
