@@ -324,11 +324,12 @@ void finish_tc_plan(HostPlan* hp, const std::vector<long long>& cost, int n_sm,
 
 // Budget packing of the tensor-core work.  A unit is one kv head of either a
 // fork's suffix (cut only when it alone exceeds the budget) or a group of forks'
-// shared prefix (cut freely at page boundaries).  Under a per-CTA budget T, in
+// shared prefix (cut freely at tile boundaries).  Under a per-CTA budget T, in
 // token-equivalents with kItemCost per item, one pass deals the suffix pieces
 // (longest first) over the CTAs in snake order, then visits the CTAs from the
 // least loaded up and fills each one's spare budget with prefix chunks.  The
-// plan takes the smallest budget for which the prefix fits.
+// plan takes the smallest budget for which the prefix fits.  An item costs its
+// whole tiles: a partial tile takes the pipeline as long as a full one.
 constexpr long long kItemCost = 384;  // fixed cost of an item (Q staging, merge, pipeline refill)
 constexpr int kMinChunk = 128;        // smallest prefix chunk carved into a CTA's spare budget
 
@@ -344,14 +345,15 @@ struct TcPlacement {
 // One packing pass under budget T.  `load` and `order` are caller-owned
 // scratch; `out` (when given) receives the items with their CTAs.
 bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int n_cta,
-             long long T, int page, std::vector<long long>* load, std::vector<int>* order,
+             long long T, int tt, std::vector<long long>* load, std::vector<int>* order,
              std::vector<TcPlacement>* out) {
   load->assign(n_cta, 0);
   if (out) out->clear();
-  const long long lmax = (T - kItemCost) / page * page;
-  if (lmax < page) return false;
+  const long long lmax = (T - kItemCost) / tt * tt;
+  if (lmax < tt) return false;
+  auto tiles = [&](long long n) { return (n + tt - 1) / tt * tt; };  // tokens of whole tiles
   auto place = [&](int cta, const TcUnit& u, int b, int e, int part) {
-    (*load)[cta] += (e - b) + kItemCost;
+    (*load)[cta] += tiles(e - b) + kItemCost;
     if (!out) return;
     TcPlacement pl;
     pl.cta = cta;
@@ -371,7 +373,7 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
   long long k_dealt = 0;  // suffix pieces dealt so far (snake order over the CTAs)
   for (const TcUnit& u : sfx) {
     const long long k = (u.len + lmax - 1) / lmax;
-    const int piece = (int)(((u.len + k - 1) / k + page - 1) / page * page);
+    const int piece = (int)tiles((u.len + k - 1) / k);
     for (int c = 0, pos = 0; pos < u.len; ++c, pos += piece, ++k_dealt) {
       const long long round = k_dealt / n_cta, i = k_dealt % n_cta;
       place((int)(round & 1 ? n_cta - 1 - i : i), u, pos, std::min(u.len, pos + piece), c);
@@ -388,7 +390,7 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
     while (ui < pfx.size()) {
       const TcUnit& u = pfx[ui];
       const int rem = u.len - pos;
-      const long long spare = (T - (*load)[cta] - kItemCost) / page * page;
+      const long long spare = (T - (*load)[cta] - kItemCost) / tt * tt;
       if (spare < std::min(kMinChunk, rem)) break;  // this CTA is full
       long long len = std::min<long long>(rem, spare);
       if (rem - len < kMinChunk / 2) len = rem;  // leave no sliver behind
@@ -406,7 +408,7 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
 }
 
 void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
-  const int page = fork_tc_page_size();
+  const int tt = fork_tc_tile_tokens();
   const int forks_per_item = std::max(1, 128 / s.G);
   const int R = (int)rows.seq.size();
   // Prefix units: the rows of a segment in groups of forks_per_item, on the grid
@@ -431,7 +433,7 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   for (int g = 0; g < s.hkv; ++g)
     for (int f = 0; f < R; ++f)
       if (rows.len[f] > 0) sfx.push_back(TcUnit{1, rows.seq[f], g, f, 1, rows.len[f]});
-  for (const TcUnit& u : sfx) total += u.len;
+  for (const TcUnit& u : sfx) total += (u.len + tt - 1) / tt * tt;
   for (const TcUnit& u : pfx) total += u.len;
   auto longer = [](const TcUnit& a, const TcUnit& b) { return a.len > b.len; };
   std::stable_sort(sfx.begin(), sfx.end(), longer);
@@ -446,20 +448,20 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     std::vector<long long> load;
     std::vector<int> order;
     const long long n_items = (long long)sfx.size() + std::max<long long>((long long)pfx.size(), n_cta);
-    long long lo = std::max<long long>(kItemCost + page, (total + kItemCost * n_items) / n_cta);
+    long long lo = std::max<long long>(kItemCost + tt, (total + kItemCost * n_items) / n_cta);
     long long hi = lo;
-    while (!pack_tc(sfx, pfx, n_cta, hi, page, &load, &order, nullptr)) {
+    while (!pack_tc(sfx, pfx, n_cta, hi, tt, &load, &order, nullptr)) {
       lo = hi;
-      hi += std::max<long long>(page, hi / 32);
+      hi += std::max<long long>(tt, hi / 32);
     }
-    while (hi - lo > std::max<long long>(page, hi / 256)) {
+    while (hi - lo > std::max<long long>(16, hi / 256)) {
       const long long mid = (lo + hi) / 2;
-      if (pack_tc(sfx, pfx, n_cta, mid, page, &load, &order, nullptr))
+      if (pack_tc(sfx, pfx, n_cta, mid, tt, &load, &order, nullptr))
         hi = mid;
       else
         lo = mid;
     }
-    pack_tc(sfx, pfx, n_cta, hi, page, &load, &order, &placed);
+    pack_tc(sfx, pfx, n_cta, hi, tt, &load, &order, &placed);
   }
   // Partial slots: per (row, head group) the prefix chunks come first (segment
   // by segment, enclosing segments first), then the suffix pieces; a row owns
