@@ -63,8 +63,11 @@ constexpr int kThreads = 32 * (kVWarp + 1);  // warp 0 K copies, warp 1 MMA, 4 w
 constexpr uint32_t kTmemCols = 512;          // S[0] [0,TT) S[1] [TT,2TT) O[0] [256,..) O[1] [384,..)
 constexpr uint32_t kTmemO = 256;
 constexpr float kRescaleLog2 = 8.0f;         // lazy-rescale threshold (factor 256)
-constexpr int kMaxStages = 4;
-constexpr int kTile = 128;                   // tokens per pipeline tile (8 pages)
+constexpr int kMaxStages = 6;
+// tokens per pipeline tile: 8 pages for D = 128 (three stages per ring); 4 pages
+// for D = 64 (six stages), where the shorter tiles fill the pipeline sooner
+constexpr int kTile128 = 128;
+constexpr int kTile64 = 64;
 
 // Shared memory of one CTA: Q (128 rows x D, non-swizzled 8x8 core matrices:
 // LBO 128 B along d, SBO D*16 B per 8 rows), a ring of `ST` K stages and one of
@@ -84,7 +87,7 @@ struct Smem {
   static constexpr uint32_t kOffK = kQ;
   static constexpr uint32_t kOffV = kOffK + ST * kKV;
   static constexpr uint32_t kOffBar = kOffV + ST * kKV;
-  static constexpr uint32_t kOffML = kOffBar + 320;        // 128 x (m, l) of the second group
+  static constexpr uint32_t kOffML = kOffBar + 384;        // 128 x (m, l) of the second group
   static constexpr uint32_t kOffItems = kOffML + 128 * 8;
   static constexpr uint32_t kAlign = TL ? 128u : 1024u;    // 128B-swizzled tiles: 1024-B aligned
   static constexpr uint32_t kBytes = kOffItems + kItemCache * (uint32_t)sizeof(TcItem) + kAlign;
@@ -180,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // the start the copies leave in the order the tiles are consumed
   volatile int* k_issued =
       reinterpret_cast<volatile int*>(gbase + L::kOffBar + kMisc + 16 + 4 * kMaxStages);
-  static_assert(kMisc + 20 + 4 * kMaxStages <= 320, "barrier block");
+  static_assert(kMisc + 20 + 4 * kMaxStages <= 384, "barrier block");
   float2* ml1 = reinterpret_cast<float2*>(gbase + L::kOffML);  // second group's (m, l) per row
   TcItem* items = reinterpret_cast<TcItem*>(gbase + L::kOffItems);
   auto sK = [&](int s) { return base + L::kOffK + s * L::kKV; };
@@ -837,7 +840,7 @@ bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G) {
   return !latent && dqk == dv && (dqk == 64 || dqk == 128) && page_size == kPB && G <= 128;
 }
 
-int fork_tc_tile_tokens() { return kTile; }
+int fork_tc_tile_tokens(int dqk) { return dqk == 64 ? kTile64 : kTile128; }
 int fork_tc_page_size() { return kPB; }
 
 cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
@@ -850,15 +853,15 @@ cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v
     memset(&mv, 0, sizeof(mv));
     if (reinterpret_cast<uintptr_t>(k_pages) % 16 || reinterpret_cast<uintptr_t>(v_pages) % 16)
       return cudaErrorInvalidValue;
-    if (dqk == 128) return launch_d<128, kTile, 3, true>(p, mk, mv, grid, stream);
-    if (dqk == 64) return launch_d<64, kTile, 4, true>(p, mk, mv, grid, stream);
+    if (dqk == 128) return launch_d<128, kTile128, 3, true>(p, mk, mv, grid, stream);
+    if (dqk == 64) return launch_d<64, kTile64, 6, true>(p, mk, mv, grid, stream);
     return cudaErrorInvalidValue;
   }
   if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
       !make_pool_map_v(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
     return cudaErrorInvalidValue;
-  if (dqk == 128) return launch_d<128, kTile, 3, false>(p, mk, mv, grid, stream);
-  if (dqk == 64) return launch_d<64, kTile, 4, false>(p, mk, mv, grid, stream);
+  if (dqk == 128) return launch_d<128, kTile128, 3, false>(p, mk, mv, grid, stream);
+  if (dqk == 64) return launch_d<64, kTile64, 6, false>(p, mk, mv, grid, stream);
   return cudaErrorInvalidValue;
 }
 

@@ -330,7 +330,7 @@ void finish_tc_plan(HostPlan* hp, const std::vector<long long>& cost, int n_sm,
 // least loaded up and fills each one's spare budget with prefix chunks.  The
 // plan takes the smallest budget for which the prefix fits.  An item costs its
 // whole tiles: a partial tile takes the pipeline as long as a full one.
-constexpr long long kItemCost = 384;  // fixed cost of an item (Q staging, merge, pipeline refill)
+constexpr long long kItemCost = 256;  // fixed cost of an item (Q staging, merge, pipeline refill)
 constexpr int kMinChunk = 128;        // smallest prefix chunk carved into a CTA's spare budget
 
 struct TcUnit {
@@ -408,7 +408,7 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
 }
 
 void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
-  const int tt = fork_tc_tile_tokens();
+  const int tt = fork_tc_tile_tokens(s.dqk);
   const int forks_per_item = std::max(1, 128 / s.G);
   const int R = (int)rows.seq.size();
   // Prefix units: the rows of a segment in groups of forks_per_item, on the grid
