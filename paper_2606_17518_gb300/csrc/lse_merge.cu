@@ -43,15 +43,18 @@ __global__ void __launch_bounds__(kMergeThreads) merge_parts_kernel(const MergeP
   // the next kernel of the stream may get launched now (it waits for this grid
   // before it uses anything this grid writes or reads)
   asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-  asm volatile("griddepcontrol.wait;\n" ::: "memory");
   const int c4n = p.dv / 4;
   const int gid = blockIdx.x * kMergeThreads + threadIdx.x;
-  if (gid >= p.n_rows * c4n) return;
+  const bool live = gid < p.n_rows * c4n;
   const int h = gid % p.hq, rest = gid / p.hq;
   const int c4 = rest % c4n, f = rest / c4n;
   const int row = f * p.hq + h;
-  const int base = p.part_base[f];
-  const int n = p.n_parts[f * p.n_groups + h / (p.hq / p.n_groups)];
+  // the plan is written by a host copy, never by a kernel: read it before the
+  // wait, so that only the partials' loads follow the producing grid
+  const int base = live ? p.part_base[f] : 0;
+  const int n = live ? p.n_parts[f * p.n_groups + h / (p.hq / p.n_groups)] : 0;
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  if (!live) return;
   const RowMerge mr = merge_row(
       p.part_lse + (size_t)base * p.hq + h, (size_t)p.hq,
       reinterpret_cast<const float4*>(p.part_o) + part_o_f4(base, h, c4, p.hq, p.dv),
