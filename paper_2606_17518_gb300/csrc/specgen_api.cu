@@ -572,10 +572,44 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
       for (int sg : serving[f]) keys += rows.segs[sg].len;
       work += 2LL * keys;
     }
-    long long chunk = (work + n_sm - 1) / std::max(1, n_sm);
-    chunk = std::max<long long>(4 * tt, (chunk + tt - 1) / tt * tt);
-    std::vector<long long> cost;
     const long long item_overhead = 128;
+    // Chunk length: near work / n_sm, chosen among whole-tile lengths for the
+    // smallest longest-CTA load under the longest-first assignment (one CTA
+    // with a second item would otherwise set the kernel's end).
+    auto makespan = [&](long long c) {
+      std::vector<long long> costs;
+      for (int f = 0; f < R; ++f) {
+        std::vector<long long> lens(1, rows.len[f]);
+        for (int sg : serving[f]) lens.push_back(rows.segs[sg].len);
+        for (long long len : lens)
+          for (long long b = 0; b < len; b += c) {
+            const long long n = std::min(len, b + c) - b;
+            costs.push_back((n + tt - 1) / tt * tt + item_overhead);
+            costs.push_back((n + tt - 1) / tt * tt + item_overhead);
+          }
+      }
+      std::sort(costs.begin(), costs.end(), std::greater<long long>());
+      std::priority_queue<long long, std::vector<long long>, std::greater<long long>> heap;
+      for (int i = 0; i < std::max(1, n_sm); ++i) heap.push(0);
+      long long worst = 0;
+      for (long long x : costs) {
+        const long long l = heap.top() + x;
+        heap.pop();
+        heap.push(l);
+        worst = std::max(worst, l);
+      }
+      return worst;
+    };
+    const long long c0 = std::max<long long>(4 * tt, ((work + n_sm - 1) / std::max(1, n_sm) + tt - 1) / tt * tt);
+    long long chunk = c0, best = makespan(c0);
+    for (long long c = std::max<long long>(4 * tt, c0 / 2 / tt * tt); c <= c0 * 3 / 2; c += tt) {
+      const long long m = makespan(c);
+      if (m < best || (m == best && c > chunk)) {
+        best = m;
+        chunk = c;
+      }
+    }
+    std::vector<long long> cost;
     auto emit = [&](int kind, int seq, int f, int len, int part0) {
       const int n = (int)((len + chunk - 1) / chunk);
       for (int c = 0; c < n; ++c)
