@@ -39,7 +39,10 @@ __device__ __forceinline__ float warp_sum(float v) {
 // producing the partials is still running and waits for it here.
 constexpr int kMergeThreads = 128;  // small blocks can sit beside a running tensor-core CTA
 
-__global__ void __launch_bounds__(kMergeThreads) merge_parts_kernel(const MergeParams p) {
+// BATCH parts are loaded together; MIN_BLOCKS bounds the registers so that
+// grids of several waves keep enough rows in flight per SM.
+template <int BATCH, int MIN_BLOCKS>
+__global__ void __launch_bounds__(kMergeThreads, MIN_BLOCKS) merge_parts_kernel(const MergeParams p) {
   // the next kernel of the stream may get launched now (it waits for this grid
   // before it uses anything this grid writes or reads)
   asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
@@ -55,7 +58,7 @@ __global__ void __launch_bounds__(kMergeThreads) merge_parts_kernel(const MergeP
   const int n = live ? p.n_parts[f * p.n_groups + h / (p.hq / p.n_groups)] : 0;
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
   if (!live) return;
-  const RowMerge mr = merge_row(
+  const RowMerge mr = merge_row<BATCH>(
       p.part_lse + (size_t)base * p.hq + h, (size_t)p.hq,
       reinterpret_cast<const float4*>(p.part_o) + part_o_f4(base, h, c4, p.hq, p.dv),
       (size_t)c4n * p.hq, n);
@@ -108,21 +111,34 @@ __global__ void __launch_bounds__(256) lse_merge2_kernel(const T* oa, const floa
 
 cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool after_dependent) {
   if (p.n_rows == 0) return cudaSuccess;
-  // keep the SMs in the shared-memory-heavy configuration of the kernels around
-  // this one, so that no L1/shared-memory reconfiguration is needed between them
-  static thread_local int configured = -1;
+  // Wide batches (one memory round trip for up to 16 parts) need many
+  // registers, so few blocks fit on an SM.  A grid of several such waves takes
+  // 4-part batches at 8 blocks per SM (one wave, more round trips); a one-wave
+  // grid whose rows have at most 8 parts takes 8-part batches.
+  static thread_local int configured = -1, sms = 0;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (configured != dev) {
-    e = cudaFuncSetAttribute(merge_parts_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                             (int)cudaSharedmemCarveoutMaxShared);
+    const void* kernels[3] = {reinterpret_cast<const void*>(merge_parts_kernel<16, 1>),
+                              reinterpret_cast<const void*>(merge_parts_kernel<8, 4>),
+                              reinterpret_cast<const void*>(merge_parts_kernel<4, 8>)};
+    // keep the SMs in the shared-memory-heavy configuration of the kernels
+    // around this one, so that no L1/shared-memory reconfiguration is needed
+    for (const void* k : kernels) {
+      e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               (int)cudaSharedmemCarveoutMaxShared);
+      if (e != cudaSuccess) return e;
+    }
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
     configured = dev;
   }
   const long long threads = (long long)p.n_rows * (p.dv / 4);
+  const long long blocks = (threads + kMergeThreads - 1) / kMergeThreads;
+  const int form = blocks > 3LL * sms ? 2 : (p.max_parts <= 8 ? 1 : 0);
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)((threads + kMergeThreads - 1) / kMergeThreads));
+  cfg.gridDim = dim3((unsigned)blocks);
   cfg.blockDim = dim3(kMergeThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
@@ -131,7 +147,9 @@ cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool a
   attr[0].val.programmaticStreamSerializationAllowed = after_dependent ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, merge_parts_kernel, p);
+  if (form == 2) return cudaLaunchKernelEx(&cfg, merge_parts_kernel<4, 8>, p);
+  if (form == 1) return cudaLaunchKernelEx(&cfg, merge_parts_kernel<8, 4>, p);
+  return cudaLaunchKernelEx(&cfg, merge_parts_kernel<16, 1>, p);
 }
 
 cudaError_t launch_lse_merge2(const void* oa, const float* la, const void* ob, const float* lb,

@@ -14,6 +14,7 @@ struct MergeParams {
   __nv_bfloat16* out;        // [forks][hq][dv]
   float* lse;                // [forks][hq]
   int n_rows, hq, dv, n_groups;
+  int max_parts;             // the most parts any row has (picks the batch width)
 };
 
 // after_dependent: launch as a programmatic dependent of the previous kernel on

@@ -1,7 +1,7 @@
 // Combining a row's partial attentions, latency-tolerant form (device helper).
 //
 // A row owns n partials (O_i normalised by its own sum, LSE_i).  They are
-// combined online in batches of kMergeBatch: the batch's LSE words and float4
+// combined online in batches of BATCH: the batch's LSE words and float4
 // output slices are loaded together (independent loads, one memory round trip
 // per batch), the running maximum moves to the batch maximum and the accumulated
 // sum is rescaled, exactly as in an online softmax:
@@ -13,8 +13,6 @@
 
 namespace specgen {
 
-constexpr int kMergeBatch = 16;
-
 struct RowMerge {
   float4 acc;
   float w, m;
@@ -22,24 +20,25 @@ struct RowMerge {
 
 // lse_p[i * lse_stride], o_p[i * o_stride] (float4 units) for i < n; L2 loads
 // (the partials may have been written by other SMs during this kernel).
+template <int BATCH>
 __device__ __forceinline__ RowMerge merge_row(const float* lse_p, size_t lse_stride,
                                               const float4* o_p, size_t o_stride, int n) {
   RowMerge r;
   r.acc = make_float4(0.f, 0.f, 0.f, 0.f);
   r.w = 0.f;
   r.m = -INFINITY;
-  for (int i0 = 0; i0 < n; i0 += kMergeBatch) {
-    float li[kMergeBatch];
-    float4 v[kMergeBatch];
+  for (int i0 = 0; i0 < n; i0 += BATCH) {
+    float li[BATCH];
+    float4 v[BATCH];
 #pragma unroll
-    for (int e = 0; e < kMergeBatch; ++e) {
+    for (int e = 0; e < BATCH; ++e) {
       const bool in = i0 + e < n;
       li[e] = in ? __ldcg(lse_p + (size_t)(i0 + e) * lse_stride) : -INFINITY;
       v[e] = in ? __ldcg(o_p + (size_t)(i0 + e) * o_stride) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
     float mb = r.m;
 #pragma unroll
-    for (int e = 0; e < kMergeBatch; ++e) mb = fmaxf(mb, li[e]);
+    for (int e = 0; e < BATCH; ++e) mb = fmaxf(mb, li[e]);
     if (mb == -INFINITY) continue;  // nothing yet
     const float sc = r.m == -INFINITY ? 0.f : fast_exp2((r.m - mb) * kLog2e);
     r.acc.x *= sc;
@@ -49,7 +48,7 @@ __device__ __forceinline__ RowMerge merge_row(const float* lse_p, size_t lse_str
     r.w *= sc;
     r.m = mb;
 #pragma unroll
-    for (int e = 0; e < kMergeBatch; ++e) {
+    for (int e = 0; e < BATCH; ++e) {
       if (li[e] == -INFINITY) continue;
       const float we = fast_exp2((li[e] - mb) * kLog2e);
       r.w += we;

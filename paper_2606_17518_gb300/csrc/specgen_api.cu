@@ -847,6 +847,7 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
   plan->offsets[3] = (int64_t)L.cta_offsets_off;
   plan->offsets[4] = (int64_t)L.part_base_off;
   plan->offsets[5] = (int64_t)L.n_parts_off;
+  plan->offsets[6] = t_plan.n_parts.empty() ? 0 : (int64_t)*std::max_element(t_plan.n_parts.begin(), t_plan.n_parts.end());
   return SPECGEN_OK;
 }
 
@@ -1013,6 +1014,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     mp.part_lse = part_lse;
     mp.part_base = reinterpret_cast<const int32_t*>(pl + plan->offsets[4]);
     mp.n_parts = reinterpret_cast<const int32_t*>(pl + plan->offsets[5]);
+    mp.max_parts = (int)plan->offsets[6];
     mp.out = static_cast<__nv_bfloat16*>(args->out);
     mp.lse = args->lse;
     mp.n_rows = plan->n_rows;
