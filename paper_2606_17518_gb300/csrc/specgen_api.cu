@@ -345,7 +345,7 @@ struct TcPlacement {
 // One packing pass under budget T.  `load` and `order` are caller-owned
 // scratch; `out` (when given) receives the items with their CTAs.
 bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int n_cta,
-             long long T, int tt, std::vector<long long>* load, std::vector<int>* order,
+             long long T, int tt, std::vector<long long>* load, std::vector<long long>* order,
              std::vector<TcPlacement>* out) {
   load->assign(n_cta, 0);
   if (out) out->clear();
@@ -379,14 +379,14 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
       place((int)(round & 1 ? n_cta - 1 - i : i), u, pos, std::min(u.len, pos + piece), c);
     }
   }
+  // CTAs from the least loaded up (ties by index): sort (load, cta) keys
   order->resize(n_cta);
-  for (int c = 0; c < n_cta; ++c) (*order)[c] = c;
-  std::sort(order->begin(), order->end(),
-            [&](int x, int y) { return (*load)[x] < (*load)[y] || ((*load)[x] == (*load)[y] && x < y); });
+  for (int c = 0; c < n_cta; ++c) (*order)[c] = ((*load)[c] << 20) | c;
+  std::sort(order->begin(), order->end());
   size_t ui = 0;
   int pos = 0, part = 0;
   for (int oc = 0; oc < n_cta && ui < pfx.size(); ++oc) {
-    const int cta = (*order)[oc];
+    const int cta = (int)((*order)[oc] & 0xFFFFF);
     while (ui < pfx.size()) {
       const TcUnit& u = pfx[ui];
       const int rem = u.len - pos;
@@ -442,26 +442,27 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   const int n_units = (int)(sfx.size() + pfx.size());
   const int n_cta = std::max(1, n_sm);
   if (n_units > 0) {
-    // Budget search.  Start from the average load with one item per suffix
-    // unit and about one prefix chunk per CTA, step up by 1/32 until the
-    // packing fits, then bisect the last step (a few linear passes in all).
-    std::vector<long long> load;
-    std::vector<int> order;
+    // Budget search.  Loads and item costs are whole tiles, so feasibility only
+    // changes at multiples of the tile: search the budget in tiles.  Start
+    // from the average load with one item per suffix unit and about one prefix
+    // chunk per CTA, step up by 1/16 until the packing fits, then bisect the
+    // last step (a few linear passes in all).
+    static thread_local std::vector<long long> load, order;
     const long long n_items = (long long)sfx.size() + std::max<long long>((long long)pfx.size(), n_cta);
-    long long lo = std::max<long long>(kItemCost + tt, (total + kItemCost * n_items) / n_cta);
+    long long lo = std::max<long long>(kItemCost + tt, (total + kItemCost * n_items) / n_cta) / tt;
     long long hi = lo;
-    while (!pack_tc(sfx, pfx, n_cta, hi, tt, &load, &order, nullptr)) {
+    while (!pack_tc(sfx, pfx, n_cta, hi * tt, tt, &load, &order, nullptr)) {
       lo = hi;
-      hi += std::max<long long>(tt, hi / 32);
+      hi += std::max<long long>(1, hi / 16);
     }
-    while (hi - lo > std::max<long long>(16, hi / 256)) {
+    while (hi - lo > 1) {
       const long long mid = (lo + hi) / 2;
-      if (pack_tc(sfx, pfx, n_cta, mid, tt, &load, &order, nullptr))
+      if (pack_tc(sfx, pfx, n_cta, mid * tt, tt, &load, &order, nullptr))
         hi = mid;
       else
         lo = mid;
     }
-    pack_tc(sfx, pfx, n_cta, hi, tt, &load, &order, &placed);
+    pack_tc(sfx, pfx, n_cta, hi * tt, tt, &load, &order, &placed);
   }
   // Partial slots: per (row, head group) the prefix chunks come first (segment
   // by segment, enclosing segments first), then the suffix pieces; a row owns
@@ -469,12 +470,16 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   // chunk index plus the chunks of the enclosing segments' same-row groups.
   hp->n_groups = s.hkv;
   hp->n_parts.assign((size_t)s.F * s.hkv, 0);
-  std::map<std::tuple<int, int, int>, int> chunks;  // (segment, head, group) -> chunk count
+  const int n_grp = (R + forks_per_item - 1) / forks_per_item;
+  std::vector<int> chunks(rows.segs.size() * s.hkv * std::max(1, n_grp), 0);  // (segment, head, group)
+  auto chunk_at = [&](int seg, int g, int grp) -> int& {
+    return chunks[((size_t)seg * s.hkv + g) * std::max(1, n_grp) + grp];
+  };
   std::vector<int32_t> n_pre((size_t)s.F * s.hkv, 0), n_suf((size_t)s.F * s.hkv, 0);
   for (const TcPlacement& pl : placed) {
     const TcItem& it = pl.item;
     if (it.table_kind == 0) {
-      int& c = chunks[std::make_tuple(it.seq, it.kv_head, group_of(it.seq, it.fork0))];
+      int& c = chunk_at(it.seq, it.kv_head, group_of(it.seq, it.fork0));
       c = std::max(c, it.part + 1);
     } else {
       int32_t& n = n_suf[(size_t)it.fork0 * s.hkv + it.kv_head];
@@ -483,15 +488,11 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   }
   auto base_of = [&](int seg, int g, int f) {  // chunks of the enclosing segments for row f
     int b = 0;
-    for (int a : rows.anc[seg]) {
-      auto q = chunks.find(std::make_tuple(a, g, group_of(a, f)));
-      if (q != chunks.end()) b += q->second;
-    }
+    for (int a : rows.anc[seg]) b += chunk_at(a, g, group_of(a, f));
     return b;
   };
   for (const TcUnit& u : pfx) {
-    auto q = chunks.find(std::make_tuple(u.seq, u.g, group_of(u.seq, u.fork0)));
-    const int c = q == chunks.end() ? 0 : q->second;
+    const int c = chunk_at(u.seq, u.g, group_of(u.seq, u.fork0));
     for (int f = u.fork0; f < u.fork0 + u.nforks; ++f) n_pre[(size_t)f * s.hkv + u.g] += c;
   }
   int slot = 0;
@@ -576,33 +577,51 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
     // Chunk length: near work / n_sm, chosen among whole-tile lengths for the
     // smallest longest-CTA load under the longest-first assignment (one CTA
     // with a second item would otherwise set the kernel's end).
+    std::vector<long long> costs, heap;
     auto makespan = [&](long long c) {
-      std::vector<long long> costs;
+      costs.clear();
       for (int f = 0; f < R; ++f) {
-        std::vector<long long> lens(1, rows.len[f]);
-        for (int sg : serving[f]) lens.push_back(rows.segs[sg].len);
-        for (long long len : lens)
+        auto add = [&](long long len) {
           for (long long b = 0; b < len; b += c) {
-            const long long n = std::min(len, b + c) - b;
-            costs.push_back((n + tt - 1) / tt * tt + item_overhead);
-            costs.push_back((n + tt - 1) / tt * tt + item_overhead);
+            const long long n = (std::min(len, b + c) - b + tt - 1) / tt * tt + item_overhead;
+            costs.push_back(n);
+            costs.push_back(n);
           }
+        };
+        add(rows.len[f]);
+        for (int sg : serving[f]) add(rows.segs[sg].len);
       }
       std::sort(costs.begin(), costs.end(), std::greater<long long>());
-      std::priority_queue<long long, std::vector<long long>, std::greater<long long>> heap;
-      for (int i = 0; i < std::max(1, n_sm); ++i) heap.push(0);
+      heap.assign(std::max(1, n_sm), 0);  // a min-heap of CTA loads (all zero is a heap)
       long long worst = 0;
       for (long long x : costs) {
-        const long long l = heap.top() + x;
-        heap.pop();
-        heap.push(l);
-        worst = std::max(worst, l);
+        std::pop_heap(heap.begin(), heap.end(), std::greater<long long>());
+        heap.back() += x;
+        worst = std::max(worst, heap.back());
+        std::push_heap(heap.begin(), heap.end(), std::greater<long long>());
       }
       return worst;
     };
     const long long c0 = std::max<long long>(4 * tt, ((work + n_sm - 1) / std::max(1, n_sm) + tt - 1) / tt * tt);
+    // candidates: every whole-tile length between half and one and a half
+    // times the average, and the lengths at which a prefix segment's chunk
+    // count changes in that range
+    std::vector<long long> cand;
+    for (long long c = std::max<long long>(4 * tt, c0 / 2 / tt * tt); c <= c0 * 3 / 2; c += tt)
+      cand.push_back(c);
+    for (const Segment& sg : rows.segs) {
+      if (sg.len <= 0) continue;
+      const long long k0 = std::max<long long>(1, (sg.len + c0 * 3 / 2 - 1) / (c0 * 3 / 2));
+      for (long long k = k0; k <= k0 + 16; ++k) {
+        const long long c = ((sg.len + k - 1) / k + tt - 1) / tt * tt;
+        if (c < std::max<long long>(4 * tt, c0 / 2)) break;
+        cand.push_back(c);
+      }
+    }
+    std::sort(cand.begin(), cand.end());
+    cand.erase(std::unique(cand.begin(), cand.end()), cand.end());
     long long chunk = c0, best = makespan(c0);
-    for (long long c = std::max<long long>(4 * tt, c0 / 2 / tt * tt); c <= c0 * 3 / 2; c += tt) {
+    for (long long c : cand) {
       const long long m = makespan(c);
       if (m < best || (m == best && c > chunk)) {
         best = m;
@@ -718,6 +737,7 @@ Layout layout_of(const Shape& s, const HostPlan& hp) {
 thread_local HostPlan t_plan;
 thread_local std::vector<unsigned char> t_plan_bytes;
 
+
 specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
                          specgen_plan* plan, void* cuda_stream);
 
@@ -797,7 +817,7 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
   const Layout L = layout_of(s, t_plan);
   if (args->workspace_bytes < L.ws_end) return SPECGEN_ERR_WORKSPACE;
 
-  t_plan_bytes.assign(L.plan_bytes, 0);
+  t_plan_bytes.assign(L.ws_plan + L.plan_bytes, 0);  // zeroed header, then the plan
   PlanHeader h;
   h.n_split = (int32_t)t_plan.split.size();
   h.n_tc = (int32_t)t_plan.tc.size();
@@ -809,7 +829,7 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
   h.cta_offsets_off = (int32_t)L.cta_offsets_off;
   h.part_base_off = (int32_t)L.part_base_off;
   h.n_parts_off = (int32_t)L.n_parts_off;
-  unsigned char* b = t_plan_bytes.data();
+  unsigned char* b = t_plan_bytes.data() + L.ws_plan;
   memcpy(b, &h, sizeof(h));
   auto put = [&](size_t off, const void* src, size_t bytes) {
     if (bytes) memcpy(b + off, src, bytes);
@@ -823,8 +843,9 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
 
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   unsigned char* ws = static_cast<unsigned char*>(args->workspace);
-  if (cudaMemsetAsync(ws, 0, L.ws_plan, stream) != cudaSuccess) return SPECGEN_ERR_CUDA;
-  if (cudaMemcpyAsync(ws + L.ws_plan, b, L.plan_bytes, cudaMemcpyHostToDevice, stream) !=
+  // one upload: the zeroed header (status word), then the plan
+  if (cudaMemcpyAsync(ws, t_plan_bytes.data(), L.ws_plan + L.plan_bytes, cudaMemcpyHostToDevice,
+                      stream) !=
       cudaSuccess)
     return SPECGEN_ERR_CUDA;
 

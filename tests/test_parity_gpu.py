@@ -274,3 +274,32 @@ def test_stages_equal_one_run(name):
     torch.cuda.synchronize()
     o2, l2 = fd.results()
     assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
+
+
+def test_back_to_back_plans_with_changing_lengths():
+    """Twelve plan + run calls on one stream with no host synchronisation in
+    between, each with different suffix lengths: the plan uploads come from a
+    ring of pinned staging buffers that wraps around while earlier copies may
+    still be pending, and every call must still see its own plan."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload("tiny_p512_f4")
+    fd = ForkDecode(w)
+    base = np.asarray(w["suffix_lens"], dtype=np.int32)
+    outs, cuts = [], []
+    stream = torch.cuda.current_stream().cuda_stream
+    for i in range(12):
+        cut = np.maximum(base - (i * 5) % 17 - np.arange(len(base)) * (i % 3), 0).astype(np.int32)
+        fd.set_suffix_lens(cut)
+        fd.plan(stream)
+        fd.run(stream)
+        outs.append((fd.out.clone(), fd.lse.clone()))
+        cuts.append(cut)
+    torch.cuda.synchronize()
+    assert fd.status() == _lib.SPECGEN_OK
+    for cut, (o, lse) in zip(cuts, outs):
+        wc = dict(w)
+        wc["suffix_lens"] = cut
+        o_ref, lse_ref = oracle.fork_attn_decode(wc)
+        _compare(o.float().cpu().numpy().astype(np.float64), lse.cpu().numpy().astype(np.float64),
+                 o_ref, lse_ref, f"cut {cut.tolist()}")
