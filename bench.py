@@ -578,29 +578,46 @@ def run_decode_steps():
 
     st, fd, offs, free = prepare(n)
     n_free = len(st["free_pages"])
-    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).pin_memory()
-    h_q = pin(st["q"])
-    h_k = pin(st["k_new"])
-    h_v = None if st["v_new"] is None else pin(st["v_new"])
-    d_k = torch.empty(h_k.shape[1:], dtype=torch.int16, device=dev)
-    d_v = None if h_v is None else torch.empty(h_v.shape[1:], dtype=torch.int16, device=dev)
-    h_o = torch.empty(fd.out.shape, dtype=fd.out.dtype).pin_memory()
-    h_l = torch.empty(fd.lse.shape, dtype=fd.lse.dtype).pin_memory()
+    # a step's inputs (Q, then the new K and V rows) travel as one packed buffer
+    # and its outputs (O, then LSE) as another: one copy each way per step,
+    # each part at a 256-byte boundary; the library reads views of them
+    align = lambda x: (x + 255) // 256 * 256
+    i16 = lambda a: np.ascontiguousarray(a).view(np.int16).reshape(-1)
+    parts_in = [i16(st["q"]), i16(st["k_new"][0])] + \
+        ([] if st["v_new"] is None else [i16(st["v_new"][0])])
+    off_in, nb_in = [], 0
+    for a in parts_in:
+        off_in.append(nb_in)
+        nb_in = align(nb_in + a.size * 2)
+    h_in = torch.zeros((n, nb_in // 2), dtype=torch.int16).pin_memory()
+    for s_ in range(n):
+        h_in[s_, 0:parts_in[0].size] = torch.from_numpy(parts_in[0])
+        h_in[s_, off_in[1] // 2:off_in[1] // 2 + parts_in[1].size] = torch.from_numpy(i16(st["k_new"][s_]))
+        if st["v_new"] is not None:
+            h_in[s_, off_in[2] // 2:off_in[2] // 2 + parts_in[2].size] = \
+                torch.from_numpy(i16(st["v_new"][s_]))
+    d_in = torch.empty(nb_in // 2, dtype=torch.int16, device=dev)
+    view_in = lambda k, shape: d_in[off_in[k] // 2:off_in[k] // 2 + int(np.prod(shape))].view(
+        torch.bfloat16).view(shape)
+    fd.q = view_in(0, tuple(st["q"].shape))
+    d_k = view_in(1, tuple(st["k_new"].shape[1:]))
+    d_v = None if st["v_new"] is None else view_in(2, tuple(st["v_new"].shape[1:]))
+    o_bytes = fd.out.numel() * 2
+    nb_out = align(o_bytes) + fd.lse.numel() * 4
+    d_out = torch.empty(nb_out, dtype=torch.uint8, device=dev)
+    fd.out = d_out[:o_bytes].view(torch.bfloat16).view(fd.out.shape)
+    fd.lse = d_out[align(o_bytes):].view(torch.float32).view(fd.lse.shape)
+    h_out = torch.empty(nb_out, dtype=torch.uint8).pin_memory()
     with torch.cuda.stream(stream):
         fd.run(sp)  # first launches configure the kernels outside any capture
     torch.cuda.synchronize(dev)
 
     def step(s):
-        fd.q.view(torch.int16).copy_(h_q, non_blocking=True)
-        d_k.copy_(h_k[s], non_blocking=True)
-        if d_v is not None:
-            d_v.copy_(h_v[s], non_blocking=True)
-        fd.append_kv(d_k.view(torch.bfloat16), None if d_v is None else d_v.view(torch.bfloat16),
-                     free[offs[s]:], n_free - offs[s], sp)
+        d_in.copy_(h_in[s], non_blocking=True)
+        fd.append_kv(d_k, d_v, free[offs[s]:], n_free - offs[s], sp)
         fd.suffix_lens_dev.add_(1)
         fd.run(sp)
-        h_o.copy_(fd.out, non_blocking=True)
-        h_l.copy_(fd.lse, non_blocking=True)
+        h_out.copy_(d_out, non_blocking=True)
 
     graphs = []
     for g0 in range(0, n, per_graph):
@@ -683,7 +700,6 @@ def run_decode_steps():
         roof = {"bound": "hbm", "kernel": attn, "achieved": achieved, "peak": hbm,
                 "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
                 "peak_source": peak_src, "algorithmic_bytes_per_launch": att_bytes}
-    row_bytes = F * w["hkv"] * (w["dqk"] + (w["dv"] if w["v_pages"] is not None else 0)) * 2
     kern = {"append_kv": app_ms, attn: part_ms, "lse_merge": merge_ms}
     line = {
         "metric": "fork-decode step tokens/s (append + attention, growing suffixes)",
@@ -702,8 +718,8 @@ def run_decode_steps():
         "roofline": roof,
         "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
         "e2e": {"value": world * F / (ms_per_step * 1e-3), "unit": "tokens/s",
-                "h2d_bytes_per_step": int(h_q.numel() * 2 + row_bytes),
-                "d2h_bytes_per_step": int(h_o.numel() * 2 + h_l.numel() * 4),
+                "h2d_bytes_per_step": int(nb_in),
+                "d2h_bytes_per_step": int(nb_out),
                 "note": "every timed step includes its own host copies"},
     }
     if rank == 0:
