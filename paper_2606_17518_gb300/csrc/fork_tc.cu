@@ -236,7 +236,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   // kernel of the stream is still running: everything above touches only this
   // CTA's own resources and the plan.  The inputs (device lengths, block tables,
   // Q, K/V, possibly written by that kernel) and the partial buffers (possibly
-  // still read by it) are used only after this wait.
+  // still read by it) are used only after this wait.  Before it, the two copy
+  // warps only ask L2 for the first item's first two tiles: the page ids they
+  // read here serve as prefetch addresses (in-range ids only) and nothing else,
+  // so a table the previous kernel rewrites costs bandwidth, never correctness.
+  // Only plans with host-resolved table offsets take part: then every read
+  // here is of the plan or of table entries at positions the plan was built
+  // for.
+  if ((warp == 0 || warp == kVWarp) && n_items > 0) {
+    const TcItem it = p.items[it_begin];  // from the plan itself, not the cache
+    const int npages = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
+    if (it.table_off >= 0 && lane < 2 * kPagesPerTile && lane < npages) {
+      const int page = page_batch(p, it, 0, lane);
+      if (page >= 0 && page < p.num_pages) {
+        const __nv_bfloat16* blk = (warp == 0 ? p.k_pages : p.v_pages) +
+                                   ((size_t)page * p.hkv + it.kv_head) * (kPB * D);
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(blk), "r"(L::kBlk)
+                     : "memory");
+      }
+    }
+  }
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
   if (warp == 0) {
     __syncwarp();
