@@ -140,7 +140,9 @@ __device__ __forceinline__ int page_batch(const TcParams& p, const TcItem& it, i
   return bt[off + it.tok_begin / kPB + pb + lane];
 }
 
-template <int D, int TT, int ST, bool TL>
+// CAUSAL: the plan has causal suffix items (prefill chunks), each row masked at
+// its own length; decode plans take the kernel without that per-row limit.
+template <int D, int TT, int ST, bool TL, bool CAUSAL>
 __global__ void __launch_bounds__(kThreads, 1)
     fork_tc_kernel(const __grid_constant__ TcParams p, const __grid_constant__ CUtensorMap tmk,
                    const __grid_constant__ CUtensorMap tmv) {
@@ -543,6 +545,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int head = it.kv_head * p.G + gi;
       // this row's partial slot base, fetched now and used at the item's end
       const int pbase = p.part_base[it.fork0 + (row_ok ? fl : 0)];
+      // causal items: tokens past this row's own length (relative to the item)
+      // are masked; everything else sees the whole item
+      const int row_end = CAUSAL && it.row_limit0 > 0 ? it.row_limit0 + fl - it.tok_begin
+                                                      : 0x7fffffff;
 
       // group 1 stores Q of the first item here, of every later item at the end
       // of the previous one (as soon as that item's last S has finished)
@@ -588,11 +594,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
               for (int i = 0; i < 32; ++i) sc[c * 32 + i] = __uint_as_float(r[c][i]);
           }
-          const bool full_tile = nt == TT && pv == (1u << kPagesPerTile) - 1u;
+          // tokens this row may see in the tile: the item's, and for a causal
+          // item (prefill chunk) those before the row's own limit
+          int lim = nt;
+          if constexpr (CAUSAL) lim = max(0, min(nt, row_end - j * TT));
+          const bool full_tile = lim == TT && pv == (1u << kPagesPerTile) - 1u;
           if (!full_tile) {
 #pragma unroll
             for (int i = 0; i < TT; ++i)
-              if (!(i < nt && ((pv >> (i / kPB)) & 1u))) sc[i] = -INFINITY;
+              if (!(i < lim && ((pv >> (i / kPB)) & 1u))) sc[i] = -INFINITY;
           }
           float mx0 = sc[0], mx1 = sc[1], mx2 = sc[2], mx3 = sc[3];
 #pragma unroll
@@ -818,14 +828,14 @@ bool make_pool_map_v(CUtensorMap* map, const void* pool, int D, int page, int hk
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int D, int TT, int ST, bool TL>
+template <int D, int TT, int ST, bool TL, bool CAUSAL>
 cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap& mv, int grid,
                      cudaStream_t stream) {
   constexpr int smem = (int)Smem<D, TT, ST, TL>::kBytes;
   static_assert(smem <= 232448, "fork_tc kernel shared memory exceeds 227 KB");
   static_assert(ST <= kMaxStages && (TT == 64 || TT == 128), "unsupported pipeline shape");
   static_assert(kTmemO + 128u * kWG <= kTmemCols && 2 * TT <= (int)kTmemO, "TMEM layout");
-  auto kern = fork_tc_kernel<D, TT, ST, TL>;
+  auto kern = fork_tc_kernel<D, TT, ST, TL, CAUSAL>;
   static thread_local int configured = -1;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -862,8 +872,9 @@ bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G) {
 int fork_tc_tile_tokens(int dqk) { return dqk == 64 ? kTile64 : kTile128; }
 int fork_tc_page_size() { return kPB; }
 
-cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
-                           int dqk, bool tiled, cudaStream_t stream) {
+template <bool CAUSAL>
+static cudaError_t launch_layout(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
+                          int dqk, bool tiled, cudaStream_t stream) {
   if (grid == 0) return cudaSuccess;
   CUtensorMap mk, mv;
   if (tiled) {
@@ -872,16 +883,22 @@ cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v
     memset(&mv, 0, sizeof(mv));
     if (reinterpret_cast<uintptr_t>(k_pages) % 16 || reinterpret_cast<uintptr_t>(v_pages) % 16)
       return cudaErrorInvalidValue;
-    if (dqk == 128) return launch_d<128, kTile128, 3, true>(p, mk, mv, grid, stream);
-    if (dqk == 64) return launch_d<64, kTile64, 6, true>(p, mk, mv, grid, stream);
+    if (dqk == 128) return launch_d<128, kTile128, 3, true, CAUSAL>(p, mk, mv, grid, stream);
+    if (dqk == 64) return launch_d<64, kTile64, 6, true, CAUSAL>(p, mk, mv, grid, stream);
     return cudaErrorInvalidValue;
   }
   if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
       !make_pool_map_v(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
     return cudaErrorInvalidValue;
-  if (dqk == 128) return launch_d<128, kTile128, 3, false>(p, mk, mv, grid, stream);
-  if (dqk == 64) return launch_d<64, kTile64, 6, false>(p, mk, mv, grid, stream);
+  if (dqk == 128) return launch_d<128, kTile128, 3, false, CAUSAL>(p, mk, mv, grid, stream);
+  if (dqk == 64) return launch_d<64, kTile64, 6, false, CAUSAL>(p, mk, mv, grid, stream);
   return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
+                           int dqk, bool tiled, bool causal, cudaStream_t stream) {
+  return causal ? launch_layout<true>(p, k_pages, v_pages, grid, dqk, tiled, stream)
+                : launch_layout<false>(p, k_pages, v_pages, grid, dqk, tiled, stream);
 }
 
 }  // namespace specgen

@@ -30,7 +30,8 @@ struct TcParams {
 bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G);
 int fork_tc_tile_tokens(int dqk);
 int fork_tc_page_size();
+// causal: the plan holds causal suffix items (TcItem::row_limit0 > 0)
 cudaError_t launch_fork_tc(const TcParams& p, const void* k_pages, const void* v_pages, int grid,
-                           int dqk, bool tiled, cudaStream_t stream);
+                           int dqk, bool tiled, bool causal, cudaStream_t stream);
 
 }  // namespace specgen

@@ -57,6 +57,8 @@ struct TcItem {
   int32_t dv0;         // first value column this item produces (latent KV: 0 or 256)
   int32_t table_off;   // index of the sequence's first page in its block table, or -1
                        // (then the kernel reads it from the device offset array)
+  int32_t row_limit0;  // causal suffix items (prefill chunks): query row r of the item
+                       // sees only tokens < row_limit0 + r / G; 0 = every token
 };
 
 // Plan header at the start of the plan region.

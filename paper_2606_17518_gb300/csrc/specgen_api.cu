@@ -335,6 +335,7 @@ constexpr int kMinChunk = 128;        // smallest prefix chunk carved into a CTA
 
 struct TcUnit {
   int kind, seq, g, fork0, nforks, len;
+  int row_limit0;  // causal rows (a prefill chunk): row i of the unit sees row_limit0 + i tokens
 };
 
 struct TcPlacement {
@@ -368,6 +369,7 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
     it.part = part;
     it.dv0 = 0;
     it.table_off = -1;
+    it.row_limit0 = u.row_limit0;
     out->push_back(pl);
   };
   long long k_dealt = 0;  // suffix pieces dealt so far (snake order over the CTAs)
@@ -426,13 +428,32 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     for (int g = 0; g < s.hkv; ++g)
       for (int f0 = seg.row_begin; f0 < seg.row_end;) {
         const int f1 = std::min(seg.row_end, r0 + (group_of(sg, f0) + 1) * forks_per_item);
-        pfx.push_back(TcUnit{0, sg, g, f0, f1 - f0, seg.len});
+        pfx.push_back(TcUnit{0, sg, g, f0, f1 - f0, seg.len, 0});
         f0 = f1;
       }
   }
+  // Suffix units: a row's own suffix, or -- for consecutive rows of one fork whose
+  // lengths grow by one (the tokens of a prefill chunk, causal) -- one unit for up
+  // to forks_per_item of them inside one prefix row group: the fork's suffix
+  // pages are then read once for the whole group, each row masked at its own
+  // length.
+  std::vector<int> group_id(R, -1);  // prefix row group of each row
+  for (int sg = 0; sg < (int)rows.segs.size(); ++sg)
+    if (rows.root[sg] == sg)
+      for (int f = rows.segs[sg].row_begin; f < rows.segs[sg].row_end; ++f)
+        group_id[f] = sg * (R / forks_per_item + 2) + group_of(sg, f);
   for (int g = 0; g < s.hkv; ++g)
-    for (int f = 0; f < R; ++f)
-      if (rows.len[f] > 0) sfx.push_back(TcUnit{1, rows.seq[f], g, f, 1, rows.len[f]});
+    for (int f = 0; f < R;) {
+      int f1 = f + 1;
+      while (f1 < R && f1 - f < forks_per_item && rows.seq[f1] == rows.seq[f] &&
+             rows.len[f1] == rows.len[f1 - 1] + 1 && group_id[f1] == group_id[f] &&
+             group_id[f] >= 0)
+        ++f1;
+      if (rows.len[f1 - 1] > 0)
+        sfx.push_back(TcUnit{1, rows.seq[f], g, f, f1 - f, rows.len[f1 - 1],
+                             f1 - f > 1 ? rows.len[f] : 0});
+      f = f1;
+    }
   for (const TcUnit& u : sfx) total += (u.len + tt - 1) / tt * tt;
   for (const TcUnit& u : pfx) total += u.len;
   auto longer = [](const TcUnit& a, const TcUnit& b) { return a.len > b.len; };
@@ -482,8 +503,10 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
       int& c = chunk_at(it.seq, it.kv_head, group_of(it.seq, it.fork0));
       c = std::max(c, it.part + 1);
     } else {
-      int32_t& n = n_suf[(size_t)it.fork0 * s.hkv + it.kv_head];
-      n = std::max(n, it.part + 1);
+      for (int f = it.fork0; f < it.fork0 + it.nforks; ++f) {
+        int32_t& n = n_suf[(size_t)f * s.hkv + it.kv_head];
+        n = std::max(n, it.part + 1);
+      }
     }
   }
   auto base_of = [&](int seg, int g, int f) {  // chunks of the enclosing segments for row f
@@ -643,6 +666,7 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
           it.tok_end = (int)std::min<long long>(len, (c + 1) * chunk);
           it.part = part0 + c;
           it.dv0 = half * 256;
+          it.row_limit0 = 0;
           hp->tc.push_back(it);
           cost.push_back(it.tok_end - it.tok_begin + item_overhead);
         }
@@ -856,7 +880,10 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
   plan->n_rows = s.F * s.hq;
   plan->total_slots = t_plan.total_slots;
   plan->n_part_groups = t_plan.n_groups;
-  plan->flags = (s.latent ? 1 : 0) | (args->kv_layout == SPECGEN_KV_TILED ? 2 : 0);
+  bool causal = false;  // causal suffix items (prefill chunks) need the per-row limit
+  for (const TcItem& it : t_plan.tc) causal = causal || it.row_limit0 > 0;
+  plan->flags = (s.latent ? 1 : 0) | (args->kv_layout == SPECGEN_KV_TILED ? 2 : 0) |
+                (causal ? 4 : 0);
   plan->plan_bytes = (int64_t)L.plan_bytes;
   plan->ws_plan_off = (int64_t)L.ws_plan;
   plan->ws_part_o_off = (int64_t)L.ws_part_o;
@@ -1017,7 +1044,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
       tp.k_pages = static_cast<const __nv_bfloat16*>(args->k_pages);
       tp.v_pages = static_cast<const __nv_bfloat16*>(args->v_pages);
       e = launch_fork_tc(tp, args->k_pages, args->v_pages, plan->n_tc_ctas, args->head_dim_qk,
-                         args->kv_layout == SPECGEN_KV_TILED, stream);
+                         args->kv_layout == SPECGEN_KV_TILED, (plan->flags & 4) != 0, stream);
     }
     if (e != cudaSuccess) return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
