@@ -59,3 +59,16 @@ def test_prefill_fuzz(case):
     if w["suffix_lens"].sum() == 0:
         pytest.skip("no suffix tokens to prefill in this draw")
     _check(w, int(rng.integers(1, 40)))
+
+
+@pytest.mark.parametrize("dqk,G", [(128, 4), (64, 8)])
+def test_prefill_long_suffix_groups_cut(dqk, G):
+    """Long suffixes behind a short prefix: a fork's chunk tokens share causal
+    suffix items (up to 128/G rows each, split where the rows leave a prefix row
+    group), and the small total work makes the planner cut those items into
+    several token pieces, so rows see pieces that end before, inside and after
+    their own causal limit."""
+    spec = wl.WorkloadSpec(name="pf_long", num_traces=1, prefix_len=(64, 64), forks=(2, 2),
+                           suffix_len=(1200, 1400), hq=G * 2, hkv=2, dqk=dqk, dv=dqk,
+                           page_size=16, seed=91 + G)
+    _check(wl.make_workload(spec), 48)
