@@ -40,6 +40,11 @@
 // item, past the sequence or on an invalid page are masked to -inf, and value
 // rows past the sequence inside its last page are zeroed in shared memory
 // before the PV product, so nothing stored there (even NaN) reaches the output.
+// Head dim 64 uses 64-token tiles (four pages) with six stages per ring.  A
+// causal instantiation serves prefill plans, whose suffix items hold several
+// query rows of one fork, each masked at its own length.  The kernel is a
+// programmatic dependent of the previous kernel of the stream: its prologue
+// (and an L2 prefetch of its first tiles) runs before it waits for that kernel.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
