@@ -433,6 +433,14 @@ def run_ours():
         "kernels": {n: {"ms_per_launch": t, "share": t / max(1e-12, sum(kernel_ms))}
                     for n, t in zip(kernel_names, kernel_ms)},
         "achieved_gbs_whole_step": nbytes["total"] / (ms_per_step * 1e-3) / 1e9,
+        # the metric's other two parts: the dominant kernel's algorithmic GB/s
+        # against the nominal 8 TB/s of HBM3e, and the prefix read amplification
+        # (DRAM bytes of the recorded ncu capture, less the suffix, Q and output
+        # bytes, over the unique prefix bytes; null without a current record)
+        "hbm_vs_8tbs": (achieved / 8000.0) if achieved else None,
+        "prefix_read_amplification": (
+            (traffic - nbytes["suffix"] - nbytes["q"] - nbytes["out"]) / nbytes["prefix"]
+            if traffic is not None and nbytes["prefix"] > 0 else None),
         "roofline": roofline,
         "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
         "e2e": e2e,
