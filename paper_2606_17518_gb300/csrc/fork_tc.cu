@@ -363,6 +363,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           __syncwarp();
           if (!is_v && lane == 0) *k_issued = t + 1;
+          // with an item's last V tile (about a ring of tiles before the item's
+          // end is consumed) ask L2 for the next item's Q rows, which the
+          // softmax loads on the path to that item's first score MMA; asked at
+          // the item's start they could be evicted by the KV streamed meanwhile
+          if (!CAUSAL && is_v && pb + tp + kPagesPerTile >= npages && k + 1 < n_items) {
+            const TcItem nx = get_item(items, p, it_begin, k + 1);
+            for (int r = lane; r < nx.nforks * p.G; r += 32) {
+              const char* qrow = reinterpret_cast<const char*>(
+                  p.q + ((size_t)(nx.fork0 + r / p.G) * p.hq + nx.kv_head * p.G + r % p.G) * D);
+#pragma unroll
+              for (int c = 0; c < D * 2; c += 128)
+                asm volatile("prefetch.global.L2 [%0];\n" ::"l"(qrow + c));
+            }
+          }
         }
         cur = nxt;
       }
@@ -505,9 +519,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ softmax groups
     // Group g (warps 2+4g .. 5+4g) takes the tiles j = g, g+2, ... of every item
     // with its own running max/sum and its own TMEM output O[g].  Group 1 also
-    // stages Q: it loads the next item's rows into registers after its last
-    // tile and stores them once the MMA reports the current item's last S
-    // finished.  At the end of every item the groups combine their halves,
+    // stages Q: it loads the next item's rows (asked of L2 by the V copy warp)
+    // into registers after its last tile and stores them once the MMA reports
+    // the current item's last S finished.  At the end of every item the groups combine their halves,
     // each writing half of the value columns.
     const int grp = (warp - 2) >> 2;
     const int q4 = warp & 3;
@@ -558,16 +572,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       // group 1 stores Q of the first item here, of every later item at the end
       // of the previous one (as soon as that item's last S has finished)
       if (grp == 1 && k == 0) store_q();
-      // and asks L2 for the next item's Q rows now, so that loading them at this
-      // item's end (on the path to the next item's first score MMA) hits L2
-      if (grp == 1 && k + 1 < n_items) {
-        const TcItem nx = get_item(items, p, it_begin, k + 1);
-        if (row < nx.nforks * p.G) {
-          const char* qrow = reinterpret_cast<const char*>(
-              p.q + ((size_t)(nx.fork0 + row / p.G) * p.hq + nx.kv_head * p.G + row % p.G) * D);
+      // prefill items are short: there group 1 asks L2 for the next item's Q
+      // rows itself, at this item's start
+      if constexpr (CAUSAL) {
+        if (grp == 1 && k + 1 < n_items) {
+          const TcItem nx = get_item(items, p, it_begin, k + 1);
+          if (row < nx.nforks * p.G) {
+            const char* qrow = reinterpret_cast<const char*>(
+                p.q + ((size_t)(nx.fork0 + row / p.G) * p.hq + nx.kv_head * p.G + row % p.G) * D);
 #pragma unroll
-          for (int c = 0; c < D * 2; c += 128)
-            asm volatile("prefetch.global.L2 [%0];\n" ::"l"(qrow + c));
+            for (int c = 0; c < D * 2; c += 128)
+              asm volatile("prefetch.global.L2 [%0];\n" ::"l"(qrow + c));
+          }
         }
       }
 
