@@ -155,7 +155,7 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------------------- CPU oracle
-def oracle_sample(workload: str, seconds: float):
+def oracle_sample(workload: str, seconds: float, first_fork: int = 0):
     """Time the fp64 oracle (as it stands) on whole forks until ~`seconds` pass."""
     import oracle
     from paper_2606_17518_gb300 import workloads as wl
@@ -163,7 +163,7 @@ def oracle_sample(workload: str, seconds: float):
     forks = 0
     t0 = time.perf_counter()
     while True:
-        f = forks % w["total_forks"]
+        f = (first_fork + forks) % w["total_forks"]
         oracle.fork_attn_decode_rows(w, [(f, h) for h in range(w["hq"])])
         forks += 1
         if time.perf_counter() - t0 >= seconds or forks >= 10000:
@@ -172,17 +172,65 @@ def oracle_sample(workload: str, seconds: float):
     return forks, dt
 
 
-def cpu_baseline(workload: str, seconds: float):
+def cpu_model() -> str:
+    """The host CPU as /proc/cpuinfo names it (model name, else the Arm part number)."""
+    try:
+        info = open("/proc/cpuinfo").read()
+    except OSError:
+        return "unknown"
+    for key in ("model name", "Model Name"):
+        for line in info.splitlines():
+            if line.split(":")[0].strip() == key:
+                return line.split(":", 1)[1].strip()
+    fields = {}
+    for line in info.splitlines():
+        if ":" in line:
+            k, v = (x.strip() for x in line.split(":", 1))
+            fields.setdefault(k, v)
+    parts = [f"{k} {fields[k]}" for k in ("CPU implementer", "CPU part", "CPU variant")
+             if k in fields]
+    return "Arm, " + ", ".join(parts) if parts else "unknown"
+
+
+def _oracle_children(workload: str, seconds: float, n: int):
+    """`n` single-threaded oracle processes at once, each from its own first fork."""
     env = dict(os.environ, SPECGEN_ORACLE_CHILD="1", OMP_NUM_THREADS="1",
                OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
-    code = ("import json,sys; sys.argv=['bench.py','--impl','reference']; import bench; "
-            f"f,dt=bench.oracle_sample({workload!r},{seconds}); print(json.dumps([f,dt]))")
-    res = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
-                         text=True, timeout=600)
-    forks, dt = json.loads(res.stdout.strip().splitlines()[-1])
+    procs = []
+    for i in range(n):
+        code = ("import json,sys; sys.argv=['bench.py','--impl','reference']; import bench; "
+                f"f,dt=bench.oracle_sample({workload!r},{seconds},{i}); "
+                "print(json.dumps([f,dt]))")
+        procs.append(subprocess.Popen([sys.executable, "-c", code], cwd=ROOT, env=env,
+                                      stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                      text=True))
+    out = []
+    for pr in procs:
+        stdout, _ = pr.communicate(timeout=600)
+        out.append(json.loads(stdout.strip().splitlines()[-1]))
+    return out
+
+
+def cpu_baseline(workload: str, seconds: float):
+    [(forks, dt)] = _oracle_children(workload, seconds, 1)
     return {"value": forks / dt, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "cpu": cpu_model(),
             "sample": f"{forks} whole forks (all heads) of {workload}, fp64 numpy, "
                       f"{dt:.1f} s on 1 host thread"}
+
+
+def cpu_baseline_all_cores(workload: str, seconds: float, unique_bytes: int):
+    """The same oracle on every host core at once (one single-threaded process per
+    core, up to 16, over different forks); tokens/s = the sum of their rates."""
+    n = min(16, os.cpu_count() or 1)
+    if unique_bytes > (1 << 30):  # every process holds its own copy of the workload
+        return None
+    res = _oracle_children(workload, seconds, n)
+    forks = sum(f for f, _ in res)
+    return {"value": sum(f / dt for f, dt in res), "unit": "tokens/s", "cores": n,
+            "kind": "oracle", "cpu": cpu_model(),
+            "sample": f"{forks} whole forks of {workload} over {n} single-threaded processes, "
+                      f"{max(dt for _, dt in res):.1f} s each at most"}
 
 
 # --------------------------------------------------------------------------- reference arm
@@ -233,8 +281,10 @@ def kernel_source_sha(name: str) -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(kernel: str, workload: str):
-    """DRAM bytes per launch from the committed ncu summary, if still current."""
+def recorded_profile(kernel: str, workload: str):
+    """The committed ncu record of a kernel on a workload (DRAM bytes and
+    tensor-pipe activity per launch), if the kernel's sources are unchanged
+    since it was taken; else None."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as fh:
@@ -242,9 +292,15 @@ def recorded_traffic(kernel: str, workload: str):
         rec = d[kernel][workload]
         if rec.get("source_sha") != kernel_source_sha(kernel):
             return None
-        return float(rec["dram_bytes_per_launch"])
+        return rec
     except Exception:
         return None
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if still current."""
+    rec = recorded_profile(kernel, workload)
+    return float(rec["dram_bytes_per_launch"]) if rec else None
 
 
 def run_ours():
@@ -334,15 +390,24 @@ def run_ours():
     barrier()
     torch.cuda.synchronize(dev)
     clocks.start()
+    # an event after every graph as well: per-graph step times give the median
+    # and the best step next to the mean
+    marks = [torch.cuda.Event(enable_timing=True) for _ in schedule]
     with torch.cuda.stream(stream):
         start.record(stream)
-        for graph, _ in schedule:
+        for (graph, _), mk in zip(schedule, marks):
             graph.replay()
+            mk.record(stream)
         end.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
     clk = clocks.stop()
     total_ms = start.elapsed_time(end)
+    graph_steps = [per_graph] * n_full + ([rem] if rem else [])
+    prev, per_step_us = start, []
+    for mk, n in zip(marks, graph_steps):
+        per_step_us.append(prev.elapsed_time(mk) * 1e3 / n)
+        prev = mk
     # per-kernel times: each stage alone, back to back, over the same replicas
     def stage_ms(call):
         g_list = [make_graph(g * per_graph, per_graph, call)[0]
@@ -366,6 +431,7 @@ def run_ours():
         (["split_decode"] if plans[0].n_split_items > 0 else [])
     partials_ms = stage_ms(lib.specgen_fork_attn_run_partials)
     merge_ms = stage_ms(lib.specgen_fork_attn_run_merge)
+    suffix_stage = measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes)
     # one launch per partial kernel kind (a plan uses one of them) plus the merge
     kernel_ms = [partials_ms / max(1, len(kernel_names))] * len(kernel_names) + [merge_ms]
     kernel_names = kernel_names + ["lse_merge"]
@@ -432,6 +498,8 @@ def run_ours():
         "gpu_launches": K * launches,
         "kernels": {n: {"ms_per_launch": t, "share": t / max(1e-12, sum(kernel_ms))}
                     for n, t in zip(kernel_names, kernel_ms)},
+        "step_us": {"mean": ms_per_step * 1e3, "median": float(np.median(per_step_us)),
+                    "best": float(np.min(per_step_us)), "graphs": len(per_step_us)},
         "achieved_gbs_whole_step": nbytes["total"] / (ms_per_step * 1e-3) / 1e9,
         # the metric's other two parts: the dominant kernel's algorithmic GB/s
         # against the nominal 8 TB/s of HBM3e, and the prefix read amplification
@@ -441,6 +509,11 @@ def run_ours():
         "prefix_read_amplification": (
             (traffic - nbytes["suffix"] - nbytes["q"] - nbytes["out"]) / nbytes["prefix"]
             if traffic is not None and nbytes["prefix"] > 0 else None),
+        # the suffix stage alone (diagnostic plan with empty prefixes)
+        "suffix_stage": suffix_stage,
+        # tensor-pipe activity of the dominant kernel from the recorded ncu capture
+        "tensor_pipe_pct": (recorded_profile(kernel_names[dom], f"{ARGS.workload}:{layout}")
+                            or {}).get("tensor_pipe_pct"),
         "roofline": roofline,
         "clocks": {k: clk[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
         "e2e": e2e,
@@ -448,6 +521,8 @@ def run_ours():
     if rank == 0 and world == 1 and not ARGS.no_cpu_baseline:
         try:
             line["cpu_baseline"] = cpu_baseline(ARGS.workload, ARGS.cpu_sample_seconds)
+            line["cpu_baseline_all_cores"] = cpu_baseline_all_cores(
+                ARGS.workload, ARGS.cpu_sample_seconds / 2, nbytes["total"])
         except Exception as exc:  # reported, never silently dropped
             line["cpu_baseline"] = {"error": repr(exc)[:200]}
     if rank == 0:
@@ -455,6 +530,63 @@ def run_ours():
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes):
+    """The suffix stage alone: the same forks, queries and suffix pages with empty
+    prefixes, so that the partial-attention kernel reads only the suffix KV (a
+    diagnostic plan; the step itself always runs both stages in one kernel).
+    GB/s = (suffix KV + Q bytes) / the kernel's time, against the nominal 8 TB/s
+    and the measured copy bandwidth."""
+    import ctypes as C
+
+    import torch
+
+    from paper_2606_17518_gb300 import _lib
+    if nbytes["suffix"] <= 0 or "segment_rows" in w:
+        return None
+    import copy
+    lib = _lib.load()
+    fds = []
+    for r in reps:
+        fd = copy.copy(r)  # the replica's device tensors, its own lengths and workspace
+        fd.w = dict(r.w)
+        fd.w["prefix_lens"] = np.zeros_like(r.w["prefix_lens"])
+        fd.workspace, fd.ws_bytes = None, 0
+        fd.set_suffix_lens(fd.w["suffix_lens"], update_device=False)
+        with torch.cuda.stream(stream):
+            fd.plan(stream.cuda_stream)
+        fds.append(fd)
+    torch.cuda.synchronize(dev)
+    keep = [fd.args() for fd in fds]  # the structs outlive the graph capture
+    arg_refs = [C.byref(a) for a in keep]
+    plan_refs = [C.byref(fd.plan_info) for fd in fds]
+    sp_c = C.c_void_p(stream.cuda_stream)
+    st = lib.specgen_fork_attn_run_partials(arg_refs[0], plan_refs[0], sp_c)
+    assert st == 0, _lib.status_string(st)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for k in range(per_graph):
+            st = lib.specgen_fork_attn_run_partials(arg_refs[k % len(fds)], plan_refs[k % len(fds)],
+                                                    sp_c)
+            assert st == 0, _lib.status_string(st)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize(dev)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n_rep = 32
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(n_rep):
+            graph.replay()
+        t1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = t0.elapsed_time(t1) / (n_rep * per_graph)
+    hbm, _, _, _ = measured_peaks()
+    gbs = (nbytes["suffix"] + nbytes["q"]) / (ms * 1e-3) / 1e9
+    return {"kernel_us": ms * 1e3, "bytes_per_launch": nbytes["suffix"] + nbytes["q"],
+            "gbs": gbs, "vs_8tbs": gbs / 8000.0, "vs_measured": gbs / hbm,
+            "plan": "same forks, queries and suffix pages; empty prefixes"}
 
 
 def measure_e2e(w, reps, stream, dev, K, W):
