@@ -446,7 +446,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   tc_fence_before();
-  __syncthreads();
+  // non-aligned CTA barrier: it counts every thread, so the lanes of a warp may
+  // arrive apart (lanes 1-31 of the MMA warp come here at once, its lane 0 and
+  // the copy lane only after their drains).  An aligned __syncthreads() there
+  // could complete before the softmax warps' last TMEM loads.
+  asm volatile("barrier.sync 0;\n" ::: "memory");
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
