@@ -590,16 +590,18 @@ def measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes):
 
 
 def measure_e2e(w, reps, stream, dev, K, W):
-    """tokens/s through specgen_fork_attn_decode with host-resident per-step inputs.
+    """tokens/s through specgen_fork_attn_decode_staged with host-resident inputs.
 
-    Every step copies that step's queries and block tables from pinned host
-    memory, plans (host) and runs the call, and reads O and LSE back into
-    pinned host memory.  The KV pools are the serving cache and stay resident.
-    A step's inputs travel as one packed buffer (Q, then the four table
-    arrays, each at a 256-byte boundary) and its outputs as another (O, then
-    LSE): one copy each way, as a serving loop stages them; the library reads
-    the views inside the packed device buffers.
+    Every step is one library call that copies that step's queries and block
+    tables from pinned host memory, plans (host) and runs the attention, and
+    reads O and LSE back into pinned host memory.  The KV pools are the serving
+    cache and stay resident.  A step's inputs travel as one packed buffer (Q,
+    then the four table arrays, each at a 256-byte boundary) and its outputs as
+    another (O, then LSE): one copy each way, as a serving loop stages them; the
+    library reads the views inside the packed device buffers.
     """
+    import ctypes as C
+
     import torch
 
     from paper_2606_17518_gb300 import _lib
@@ -634,13 +636,17 @@ def measure_e2e(w, reps, stream, dev, K, W):
     bi = staged[0][0].numel() + int(reps[0].plan_info.plan_bytes)
     bo = staged[0][2].numel()
 
+    lib = _lib.load()
+    staged_call = lib.specgen_fork_attn_decode_staged
+    calls = [(C.byref(args), C.byref(r.lens), C.c_void_p(hin.data_ptr()),
+              C.c_void_p(din.data_ptr()), C.c_size_t(din.numel()), C.c_void_p(dout.data_ptr()),
+              C.c_void_p(hout.data_ptr()), C.c_size_t(dout.numel()), C.c_void_p(sp))
+             for r, (din, hin, dout, hout, args) in zip(reps, staged)]
+
     def step(i):
-        r = reps[i % replicas]
-        din, hin, dout, hout, args = staged[i % replicas]
-        with torch.cuda.stream(stream):
-            din.copy_(hin, non_blocking=True)
-            _lib.specgen_fork_attn_decode(args, r.lens, sp)
-            hout.copy_(dout, non_blocking=True)
+        st = staged_call(*calls[i % replicas])
+        if st != 0:
+            raise RuntimeError(_lib.status_string(st))
 
     for i in range(W):
         step(i)

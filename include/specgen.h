@@ -182,6 +182,24 @@ specgen_status specgen_fork_attn_decode(const specgen_fork_attn_args* args,
                                         const specgen_host_lens* lens,
                                         void* cuda_stream);
 
+/* One decode step from host memory, in one call (no counterpart in the paper:
+ * a serving convenience).  On `cuda_stream`: copies in_bytes from host_in to
+ * dev_in, then does specgen_fork_attn_decode(args, lens), then copies
+ * out_bytes from dev_out to host_out.  The caller lays the step's device
+ * inputs (Q and the block-table arrays) out inside dev_in and points args at
+ * them, and likewise out / lse inside dev_out, so that each direction is a
+ * single copy.  Host buffers should be pinned for the copies to be
+ * asynchronous; host_out is valid once the stream reaches the end of the
+ * call.  in_bytes or out_bytes may be 0 (that copy is skipped).  Status codes
+ * as specgen_fork_attn_decode; SPECGEN_ERR_NULL for a missing buffer of a
+ * non-empty copy; SPECGEN_ERR_CUDA if a copy cannot be queued. */
+specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* args,
+                                               const specgen_host_lens* lens,
+                                               const void* host_in, void* dev_in,
+                                               size_t in_bytes, const void* dev_out,
+                                               void* host_out, size_t out_bytes,
+                                               void* cuda_stream);
+
 /* specgen_fork_attn_decode for callers that cannot allocate device memory.
  * (No counterpart in the paper: this is a deployment convenience.)  Some
  * callers cannot call cudaMalloc at all -- for example a plugin inside a host

@@ -37,6 +37,7 @@ EXPORTED = [
     "specgen_fork_prefill_workspace_size",
     "specgen_fork_prefill_plan",
     "specgen_fork_attn_decode",
+    "specgen_fork_attn_decode_staged",
     "specgen_fork_attn_decode_static",
     "specgen_lse_merge",
     "specgen_append_kv",
@@ -165,6 +166,10 @@ def load() -> C.CDLL:
                                                    C.c_void_p, C.c_int, P(C.c_int)]
     lib.specgen_fork_attn_decode.restype = C.c_int
     lib.specgen_fork_attn_decode.argtypes = [P(ForkAttnArgs), P(HostLens), C.c_void_p]
+    lib.specgen_fork_attn_decode_staged.restype = C.c_int
+    lib.specgen_fork_attn_decode_staged.argtypes = [
+        P(ForkAttnArgs), P(HostLens), C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p,
+        C.c_void_p, C.c_size_t, C.c_void_p]
     lib.specgen_fork_attn_decode_static.restype = C.c_int
     lib.specgen_fork_attn_decode_static.argtypes = [P(ForkAttnArgs), P(HostLens), C.c_void_p]
     lib.specgen_lse_merge.restype = C.c_int
@@ -340,6 +345,16 @@ def specgen_fork_attn_run_profiled(args: ForkAttnArgs, plan: Plan, stream: int, 
 def specgen_fork_attn_decode(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> None:
     _check(load().specgen_fork_attn_decode(C.byref(args), C.byref(lens), C.c_void_p(stream)),
            "specgen_fork_attn_decode")
+
+
+def specgen_fork_attn_decode_staged(args: ForkAttnArgs, lens: HostLens, host_in, dev_in,
+                                    in_bytes: int, dev_out, host_out, out_bytes: int,
+                                    stream: int = 0) -> None:
+    """One decode step from host memory: copy in, plan + run, copy out (one call)."""
+    _check(load().specgen_fork_attn_decode_staged(
+        C.byref(args), C.byref(lens), _ptr(host_in), _ptr(dev_in), C.c_size_t(in_bytes),
+        _ptr(dev_out), _ptr(host_out), C.c_size_t(out_bytes), C.c_void_p(stream)),
+        "specgen_fork_attn_decode_staged")
 
 
 def specgen_fork_attn_decode_static(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> None:

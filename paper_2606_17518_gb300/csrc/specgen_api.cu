@@ -1089,6 +1089,27 @@ specgen_status specgen_fork_attn_decode(const specgen_fork_attn_args* args,
   return specgen_fork_attn_run(args, &plan, cuda_stream);
 }
 
+specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* args,
+                                               const specgen_host_lens* lens,
+                                               const void* host_in, void* dev_in,
+                                               size_t in_bytes, const void* dev_out,
+                                               void* host_out, size_t out_bytes,
+                                               void* cuda_stream) {
+  if (!args || !lens) return SPECGEN_ERR_NULL;
+  if ((in_bytes > 0 && (!host_in || !dev_in)) || (out_bytes > 0 && (!dev_out || !host_out)))
+    return SPECGEN_ERR_NULL;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  if (in_bytes > 0 &&
+      cudaMemcpyAsync(dev_in, host_in, in_bytes, cudaMemcpyHostToDevice, stream) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  const specgen_status st = specgen_fork_attn_decode(args, lens, cuda_stream);
+  if (st != SPECGEN_OK) return st;
+  if (out_bytes > 0 &&
+      cudaMemcpyAsync(host_out, dev_out, out_bytes, cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
+}
+
 specgen_status specgen_append_kv(const specgen_append_args* a, void* cuda_stream) {
   if (!a) return SPECGEN_ERR_NULL;
   if (a->total_forks < 0 || a->hkv < 1 || a->page_size < 1 || a->num_pages < 0 || a->num_free < 0)

@@ -174,6 +174,14 @@ def test_null_and_workspace_errors(w):
     # run with an invalid (zeroed) plan is rejected on the host
     assert lib.specgen_fork_attn_run(C.byref(_fake_args(w)), C.byref(plan), None) == \
         S.SPECGEN_ERR_SHAPE
+    # the staged decode rejects a missing buffer of a non-empty copy before any copy
+    staged = lib.specgen_fork_attn_decode_staged
+    args = _fake_args(w)
+    assert staged(C.byref(args), C.byref(lens), None, 0x10000, 64, None, None, 0, None) == \
+        S.SPECGEN_ERR_NULL
+    assert staged(C.byref(args), C.byref(lens), None, None, 0, 0x10000, None, 64, None) == \
+        S.SPECGEN_ERR_NULL
+    assert staged(None, C.byref(lens), None, None, 0, None, None, 0, None) == S.SPECGEN_ERR_NULL
 
 
 def test_lse_merge_host_checks():

@@ -194,6 +194,55 @@ def test_invalid_page_id_is_reported_not_read():
     assert np.all(np.isfinite(o))
 
 
+def _pack_device(tensors):
+    """One device buffer holding copies of `tensors` (256-byte aligned views) and
+    a pinned host twin: (device bytes, host bytes, views)."""
+    import torch
+    offs, n = [], 0
+    for t in tensors:
+        offs.append(n)
+        n = (n + t.numel() * t.element_size() + 255) // 256 * 256
+    dbuf = torch.empty(n, dtype=torch.uint8, device="cuda")
+    views = []
+    for t, o in zip(tensors, offs):
+        v = dbuf[o:o + t.numel() * t.element_size()].view(t.dtype).view(t.shape)
+        v.copy_(t)
+        views.append(v)
+    hbuf = torch.empty(n, dtype=torch.uint8).pin_memory()
+    hbuf.copy_(dbuf)
+    return dbuf, hbuf, views, offs
+
+
+@pytest.mark.parametrize("name", ["tiny_p512_f4", "fork_p8k_f8"])
+def test_staged_decode_from_host_buffers(name):
+    """specgen_fork_attn_decode_staged: the step's inputs arrive only through its
+    host->device copy (the device copy is wiped first), and its outputs, read
+    from the pinned host buffer, equal the plain call's bits, call after call."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload(name)
+    fd = ForkDecode(w)
+    fd.decode()
+    o_ref, l_ref = fd.results()
+    din, hin, (fd.q, fd.prefix_table, fd.prefix_off, fd.suffix_table, fd.suffix_off), _ = \
+        _pack_device([fd.q, fd.prefix_table, fd.prefix_off, fd.suffix_table, fd.suffix_off])
+    dout, hout, (fd.out, fd.lse), ooff = _pack_device([fd.out, fd.lse])
+    F, hq, dv = w["total_forks"], w["hq"], w["dv"]
+    for _ in range(2):
+        din.zero_()
+        dout.zero_()
+        hout.zero_()
+        torch.cuda.synchronize()
+        _lib.specgen_fork_attn_decode_staged(fd.args(), fd.lens, hin, din, din.numel(), dout, hout,
+                                             dout.numel())
+        torch.cuda.synchronize()
+        o = hout[ooff[0]:ooff[0] + F * hq * dv * 2].view(torch.bfloat16).float().numpy()
+        lse = hout[ooff[1]:ooff[1] + F * hq * 4].view(torch.float32).numpy()
+        assert np.array_equal(o.astype(np.float64).reshape(F, hq, dv), o_ref)
+        assert np.array_equal(lse.astype(np.float64).reshape(F, hq), l_ref)
+    assert fd.status() == _lib.SPECGEN_OK
+
+
 def test_plan_once_run_many_is_deterministic():
     from paper_2606_17518_gb300.fork_attn import ForkDecode
     w = wl.make_workload("fork_p8k_f8")
