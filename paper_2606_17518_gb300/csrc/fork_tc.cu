@@ -912,9 +912,28 @@ static cudaError_t launch_layout(const TcParams& p, const void* k_pages, const v
     if (dqk == 64) return launch_d<64, kTile64, 6, true, CAUSAL>(p, mk, mv, grid, stream);
     return cudaErrorInvalidValue;
   }
-  if (!make_pool_map(&mk, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
-      !make_pool_map_v(&mv, v_pages, dqk, kPB, p.hkv, p.num_pages))
-    return cudaErrorInvalidValue;
+  // the maps depend only on the pools' addresses and shapes: encode them again
+  // only when those change (a decode loop launches over the same pools)
+  struct MapKey {
+    const void* k;
+    const void* v;
+    int dqk, hkv, num_pages;
+    bool operator==(const MapKey& o) const {
+      return k == o.k && v == o.v && dqk == o.dqk && hkv == o.hkv && num_pages == o.num_pages;
+    }
+  };
+  static thread_local MapKey cached{nullptr, nullptr, 0, 0, 0};
+  static thread_local CUtensorMap cached_k, cached_v;
+  const MapKey key{k_pages, v_pages, dqk, p.hkv, p.num_pages};
+  if (!(key == cached)) {
+    cached = MapKey{nullptr, nullptr, 0, 0, 0};
+    if (!make_pool_map(&cached_k, k_pages, dqk, kPB, p.hkv, p.num_pages) ||
+        !make_pool_map_v(&cached_v, v_pages, dqk, kPB, p.hkv, p.num_pages))
+      return cudaErrorInvalidValue;
+    cached = key;
+  }
+  mk = cached_k;
+  mv = cached_v;
   if (dqk == 128) return launch_d<128, kTile128, 3, false, CAUSAL>(p, mk, mv, grid, stream);
   if (dqk == 64) return launch_d<64, kTile64, 6, false, CAUSAL>(p, mk, mv, grid, stream);
   return cudaErrorInvalidValue;

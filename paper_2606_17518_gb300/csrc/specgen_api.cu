@@ -331,6 +331,7 @@ void finish_tc_plan(HostPlan* hp, const std::vector<long long>& cost, int n_sm,
 // plan takes the smallest budget for which the prefix fits.  An item costs its
 // whole tiles: a partial tile takes the pipeline as long as a full one.
 constexpr long long kItemCost = 256;  // fixed cost of an item (Q staging, merge, pipeline refill)
+static_assert(kItemCost % 128 == 0, "item cost in whole tiles of every tile size");
 constexpr int kMinChunk = 128;        // smallest prefix chunk carved into a CTA's spare budget
 
 struct TcUnit {
@@ -350,9 +351,13 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
              std::vector<TcPlacement>* out) {
   load->assign(n_cta, 0);
   if (out) out->clear();
-  const long long lmax = (T - kItemCost) / tt * tt;
-  if (lmax < tt) return false;
-  auto tiles = [&](long long n) { return (n + tt - 1) / tt * tt; };  // tokens of whole tiles
+  // tt (64 or 128 tokens) is a power of two: whole tiles by shifts (this runs a
+  // few times per plan)
+  int sh = 0;
+  while ((1 << sh) < tt) ++sh;
+  if (T - kItemCost < tt) return false;
+  const long long lmax = (T - kItemCost) >> sh << sh;
+  auto tiles = [&](long long n) { return (n + tt - 1) >> sh << sh; };  // tokens of whole tiles
   auto place = [&](int cta, const TcUnit& u, int b, int e, int part) {
     (*load)[cta] += tiles(e - b) + kItemCost;
     if (!out) return;
@@ -372,28 +377,42 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
     it.row_limit0 = u.row_limit0;
     out->push_back(pl);
   };
-  long long k_dealt = 0;  // suffix pieces dealt so far (snake order over the CTAs)
+  // suffix pieces in snake order over the CTAs: piece i of a round goes to CTA
+  // i, or to CTA n_cta - 1 - i in odd rounds
+  int i_snake = 0;
+  bool odd = false;
   for (const TcUnit& u : sfx) {
     const long long k = (u.len + lmax - 1) / lmax;
     const int piece = (int)tiles((u.len + k - 1) / k);
-    for (int c = 0, pos = 0; pos < u.len; ++c, pos += piece, ++k_dealt) {
-      const long long round = k_dealt / n_cta, i = k_dealt % n_cta;
-      place((int)(round & 1 ? n_cta - 1 - i : i), u, pos, std::min(u.len, pos + piece), c);
+    for (int c = 0, pos = 0; pos < u.len; ++c, pos += piece) {
+      place(odd ? n_cta - 1 - i_snake : i_snake, u, pos, std::min(u.len, pos + piece), c);
+      if (++i_snake == n_cta) {
+        i_snake = 0;
+        odd = !odd;
+      }
     }
   }
-  // CTAs from the least loaded up (ties by index): sort (load, cta) keys
+  // CTAs from the least loaded up (ties by index): a stable counting sort of
+  // the loads, which are whole tiles (tiles and kItemCost are multiples of tt)
+  static thread_local std::vector<int> count;
+  long long most = 0;
+  for (int c = 0; c < n_cta; ++c) most = std::max(most, (*load)[c]);
+  count.assign((size_t)(most >> sh) + 2, 0);
+  for (int c = 0; c < n_cta; ++c) ++count[(size_t)((*load)[c] >> sh) + 1];
+  for (size_t b = 1; b < count.size(); ++b) count[b] += count[b - 1];
   order->resize(n_cta);
-  for (int c = 0; c < n_cta; ++c) (*order)[c] = ((*load)[c] << 20) | c;
-  std::sort(order->begin(), order->end());
+  for (int c = 0; c < n_cta; ++c) (*order)[count[(size_t)((*load)[c] >> sh)]++] = c;
   size_t ui = 0;
   int pos = 0, part = 0;
   for (int oc = 0; oc < n_cta && ui < pfx.size(); ++oc) {
-    const int cta = (int)((*order)[oc] & 0xFFFFF);
+    const int cta = (int)(*order)[oc];
     while (ui < pfx.size()) {
       const TcUnit& u = pfx[ui];
       const int rem = u.len - pos;
-      const long long spare = (T - (*load)[cta] - kItemCost) / tt * tt;
-      if (spare < std::min(kMinChunk, rem)) break;  // this CTA is full
+      const long long room = T - (*load)[cta] - kItemCost;
+      if (room < std::min(kMinChunk, rem)) break;  // this CTA is full
+      const long long spare = room >> sh << sh;
+      if (spare < std::min(kMinChunk, rem)) break;
       long long len = std::min<long long>(rem, spare);
       if (rem - len < kMinChunk / 2) len = rem;  // leave no sliver behind
       place(cta, u, pos, pos + (int)len, part);
@@ -419,7 +438,13 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   auto group_of = [&](int seg, int f) {
     return (f - rows.segs[rows.root[seg]].row_begin) / forks_per_item;
   };
-  std::vector<TcUnit> sfx, pfx;
+  // scratch kept across calls (planning runs on every decode call)
+  static thread_local std::vector<TcUnit> sfx, pfx, unit_tmp;
+  static thread_local std::vector<uint64_t> unit_keys;
+  static thread_local std::vector<int> group_id;
+  static thread_local std::vector<TcPlacement> placed, trial;
+  sfx.clear();
+  pfx.clear();
   long long total = 0;
   for (int sg = 0; sg < (int)rows.segs.size(); ++sg) {
     const Segment& seg = rows.segs[sg];
@@ -437,7 +462,7 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   // to forks_per_item of them inside one prefix row group: the fork's suffix
   // pages are then read once for the whole group, each row masked at its own
   // length.
-  std::vector<int> group_id(R, -1);  // prefix row group of each row
+  group_id.assign(R, -1);  // prefix row group of each row
   for (int sg = 0; sg < (int)rows.segs.size(); ++sg)
     if (rows.root[sg] == sg)
       for (int f = rows.segs[sg].row_begin; f < rows.segs[sg].row_end; ++f)
@@ -456,10 +481,19 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     }
   for (const TcUnit& u : sfx) total += (u.len + tt - 1) / tt * tt;
   for (const TcUnit& u : pfx) total += u.len;
-  auto longer = [](const TcUnit& a, const TcUnit& b) { return a.len > b.len; };
-  std::stable_sort(sfx.begin(), sfx.end(), longer);
-  std::stable_sort(pfx.begin(), pfx.end(), longer);
-  std::vector<TcPlacement> placed;
+  // longest first, ties in their present order (a sort of (length, index) keys)
+  auto longest_first = [](std::vector<TcUnit>& v) {
+    unit_keys.resize(v.size());
+    for (size_t i = 0; i < v.size(); ++i)
+      unit_keys[i] = ((uint64_t)(0x7fffffff - v[i].len) << 32) | (uint64_t)i;
+    std::sort(unit_keys.begin(), unit_keys.end());
+    unit_tmp.resize(v.size());
+    for (size_t i = 0; i < v.size(); ++i) unit_tmp[i] = v[unit_keys[i] & 0xffffffffu];
+    v.swap(unit_tmp);
+  };
+  longest_first(sfx);
+  longest_first(pfx);
+  placed.clear();
   const int n_units = (int)(sfx.size() + pfx.size());
   const int n_cta = std::max(1, n_sm);
   if (n_units > 0) {
@@ -468,22 +502,26 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     // from the average load with one item per suffix unit and about one prefix
     // chunk per CTA, step up by 1/16 until the packing fits, then bisect the
     // last step (a few linear passes in all).
+    // Every pass records its placements; `placed` keeps those of the pass that
+    // last fitted, which is the one at the final budget.
     static thread_local std::vector<long long> load, order;
     const long long n_items = (long long)sfx.size() + std::max<long long>((long long)pfx.size(), n_cta);
     long long lo = std::max<long long>(kItemCost + tt, (total + kItemCost * n_items) / n_cta) / tt;
     long long hi = lo;
-    while (!pack_tc(sfx, pfx, n_cta, hi * tt, tt, &load, &order, nullptr)) {
+    while (!pack_tc(sfx, pfx, n_cta, hi * tt, tt, &load, &order, &trial)) {
       lo = hi;
       hi += std::max<long long>(1, hi / 16);
     }
+    placed.swap(trial);
     while (hi - lo > 1) {
       const long long mid = (lo + hi) / 2;
-      if (pack_tc(sfx, pfx, n_cta, mid * tt, tt, &load, &order, nullptr))
+      if (pack_tc(sfx, pfx, n_cta, mid * tt, tt, &load, &order, &trial)) {
         hi = mid;
-      else
+        placed.swap(trial);
+      } else {
         lo = mid;
+      }
     }
-    pack_tc(sfx, pfx, n_cta, hi * tt, tt, &load, &order, &placed);
   }
   // Partial slots: per (row, head group) the prefix chunks come first (segment
   // by segment, enclosing segments first), then the suffix pieces; a row owns
@@ -492,11 +530,15 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   hp->n_groups = s.hkv;
   hp->n_parts.assign((size_t)s.F * s.hkv, 0);
   const int n_grp = (R + forks_per_item - 1) / forks_per_item;
-  std::vector<int> chunks(rows.segs.size() * s.hkv * std::max(1, n_grp), 0);  // (segment, head, group)
+  static thread_local std::vector<int> chunks, per_cta, next;
+  static thread_local std::vector<int32_t> n_pre, n_suf;
+  static thread_local std::vector<TcItem> by_cta;
+  chunks.assign(rows.segs.size() * s.hkv * std::max(1, n_grp), 0);  // (segment, head, group)
   auto chunk_at = [&](int seg, int g, int grp) -> int& {
     return chunks[((size_t)seg * s.hkv + g) * std::max(1, n_grp) + grp];
   };
-  std::vector<int32_t> n_pre((size_t)s.F * s.hkv, 0), n_suf((size_t)s.F * s.hkv, 0);
+  n_pre.assign((size_t)s.F * s.hkv, 0);
+  n_suf.assign((size_t)s.F * s.hkv, 0);
   for (const TcPlacement& pl : placed) {
     const TcItem& it = pl.item;
     if (it.table_kind == 0) {
@@ -535,14 +577,12 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   const bool host_off = rows.prefix_bt_offsets && rows.suffix_bt_offsets;
   hp->tc.clear();
   hp->cta_offsets.assign(1, 0);
-  std::vector<int> per_cta(n_cta + 1, 0);  // counting sort of the placements by CTA
+  per_cta.assign(n_cta + 1, 0);  // counting sort of the placements by CTA
   for (const TcPlacement& pl : placed) ++per_cta[pl.cta + 1];
   for (int c = 0; c < n_cta; ++c) per_cta[c + 1] += per_cta[c];
-  std::vector<TcItem> by_cta(placed.size());
-  {
-    std::vector<int> next(per_cta.begin(), per_cta.end() - 1);
-    for (const TcPlacement& pl : placed) by_cta[next[pl.cta]++] = pl.item;
-  }
+  by_cta.resize(placed.size());
+  next.assign(per_cta.begin(), per_cta.end() - 1);
+  for (const TcPlacement& pl : placed) by_cta[next[pl.cta]++] = pl.item;
   for (int c = 0; c < n_cta; ++c) {
     if (per_cta[c + 1] == per_cta[c]) continue;  // empty CTAs are dropped
     for (int i = per_cta[c]; i < per_cta[c + 1]; ++i) {
