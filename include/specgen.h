@@ -145,6 +145,19 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
                                       const specgen_host_lens* lens,
                                       specgen_plan* plan, void* cuda_stream);
 
+/* specgen_fork_attn_plan into host memory (no counterpart in the paper: a
+ * convenience for callers that stage their own uploads, and a way to check a
+ * plan on the host).  Writes the plan region -- exactly the
+ * plan->ws_plan_off + plan->plan_bytes bytes that specgen_fork_attn_plan copies
+ * to the start of args->workspace: a zeroed header holding the status word,
+ * then the work list -- to host_dst, and fills `plan`.  Nothing is copied to
+ * the device: the caller uploads those bytes to the start of the workspace
+ * before specgen_fork_attn_run.  Same checks and status codes as
+ * specgen_fork_attn_plan; SPECGEN_ERR_WORKSPACE if host_bytes is too small. */
+specgen_status specgen_fork_attn_plan_host(const specgen_fork_attn_args* args,
+                                           const specgen_host_lens* lens, void* host_dst,
+                                           size_t host_bytes, specgen_plan* plan);
+
 /* Launch the kernels of a planned call (no host-device copies; capturable in a
  * CUDA graph).  The data pointers in args may differ from the planning call;
  * the sizes and workspace may not. */

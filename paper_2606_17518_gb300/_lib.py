@@ -28,6 +28,7 @@ SPECGEN_ERR_TIMEOUT = -7
 EXPORTED = [
     "specgen_fork_attn_workspace_size",
     "specgen_fork_attn_plan",
+    "specgen_fork_attn_plan_host",
     "specgen_fork_attn_run",
     "specgen_fork_attn_run_profiled",
     "specgen_fork_attn_run_partials",
@@ -139,6 +140,9 @@ def load() -> C.CDLL:
     lib.specgen_fork_attn_workspace_size.argtypes = [P(ForkAttnArgs), P(HostLens)]
     lib.specgen_fork_attn_plan.restype = C.c_int
     lib.specgen_fork_attn_plan.argtypes = [P(ForkAttnArgs), P(HostLens), P(Plan), C.c_void_p]
+    lib.specgen_fork_attn_plan_host.restype = C.c_int
+    lib.specgen_fork_attn_plan_host.argtypes = [P(ForkAttnArgs), P(HostLens), C.c_void_p,
+                                                C.c_size_t, P(Plan)]
     lib.specgen_fork_attn_run.restype = C.c_int
     lib.specgen_fork_attn_run.argtypes = [P(ForkAttnArgs), P(Plan), C.c_void_p]
     lib.specgen_fork_cascade_workspace_size.restype = C.c_size_t
@@ -345,6 +349,16 @@ def specgen_fork_attn_run_profiled(args: ForkAttnArgs, plan: Plan, stream: int, 
 def specgen_fork_attn_decode(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> None:
     _check(load().specgen_fork_attn_decode(C.byref(args), C.byref(lens), C.c_void_p(stream)),
            "specgen_fork_attn_decode")
+
+
+def specgen_fork_attn_plan_host(args: ForkAttnArgs, lens: HostLens, host_dst: np.ndarray) -> Plan:
+    """Plan into host memory: the plan region's bytes go to ``host_dst`` (uint8)."""
+    plan = Plan()
+    _check(load().specgen_fork_attn_plan_host(C.byref(args), C.byref(lens),
+                                              host_dst.ctypes.data, host_dst.nbytes,
+                                              C.byref(plan)),
+           "specgen_fork_attn_plan_host")
+    return plan
 
 
 def specgen_fork_attn_decode_staged(args: ForkAttnArgs, lens: HostLens, host_in, dev_in,

@@ -802,8 +802,11 @@ thread_local HostPlan t_plan;
 thread_local std::vector<unsigned char> t_plan_bytes;
 
 
+// host_dst == nullptr: upload the plan region to the workspace on cuda_stream;
+// otherwise copy it into host_dst (host_bytes long) and make no CUDA call.
 specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
-                         specgen_plan* plan, void* cuda_stream);
+                         specgen_plan* plan, void* cuda_stream, void* host_dst = nullptr,
+                         size_t host_bytes = 0);
 
 }  // namespace
 
@@ -827,6 +830,17 @@ specgen_status specgen_fork_attn_plan(const specgen_fork_attn_args* args,
   specgen_status st = check_shape(args, lens, &s);
   if (st != SPECGEN_OK) return st;
   return plan_impl(args, s, rows_for_decode(lens, s.T, s.F), plan, cuda_stream);
+}
+
+specgen_status specgen_fork_attn_plan_host(const specgen_fork_attn_args* args,
+                                           const specgen_host_lens* lens, void* host_dst,
+                                           size_t host_bytes, specgen_plan* plan) {
+  if (!plan || !host_dst) return SPECGEN_ERR_NULL;
+  memset(plan, 0, sizeof(*plan));
+  Shape s;
+  specgen_status st = check_shape(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
+  return plan_impl(args, s, rows_for_decode(lens, s.T, s.F), plan, nullptr, host_dst, host_bytes);
 }
 
 size_t specgen_fork_cascade_workspace_size(const specgen_fork_attn_args* args,
@@ -874,7 +888,8 @@ specgen_status specgen_fork_prefill_plan(const specgen_fork_attn_args* args,
 namespace {
 
 specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
-                         specgen_plan* plan, void* cuda_stream) {
+                         specgen_plan* plan, void* cuda_stream, void* host_dst,
+                         size_t host_bytes) {
   specgen_status st;
   if ((st = check_pointers(args)) != SPECGEN_OK) return st;
   build_plan(s, rows, &t_plan);
@@ -905,13 +920,17 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
   put(L.part_base_off, t_plan.part_base.data(), (size_t)s.F * 4);
   put(L.n_parts_off, t_plan.n_parts.data(), t_plan.n_parts.size() * 4);
 
-  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-  unsigned char* ws = static_cast<unsigned char*>(args->workspace);
-  // one upload: the zeroed header (status word), then the plan
-  if (cudaMemcpyAsync(ws, t_plan_bytes.data(), L.ws_plan + L.plan_bytes, cudaMemcpyHostToDevice,
-                      stream) !=
-      cudaSuccess)
-    return SPECGEN_ERR_CUDA;
+  if (host_dst) {
+    if (host_bytes < t_plan_bytes.size()) return SPECGEN_ERR_WORKSPACE;
+    memcpy(host_dst, t_plan_bytes.data(), t_plan_bytes.size());
+  } else {
+    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+    unsigned char* ws = static_cast<unsigned char*>(args->workspace);
+    // one upload: the zeroed header (status word), then the plan
+    if (cudaMemcpyAsync(ws, t_plan_bytes.data(), L.ws_plan + L.plan_bytes,
+                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
+      return SPECGEN_ERR_CUDA;
+  }
 
   plan->valid = 1;
   plan->n_tc_items = h.n_tc;

@@ -93,6 +93,26 @@ def _uniform(rng, lo_hi, n):
     return rng.integers(lo, hi + 1, size=n, dtype=np.int64)
 
 
+def _draw_lengths(rng, spec: WorkloadSpec):
+    """The first draws of a workload: prefix lengths, forks per trace, suffix lengths."""
+    prefix_lens = _uniform(rng, spec.prefix_len, spec.num_traces)
+    forks = _uniform(rng, spec.forks, spec.num_traces)
+    suffix_lens = _uniform(rng, spec.suffix_len, int(forks.sum()))
+    return prefix_lens, forks, suffix_lens
+
+
+def workload_lengths(spec: WorkloadSpec | str, seed: int | None = None):
+    """(prefix_lens, fork_offsets, suffix_lens) of make_workload(spec, seed), as int32,
+    without drawing the KV pools and queries."""
+    if isinstance(spec, str):
+        spec = WORKLOADS[spec]
+    rng = np.random.default_rng(spec.seed if seed is None else seed)
+    prefix_lens, forks, suffix_lens = _draw_lengths(rng, spec)
+    fork_offsets = np.concatenate([[0], np.cumsum(forks)])
+    return (prefix_lens.astype(np.int32), fork_offsets.astype(np.int32),
+            suffix_lens.astype(np.int32))
+
+
 def make_workload(spec: WorkloadSpec | str, seed: int | None = None,
                   fill_unused: str = "nan", **overrides) -> dict:
     """Build the host-side workload dict (numpy arrays; bf16 as uint16 bits).
@@ -108,10 +128,8 @@ def make_workload(spec: WorkloadSpec | str, seed: int | None = None,
         spec = WorkloadSpec(**{**asdict(spec), **overrides})
     rng = np.random.default_rng(spec.seed if seed is None else seed)
     T, B = spec.num_traces, spec.page_size
-    prefix_lens = _uniform(rng, spec.prefix_len, T)
-    forks = _uniform(rng, spec.forks, T)
+    prefix_lens, forks, suffix_lens = _draw_lengths(rng, spec)
     F = int(forks.sum())
-    suffix_lens = _uniform(rng, spec.suffix_len, F)
     fork_offsets = np.concatenate([[0], np.cumsum(forks)]).astype(np.int64)
 
     p_pages = -(-prefix_lens // B)

@@ -1,0 +1,236 @@
+"""Host planner invariants, on the CPU (specgen_fork_attn_plan_host).
+
+A fork-decode plan is correct when, for every query row and every kv head,
+its work items cover the row's keys -- the trace's shared prefix, then the
+fork's own suffix -- exactly once, each item writes a distinct partial slot
+inside the row's slot range, and the merge reads exactly those slots.  These
+tests parse the plan bytes the library would upload and check that, with
+fake device pointers, over the benchmark workloads and random ragged shapes
+on all three kernel paths (tensor-core GQA, latent tensor-core, split-K).
+"""
+
+import ctypes as C
+
+import numpy as np
+import pytest
+
+from paper_2606_17518_gb300 import _lib, workloads as wl
+
+FAKE = 0x10000
+TC_WORDS = 11      # TcItem: int32 fields
+SPLIT_WORDS = 10   # SplitItem: int32 fields
+
+
+def _args(T, F, hq, hkv, dqk, dv, B, latent, **kw):
+    a = _lib.make_args(num_traces=T, total_forks=F, hq=hq, hkv=hkv, head_dim_qk=dqk,
+                       head_dim_v=dv, page_size=B, num_pages=1 << 20, scale=0.1, q=FAKE,
+                       k_pages=FAKE, v_pages=None if latent else FAKE,
+                       prefix_block_table=FAKE, prefix_bt_offsets=FAKE,
+                       suffix_block_table=FAKE, suffix_bt_offsets=FAKE, out=FAKE, lse=FAKE,
+                       workspace=FAKE, workspace_bytes=1 << 40, kv_layout=_lib.KV_ROWS,
+                       suffix_lens=None)
+    for k, v in kw.items():
+        setattr(a, k, v)
+    return a
+
+
+def _plan(shape, pl, fo, sl, host_offsets=True):
+    T, F = len(pl), int(fo[-1])
+    B = shape["B"]
+    pbo = np.concatenate([[0], np.cumsum((pl + B - 1) // B)]).astype(np.int32)
+    sbo = np.concatenate([[0], np.cumsum((sl + B - 1) // B)]).astype(np.int32)
+    if host_offsets:
+        lens, keep = _lib.make_host_lens(pl, fo, sl, pbo, sbo)
+    else:
+        lens, keep = _lib.make_host_lens(pl, fo, sl)
+    args = _args(T, F, **shape)
+    need = _lib.specgen_fork_attn_workspace_size(args, lens)
+    assert need > 0
+    buf = np.zeros(need, dtype=np.uint8)
+    plan = _lib.specgen_fork_attn_plan_host(args, lens, buf)
+    return plan, buf, pbo, sbo
+
+
+def _parse(plan, buf):
+    assert plan.valid == 1
+    assert not buf[:plan.ws_plan_off].any()  # the status header goes up zeroed
+    region = buf[plan.ws_plan_off:plan.ws_plan_off + plan.plan_bytes]
+    w = region.view(np.int32)
+    n_split, n_tc, n_ctas, n_forks, so, to, _, coo, pbo_, npo = (int(x) for x in w[:10])
+    words = lambda off, n: w[off // 4: off // 4 + n]
+    return dict(
+        split=words(so, n_split * SPLIT_WORDS).reshape(n_split, SPLIT_WORDS),
+        tc=words(to, n_tc * TC_WORDS).reshape(n_tc, TC_WORDS),
+        cta_offsets=words(coo, n_ctas + 1) if n_tc else np.zeros(1, np.int32),
+        part_base=words(pbo_, n_forks),
+        n_parts=words(npo, n_forks * plan.n_part_groups).reshape(n_forks, plan.n_part_groups),
+        n_ctas=n_ctas)
+
+
+def _covers(ranges, length, what):
+    """Half-open ranges tile [0, length) exactly once."""
+    ranges = sorted(ranges)
+    pos = 0
+    for b, e in ranges:
+        assert b == pos and e > b, (what, ranges, length)
+        pos = e
+    assert pos == length, (what, ranges, length)
+
+
+def _check_slots(p, plan, F):
+    base = p["part_base"]
+    most = p["n_parts"].max(axis=1) if F else np.zeros(0)
+    assert base[0] == 0
+    ends = base + most
+    assert np.all(ends[:-1] <= base[1:])
+    assert int(ends[-1]) <= plan.total_slots
+
+
+def _check_tc(shape, pl, fo, sl, plan, p, pbo, sbo, host_offsets):
+    G = shape["hq"] // shape["hkv"]
+    F = int(fo[-1])
+    tc = p["tc"]
+    co = p["cta_offsets"]
+    assert co[0] == 0 and co[-1] == len(tc) and np.all(np.diff(co) > 0)
+    fork_trace = np.repeat(np.arange(len(pl)), np.diff(fo))
+    cover = {}
+    parts = {}
+    for kind, seq, g, f0, nf, tb, te, part, dv0, toff, rl in tc:
+        assert te > tb >= 0 and dv0 == 0 and rl == 0
+        assert 1 <= nf and nf * G <= 128 and 0 <= g < shape["hkv"]
+        if kind == 0:
+            assert np.all(fork_trace[f0:f0 + nf] == seq) and te <= pl[seq]
+            assert toff == (pbo[seq] if host_offsets else -1)
+        else:
+            assert nf == 1 and seq == f0 and te <= sl[seq]
+            assert toff == (sbo[seq] if host_offsets else -1)
+        for f in range(f0, f0 + nf):
+            cover.setdefault((f, g, kind), []).append((int(tb), int(te)))
+            parts.setdefault((f, g), []).append(int(part))
+    for f in range(F):
+        for g in range(shape["hkv"]):
+            _covers(cover.get((f, g, 0), []), int(pl[fork_trace[f]]), ("prefix", f, g))
+            _covers(cover.get((f, g, 1), []), int(sl[f]), ("suffix", f, g))
+            got = sorted(parts.get((f, g), []))
+            assert got == list(range(p["n_parts"][f, g])), (f, g, got)
+    _check_slots(p, plan, F)
+
+
+def _check_latent(pl, fo, sl, plan, p):
+    F = int(fo[-1])
+    fork_trace = np.repeat(np.arange(len(pl)), np.diff(fo))
+    cover, parts = {}, {}
+    for kind, seq, g, f0, nf, tb, te, part, dv0, toff, rl in p["tc"]:
+        assert g == 0 and nf == 1 and dv0 in (0, 256) and te > tb >= 0
+        key = (f0, dv0)
+        cover.setdefault(key + (kind,), []).append((int(tb), int(te)))
+        parts.setdefault(key, []).append(int(part))
+        if kind == 0:
+            assert seq == fork_trace[f0]
+        else:
+            assert seq == f0
+    for f in range(F):
+        for dv0 in (0, 256):
+            _covers(cover.get((f, dv0, 0), []), int(pl[fork_trace[f]]), ("prefix", f, dv0))
+            _covers(cover.get((f, dv0, 1), []), int(sl[f]), ("suffix", f, dv0))
+            assert sorted(parts.get((f, dv0), [])) == list(range(p["n_parts"][f, 0]))
+    _check_slots(p, plan, F)
+
+
+def _check_split(shape, pl, fo, sl, plan, p):
+    F = int(fo[-1])
+    fork_trace = np.repeat(np.arange(len(pl)), np.diff(fo))
+    cover, slots = {}, {}
+    for f, kind, seq, g, h0, nrows, dv0, tb, te, slot in p["split"]:
+        assert te > tb >= 0 and nrows >= 1 and 0 <= g < shape["hkv"]
+        assert seq == (fork_trace[f] if kind == 0 else f)
+        key = (f, h0, dv0)
+        cover.setdefault(key + (kind,), []).append((int(tb), int(te)))
+        slots.setdefault(key, []).append(int(slot) - int(p["part_base"][f]))
+    # every fork with keys has items for every (row block, value block), and
+    # the row blocks tile the query heads
+    blocks = sorted({(int(h0), int(nr), int(dv0)) for _, _, _, _, h0, nr, dv0, _, _, _ in p["split"]})
+    heads = sorted({(h0, nr) for h0, nr, _ in blocks})
+    _covers([(h0, h0 + nr) for h0, nr in heads], shape["hq"], "row blocks")
+    for f in range(F):
+        if pl[fork_trace[f]] + sl[f] == 0:
+            continue
+        for h0, _, dv0 in blocks:
+            _covers(cover.get((f, h0, dv0, 0), []), int(pl[fork_trace[f]]), ("prefix", f, h0))
+            _covers(cover.get((f, h0, dv0, 1), []), int(sl[f]), ("suffix", f, h0))
+            assert sorted(slots[(f, h0, dv0)]) == list(range(p["n_parts"][f, 0]))
+    _check_slots(p, plan, F)
+
+
+SHAPES = {
+    "gqa128": dict(hq=64, hkv=8, dqk=128, dv=128, B=16, latent=False),
+    "gqa64": dict(hq=8, hkv=2, dqk=64, dv=64, B=16, latent=False),
+    "mha": dict(hq=4, hkv=4, dqk=128, dv=128, B=16, latent=False),
+    "g128": dict(hq=128, hkv=1, dqk=128, dv=128, B=16, latent=False),
+    "latent": dict(hq=128, hkv=1, dqk=576, dv=512, B=64, latent=True),
+    "split_page32": dict(hq=16, hkv=2, dqk=128, dv=128, B=32, latent=False),
+    "split_latent_page16": dict(hq=16, hkv=1, dqk=576, dv=512, B=16, latent=True),
+}
+
+
+def _check(name, pl, fo, sl, host_offsets=True):
+    shape = SHAPES[name]
+    plan, buf, pbo, sbo = _plan(shape, pl, fo, sl, host_offsets)
+    p = _parse(plan, buf)
+    if plan.n_split_items:
+        assert plan.n_tc_items == 0
+        _check_split(shape, pl, fo, sl, plan, p)
+    elif shape["latent"]:
+        _check_latent(pl, fo, sl, plan, p)
+    else:
+        _check_tc(shape, pl, fo, sl, plan, p, pbo, sbo, host_offsets)
+    return plan
+
+
+@pytest.mark.parametrize("name", list(wl.WORKLOAD_ORDER))
+def test_workload_plans_cover_every_key_once(name):
+    spec = wl.WORKLOADS[name]
+    pl, fo, sl = wl.workload_lengths(name)
+    shape = dict(hq=spec.hq, hkv=spec.hkv, dqk=spec.dqk, dv=spec.dv, B=spec.page_size,
+                 latent=not spec.separate_v)
+    key = next(k for k, v in SHAPES.items() if v == shape)
+    plan = _check(key, pl, fo, sl)
+    assert plan.n_tc_items > 0 and plan.n_split_items == 0
+
+
+@pytest.mark.parametrize("case", range(24))
+def test_random_plans_cover_every_key_once(case):
+    rng = np.random.default_rng(1000 + case)
+    name = list(SHAPES)[case % len(SHAPES)]
+    T = int(rng.integers(1, 6))
+    fk = rng.integers(1, 11, T)
+    fo = np.concatenate([[0], np.cumsum(fk)]).astype(np.int32)
+    F = int(fo[-1])
+    pl = rng.integers(0, 6000, T).astype(np.int32)
+    sl = rng.integers(0, 800, F).astype(np.int32)
+    # degenerate rows: empty prefixes and suffixes, one-token sequences
+    pl[rng.random(T) < 0.2] = 0
+    sl[rng.random(F) < 0.2] = 0
+    sl[rng.random(F) < 0.1] = 1
+    _check(name, pl, fo, sl, host_offsets=bool(case % 2))
+
+
+def test_plan_host_errors():
+    shape = SHAPES["gqa128"]
+    pl = np.array([100], np.int32)
+    fo = np.array([0, 2], np.int32)
+    sl = np.array([5, 7], np.int32)
+    lens, keep = _lib.make_host_lens(pl, fo, sl)
+    args = _args(1, 2, **shape)
+    lib = _lib.load()
+    plan = _lib.Plan()
+    small = np.zeros(8, np.uint8)
+    assert lib.specgen_fork_attn_plan_host(C.byref(args), C.byref(lens), small.ctypes.data,
+                                           small.nbytes, C.byref(plan)) == \
+        _lib.SPECGEN_ERR_WORKSPACE
+    assert lib.specgen_fork_attn_plan_host(C.byref(args), C.byref(lens), None, 0,
+                                           C.byref(plan)) == _lib.SPECGEN_ERR_NULL
+    bad = _args(1, 2, **dict(shape, hq=63))
+    buf = np.zeros(1 << 16, np.uint8)
+    assert lib.specgen_fork_attn_plan_host(C.byref(bad), C.byref(lens), buf.ctypes.data,
+                                           buf.nbytes, C.byref(plan)) == _lib.SPECGEN_ERR_SHAPE
