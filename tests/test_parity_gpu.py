@@ -93,6 +93,34 @@ def test_fuzz_small_shapes(case):
     _compare(o, lse, o_ref, lse_ref, f"fuzz{case}")
 
 
+EDGE_SPECS = {
+    # the largest row tile: one fork's 128 query heads on one kv head
+    "g128_d128": dict(num_traces=1, prefix_len=(3001, 3001), forks=(3, 3), suffix_len=(0, 700),
+                      hq=128, hkv=1, dqk=128, dv=128),
+    "g64_d64": dict(num_traces=2, prefix_len=(17, 1500), forks=(1, 4), suffix_len=(1, 300),
+                    hq=128, hkv=2, dqk=64, dv=64),
+    # many forks of one trace: three prefix row groups of 16, 16 and 8 forks
+    "forks40": dict(num_traces=1, prefix_len=(2000, 2000), forks=(40, 40), suffix_len=(0, 200),
+                    hq=8, hkv=1, dqk=128, dv=128),
+    # G = 2: 64 forks per prefix item, 70 forks
+    "g2_forks70": dict(num_traces=1, prefix_len=(900, 900), forks=(70, 70), suffix_len=(5, 60),
+                       hq=4, hkv=2, dqk=128, dv=128),
+    # a 64k-token prefix (512 tiles per kv head, cut over many CTAs)
+    "prefix64k": dict(num_traces=1, prefix_len=(65543, 65543), forks=(2, 2), suffix_len=(1, 33),
+                      hq=16, hkv=2, dqk=128, dv=128),
+}
+
+
+@pytest.mark.parametrize("name", list(EDGE_SPECS))
+def test_edge_sizes_against_oracle(name):
+    """Row tiles of 128 heads, many forks per trace and long prefixes, every row."""
+    spec = wl.WorkloadSpec(name=name, page_size=16, seed=77, **EDGE_SPECS[name])
+    w = wl.make_workload(spec)
+    o, lse, _ = _gpu(w)
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, name)
+
+
 @pytest.mark.parametrize("name", ["tiny_p512_f4", "fork_p8k_f8"])
 def test_tiled_layout_workload_full(name):
     """K/V pools in the 8x8-tiled layout (one bulk copy per page and head)."""
