@@ -275,6 +275,11 @@ size_t specgen_fork_prefill_workspace_size(const specgen_fork_attn_args* args,
 specgen_status specgen_fork_prefill_plan(const specgen_fork_attn_args* args,
                                          const specgen_prefill_lens* lens, specgen_plan* plan,
                                          void* cuda_stream);
+/* specgen_fork_prefill_plan into host memory, as specgen_fork_attn_plan_host
+ * does for decode (no counterpart in the paper). */
+specgen_status specgen_fork_prefill_plan_host(const specgen_fork_attn_args* args,
+                                              const specgen_prefill_lens* lens, void* host_dst,
+                                              size_t host_bytes, specgen_plan* plan);
 
 /* ---- Nested-prefix cascade -------------------------------------------------
  * Fork events taken repeatedly along one reasoning trace, at growing prefixes
@@ -304,6 +309,11 @@ size_t specgen_fork_cascade_workspace_size(const specgen_fork_attn_args* args,
 specgen_status specgen_fork_cascade_plan(const specgen_fork_attn_args* args,
                                          const specgen_cascade_lens* lens, specgen_plan* plan,
                                          void* cuda_stream);
+/* specgen_fork_cascade_plan into host memory, as specgen_fork_attn_plan_host
+ * does for decode (no counterpart in the paper). */
+specgen_status specgen_fork_cascade_plan_host(const specgen_fork_attn_args* args,
+                                              const specgen_cascade_lens* lens, void* host_dst,
+                                              size_t host_bytes, specgen_plan* plan);
 
 /* ---- Decode-step append --------------------------------------------------
  * After a fork event every fork decodes its own continuation while the prefix

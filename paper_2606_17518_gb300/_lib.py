@@ -35,8 +35,10 @@ EXPORTED = [
     "specgen_fork_attn_run_merge",
     "specgen_fork_cascade_workspace_size",
     "specgen_fork_cascade_plan",
+    "specgen_fork_cascade_plan_host",
     "specgen_fork_prefill_workspace_size",
     "specgen_fork_prefill_plan",
+    "specgen_fork_prefill_plan_host",
     "specgen_fork_attn_decode",
     "specgen_fork_attn_decode_staged",
     "specgen_fork_attn_decode_static",
@@ -155,6 +157,11 @@ def load() -> C.CDLL:
     lib.specgen_fork_prefill_plan.restype = C.c_int
     lib.specgen_fork_prefill_plan.argtypes = [P(ForkAttnArgs), P(PrefillLens), P(Plan),
                                               C.c_void_p]
+    for name, lens_t in (("specgen_fork_prefill_plan_host", PrefillLens),
+                         ("specgen_fork_cascade_plan_host", CascadeLens)):
+        fn = getattr(lib, name)
+        fn.restype = C.c_int
+        fn.argtypes = [P(ForkAttnArgs), P(lens_t), C.c_void_p, C.c_size_t, P(Plan)]
     lib.specgen_append_kv.restype = C.c_int
     lib.specgen_append_kv.argtypes = [P(AppendArgs), C.c_void_p]
     lib.specgen_packed_bytes.restype = C.c_size_t
@@ -358,6 +365,26 @@ def specgen_fork_attn_plan_host(args: ForkAttnArgs, lens: HostLens, host_dst: np
                                               host_dst.ctypes.data, host_dst.nbytes,
                                               C.byref(plan)),
            "specgen_fork_attn_plan_host")
+    return plan
+
+
+def specgen_fork_prefill_plan_host(args: ForkAttnArgs, lens, host_dst: np.ndarray) -> Plan:
+    """Prefill plan into host memory (``host_dst``, uint8)."""
+    plan = Plan()
+    _check(load().specgen_fork_prefill_plan_host(C.byref(args), C.byref(lens),
+                                                 host_dst.ctypes.data, host_dst.nbytes,
+                                                 C.byref(plan)),
+           "specgen_fork_prefill_plan_host")
+    return plan
+
+
+def specgen_fork_cascade_plan_host(args: ForkAttnArgs, lens, host_dst: np.ndarray) -> Plan:
+    """Cascade plan into host memory (``host_dst``, uint8)."""
+    plan = Plan()
+    _check(load().specgen_fork_cascade_plan_host(C.byref(args), C.byref(lens),
+                                                 host_dst.ctypes.data, host_dst.nbytes,
+                                                 C.byref(plan)),
+           "specgen_fork_cascade_plan_host")
     return plan
 
 

@@ -863,6 +863,17 @@ specgen_status specgen_fork_cascade_plan(const specgen_fork_attn_args* args,
   return plan_impl(args, s, rows_for_cascade(lens, s.F), plan, cuda_stream);
 }
 
+specgen_status specgen_fork_cascade_plan_host(const specgen_fork_attn_args* args,
+                                              const specgen_cascade_lens* lens, void* host_dst,
+                                              size_t host_bytes, specgen_plan* plan) {
+  if (!plan || !host_dst) return SPECGEN_ERR_NULL;
+  memset(plan, 0, sizeof(*plan));
+  Shape s;
+  specgen_status st = check_cascade(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
+  return plan_impl(args, s, rows_for_cascade(lens, s.F), plan, nullptr, host_dst, host_bytes);
+}
+
 size_t specgen_fork_prefill_workspace_size(const specgen_fork_attn_args* args,
                                            const specgen_prefill_lens* lens) {
   Shape s;
@@ -881,6 +892,17 @@ specgen_status specgen_fork_prefill_plan(const specgen_fork_attn_args* args,
   specgen_status st = check_prefill(args, lens, &s);
   if (st != SPECGEN_OK) return st;
   return plan_impl(args, s, rows_for_prefill(lens, s.T), plan, cuda_stream);
+}
+
+specgen_status specgen_fork_prefill_plan_host(const specgen_fork_attn_args* args,
+                                              const specgen_prefill_lens* lens, void* host_dst,
+                                              size_t host_bytes, specgen_plan* plan) {
+  if (!plan || !host_dst) return SPECGEN_ERR_NULL;
+  memset(plan, 0, sizeof(*plan));
+  Shape s;
+  specgen_status st = check_prefill(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
+  return plan_impl(args, s, rows_for_prefill(lens, s.T), plan, nullptr, host_dst, host_bytes);
 }
 
 }  // extern "C"

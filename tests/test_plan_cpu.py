@@ -234,3 +234,134 @@ def test_plan_host_errors():
     buf = np.zeros(1 << 16, np.uint8)
     assert lib.specgen_fork_attn_plan_host(C.byref(bad), C.byref(lens), buf.ctypes.data,
                                            buf.nbytes, C.byref(plan)) == _lib.SPECGEN_ERR_SHAPE
+
+
+# ---- fork prefill: one query row per chunk token, causal suffix lengths ------
+
+def _prefill_plan(shape, pl, fo, sl, cl):
+    B = shape["B"]
+    pbo = np.concatenate([[0], np.cumsum((pl + B - 1) // B)]).astype(np.int32)
+    sbo = np.concatenate([[0], np.cumsum((sl + cl + B - 1) // B)]).astype(np.int32)
+    lens, keep = _lib.make_prefill_lens(pl, fo, sl, cl, pbo, sbo)
+    args = _args(len(pl), int(cl.sum()), **shape)
+    need = _lib.specgen_fork_prefill_workspace_size(args, lens)
+    assert need > 0
+    buf = np.zeros(need, dtype=np.uint8)
+    plan = _lib.specgen_fork_prefill_plan_host(args, lens, buf)
+    return plan, _parse(plan, buf), pbo, sbo
+
+
+@pytest.mark.parametrize("case", range(10))
+def test_prefill_plans_cover_every_causal_key_once(case):
+    """Row r (chunk token j of fork f) must see the trace's prefix and suffix keys
+    [0, S_f + j + 1) exactly once; a suffix item of several rows masks row i of
+    the item at row_limit0 + i keys."""
+    rng = np.random.default_rng(2000 + case)
+    shape = [SHAPES["gqa128"], SHAPES["gqa64"], SHAPES["g128"], SHAPES["mha"]][case % 4]
+    G = shape["hq"] // shape["hkv"]
+    T = int(rng.integers(1, 4))
+    fk = rng.integers(1, 5, T)
+    fo = np.concatenate([[0], np.cumsum(fk)]).astype(np.int32)
+    nf = int(fo[-1])
+    pl = rng.integers(0, 3000, T).astype(np.int32)
+    sl = rng.integers(0, 400, nf).astype(np.int32)
+    cl = rng.integers(0, 90, nf).astype(np.int32)
+    cl[0] = max(int(cl[0]), 1)
+    plan, p, pbo, sbo = _prefill_plan(shape, pl, fo, sl, cl)
+    assert plan.n_split_items == 0
+    # the query rows: fork by fork, one per chunk token
+    row_fork = np.repeat(np.arange(nf), cl)
+    row_len = np.concatenate([sl[f] + np.arange(1, cl[f] + 1) for f in range(nf)]).astype(int)
+    fork_trace = np.repeat(np.arange(T), np.diff(fo))
+    R = len(row_fork)
+    cover, parts = {}, {}
+    for kind, seq, g, f0, n, tb, te, part, dv0, toff, rl in p["tc"]:
+        assert te > tb >= 0 and 1 <= n and n * G <= 128
+        rows = range(f0, f0 + n)
+        if kind == 0:
+            assert all(fork_trace[row_fork[r]] == seq for r in rows) and te <= pl[seq]
+            assert rl == 0 and toff == pbo[seq]
+            for r in rows:
+                cover.setdefault((r, g, 0), []).append((int(tb), int(te)))
+        else:
+            assert all(row_fork[r] == seq for r in rows) and toff == sbo[seq]
+            assert (rl > 0) == (n > 1)
+            if n > 1:
+                assert rl == row_len[f0] and all(row_len[r] == rl + (r - f0) for r in rows)
+            for i, r in enumerate(rows):
+                end = min(int(te), int(rl) + i) if n > 1 else int(te)
+                assert end <= row_len[r]
+                if end > tb:
+                    cover.setdefault((r, g, 1), []).append((int(tb), end))
+        for r in rows:
+            parts.setdefault((r, g), []).append(int(part))
+    for r in range(R):
+        for g in range(shape["hkv"]):
+            _covers(cover.get((r, g, 0), []), int(pl[fork_trace[row_fork[r]]]), ("prefix", r, g))
+            _covers(cover.get((r, g, 1), []), int(row_len[r]), ("suffix", r, g))
+            assert sorted(parts.get((r, g), [])) == list(range(p["n_parts"][r, g]))
+    _check_slots(p, plan, R)
+
+
+# ---- nested-prefix cascade: laminar shared segments --------------------------
+
+def _laminar(rng, b, e, depth, out):
+    """Random laminar segments over forks [b, e): this range, then children that
+    partition parts of it."""
+    out.append((b, e))
+    if depth == 0 or e - b < 2:
+        return
+    cuts = np.sort(rng.choice(np.arange(b + 1, e), size=min(e - b - 1, int(rng.integers(1, 3))),
+                              replace=False))
+    edges = [b] + [int(c) for c in cuts] + [e]
+    for lo, hi in zip(edges[:-1], edges[1:]):
+        if rng.random() < 0.7:
+            _laminar(rng, lo, hi, depth - 1, out)
+
+
+@pytest.mark.parametrize("case", range(10))
+def test_cascade_plans_cover_every_segment_once(case):
+    """Fork f must see every segment that serves it, each exactly once, then its
+    suffix; the slots of its items are distinct and dense."""
+    rng = np.random.default_rng(3000 + case)
+    shape = [SHAPES["gqa128"], SHAPES["gqa64"], SHAPES["mha"], SHAPES["latent"]][case % 4]
+    F = int(rng.integers(2, 24))
+    segs = []
+    _laminar(rng, 0, F, 3, segs)
+    seg_lens = rng.integers(0, 2500, len(segs)).astype(np.int32)
+    seg_rows = np.array([x for s in segs for x in s], np.int32)
+    sl = rng.integers(0, 500, F).astype(np.int32)
+    B = shape["B"]
+    sgbo = np.concatenate([[0], np.cumsum((seg_lens + B - 1) // B)]).astype(np.int32)
+    sbo = np.concatenate([[0], np.cumsum((sl + B - 1) // B)]).astype(np.int32)
+    lens, keep = _lib.make_cascade_lens(seg_lens, seg_rows, sl, sgbo, sbo)
+    args = _args(len(segs), F, **shape)
+    need = _lib.specgen_fork_cascade_workspace_size(args, lens)
+    assert need > 0
+    buf = np.zeros(need, dtype=np.uint8)
+    plan = _lib.specgen_fork_cascade_plan_host(args, lens, buf)
+    p = _parse(plan, buf)
+    groups = shape["hkv"] if not shape["latent"] else 1
+    cover, parts = {}, {}
+    for kind, seq, g, f0, n, tb, te, part, dv0, toff, rl in p["tc"]:
+        assert te > tb >= 0 and rl == 0
+        key_g = dv0 if shape["latent"] else g
+        for f in range(f0, f0 + n):
+            if kind == 0:
+                assert segs[seq][0] <= f < segs[seq][1] and te <= seg_lens[seq]
+                assert toff == sgbo[seq]
+            else:
+                assert seq == f and te <= sl[f] and toff == sbo[seq]
+            cover.setdefault((f, key_g, kind, int(seq) if kind == 0 else -1), []).append(
+                (int(tb), int(te)))
+            parts.setdefault((f, key_g), []).append(int(part))
+    keys_g = (0, 256) if shape["latent"] else range(groups)
+    for f in range(F):
+        for g in keys_g:
+            for si, (b, e) in enumerate(segs):
+                want = int(seg_lens[si]) if b <= f < e else 0
+                _covers(cover.get((f, g, 0, si), []), want, ("segment", f, g, si))
+            _covers(cover.get((f, g, 1, -1), []), int(sl[f]), ("suffix", f, g))
+            n_parts = p["n_parts"][f, 0 if shape["latent"] else g]
+            assert sorted(parts.get((f, g), [])) == list(range(n_parts)), (f, g)
+    _check_slots(p, plan, F)
