@@ -640,23 +640,36 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
     // Chunk length: near work / n_sm, chosen among whole-tile lengths for the
     // smallest longest-CTA load under the longest-first assignment (one CTA
     // with a second item would otherwise set the kernel's end).
-    std::vector<long long> costs, heap;
+    // Longest-first assignment of every item cost (two per chunk, one per value
+    // half) to n_sm CTAs; its largest load.  All whole chunks cost the same and
+    // are the longest items, so they come first and leave the loads at q or q + 1
+    // times their cost; only the shorter last chunks of the sequences go through
+    // the heap.
+    static thread_local std::vector<long long> costs, heap;
+    const int m = std::max(1, n_sm);
     auto makespan = [&](long long c) {
+      const long long full = c + item_overhead;  // c is whole tiles
+      long long n_full = 0;
       costs.clear();
+      auto add = [&](long long len) {
+        n_full += 2 * (len / c);
+        const long long rest = len % c;
+        if (rest > 0) {
+          const long long n = (rest + tt - 1) / tt * tt + item_overhead;
+          costs.push_back(n);
+          costs.push_back(n);
+        }
+      };
       for (int f = 0; f < R; ++f) {
-        auto add = [&](long long len) {
-          for (long long b = 0; b < len; b += c) {
-            const long long n = (std::min(len, b + c) - b + tt - 1) / tt * tt + item_overhead;
-            costs.push_back(n);
-            costs.push_back(n);
-          }
-        };
         add(rows.len[f]);
         for (int sg : serving[f]) add(rows.segs[sg].len);
       }
       std::sort(costs.begin(), costs.end(), std::greater<long long>());
-      heap.assign(std::max(1, n_sm), 0);  // a min-heap of CTA loads (all zero is a heap)
-      long long worst = 0;
+      const long long q = n_full / m, r = n_full % m;
+      heap.assign(m, q * full);
+      for (long long i = 0; i < r; ++i) heap[i] += full;
+      std::make_heap(heap.begin(), heap.end(), std::greater<long long>());
+      long long worst = (r > 0 ? q + 1 : q) * full;
       for (long long x : costs) {
         std::pop_heap(heap.begin(), heap.end(), std::greater<long long>());
         heap.back() += x;
