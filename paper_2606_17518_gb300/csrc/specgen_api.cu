@@ -9,6 +9,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <climits>
 #include <map>
 #include <tuple>
 #include <queue>
@@ -647,7 +648,9 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
     // the heap.
     static thread_local std::vector<long long> costs, heap;
     const int m = std::max(1, n_sm);
-    auto makespan = [&](long long c) {
+    // `bound`: a candidate whose lower bound (the largest item, or the average
+    // CTA load) already exceeds it cannot be chosen, and is not simulated
+    auto makespan = [&](long long c, long long bound) {
       const long long full = c + item_overhead;  // c is whole tiles
       long long n_full = 0;
       costs.clear();
@@ -664,6 +667,13 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
         add(rows.len[f]);
         for (int sg : serving[f]) add(rows.segs[sg].len);
       }
+      long long total = n_full * full, largest = n_full > 0 ? full : 0;
+      for (long long x : costs) {
+        total += x;
+        largest = std::max(largest, x);
+      }
+      const long long lower = std::max(largest, (total + m - 1) / m);
+      if (lower > bound) return lower;
       std::sort(costs.begin(), costs.end(), std::greater<long long>());
       const long long q = n_full / m, r = n_full % m;
       heap.assign(m, q * full);
@@ -696,9 +706,9 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
     }
     std::sort(cand.begin(), cand.end());
     cand.erase(std::unique(cand.begin(), cand.end()), cand.end());
-    long long chunk = c0, best = makespan(c0);
+    long long chunk = c0, best = makespan(c0, LLONG_MAX);
     for (long long c : cand) {
-      const long long m = makespan(c);
+      const long long m = makespan(c, best);
       if (m < best || (m == best && c > chunk)) {
         best = m;
         chunk = c;
