@@ -54,9 +54,10 @@ def parse_args():
                          "decode over nested prefixes (fork events at 4096 and 8192 tokens, "
                          "8 forks each), timed beside the same forks as flat traces")
     ap.add_argument("--chunk", type=int, default=64, help="prefill chunk tokens per fork")
-    ap.add_argument("--kv-layout", choices=["rows", "tiled"], default="rows",
-                    help="K/V pool layout: token-major rows (default) or 8x8 core-matrix tiles "
-                         "(tensor-core shapes only)")
+    ap.add_argument("--kv-layout", choices=["rows", "tiled"], default="tiled",
+                    help="K/V pool layout: 8x8 core-matrix tiles (default; one bulk copy per "
+                         "page and head, the faster layout on the default workload) or "
+                         "token-major rows; latent (MLA) pools are always rows")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
     return ap.parse_args()
