@@ -365,3 +365,12 @@ def test_cascade_plans_cover_every_segment_once(case):
             n_parts = p["n_parts"][f, 0 if shape["latent"] else g]
             assert sorted(parts.get((f, g), [])) == list(range(n_parts)), (f, g)
     _check_slots(p, plan, F)
+
+
+@pytest.mark.parametrize("name", ["tiny_p512_f4", "fork_p8k_f8", "mla_p16k_f8"])
+def test_workload_lengths_match_the_workload(name):
+    """The lengths the planner tests draw are the ones the full workload uses."""
+    w = wl.make_workload(name)
+    pl, fo, sl = wl.workload_lengths(name)
+    assert np.array_equal(pl, w["prefix_lens"]) and np.array_equal(fo, w["fork_offsets"])
+    assert np.array_equal(sl, w["suffix_lens"])
