@@ -250,3 +250,35 @@ def test_pack_host_checks():
     assert pk(d(), 2, packed=fake + 4) == S.SPECGEN_ERR_SHAPE    # not 16-byte aligned
     assert pk(d(hkv=1, page_size=1, head_dim_qk=4, v_pages=None), 2) == S.SPECGEN_ERR_UNSUPPORTED
     assert lib.specgen_pack_pages(None, fake, 1, fake, None) == S.SPECGEN_ERR_NULL
+
+
+def test_header_is_plain_c_and_links(tmp_path):
+    """include/specgen.h compiles as C99 and a C program links against the
+    library and calls it (host-side checks only: no device work)."""
+    import os
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not found")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    src = tmp_path / "abi.c"
+    src.write_text(
+        '#include <stdio.h>\n#include <string.h>\n#include "specgen.h"\n'
+        "int main(void) {\n"
+        "  specgen_plan plan;\n"
+        "  memset(&plan, 0, sizeof(plan));\n"
+        "  if (specgen_fork_attn_plan(NULL, NULL, &plan, NULL) != SPECGEN_ERR_NULL) return 1;\n"
+        "  if (specgen_fork_attn_decode_staged(NULL, NULL, NULL, NULL, 0, NULL, NULL, 0, NULL)\n"
+        "      != SPECGEN_ERR_NULL) return 2;\n"
+        '  printf("%d %s\\n", specgen_version(), specgen_status_string(SPECGEN_ERR_SHAPE));\n'
+        "  return 0;\n}\n")
+    exe = tmp_path / "abi"
+    lib_dir = os.path.dirname(_lib.LIB_PATH)
+    cmd = [gcc, "-std=c99", "-Wall", "-Werror", "-I", os.path.join(root, "include"), str(src),
+           "-o", str(exe), "-L", lib_dir, "-lspecgen", "-Wl,-rpath," + lib_dir]
+    res = subprocess.run(cmd, capture_output=True, text=True)
+    assert res.returncode == 0, res.stderr
+    run = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert run.returncode == 0, (run.returncode, run.stderr)
+    assert run.stdout.split()[0].isdigit()
