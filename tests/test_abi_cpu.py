@@ -282,3 +282,22 @@ def test_header_is_plain_c_and_links(tmp_path):
     run = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
     assert run.returncode == 0, (run.returncode, run.stderr)
     assert run.stdout.split()[0].isdigit()
+
+
+def test_static_decode_refuses_oversized_calls_on_the_host():
+    """The allocation-free decode refuses a call whose workspace would exceed its
+    fixed scratch array before it touches the device."""
+    lib = _lib.load()
+    F = 2000
+    pl = np.array([64], np.int32)
+    fo = np.array([0, F], np.int32)
+    sl = np.ones(F, np.int32)
+    lens, keep = _lib.make_host_lens(pl, fo, sl)
+    w = dict(num_traces=1, total_forks=F, hq=64, hkv=8, dqk=128, dv=128, page_size=16,
+             num_pages=1 << 16, scale=0.088, v_pages=1, prefix_lens=pl, fork_offsets=fo,
+             suffix_lens=sl)
+    args = _fake_args(w)
+    assert _lib.specgen_fork_attn_workspace_size(args, lens) > (16 << 20)
+    assert lib.specgen_fork_attn_decode_static(C.byref(args), C.byref(lens), None) == \
+        _lib.SPECGEN_ERR_WORKSPACE
+    assert lib.specgen_fork_attn_decode_static(None, C.byref(lens), None) == _lib.SPECGEN_ERR_NULL
