@@ -6,8 +6,11 @@
 A step is one complete fork-decode call (prefix stage + suffix stage + merge)
 for every fork of the workload: one decode token per fork, one attention layer.
 Metric: tokens/s = forks per step / seconds per step.  The default workload is
-the reasoning-trace fork: one 8192-token shared prefix, 8 forks with suffixes
-in [64, 512], Hq=64, Hkv=8, head dim 128, page 16, shuffled pages.
+the largest one, the ragged multi-trace batch: 8 independent reasoning traces
+with prefixes uniform in [4096, 32768] tokens, each forked into 4-16 branches
+with suffixes uniform in [32, 1024], Hq=64, Hkv=8, head dim 128, page 16,
+shuffled pages (708 MB of unique KV with its seed); ``--workload`` picks the
+others.
 
 Timing: W untimed warm-up steps, then K steps between CUDA events on the
 launching stream, bracketed by a barrier and a device synchronise.  Inputs
@@ -34,7 +37,7 @@ import sys
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
-DEFAULT_WORKLOAD = "fork_p8k_f8"
+DEFAULT_WORKLOAD = "ragged_t8"
 
 
 def parse_args():

@@ -221,18 +221,29 @@ specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* arg
  * so they cannot supply args->workspace.  This entry point ignores
  * args->workspace / workspace_bytes and uses a library-owned scratch array of
  * 16 MiB (SPECGEN_STATIC_WORKSPACE_BYTES) that every GPU loading the library
- * keeps until the process exits; it allocates nothing.  A call whose
- * specgen_fork_attn_workspace_size exceeds that returns SPECGEN_ERR_WORKSPACE.
- * The first call on a device looks up the array's device address (a CUDA
- * runtime query), so make that first call before any stream capture.  All calls
- * share the one array: calls that may overlap on the GPU (different streams,
- * or host threads) race and must be serialised by the caller.  The status word
- * read by specgen_workspace_status lives in that array too and is not exposed
- * here: an out-of-range page id is skipped silently. */
+ * keeps until the process exits; it allocates nothing.  Each call is planned
+ * once on the host; a call that needs more scratch than the array holds
+ * (specgen_fork_attn_workspace_size above 16 MiB) returns SPECGEN_ERR_WORKSPACE
+ * before any CUDA call.  Every call then asks the runtime for the array's
+ * device address on the calling thread's current device (a host-side query;
+ * nothing is cached, so a context created again is handled).  All calls share
+ * the one array and each leaves its contents behind (the plan upload resets
+ * the status word): calls that may overlap on the GPU (different streams, or
+ * host threads) race and must be serialised by the caller.  The status word of
+ * the array (a page id outside the pool was skipped, or a device-side wait hit
+ * its limit and the outputs are not valid) is read with
+ * specgen_static_workspace_status; without that read both go unnoticed. */
 #define SPECGEN_STATIC_WORKSPACE_BYTES (16u << 20)
 specgen_status specgen_fork_attn_decode_static(const specgen_fork_attn_args* args,
                                                const specgen_host_lens* lens,
                                                void* cuda_stream);
+
+/* specgen_workspace_status for the scratch array of
+ * specgen_fork_attn_decode_static on the current device: synchronises
+ * `cuda_stream` and returns SPECGEN_OK, SPECGEN_ERR_INDEX or
+ * SPECGEN_ERR_TIMEOUT for the last static call that ran (SPECGEN_ERR_CUDA if
+ * the array's address cannot be had).  (No counterpart in the paper.) */
+specgen_status specgen_static_workspace_status(void* cuda_stream);
 
 /* Standalone log-sum-exp merge of two partial attentions over disjoint key
  * sets (the combination step of the split computation):

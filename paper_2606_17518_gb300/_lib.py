@@ -48,6 +48,7 @@ EXPORTED = [
     "specgen_pack_pages",
     "specgen_unpack_pages",
     "specgen_workspace_status",
+    "specgen_static_workspace_status",
     "specgen_status_string",
     "specgen_version",
 ]
@@ -187,6 +188,8 @@ def load() -> C.CDLL:
     lib.specgen_lse_merge.argtypes = [C.c_void_p] * 6 + [C.c_int, C.c_int, C.c_int, C.c_void_p]
     lib.specgen_workspace_status.restype = C.c_int
     lib.specgen_workspace_status.argtypes = [C.c_void_p, C.c_void_p]
+    lib.specgen_static_workspace_status.restype = C.c_int
+    lib.specgen_static_workspace_status.argtypes = [C.c_void_p]
     lib.specgen_status_string.restype = C.c_char_p
     lib.specgen_status_string.argtypes = [C.c_int]
     lib.specgen_version.restype = C.c_int
@@ -414,6 +417,11 @@ def specgen_lse_merge(out_a, lse_a, out_b, lse_b, out, lse, rows: int, dv: int, 
 
 def specgen_workspace_status(workspace, stream: int = 0) -> int:
     return int(load().specgen_workspace_status(_ptr(workspace), C.c_void_p(stream)))
+
+
+def specgen_static_workspace_status(stream: int = 0) -> int:
+    """Status word of the scratch array used by specgen_fork_attn_decode_static."""
+    return int(load().specgen_static_workspace_status(C.c_void_p(stream)))
 
 
 def specgen_version() -> int:

@@ -825,8 +825,15 @@ thread_local HostPlan t_plan;
 thread_local std::vector<unsigned char> t_plan_bytes;
 
 
-// host_dst == nullptr: upload the plan region to the workspace on cuda_stream;
-// otherwise copy it into host_dst (host_bytes long) and make no CUDA call.
+// Plans one call on the host: the plan region (zeroed header, then the work
+// list) into t_plan_bytes and the launch shapes into *plan.  No CUDA call;
+// SPECGEN_ERR_WORKSPACE when args->workspace_bytes is below what the call needs.
+specgen_status plan_build(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
+                          specgen_plan* plan);
+
+// plan_build, then: host_dst == nullptr uploads the plan region to the workspace
+// on cuda_stream; otherwise it is copied into host_dst (host_bytes long) and no
+// CUDA call is made.
 specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
                          specgen_plan* plan, void* cuda_stream, void* host_dst = nullptr,
                          size_t host_bytes = 0);
@@ -932,11 +939,8 @@ specgen_status specgen_fork_prefill_plan_host(const specgen_fork_attn_args* args
 
 namespace {
 
-specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
-                         specgen_plan* plan, void* cuda_stream, void* host_dst,
-                         size_t host_bytes) {
-  specgen_status st;
-  if ((st = check_pointers(args)) != SPECGEN_OK) return st;
+specgen_status plan_build(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
+                          specgen_plan* plan) {
   build_plan(s, rows, &t_plan);
   const Layout L = layout_of(s, t_plan);
   if (args->workspace_bytes < L.ws_end) return SPECGEN_ERR_WORKSPACE;
@@ -965,18 +969,6 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
   put(L.part_base_off, t_plan.part_base.data(), (size_t)s.F * 4);
   put(L.n_parts_off, t_plan.n_parts.data(), t_plan.n_parts.size() * 4);
 
-  if (host_dst) {
-    if (host_bytes < t_plan_bytes.size()) return SPECGEN_ERR_WORKSPACE;
-    memcpy(host_dst, t_plan_bytes.data(), t_plan_bytes.size());
-  } else {
-    cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-    unsigned char* ws = static_cast<unsigned char*>(args->workspace);
-    // one upload: the zeroed header (status word), then the plan
-    if (cudaMemcpyAsync(ws, t_plan_bytes.data(), L.ws_plan + L.plan_bytes,
-                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
-      return SPECGEN_ERR_CUDA;
-  }
-
   plan->valid = 1;
   plan->n_tc_items = h.n_tc;
   plan->n_tc_ctas = h.n_tc_ctas;
@@ -1001,6 +993,36 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
   plan->offsets[5] = (int64_t)L.n_parts_off;
   plan->offsets[6] = t_plan.n_parts.empty() ? 0 : (int64_t)*std::max_element(t_plan.n_parts.begin(), t_plan.n_parts.end());
   return SPECGEN_OK;
+}
+
+// One upload of the plan region built last on this thread: the zeroed header
+// (status word), then the plan.
+specgen_status upload_plan(void* workspace, void* cuda_stream) {
+  if (cudaMemcpyAsync(workspace, t_plan_bytes.data(), t_plan_bytes.size(), cudaMemcpyHostToDevice,
+                      static_cast<cudaStream_t>(cuda_stream)) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
+}
+
+specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
+                         specgen_plan* plan, void* cuda_stream, void* host_dst,
+                         size_t host_bytes) {
+  specgen_status st;
+  if ((st = check_pointers(args)) != SPECGEN_OK) return st;
+  if ((st = plan_build(args, s, rows, plan)) != SPECGEN_OK) {
+    memset(plan, 0, sizeof(*plan));
+    return st;
+  }
+  if (host_dst) {
+    if (host_bytes < t_plan_bytes.size()) {
+      memset(plan, 0, sizeof(*plan));
+      return SPECGEN_ERR_WORKSPACE;
+    }
+    memcpy(host_dst, t_plan_bytes.data(), t_plan_bytes.size());
+    return SPECGEN_OK;
+  }
+  if ((st = upload_plan(args->workspace, cuda_stream)) != SPECGEN_OK) memset(plan, 0, sizeof(*plan));
+  return st;
 }
 
 }  // namespace
@@ -1378,22 +1400,15 @@ namespace {
 constexpr size_t kStaticWorkspaceBytes = 16u << 20;  // 16 MiB
 static __device__ __align__(256) unsigned char g_static_workspace[kStaticWorkspaceBytes];
 
-constexpr int kMaxDevices = 64;
-void* g_static_ws_ptr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device.  Host code may
-// not use the symbol itself as a device pointer, so the address is looked up
-// once per device (with that device current) and cached.
+// Device address of the scratch array on the current device.  In host code
+// the symbol names a host-side stand-in, not device memory, so the address is
+// asked of the runtime with the device current, on every call: it is a host
+// query, and an address kept from an earlier call could belong to a context
+// that has since been torn down and created again.
 specgen_status static_workspace(void** ptr) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return SPECGEN_ERR_CUDA;
-  if (dev < 0 || dev >= kMaxDevices) return SPECGEN_ERR_UNSUPPORTED;
-  if (!g_static_ws_ptr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_static_workspace) != cudaSuccess || !p) return SPECGEN_ERR_CUDA;
-    g_static_ws_ptr[dev] = p;
-  }
-  *ptr = g_static_ws_ptr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_static_workspace) != cudaSuccess || !p) return SPECGEN_ERR_CUDA;
+  *ptr = p;
   return SPECGEN_OK;
 }
 
@@ -1405,20 +1420,31 @@ specgen_status specgen_fork_attn_decode_static(const specgen_fork_attn_args* arg
                                                const specgen_host_lens* lens,
                                                void* cuda_stream) {
   if (!args) return SPECGEN_ERR_NULL;
-  const size_t need = specgen_fork_attn_workspace_size(args, lens);
-  if (need == 0) {
-    Shape s;
-    const specgen_status st = check_shape(args, lens, &s);
-    return st == SPECGEN_OK ? SPECGEN_ERR_SHAPE : st;
-  }
-  if (need > kStaticWorkspaceBytes) return SPECGEN_ERR_WORKSPACE;
-  void* ws = nullptr;
-  specgen_status st = static_workspace(&ws);
+  Shape s;
+  specgen_status st = check_shape(args, lens, &s);
   if (st != SPECGEN_OK) return st;
   specgen_fork_attn_args a = *args;
-  a.workspace = ws;
   a.workspace_bytes = kStaticWorkspaceBytes;
-  return specgen_fork_attn_decode(&a, lens, cuda_stream);
+  // the other pointers are checked as for every call; the workspace is ours
+  a.workspace = reinterpret_cast<void*>(kAlign);
+  if ((st = check_pointers(&a)) != SPECGEN_OK) return st;
+  // planned once, on the host: a call that needs more than the array is
+  // refused here, before any CUDA call
+  specgen_plan plan;
+  memset(&plan, 0, sizeof(plan));
+  if ((st = plan_build(&a, s, rows_for_decode(lens, s.T, s.F), &plan)) != SPECGEN_OK) return st;
+  void* ws = nullptr;
+  if ((st = static_workspace(&ws)) != SPECGEN_OK) return st;
+  a.workspace = ws;
+  if ((st = upload_plan(ws, cuda_stream)) != SPECGEN_OK) return st;
+  return specgen_fork_attn_run(&a, &plan, cuda_stream);
+}
+
+specgen_status specgen_static_workspace_status(void* cuda_stream) {
+  void* ws = nullptr;
+  const specgen_status st = static_workspace(&ws);
+  if (st != SPECGEN_OK) return st;
+  return specgen_workspace_status(ws, cuda_stream);
 }
 
 }  // extern "C"

@@ -301,3 +301,47 @@ def test_static_decode_refuses_oversized_calls_on_the_host():
     assert lib.specgen_fork_attn_decode_static(C.byref(args), C.byref(lens), None) == \
         _lib.SPECGEN_ERR_WORKSPACE
     assert lib.specgen_fork_attn_decode_static(None, C.byref(lens), None) == _lib.SPECGEN_ERR_NULL
+
+
+def test_static_decode_plans_once():
+    """The allocation-free decode plans a call once: on a host without a GPU it
+    stops at its first CUDA call (the scratch array's address), after planning,
+    and takes about the host time of one plan -- not the two plans of a size
+    query followed by a planning decode."""
+    from conftest import cuda_available
+    if cuda_available():
+        pytest.skip("with a GPU the call would go on to launch kernels on the fake pointers")
+    import time
+    lib = _lib.load()
+    rng = np.random.default_rng(0)
+    T = 8  # a ragged batch: 8 traces of 4-16 forks, planning takes ~0.1 ms
+    pl = rng.integers(4096, 32769, T).astype(np.int32)
+    fo = np.concatenate([[0], np.cumsum(rng.integers(4, 17, T))]).astype(np.int32)
+    F = int(fo[-1])
+    sl = rng.integers(32, 1025, F).astype(np.int32)
+    lens, keep = _lib.make_host_lens(pl, fo, sl)
+    w = dict(num_traces=T, total_forks=F, hq=64, hkv=8, dqk=128, dv=128, page_size=16,
+             num_pages=1 << 20, scale=0.088, v_pages=1, prefix_lens=pl, fork_offsets=fo,
+             suffix_lens=sl)
+    args = _fake_args(w)
+    assert _lib.specgen_fork_attn_workspace_size(args, lens) <= (16 << 20)
+    dst = np.zeros(1 << 22, np.uint8)
+    plan = _lib.Plan()
+
+    def one_plan():
+        t = time.perf_counter()
+        st = lib.specgen_fork_attn_plan_host(C.byref(args), C.byref(lens), dst.ctypes.data,
+                                             dst.nbytes, C.byref(plan))
+        assert st == _lib.SPECGEN_OK
+        return time.perf_counter() - t
+
+    def static_call():
+        t = time.perf_counter()
+        st = lib.specgen_fork_attn_decode_static(C.byref(args), C.byref(lens), None)
+        assert st == _lib.SPECGEN_ERR_CUDA  # planned, then no device
+        return time.perf_counter() - t
+
+    static_call()
+    t_plan = np.median([one_plan() for _ in range(300)])
+    t_static = np.median([static_call() for _ in range(300)])
+    assert t_static < 1.5 * t_plan, (t_static, t_plan)

@@ -4,7 +4,9 @@ It serves callers that cannot allocate device memory (a plugin inside an
 engine that owns the device memory pool, or a latency-critical path where an
 allocation is not allowed): it takes no workspace and uses the library's
 fixed 16 MiB scratch array instead.  Its output must match the ordinary entry
-point's, call after call.  This file is collected last on purpose, so that a
+point's, call after call, and its status word (kept in that array) must be
+readable.  The refusal of oversized calls happens on the host and is checked
+by the CPU tests.  This file is collected last on purpose, so that a
 run that stops at the first failure has already run every other test.
 """
 
@@ -45,17 +47,25 @@ def test_static_matches_workspace_entry_point_twice(name):
         fin = np.isfinite(l_ref)
         assert np.array_equal(np.isfinite(lse), fin)
         assert np.max(np.abs(lse[fin] - l_ref[fin])) <= TOL_LSE
+        # the status word lives in the library's array: readable, and clean
+        assert _lib.specgen_static_workspace_status() == _lib.SPECGEN_OK
 
 
-def test_static_rejects_oversized_calls():
-    """A consistent workload whose workspace exceeds 16 MiB is refused on the host."""
+def test_static_status_reports_a_bad_page_id():
+    """A page id outside the pool is skipped by the kernels and reported in the
+    scratch array's status word; the next clean call resets it."""
+    import torch
     from paper_2606_17518_gb300.fork_attn import ForkDecode
-    spec = wl.WorkloadSpec(name="many_forks", num_traces=1, prefix_len=(64, 64),
-                           forks=(2000, 2000), suffix_len=(1, 1), hq=64, hkv=8, dqk=128,
-                           dv=128, page_size=16, seed=7)
-    w = wl.make_workload(spec)
-    fd = ForkDecode(w)
-    assert fd.ws_bytes > (16 << 20)
-    with pytest.raises(_lib.SpecgenError) as err:
-        _lib.specgen_fork_attn_decode_static(fd.args(with_ws=False), fd.lens)
-    assert err.value.status == _lib.SPECGEN_ERR_WORKSPACE
+    w = dict(wl.make_workload("tiny_p512_f4"))
+    good = ForkDecode(w)
+    w["suffix_table"] = w["suffix_table"].copy()
+    w["suffix_table"][0] = w["num_pages"] + 5
+    bad = ForkDecode(w)
+    _lib.specgen_fork_attn_decode_static(bad.args(with_ws=False), bad.lens)
+    torch.cuda.synchronize()
+    assert _lib.specgen_static_workspace_status() == _lib.SPECGEN_ERR_INDEX
+    o, _ = bad.results()
+    assert np.all(np.isfinite(o))
+    _lib.specgen_fork_attn_decode_static(good.args(with_ws=False), good.lens)
+    torch.cuda.synchronize()
+    assert _lib.specgen_static_workspace_status() == _lib.SPECGEN_OK
