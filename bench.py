@@ -274,12 +274,18 @@ def run_reference():
 
 
 # --------------------------------------------------------------------------- GPU arm
+# source files of each kernel (a stage of concurrent kernels is named "a+b")
+KERNEL_SOURCES = {"fork_tc": "fork_tc", "fork_suffix": "suffix_stage", "mla_tc": "mla_tc",
+                  "split_decode": "split_decode", "lse_merge": "lse_merge"}
+
+
 def kernel_source_sha(name: str) -> str:
     import hashlib
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2606_17518_gb300", "csrc")
+    stems = [KERNEL_SOURCES.get(k, k) for k in name.split("+")]
     for fn in sorted(os.listdir(csrc)):
-        if fn.startswith(name) or fn in ("common.cuh", "plan.h", "tc_common.cuh"):
+        if any(fn.startswith(st) for st in stems) or fn in ("common.cuh", "plan.h", "tc_common.cuh"):
             with open(os.path.join(csrc, fn), "rb") as fh:
                 h.update(fh.read())
     return h.hexdigest()[:16]
@@ -431,15 +437,18 @@ def run_ours():
         return t0.elapsed_time(t1) / (n_rep * len(g_list) * per_graph)
 
     tc_name = "mla_tc" if w["v_pages"] is None else "fork_tc"
-    kernel_names = ([tc_name] if plans[0].n_tc_items > 0 else []) + \
+    # the partial-attention kernels of a step: the prefix kernel and, beside it
+    # on the SMs it leaves free, the suffix stage (they run concurrently, so
+    # they are timed together as one stage), or the split-K kernel
+    part_kernels = ([tc_name] if plans[0].n_tc_ctas > 0 else []) + \
+        (["fork_suffix"] if plans[0].n_sfx_ctas > 0 else []) + \
         (["split_decode"] if plans[0].n_split_items > 0 else [])
     partials_ms = stage_ms(lib.specgen_fork_attn_run_partials)
     merge_ms = stage_ms(lib.specgen_fork_attn_run_merge)
     suffix_stage = measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes)
-    # one launch per partial kernel kind (a plan uses one of them) plus the merge
-    kernel_ms = [partials_ms / max(1, len(kernel_names))] * len(kernel_names) + [merge_ms]
-    kernel_names = kernel_names + ["lse_merge"]
-    launches = len(kernel_names)
+    kernel_names = ["+".join(part_kernels), "lse_merge"]
+    kernel_ms = [partials_ms, merge_ms]
+    launches = len(part_kernels) + 1
     n_slots = per_graph * max(1, min(8, K // per_graph))
     status = reps[0].status(sp)
     if status != 0:
@@ -460,14 +469,14 @@ def run_ours():
     hbm, tf_burst, tf_sus, peak_src = measured_peaks()
     # algorithmic bytes of the dominant launch: what that kernel must read/write once
     dom_name = kernel_names[dom] if kernel_names else None
-    if dom_name in ("fork_tc", "mla_tc", "split_decode"):
+    if dom_name != "lse_merge":
         # the kernel that reads the KV: unique prefix + every suffix + Q
         dom_bytes = nbytes["prefix"] + nbytes["suffix"] + nbytes["q"]
     else:
         dom_bytes = nbytes["total"]
     achieved = dom_bytes / (kernel_ms[dom] * 1e-3) / 1e9 if kernel_ms else None
     traffic = recorded_traffic(kernel_names[dom], f"{ARGS.workload}:{layout}")
-    if dom_name == "mla_tc":
+    if dom_name.startswith("mla_tc"):
         # latent attention is a dense contraction (the 128 heads of a fork share
         # every latent key): bound by the bf16 tensor pipe, timed inside a long
         # loop of steps, so against the sustained bf16 peak

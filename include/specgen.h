@@ -70,7 +70,8 @@ typedef struct {
   int page_size;                /* 16 or 64 tokens */
   int num_pages;                /* pool size; page ids are checked against it */
   float scale;                  /* softmax scale sigma applied to q.k, finite and > 0 */
-  const void* q;                /* bf16 [total_forks][hq][head_dim_qk] */
+  const void* q;                /* bf16 [total_forks][hq][head_dim_qk]; q and the pools
+                                   16-byte aligned (else SPECGEN_ERR_SHAPE) */
   const void* k_pages;          /* bf16, layout above */
   const void* v_pages;          /* bf16, layout above, or NULL (latent KV) */
   const int32_t* prefix_block_table;
@@ -130,6 +131,9 @@ typedef struct {
   int64_t plan_bytes;           /* plan bytes copied into the workspace */
   int64_t ws_plan_off, ws_part_o_off, ws_part_lse_off, ws_end;
   int64_t offsets[8];           /* internal offsets inside the plan region */
+  int32_t n_sfx_items;          /* suffix-stage work items (per-fork suffix page ranges) */
+  int32_t n_sfx_ctas;           /* CTAs of the suffix-stage kernel */
+  int64_t sfx_offsets[2];       /* internal offsets inside the plan region */
 } specgen_plan;
 
 /* Bytes of workspace one call needs (0 on invalid input).  Depends only on the

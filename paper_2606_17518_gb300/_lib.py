@@ -117,6 +117,7 @@ class Plan(C.Structure):
         ("flags", C.c_int32), ("n_part_groups", C.c_int32),
         ("plan_bytes", C.c_int64), ("ws_plan_off", C.c_int64), ("ws_part_o_off", C.c_int64),
         ("ws_part_lse_off", C.c_int64), ("ws_end", C.c_int64), ("offsets", C.c_int64 * 8),
+        ("n_sfx_items", C.c_int32), ("n_sfx_ctas", C.c_int32), ("sfx_offsets", C.c_int64 * 2),
     ]
 
 

@@ -199,9 +199,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
   const int n_items = it_end - it_begin;
-  // let the merge grid (a programmatic dependent) get launched early; it waits
-  // for this grid's completion before it reads anything
-  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
   // the CTA's first items, one per lane (40-byte records): the plan is written
   // by a host copy, never by a kernel, so it is read before the wait below
@@ -264,6 +261,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  // The next kernel of the stream (the suffix stage, or the merge: a
+  // programmatic dependent) may be launched once every CTA is past this wait,
+  // i.e. once the previous kernel has finished: the suffix stage runs beside
+  // this grid and relies on that ordering; the merge waits for this grid's
+  // completion before it reads any partial.
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   if (warp == 0) {
     __syncwarp();
     for (int k = lane; k < n_cached; k += 32) items[k] = clamp_item(items[k], p.suffix_lens);
@@ -889,6 +892,10 @@ cudaError_t launch_d(const TcParams& p, const CUtensorMap& mk, const CUtensorMap
 }
 
 }  // namespace
+
+bool fork_tc_block_map(CUtensorMap* map, const void* pool, int D, int hkv, int num_pages) {
+  return make_pool_map_v(map, pool, D, kPB, hkv, num_pages);
+}
 
 bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G) {
   return !latent && dqk == dv && (dqk == 64 || dqk == 128) && page_size == kPB && G <= 128;

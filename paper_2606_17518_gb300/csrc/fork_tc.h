@@ -1,5 +1,6 @@
 // Host-visible interface of the tensor-core fork-decode kernel (internal).
 #pragma once
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -28,6 +29,9 @@ struct TcParams {
 };
 
 bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G);
+// Tensor map of a paged pool [num_pages][hkv][16][D] bf16 whose box is one whole
+// (page, head) block, landing as [D/64 panels][16 rows][128 B], 128-byte swizzled.
+bool fork_tc_block_map(CUtensorMap* map, const void* pool, int D, int hkv, int num_pages);
 int fork_tc_tile_tokens(int dqk);
 int fork_tc_page_size();
 // causal: the plan holds causal suffix items (TcItem::row_limit0 > 0)

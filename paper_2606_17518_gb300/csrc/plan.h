@@ -65,6 +65,9 @@ struct TcItem {
 struct PlanHeader {
   int32_t n_split, n_tc, n_tc_ctas, n_forks;
   int32_t split_off, tc_off, cta_items_off, cta_offsets_off, part_base_off, n_parts_off;
+  // suffix-stage items (TcItem records, worker order) and the worker ranges
+  // ([n_sfx_ctas * suffix warps + 1] offsets)
+  int32_t n_sfx, n_sfx_ctas, sfx_off, sfx_offsets_off;
 };
 
 }  // namespace specgen

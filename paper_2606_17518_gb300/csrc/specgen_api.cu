@@ -24,6 +24,7 @@
 #include "fork_tc.h"
 #include "mla_tc.h"
 #include "split_decode.h"
+#include "suffix_stage.h"
 
 using namespace specgen;
 
@@ -131,6 +132,10 @@ specgen_status check_pointers(const specgen_fork_attn_args* a) {
       !a->suffix_block_table || !a->suffix_bt_offsets || !a->out || !a->lse || !a->workspace)
     return SPECGEN_ERR_NULL;
   if (reinterpret_cast<uintptr_t>(a->workspace) % kAlign != 0) return SPECGEN_ERR_WORKSPACE;
+  // queries and pools move in 16-byte pieces and bulk copies
+  const void* rows16[3] = {a->q, a->k_pages, a->v_pages};
+  for (const void* r : rows16)
+    if (reinterpret_cast<uintptr_t>(r) % 16 != 0) return SPECGEN_ERR_SHAPE;
   return SPECGEN_OK;
 }
 
@@ -139,6 +144,10 @@ struct HostPlan {
   std::vector<SplitItem> split;
   std::vector<TcItem> tc;
   std::vector<int32_t> cta_items, cta_offsets;
+  // suffix-stage items in worker order, worker w taking [sfx_offsets[w], [w+1])
+  std::vector<TcItem> sfx;
+  std::vector<int32_t> sfx_offsets;
+  int n_sfx_ctas = 0;
   std::vector<int32_t> part_base;
   std::vector<int32_t> n_parts;  // [forks][n_groups]: partial slots used by each head group
   int n_groups = 1;
@@ -334,6 +343,14 @@ void finish_tc_plan(HostPlan* hp, const std::vector<long long>& cost, int n_sm,
 constexpr long long kItemCost = 256;  // fixed cost of an item (Q staging, merge, pipeline refill)
 static_assert(kItemCost % 128 == 0, "item cost in whole tiles of every tile size");
 constexpr int kMinChunk = 128;        // smallest prefix chunk carved into a CTA's spare budget
+// Suffix stage (its own kernel beside the prefix CTAs, kSuffixWarps workers per
+// CTA): an item's fixed cost in pages (query rows in, partial out), and the
+// smallest load in pages worth a worker, which bounds the suffix CTAs of small
+// calls.
+constexpr long long kSfxItemPages = 1;
+constexpr long long kSfxMinWorkerPages = 2;
+constexpr long long kSfxMinPiecePages = 2;
+constexpr long long kSfxSplitMinPages = 8;  // beside a prefix: the least worker load that pays
 
 struct TcUnit {
   int kind, seq, g, fork0, nforks, len;
@@ -429,6 +446,52 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
   return ui == pfx.size();
 }
 
+// The suffix units over n_workers suffix-stage workers (cta = -1 - worker), in
+// one pass.  Every unit is laid on a ribbon as its item cost (kSfxItemPages)
+// followed by its pages, the units end to end; the ribbon of length T is cut
+// into n_workers runs of equal length (worker w takes positions
+// [T w / n, T (w+1) / n)), so the loads differ by at most a page or two.  A
+// unit is cut at page boundaries where a run ends, and no piece is shorter
+// than kSfxMinPiecePages unless its unit is.
+void place_suffix_stage(const std::vector<TcUnit>& sfx, int n_workers, int page,
+                        std::vector<TcPlacement>* placed) {
+  auto pages = [&](long long n) { return (n + page - 1) / page; };
+  long long T = 0;
+  for (const TcUnit& u : sfx) T += kSfxItemPages + pages(u.len);
+  auto bound = [&](long long w) { return T * w / n_workers; };  // first position of run w
+  long long g = 0;  // position on the ribbon
+  int w = 0;        // the worker whose run holds g
+  for (const TcUnit& u : sfx) {
+    const long long p0 = g + kSfxItemPages, end = p0 + pages(u.len);  // the unit's pages
+    int part = 0;
+    while (g < end) {
+      while (w + 1 < n_workers && bound(w + 1) <= g) ++w;
+      long long stop = std::min(end, w + 1 < n_workers ? bound(w + 1) : end);
+      stop = std::max(stop, std::min(end, p0 + 1));  // a piece holds at least a page
+      if (end - stop < kSfxMinPiecePages)
+        stop = end;  // no sliver at the unit's end
+      else if (stop - std::max(g, p0) < kSfxMinPiecePages)
+        stop = std::min(end, std::max(g, p0) + kSfxMinPiecePages);  // nor anywhere else
+      TcPlacement pl;
+      pl.cta = -1 - w;
+      TcItem& it = pl.item;
+      it.table_kind = 1;
+      it.seq = u.seq;
+      it.kv_head = u.g;
+      it.fork0 = u.fork0;
+      it.nforks = 1;
+      it.tok_begin = (int)((std::max(g, p0) - p0) * page);
+      it.tok_end = (int)std::min<long long>(u.len, (stop - p0) * page);
+      it.part = part++;
+      it.dv0 = 0;
+      it.table_off = -1;
+      it.row_limit0 = 0;
+      placed->push_back(pl);
+      g = stop;
+    }
+  }
+}
+
 void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   const int tt = fork_tc_tile_tokens(s.dqk);
   const int forks_per_item = std::max(1, 128 / s.G);
@@ -480,7 +543,44 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
                              f1 - f > 1 ? rows.len[f] : 0});
       f = f1;
     }
-  for (const TcUnit& u : sfx) total += (u.len + tt - 1) / tt * tt;
+  // The suffix stage takes the suffix units when each serves one query row
+  // (decode and cascade; prefill only when no chunk shares an item) and the
+  // group fits its n-tiles.  The grid is then split between the prefix CTAs
+  // and the suffix-stage CTAs in proportion to their work.
+  bool use_sfx = !sfx.empty() && suffix_stage_supported(s.dqk, s.dv, s.latent, s.B, s.G);
+  for (const TcUnit& u : sfx) use_sfx = use_sfx && u.nforks == 1 && u.row_limit0 == 0;
+  int n_sfx_sm = 0;
+  if (use_sfx) {
+    const int pg = fork_tc_page_size();
+    long long ws = 0, wp = 0, sfx_pages = 0;
+    for (const TcUnit& u : sfx) {
+      sfx_pages += (u.len + pg - 1) / pg;
+      ws += ((u.len + pg - 1) / pg + kSfxItemPages) * pg;
+    }
+    for (const TcUnit& u : pfx) wp += (u.len + tt - 1) / tt * tt + kItemCost;
+    const int n_all = std::max(1, n_sm);
+    constexpr long long kWorkersPerSm = kSuffixWarps * kSuffixCtasPerSm;
+    const long long most = std::max<long long>(
+        1, (sfx_pages + kWorkersPerSm * kSfxMinWorkerPages - 1) / (kWorkersPerSm * kSfxMinWorkerPages));
+    if (wp == 0) {
+      n_sfx_sm = (int)std::min<long long>(n_all, most);
+    } else if (n_all < 2) {
+      use_sfx = false;
+    } else {
+      long long n = (long long)llround((double)n_all * (double)ws / (double)(ws + wp));
+      n = std::max<long long>(1, std::min<long long>(std::min<long long>(n, n_all - 1), most));
+      n_sfx_sm = (int)n;
+      // a kernel of its own pays (one more launch in the chain, more partials to
+      // merge) only when each worker streams enough pages
+      if (sfx_pages < n * kWorkersPerSm * kSfxSplitMinPages) {
+        use_sfx = false;
+        n_sfx_sm = 0;
+      }
+    }
+  }
+  static thread_local std::vector<TcUnit> no_units;
+  std::vector<TcUnit>& tc_sfx = use_sfx ? no_units : sfx;
+  for (const TcUnit& u : tc_sfx) total += (u.len + tt - 1) / tt * tt;
   for (const TcUnit& u : pfx) total += u.len;
   // longest first, ties in their present order (a sort of (length, index) keys)
   auto longest_first = [](std::vector<TcUnit>& v) {
@@ -495,8 +595,8 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   longest_first(sfx);
   longest_first(pfx);
   placed.clear();
-  const int n_units = (int)(sfx.size() + pfx.size());
-  const int n_cta = std::max(1, n_sm);
+  const int n_units = (int)(tc_sfx.size() + pfx.size());
+  const int n_cta = std::max(1, n_sm - n_sfx_sm);
   if (n_units > 0) {
     // Budget search.  Loads and item costs are whole tiles, so feasibility only
     // changes at multiples of the tile: search the budget in tiles.  Start
@@ -506,17 +606,17 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     // Every pass records its placements; `placed` keeps those of the pass that
     // last fitted, which is the one at the final budget.
     static thread_local std::vector<long long> load, order;
-    const long long n_items = (long long)sfx.size() + std::max<long long>((long long)pfx.size(), n_cta);
+    const long long n_items = (long long)tc_sfx.size() + std::max<long long>((long long)pfx.size(), n_cta);
     long long lo = std::max<long long>(kItemCost + tt, (total + kItemCost * n_items) / n_cta) / tt;
     long long hi = lo;
-    while (!pack_tc(sfx, pfx, n_cta, hi * tt, tt, &load, &order, &trial)) {
+    while (!pack_tc(tc_sfx, pfx, n_cta, hi * tt, tt, &load, &order, &trial)) {
       lo = hi;
       hi += std::max<long long>(1, hi / 16);
     }
     placed.swap(trial);
     while (hi - lo > 1) {
       const long long mid = (lo + hi) / 2;
-      if (pack_tc(sfx, pfx, n_cta, mid * tt, tt, &load, &order, &trial)) {
+      if (pack_tc(tc_sfx, pfx, n_cta, mid * tt, tt, &load, &order, &trial)) {
         hi = mid;
         placed.swap(trial);
       } else {
@@ -524,6 +624,10 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
       }
     }
   }
+  // the suffix-stage grid has kSuffixCtasPerSm CTAs on each of its n_sfx_sm SMs
+  if (use_sfx)
+    place_suffix_stage(sfx, n_sfx_sm * kSuffixCtasPerSm * kSuffixWarps, fork_tc_page_size(),
+                       &placed);
   // Partial slots: per (row, head group) the prefix chunks come first (segment
   // by segment, enclosing segments first), then the suffix pieces; a row owns
   // as many slots as its busiest head group.  A prefix chunk's part is the
@@ -578,27 +682,41 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
   const bool host_off = rows.prefix_bt_offsets && rows.suffix_bt_offsets;
   hp->tc.clear();
   hp->cta_offsets.assign(1, 0);
-  per_cta.assign(n_cta + 1, 0);  // counting sort of the placements by CTA
-  for (const TcPlacement& pl : placed) ++per_cta[pl.cta + 1];
-  for (int c = 0; c < n_cta; ++c) per_cta[c + 1] += per_cta[c];
+  // lists 0 .. n_cta-1: the prefix CTAs; then one per suffix-stage worker
+  const int n_workers = n_sfx_sm * kSuffixCtasPerSm * kSuffixWarps;
+  const int n_lists = n_cta + n_workers;
+  auto list_of = [&](const TcPlacement& pl) { return pl.cta >= 0 ? pl.cta : n_cta + (-1 - pl.cta); };
+  per_cta.assign(n_lists + 1, 0);  // counting sort of the placements by list
+  for (const TcPlacement& pl : placed) ++per_cta[list_of(pl) + 1];
+  for (int c = 0; c < n_lists; ++c) per_cta[c + 1] += per_cta[c];
   by_cta.resize(placed.size());
   next.assign(per_cta.begin(), per_cta.end() - 1);
-  for (const TcPlacement& pl : placed) by_cta[next[pl.cta]++] = pl.item;
+  for (const TcPlacement& pl : placed) by_cta[next[list_of(pl)]++] = pl.item;
+  auto finish = [&](TcItem it) {
+    if (it.table_kind == 1)
+      it.part += n_pre[(size_t)it.fork0 * s.hkv + it.kv_head];
+    else
+      it.part += base_of(it.seq, it.kv_head, it.fork0);
+    it.table_off = host_off ? (it.table_kind == 0 ? rows.prefix_bt_offsets[it.seq]
+                                                  : rows.suffix_bt_offsets[it.seq])
+                            : -1;
+    return it;
+  };
   for (int c = 0; c < n_cta; ++c) {
     if (per_cta[c + 1] == per_cta[c]) continue;  // empty CTAs are dropped
-    for (int i = per_cta[c]; i < per_cta[c + 1]; ++i) {
-      TcItem it = by_cta[i];
-      if (it.table_kind == 1)
-        it.part += n_pre[(size_t)it.fork0 * s.hkv + it.kv_head];
-      else
-        it.part += base_of(it.seq, it.kv_head, it.fork0);
-      it.table_off = host_off ? (it.table_kind == 0 ? rows.prefix_bt_offsets[it.seq]
-                                                    : rows.suffix_bt_offsets[it.seq])
-                              : -1;
-      hp->tc.push_back(it);
-    }
+    for (int i = per_cta[c]; i < per_cta[c + 1]; ++i) hp->tc.push_back(finish(by_cta[i]));
     hp->cta_offsets.push_back((int32_t)hp->tc.size());
   }
+  // every worker keeps its place (worker w is warp w % kSuffixWarps of CTA
+  // w / kSuffixWarps), empty or not
+  hp->sfx.clear();
+  hp->sfx_offsets.assign(1, 0);
+  for (int w = 0; w < n_workers; ++w) {
+    for (int i = per_cta[n_cta + w]; i < per_cta[n_cta + w + 1]; ++i)
+      hp->sfx.push_back(finish(by_cta[i]));
+    hp->sfx_offsets.push_back((int32_t)hp->sfx.size());
+  }
+  hp->n_sfx_ctas = n_sfx_sm * kSuffixCtasPerSm;
   hp->cta_items.clear();
 }
 
@@ -608,6 +726,9 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
   const int R = (int)rows.seq.size();
   hp->split.clear();
   hp->tc.clear();
+  hp->sfx.clear();
+  hp->sfx_offsets.assign(1, 0);
+  hp->n_sfx_ctas = 0;
   hp->cta_items.clear();
   hp->cta_offsets.assign(1, 0);
   hp->part_base.assign(s.F, 0);
@@ -801,6 +922,7 @@ void build_plan(const Shape& s, const Rows& rows, HostPlan* hp) {
 
 struct Layout {
   size_t split_off, tc_off, cta_items_off, cta_offsets_off, part_base_off, n_parts_off, plan_bytes;
+  size_t sfx_off, sfx_offsets_off;
   size_t ws_plan, ws_part_o, ws_part_lse, ws_end;
 };
 
@@ -810,7 +932,9 @@ Layout layout_of(const Shape& s, const HostPlan& hp) {
   L.tc_off = align_up(L.split_off + hp.split.size() * sizeof(SplitItem), 16);
   L.cta_items_off = align_up(L.tc_off + hp.tc.size() * sizeof(TcItem), 16);
   L.cta_offsets_off = align_up(L.cta_items_off + hp.cta_items.size() * 4, 16);
-  L.part_base_off = align_up(L.cta_offsets_off + hp.cta_offsets.size() * 4, 16);
+  L.sfx_off = align_up(L.cta_offsets_off + hp.cta_offsets.size() * 4, 16);
+  L.sfx_offsets_off = align_up(L.sfx_off + hp.sfx.size() * sizeof(TcItem), 16);
+  L.part_base_off = align_up(L.sfx_offsets_off + hp.sfx_offsets.size() * 4, 16);
   L.n_parts_off = align_up(L.part_base_off + (size_t)s.F * 4, 16);
   L.plan_bytes = L.n_parts_off + hp.n_parts.size() * 4;
   L.ws_plan = kHeaderBytes;
@@ -957,6 +1081,10 @@ specgen_status plan_build(const specgen_fork_attn_args* args, const Shape& s, co
   h.cta_offsets_off = (int32_t)L.cta_offsets_off;
   h.part_base_off = (int32_t)L.part_base_off;
   h.n_parts_off = (int32_t)L.n_parts_off;
+  h.n_sfx = (int32_t)t_plan.sfx.size();
+  h.n_sfx_ctas = t_plan.n_sfx_ctas;
+  h.sfx_off = (int32_t)L.sfx_off;
+  h.sfx_offsets_off = (int32_t)L.sfx_offsets_off;
   unsigned char* b = t_plan_bytes.data() + L.ws_plan;
   memcpy(b, &h, sizeof(h));
   auto put = [&](size_t off, const void* src, size_t bytes) {
@@ -966,6 +1094,8 @@ specgen_status plan_build(const specgen_fork_attn_args* args, const Shape& s, co
   put(L.tc_off, t_plan.tc.data(), t_plan.tc.size() * sizeof(TcItem));
   put(L.cta_items_off, t_plan.cta_items.data(), t_plan.cta_items.size() * 4);
   put(L.cta_offsets_off, t_plan.cta_offsets.data(), t_plan.cta_offsets.size() * 4);
+  put(L.sfx_off, t_plan.sfx.data(), t_plan.sfx.size() * sizeof(TcItem));
+  put(L.sfx_offsets_off, t_plan.sfx_offsets.data(), t_plan.sfx_offsets.size() * 4);
   put(L.part_base_off, t_plan.part_base.data(), (size_t)s.F * 4);
   put(L.n_parts_off, t_plan.n_parts.data(), t_plan.n_parts.size() * 4);
 
@@ -992,6 +1122,10 @@ specgen_status plan_build(const specgen_fork_attn_args* args, const Shape& s, co
   plan->offsets[4] = (int64_t)L.part_base_off;
   plan->offsets[5] = (int64_t)L.n_parts_off;
   plan->offsets[6] = t_plan.n_parts.empty() ? 0 : (int64_t)*std::max_element(t_plan.n_parts.begin(), t_plan.n_parts.end());
+  plan->n_sfx_items = h.n_sfx;
+  plan->n_sfx_ctas = h.n_sfx_ctas;
+  plan->sfx_offsets[0] = (int64_t)L.sfx_off;
+  plan->sfx_offsets[1] = (int64_t)L.sfx_offsets_off;
   return SPECGEN_OK;
 }
 
@@ -1175,6 +1309,32 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     if (e != cudaSuccess) return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
   }
+  if ((stages & 1) && plan->n_sfx_ctas > 0) {
+    SfxParams xp;
+    xp.q = sp.q;
+    xp.k_pages = static_cast<const __nv_bfloat16*>(args->k_pages);
+    xp.v_pages = static_cast<const __nv_bfloat16*>(args->v_pages);
+    xp.suffix_bt = args->suffix_block_table;
+    xp.suffix_bt_off = args->suffix_bt_offsets;
+    xp.items = reinterpret_cast<const TcItem*>(pl + plan->sfx_offsets[0]);
+    xp.worker_offsets = reinterpret_cast<const int32_t*>(pl + plan->sfx_offsets[1]);
+    xp.part_base = reinterpret_cast<const int32_t*>(pl + plan->offsets[4]);
+    xp.part_o = part_o;
+    xp.part_lse = part_lse;
+    xp.status = sp.status;
+    xp.suffix_lens = args->suffix_lens;
+    xp.hq = args->hq;
+    xp.hkv = args->hkv;
+    xp.G = args->hq / args->hkv;
+    xp.dv = args->head_dim_v;
+    xp.num_pages = args->num_pages;
+    xp.scale_log2 = sp.scale_log2;
+    xp.wait_first = plan->n_tc_ctas > 0 ? 0 : 1;
+    if (launch_suffix_stage(xp, args->k_pages, args->v_pages, plan->n_sfx_ctas, args->head_dim_qk,
+                            args->kv_layout == SPECGEN_KV_TILED, stream) != cudaSuccess)
+      return SPECGEN_ERR_CUDA;
+    if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
+  }
   if ((stages & 1) && plan->n_split_items > 0) {
     if (launch_split_decode(sp, plan->n_split_items, args->v_pages == nullptr, stream) !=
         cudaSuccess)
@@ -1195,7 +1355,8 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     mp.n_groups = plan->n_part_groups;
     mp.hq = args->hq;
     mp.dv = args->head_dim_v;
-    if (launch_merge_parts(mp, stream, plan->n_tc_ctas > 0 && plan->n_split_items == 0) !=
+    if (launch_merge_parts(mp, stream,
+                           (plan->n_tc_ctas > 0 || plan->n_sfx_ctas > 0) && plan->n_split_items == 0) !=
         cudaSuccess)
       return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;

@@ -164,6 +164,10 @@ def test_null_and_workspace_errors(w):
     assert _plan_status(_fake_args(w, q=None), lens) == S.SPECGEN_ERR_NULL
     assert _plan_status(_fake_args(w, out=None), lens) == S.SPECGEN_ERR_NULL
     assert _plan_status(_fake_args(w, workspace=0x10010), lens) == S.SPECGEN_ERR_WORKSPACE
+    # queries and pools move in 16-byte pieces and bulk copies
+    assert _plan_status(_fake_args(w, q=0x10008), lens) == S.SPECGEN_ERR_SHAPE
+    assert _plan_status(_fake_args(w, k_pages=0x10004), lens) == S.SPECGEN_ERR_SHAPE
+    assert _plan_status(_fake_args(w, v_pages=0x10002), lens) == S.SPECGEN_ERR_SHAPE
     assert _plan_status(_fake_args(w, workspace_bytes=1024), lens) == S.SPECGEN_ERR_WORKSPACE
     plan = _lib.Plan()
     lib = _lib.load()

@@ -19,6 +19,7 @@ from paper_2606_17518_gb300 import _lib, workloads as wl
 FAKE = 0x10000
 TC_WORDS = 11      # TcItem: int32 fields
 SPLIT_WORDS = 10   # SplitItem: int32 fields
+SUFFIX_WARPS = 8   # worker warps per suffix-stage CTA
 
 
 def _args(T, F, hq, hkv, dqk, dv, B, latent, **kw):
@@ -56,11 +57,22 @@ def _parse(plan, buf):
     assert not buf[:plan.ws_plan_off].any()  # the status header goes up zeroed
     region = buf[plan.ws_plan_off:plan.ws_plan_off + plan.plan_bytes]
     w = region.view(np.int32)
-    n_split, n_tc, n_ctas, n_forks, so, to, _, coo, pbo_, npo = (int(x) for x in w[:10])
+    (n_split, n_tc, n_ctas, n_forks, so, to, _, coo, pbo_, npo,
+     n_sfx, n_sfx_ctas, sfo, sfoo) = (int(x) for x in w[:14])
     words = lambda off, n: w[off // 4: off // 4 + n]
+    tc_only = words(to, n_tc * TC_WORDS).reshape(n_tc, TC_WORDS)
+    sfx = words(sfo, n_sfx * TC_WORDS).reshape(n_sfx, TC_WORDS)
+    n_workers = n_sfx_ctas * SUFFIX_WARPS
+    sfx_offsets = words(sfoo, n_workers + 1)
+    # the suffix-stage workers: every item in exactly one worker's range, in order
+    assert plan.n_sfx_items == n_sfx and plan.n_sfx_ctas == n_sfx_ctas
+    assert sfx_offsets[0] == 0 and sfx_offsets[-1] == n_sfx and np.all(np.diff(sfx_offsets) >= 0)
+    for kind, seq, g, f0, nf, tb, te, part, dv0, toff, rl in sfx:
+        assert kind == 1 and nf == 1 and rl == 0 and dv0 == 0
     return dict(
         split=words(so, n_split * SPLIT_WORDS).reshape(n_split, SPLIT_WORDS),
-        tc=words(to, n_tc * TC_WORDS).reshape(n_tc, TC_WORDS),
+        tc=np.concatenate([tc_only, sfx]) if n_sfx else tc_only,
+        tc_only=tc_only, sfx=sfx, sfx_offsets=sfx_offsets,
         cta_offsets=words(coo, n_ctas + 1) if n_tc else np.zeros(1, np.int32),
         part_base=words(pbo_, n_forks),
         n_parts=words(npo, n_forks * plan.n_part_groups).reshape(n_forks, plan.n_part_groups),
@@ -91,7 +103,8 @@ def _check_tc(shape, pl, fo, sl, plan, p, pbo, sbo, host_offsets):
     F = int(fo[-1])
     tc = p["tc"]
     co = p["cta_offsets"]
-    assert co[0] == 0 and co[-1] == len(tc) and np.all(np.diff(co) > 0)
+    assert co[0] == 0 and co[-1] == len(p["tc_only"]) and np.all(np.diff(co) > 0)
+    assert plan.n_tc_ctas + plan.n_sfx_ctas <= 148  # the grids share the SMs (148: no device)
     fork_trace = np.repeat(np.arange(len(pl)), np.diff(fo))
     cover = {}
     parts = {}
