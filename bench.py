@@ -446,6 +446,8 @@ def run_ours():
     partials_ms = stage_ms(lib.specgen_fork_attn_run_partials)
     merge_ms = stage_ms(lib.specgen_fork_attn_run_merge)
     suffix_stage = measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes)
+    suffix_steady = (measure_suffix_steady(stream, dev, kv_layout)
+                     if w["v_pages"] is not None else None)
     kernel_names = ["+".join(part_kernels), "lse_merge"]
     kernel_ms = [partials_ms, merge_ms]
     launches = len(part_kernels) + 1
@@ -522,8 +524,11 @@ def run_ours():
         "prefix_read_amplification": (
             (traffic - nbytes["suffix"] - nbytes["q"] - nbytes["out"]) / nbytes["prefix"]
             if traffic is not None and nbytes["prefix"] > 0 else None),
-        # the suffix stage alone (diagnostic plan with empty prefixes)
+        # the suffix stage alone (diagnostic plan with empty prefixes), and the
+        # suffix-stage kernel's streaming rate on a call large enough to amortise
+        # its fixed per-call latency
         "suffix_stage": suffix_stage,
+        "suffix_stage_steady": suffix_steady,
         # tensor-pipe activity of the dominant kernel from the recorded ncu capture
         "tensor_pipe_pct": (recorded_profile(kernel_names[dom], f"{ARGS.workload}:{layout}")
                             or {}).get("tensor_pipe_pct"),
@@ -600,6 +605,65 @@ def measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes):
     return {"kernel_us": ms * 1e3, "bytes_per_launch": nbytes["suffix"] + nbytes["q"],
             "gbs": gbs, "vs_8tbs": gbs / 8000.0, "vs_measured": gbs / hbm,
             "plan": "same forks, queries and suffix pages; empty prefixes"}
+
+
+def measure_suffix_steady(stream, dev, kv_layout):
+    """The suffix-stage kernel alone on a suffix-only call large enough that its
+    fixed per-call latency (start, ramp, tail: a few microseconds) is amortised:
+    64 forks of one trace with 2048-token suffixes and no prefix (538 MB of KV,
+    Hq=64, Hkv=8, head dim 128, page 16).  Its GB/s is the kernel's streaming
+    rate, against the nominal 8 TB/s and the measured copy bandwidth."""
+    import ctypes as C
+
+    import torch
+
+    from paper_2606_17518_gb300 import _lib, workloads as wl
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    spec = wl.WorkloadSpec(name="suffix_only_f64_s2048", num_traces=1, prefix_len=(0, 0),
+                           forks=(64, 64), suffix_len=(2048, 2048), hq=64, hkv=8, dqk=128,
+                           dv=128, page_size=16, seed=5)
+    w = wl.make_workload(spec)
+    fd = ForkDecode(w, device=dev, kv_layout=kv_layout)
+    sp = stream.cuda_stream
+    with torch.cuda.stream(stream):
+        fd.plan(sp)
+    torch.cuda.synchronize(dev)
+    if fd.plan_info.n_sfx_ctas == 0:
+        return None
+    lib = _lib.load()
+    args = fd.args()
+    ref = (C.byref(args), C.byref(fd.plan_info), C.c_void_p(sp))
+    st = lib.specgen_fork_attn_run_partials(*ref)
+    assert st == 0, _lib.status_string(st)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for _ in range(8):
+            st = lib.specgen_fork_attn_run_partials(*ref)
+            assert st == 0, _lib.status_string(st)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize(dev)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n_rep = 8
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(n_rep):
+            graph.replay()
+        t1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = t0.elapsed_time(t1) / (n_rep * 8)
+    nb = wl.algorithmic_bytes(w)
+    nbytes = nb["suffix"] + nb["q"]
+    hbm, _, _, _ = measured_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    status = fd.status(sp)
+    del fd
+    torch.cuda.empty_cache()
+    if status != 0:
+        raise RuntimeError(f"workspace status {status}")
+    return {"kernel_us": ms * 1e3, "bytes_per_launch": nbytes, "gbs": gbs, "vs_8tbs": gbs / 8000.0,
+            "vs_measured": gbs / hbm, "workload": spec.name,
+            "plan": "64 forks x 2048 suffix tokens, no prefix: the suffix-stage kernel alone"}
 
 
 def measure_e2e(w, reps, stream, dev, K, W):

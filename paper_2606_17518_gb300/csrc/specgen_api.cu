@@ -347,10 +347,16 @@ constexpr int kMinChunk = 128;        // smallest prefix chunk carved into a CTA
 // CTA): an item's fixed cost in pages (query rows in, partial out), and the
 // smallest load in pages worth a worker, which bounds the suffix CTAs of small
 // calls.
-constexpr long long kSfxItemPages = 1;
+constexpr long long kSfxItemPages = 3;
 constexpr long long kSfxMinWorkerPages = 2;
 constexpr long long kSfxMinPiecePages = 2;
 constexpr long long kSfxSplitMinPages = 8;  // beside a prefix: the least worker load that pays
+// beside a prefix: the largest mean suffix (in pages) for which the split pays;
+// longer suffixes stream as well on the tensor-core kernel, which then keeps
+// every SM and one kernel less in the chain
+constexpr long long kSfxSplitMaxUnitPages = 48;
+// weight of a suffix page against a prefix token-page in the SM split (percent)
+constexpr long long kSfxWeightPct = 80;
 
 struct TcUnit {
   int kind, seq, g, fork0, nforks, len;
@@ -453,8 +459,16 @@ bool pack_tc(const std::vector<TcUnit>& sfx, const std::vector<TcUnit>& pfx, int
 // [T w / n, T (w+1) / n)), so the loads differ by at most a page or two.  A
 // unit is cut at page boundaries where a run ends, and no piece is shorter
 // than kSfxMinPiecePages unless its unit is.
-void place_suffix_stage(const std::vector<TcUnit>& sfx, int n_workers, int page,
+void place_suffix_stage(const std::vector<TcUnit>& units, int n_workers, int page,
                         std::vector<TcPlacement>* placed) {
+  // in row order (fork, then kv head): every run then holds suffixes of mixed
+  // lengths, and no worker is left with all the short ones (whose item costs
+  // are real time on the GPU)
+  static thread_local std::vector<TcUnit> sfx;
+  sfx.assign(units.begin(), units.end());
+  std::sort(sfx.begin(), sfx.end(), [](const TcUnit& a, const TcUnit& b) {
+    return a.fork0 < b.fork0 || (a.fork0 == b.fork0 && a.g < b.g);
+  });
   auto pages = [&](long long n) { return (n + page - 1) / page; };
   long long T = 0;
   for (const TcUnit& u : sfx) T += kSfxItemPages + pages(u.len);
@@ -567,12 +581,14 @@ void build_tc_plan(const Shape& s, const Rows& rows, int n_sm, HostPlan* hp) {
     } else if (n_all < 2) {
       use_sfx = false;
     } else {
-      long long n = (long long)llround((double)n_all * (double)ws / (double)(ws + wp));
+      const double wsw = (double)ws * kSfxWeightPct / 100.0;
+      long long n = (long long)llround((double)n_all * wsw / (wsw + (double)wp));
       n = std::max<long long>(1, std::min<long long>(std::min<long long>(n, n_all - 1), most));
       n_sfx_sm = (int)n;
       // a kernel of its own pays (one more launch in the chain, more partials to
       // merge) only when each worker streams enough pages
-      if (sfx_pages < n * kWorkersPerSm * kSfxSplitMinPages) {
+      if (sfx_pages < n * kWorkersPerSm * kSfxSplitMinPages ||
+          sfx_pages > (long long)sfx.size() * kSfxSplitMaxUnitPages) {
         use_sfx = false;
         n_sfx_sm = 0;
       }

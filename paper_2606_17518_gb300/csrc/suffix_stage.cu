@@ -4,7 +4,7 @@
 //
 // The suffix of one fork is private to that fork, so its keys serve only the
 // G = hq / hkv query heads of one kv head: a 128-row tensor-core tile would
-// carry G live rows.  Here every warp of a suffix-role CTA is an independent
+// carry G live rows.  Here every warp of a suffix-stage CTA is an independent
 // worker with its own list of (fork, kv head, page range) items and its own
 // ring of page slots:
 //
@@ -50,7 +50,7 @@ namespace {
 using namespace tc;
 
 constexpr int kPage = 16;                    // tokens per page (the tensor-core path's page size)
-constexpr int kSlots = 3;                    // ring slots (pages) per warp
+constexpr int kSlots = kSuffixSlots;         // ring slots (pages) per warp
 constexpr float kRescale = 8.0f;             // lazy-rescale threshold, log2 units
 
 __device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a) {
@@ -70,7 +70,8 @@ struct Layout {
   static constexpr uint32_t kQ = 8u * NT * D * 2u;
   static constexpr uint32_t kWarp = kSlots * kSlot + kQ;
   static constexpr uint32_t kBar = kSuffixWarps * kWarp;
-  static constexpr uint32_t kWarpBar = 64u;
+  // kSlots + 1 mbarriers and kSlots flags, in 64-byte units
+  static constexpr uint32_t kWarpBar = (8u * (kSlots + 1) + 4u * kSlots + 63u) / 64u * 64u;
   static constexpr int kCache = NT == 1 ? 16 : 4;
   static constexpr uint32_t kItems = kBar + kSuffixWarps * kWarpBar;
   static constexpr uint32_t kAbort = kItems + kSuffixWarps * kCache * (uint32_t)sizeof(TcItem);
@@ -348,16 +349,30 @@ __device__ __forceinline__ void suffix_warp(const SfxParams& p, const CUtensorMa
         }
         __syncwarp();
       }
-      // S^T = K Q^T (16 tokens x 8 heads per n-tile)
-      float sc[NT][4];
+      // S^T = K Q^T (16 tokens x 8 heads per n-tile); with one n-tile the
+      // k-steps run in two independent accumulator chains (even and odd k-steps,
+      // added at the end), with two the n-tiles are the two chains
+      float sc[NT][4], sc2[4];
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) sc[nt][0] = sc[nt][1] = sc[nt][2] = sc[nt][3] = 0.f;
+      for (int e = 0; e < 4; ++e) {
+        sc2[e] = 0.f;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) sc[nt][e] = 0.f;
+      }
 #pragma unroll
       for (int ks = 0; ks < KS; ++ks) {
         uint32_t a[4];
         ldmatrix_x4(sK + piece<D, TL>(tk, 2 * ks + ck), a[0], a[1], a[2], a[3]);
+        if constexpr (NT == 1) {
+          mma_bf16_16816((ks & 1) ? sc2 : sc[0], a, qf[0][ks][0], qf[0][ks][1]);
+        } else {
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(sc[nt], a, qf[nt][ks][0], qf[nt][ks][1]);
+          for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(sc[nt], a, qf[nt][ks][0], qf[nt][ks][1]);
+        }
+      }
+      if constexpr (NT == 1) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sc[0][e] += sc2[e];
       }
       // tokens g8 and g8 + 8 of the page, heads 2*tig and 2*tig + 1 (+ 8 nt)
       const bool v0 = valid && g8 < ntok, v1 = valid && g8 + 8 < ntok;

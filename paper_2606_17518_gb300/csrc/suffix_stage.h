@@ -8,9 +8,10 @@
 
 namespace specgen {
 
-// Worker warps of a suffix-stage CTA (each walks its own list of items) and
-// suffix-stage CTAs resident on one SM.
+// Worker warps of a suffix-stage CTA (each walks its own list of items), page
+// slots in each worker's ring, and suffix-stage CTAs resident on one SM.
 constexpr int kSuffixWarps = 8;
+constexpr int kSuffixSlots = 3;
 constexpr int kSuffixCtasPerSm = 1;
 // Group sizes served (one or two n-tiles of 8 query heads).
 constexpr int kSuffixMaxG = 16;
