@@ -199,6 +199,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
   const int n_items = it_end - it_begin;
+  // dependents released at the start (see late_trigger)
+  if (!p.late_trigger && threadIdx.x == 0)
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
   // the CTA's first items, one per lane (40-byte records): the plan is written
   // by a host copy, never by a kernel, so it is read before the wait below
@@ -261,12 +264,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
-  // The next kernel of the stream (the suffix stage, or the merge: a
-  // programmatic dependent) may be launched once every CTA is past this wait,
-  // i.e. once the previous kernel has finished: the suffix stage runs beside
-  // this grid and relies on that ordering; the merge waits for this grid's
-  // completion before it reads any partial.
-  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  // With the suffix stage behind it, the next kernel of the stream may be
+  // launched only once every CTA is past this wait, i.e. once the previous
+  // kernel has finished: the suffix stage runs beside this grid and relies on
+  // that ordering for its inputs.
+  if (p.late_trigger && threadIdx.x == 0)
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   if (warp == 0) {
     __syncwarp();
     for (int k = lane; k < n_cached; k += 32) items[k] = clamp_item(items[k], p.suffix_lens);

@@ -26,6 +26,11 @@ struct TcParams {
   const int32_t* suffix_lens;  // device lengths that clamp suffix items, or nullptr
   int hq, hkv, G, dv, num_pages;
   float scale_log2;            // softmax scale * log2(e), > 0
+  // 1: the suffix-stage kernel follows this grid in the stream and runs beside
+  // it, so its dependents are released only once every CTA has passed the wait
+  // for the previous kernel; 0: they are released at the start (the merge
+  // waits for this grid's completion anyway)
+  int late_trigger;
 };
 
 bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G);

@@ -481,11 +481,10 @@ void place_suffix_stage(const std::vector<TcUnit>& units, int n_workers, int pag
     while (g < end) {
       while (w + 1 < n_workers && bound(w + 1) <= g) ++w;
       long long stop = std::min(end, w + 1 < n_workers ? bound(w + 1) : end);
-      stop = std::max(stop, std::min(end, p0 + 1));  // a piece holds at least a page
-      if (end - stop < kSfxMinPiecePages)
-        stop = end;  // no sliver at the unit's end
-      else if (stop - std::max(g, p0) < kSfxMinPiecePages)
-        stop = std::min(end, std::max(g, p0) + kSfxMinPiecePages);  // nor anywhere else
+      // no piece shorter than kSfxMinPiecePages (or the rest of the unit), and
+      // no shorter remainder left behind at the unit's end
+      stop = std::max(stop, std::min(end, std::max(g, p0) + kSfxMinPiecePages));
+      if (end - stop < kSfxMinPiecePages) stop = end;
       TcPlacement pl;
       pl.cta = -1 - w;
       TcItem& it = pl.item;
@@ -1297,6 +1296,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     tp.num_pages = args->num_pages;
     tp.scale_log2 = sp.scale_log2;
     tp.suffix_lens = args->suffix_lens;
+    tp.late_trigger = plan->n_sfx_ctas > 0 ? 1 : 0;
     cudaError_t e;
     if (args->v_pages == nullptr) {
       MlaParams mp;

@@ -387,3 +387,78 @@ def test_workload_lengths_match_the_workload(name):
     pl, fo, sl = wl.workload_lengths(name)
     assert np.array_equal(pl, w["prefix_lens"]) and np.array_equal(fo, w["fork_offsets"])
     assert np.array_equal(sl, w["suffix_lens"])
+
+
+# ---- suffix stage: per-fork suffix pages on the split-K worker warps ---------
+
+def _sfx_pieces(p):
+    """(fork, kv head) -> sorted token ranges of its suffix-stage items, and the
+    per-worker page loads."""
+    pieces, loads = {}, []
+    so = p["sfx_offsets"]
+    for w in range(len(so) - 1):
+        load = 0
+        for it in p["sfx"][so[w]:so[w + 1]]:
+            kind, seq, g, f0, nf, tb, te = (int(x) for x in it[:7])
+            pieces.setdefault((f0, g), []).append((tb, te))
+            load += (te - tb + 15) // 16
+        loads.append(load)
+    return pieces, np.array(loads)
+
+
+@pytest.mark.parametrize("case", range(12))
+def test_suffix_only_plans_use_the_suffix_stage(case):
+    """With no prefix the whole call is the suffix stage: every suffix key is
+    covered once (checked with the tensor-core items' rules), items are page
+    aligned, no piece is shorter than two pages unless its suffix is, and the
+    workers' page loads are within a few pages of each other."""
+    rng = np.random.default_rng(4000 + case)
+    G = [1, 2, 3, 4, 5, 8, 12, 16][case % 8]
+    hkv = [1, 2, 4][case % 3]
+    dqk = [64, 128][case % 2]
+    shape = dict(hq=G * hkv, hkv=hkv, dqk=dqk, dv=dqk, B=16, latent=False)
+    T = int(rng.integers(1, 4))
+    fo = np.concatenate([[0], np.cumsum(rng.integers(1, 12, T))]).astype(np.int32)
+    F = int(fo[-1])
+    pl = np.zeros(T, np.int32)
+    sl = rng.integers(0, 3000, F).astype(np.int32)
+    sl[rng.random(F) < 0.15] = 0
+    sl[rng.random(F) < 0.1] = 1
+    if sl.sum() == 0:
+        sl[0] = 40
+    plan, buf, pbo, sbo = _plan(shape, pl, fo, sl)
+    p = _parse(plan, buf)
+    assert plan.n_tc_ctas == 0 and plan.n_sfx_ctas > 0 and plan.n_split_items == 0
+    _check_tc(shape, pl, fo, sl, plan, p, pbo, sbo, True)
+    pieces, loads = _sfx_pieces(p)
+    for (f, g), rs in pieces.items():
+        rs = sorted(rs)
+        for tb, te in rs:
+            assert tb % 16 == 0                       # page aligned
+            # no piece shorter than two pages unless the whole suffix is
+            assert (te - tb + 15) // 16 >= min(2, (int(sl[f]) + 15) // 16)
+    assert loads.max() - loads.min() <= 3 + 2 * 3, (loads.min(), loads.max())
+
+
+def test_split_rules():
+    """The suffix stage runs beside the prefix only where it pays: many short
+    suffixes (the ragged batch) split, long suffixes (32k prefix, 256-2048-token
+    suffixes) and small calls (8k prefix, 8 forks) stay on the tensor-core kernel."""
+    def plan_of(name):
+        spec = wl.WORKLOADS[name]
+        pl, fo, sl = wl.workload_lengths(name)
+        shape = dict(hq=spec.hq, hkv=spec.hkv, dqk=spec.dqk, dv=spec.dv, B=spec.page_size,
+                     latent=not spec.separate_v)
+        plan, buf, pbo, sbo = _plan(shape, pl, fo, sl)
+        return plan, _parse(plan, buf), (shape, pl, fo, sl, pbo, sbo)
+    plan, p, (shape, pl, fo, sl, pbo, sbo) = plan_of("ragged_t8")
+    assert plan.n_tc_ctas > 0 and plan.n_sfx_ctas > 0
+    assert plan.n_tc_ctas + plan.n_sfx_ctas <= 148
+    # the prefix kernel takes no suffix item, the suffix stage every one
+    assert np.all(p["tc_only"][:, 0] == 0) and np.all(p["sfx"][:, 0] == 1)
+    # SMs split about in proportion to the work (suffix pages weighted 0.8)
+    share = plan.n_sfx_ctas / (plan.n_tc_ctas + plan.n_sfx_ctas)
+    assert 0.1 < share < 0.3, share
+    for name in ("long_p32k_f16", "fork_p8k_f8", "tiny_p512_f4"):
+        plan, p, _ = plan_of(name)
+        assert plan.n_sfx_ctas == 0, name
