@@ -307,12 +307,12 @@ __device__ __forceinline__ void suffix_warp(const SfxParams& p, const CUtensorMa
         qf[nt][2 * kk + 1][1] = live ? r3 : kZero;
       }
     }
-    __syncwarp();
-    // the buffer is free: the next item's query rows go in now
-    if (cnk < n_items) {
-      issue_q(cnext);
-      cnk = next_nonempty(cnk + 1, cnext);
-    }
+    // The next item's query rows go into the buffer only after the first page's
+    // S^T MMAs have consumed these fragments: an ldmatrix result that no
+    // instruction has used yet may still be in flight, and the bulk copy could
+    // overwrite the buffer before it is read (seen as run-to-run differences in
+    // the second n-tile's rows).
+    bool next_q = cnk < n_items;
 
     float acc[NT][KS][4];
     float m[NT][2], l[NT][2];
@@ -373,6 +373,12 @@ __device__ __forceinline__ void suffix_warp(const SfxParams& p, const CUtensorMa
       if constexpr (NT == 1) {
 #pragma unroll
         for (int e = 0; e < 4; ++e) sc[0][e] += sc2[e];
+      }
+      if (next_q) {  // every Q fragment has been consumed by an MMA issued above
+        __syncwarp();
+        issue_q(cnext);
+        cnk = next_nonempty(cnk + 1, cnext);
+        next_q = false;
       }
       // tokens g8 and g8 + 8 of the page, heads 2*tig and 2*tig + 1 (+ 8 nt)
       const bool v0 = valid && g8 < ntok, v1 = valid && g8 + 8 < ntok;

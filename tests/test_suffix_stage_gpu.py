@@ -173,15 +173,22 @@ def test_suffix_stage_items_cut_by_device_lengths(ahead):
     _compare(o, lse, o_ref, lse_ref, f"ahead {ahead}")
 
 
+@pytest.mark.parametrize("mode", ["alone", "beside"])
 @pytest.mark.parametrize("layout", ["rows", "tiled"])
-@pytest.mark.parametrize("G,hkv", [(16, 2), (8, 8)])
-def test_suffix_stage_repeatable(G, hkv, layout):
+@pytest.mark.parametrize("G,hkv", [(16, 4), (8, 8)])
+def test_suffix_stage_repeatable(G, hkv, layout, mode):
     """Twenty runs of one plan give the same bits: every partial of the suffix
-    stage is written by one worker from data it waited for (a lost wait or a
-    slot reused too early would show up here as run-to-run differences)."""
+    stage is written by one worker from data it waited for.  A buffer refilled
+    too early shows up here as run-to-run differences (it did, for the query
+    rows of the second n-tile, before the next item's rows were copied in only
+    after the current ones had been consumed)."""
     import torch
-    w = wl.make_workload(_spec(G, hkv, 128, 900 + G, traces=2, prefix=(0, 0), suffix=(20, 700),
-                               forks=(4, 8)))
+    if mode == "alone":
+        w = wl.make_workload(_spec(G, hkv, 128, 900 + G, traces=2, prefix=(0, 0),
+                                   suffix=(20, 700), forks=(4, 8)))
+    else:
+        w = wl.make_workload(_spec(G, hkv, 128, 500 + G, traces=2, prefix=(8192, 8192),
+                                   suffix=(300, 900), forks=(16, 16)))
     kv = _lib.KV_TILED if layout == "tiled" else _lib.KV_ROWS
     o1, l1, fd = _run(w, kv)
     o_ref, lse_ref = oracle.fork_attn_decode(w)
