@@ -207,9 +207,14 @@ specgen_status specgen_fork_attn_decode(const specgen_fork_attn_args* args,
  * them, and likewise out / lse inside dev_out, so that each direction is a
  * single copy.  Host buffers should be pinned for the copies to be
  * asynchronous; host_out is valid once the stream reaches the end of the
- * call.  in_bytes or out_bytes may be 0 (that copy is skipped).  Status codes
- * as specgen_fork_attn_decode; SPECGEN_ERR_NULL for a missing buffer of a
- * non-empty copy; SPECGEN_ERR_CUDA if a copy cannot be queued. */
+ * call.  in_bytes or out_bytes may be 0 (that copy is skipped).  The plan is
+ * uploaded from a page-locked staging ring that the library keeps per host
+ * thread (4 slots, grown on demand, kept until the process exits), so the call
+ * does not wait for its copies; a slot is reused only once the copy that read
+ * it has run, so the host blocks when it is 4 calls ahead of the GPU.  Status
+ * codes as specgen_fork_attn_decode (a shape error queues nothing);
+ * SPECGEN_ERR_NULL for a missing buffer of a non-empty copy; SPECGEN_ERR_CUDA
+ * if a copy cannot be queued. */
 specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* args,
                                                const specgen_host_lens* lens,
                                                const void* host_in, void* dev_in,

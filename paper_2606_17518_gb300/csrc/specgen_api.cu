@@ -971,11 +971,12 @@ specgen_status plan_build(const specgen_fork_attn_args* args, const Shape& s, co
                           specgen_plan* plan);
 
 // plan_build, then: host_dst == nullptr uploads the plan region to the workspace
-// on cuda_stream; otherwise it is copied into host_dst (host_bytes long) and no
-// CUDA call is made.
+// on cuda_stream (from this thread's page-locked ring when `pinned`, else from
+// the pageable buffer); otherwise it is copied into host_dst (host_bytes long)
+// and no CUDA call is made.
 specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
                          specgen_plan* plan, void* cuda_stream, void* host_dst = nullptr,
-                         size_t host_bytes = 0);
+                         size_t host_bytes = 0, bool pinned = false);
 
 }  // namespace
 
@@ -1153,9 +1154,71 @@ specgen_status upload_plan(void* workspace, void* cuda_stream) {
   return SPECGEN_OK;
 }
 
+// Page-locked staging for the plan uploads of the one-call step
+// (specgen_fork_attn_decode_staged): a ring of kRing host slots per host
+// thread.  A copy from page-locked memory is queued without the host staging
+// it first, so the call returns as soon as its work is queued.  A slot is
+// written again only after the copy that last read it has run (an event
+// recorded behind that copy), which lets the host run up to kRing calls ahead
+// of the GPU and holds it there.  A slot grows, to the next power of two, when
+// a plan does not fit; the slots are kept until the process exits.  If
+// page-locked memory cannot be had, the upload goes from the pageable buffer.
+struct PinnedRing {
+  static constexpr int kRing = 4;
+  void* buf[kRing] = {};
+  size_t cap[kRing] = {};
+  cudaEvent_t read[kRing] = {};
+  int dev = -1;
+  int next = 0;
+};
+thread_local PinnedRing t_ring;
+
+specgen_status upload_plan_pinned(void* workspace, void* cuda_stream) {
+  PinnedRing& r = t_ring;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return SPECGEN_ERR_CUDA;
+  if (dev != r.dev) {  // an event belongs to the device it was made on
+    for (int i = 0; i < PinnedRing::kRing; ++i) {
+      if (!r.read[i]) continue;
+      if (cudaEventSynchronize(r.read[i]) != cudaSuccess) return SPECGEN_ERR_CUDA;
+      cudaEventDestroy(r.read[i]);
+      r.read[i] = nullptr;
+    }
+    r.dev = dev;
+  }
+  const int k = r.next;
+  r.next = (k + 1) % PinnedRing::kRing;
+  if (r.read[k]) {
+    if (cudaEventSynchronize(r.read[k]) != cudaSuccess) return SPECGEN_ERR_CUDA;
+  } else if (cudaEventCreateWithFlags(&r.read[k], cudaEventDisableTiming) != cudaSuccess) {
+    r.read[k] = nullptr;
+    return SPECGEN_ERR_CUDA;
+  }
+  const size_t n = t_plan_bytes.size();
+  if (r.cap[k] < n) {
+    size_t c = 4096;
+    while (c < n) c <<= 1;
+    if (r.buf[k]) cudaFreeHost(r.buf[k]);
+    r.buf[k] = nullptr;
+    r.cap[k] = 0;
+    if (cudaHostAlloc(&r.buf[k], c, cudaHostAllocPortable) != cudaSuccess) {
+      (void)cudaGetLastError();
+      r.buf[k] = nullptr;
+      return upload_plan(workspace, cuda_stream);
+    }
+    r.cap[k] = c;
+  }
+  memcpy(r.buf[k], t_plan_bytes.data(), n);
+  if (cudaMemcpyAsync(workspace, r.buf[k], n, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+      cudaEventRecord(r.read[k], stream) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
+}
+
 specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, const Rows& rows,
                          specgen_plan* plan, void* cuda_stream, void* host_dst,
-                         size_t host_bytes) {
+                         size_t host_bytes, bool pinned) {
   specgen_status st;
   if ((st = check_pointers(args)) != SPECGEN_OK) return st;
   if ((st = plan_build(args, s, rows, plan)) != SPECGEN_OK) {
@@ -1170,7 +1233,9 @@ specgen_status plan_impl(const specgen_fork_attn_args* args, const Shape& s, con
     memcpy(host_dst, t_plan_bytes.data(), t_plan_bytes.size());
     return SPECGEN_OK;
   }
-  if ((st = upload_plan(args->workspace, cuda_stream)) != SPECGEN_OK) memset(plan, 0, sizeof(*plan));
+  st = pinned ? upload_plan_pinned(args->workspace, cuda_stream)
+              : upload_plan(args->workspace, cuda_stream);
+  if (st != SPECGEN_OK) memset(plan, 0, sizeof(*plan));
   return st;
 }
 
@@ -1402,11 +1467,18 @@ specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* arg
   if ((in_bytes > 0 && (!host_in || !dev_in)) || (out_bytes > 0 && (!dev_out || !host_out)))
     return SPECGEN_ERR_NULL;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  // shapes first: a call refused here queues nothing
+  Shape s;
+  specgen_status st = check_shape(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
   if (in_bytes > 0 &&
       cudaMemcpyAsync(dev_in, host_in, in_bytes, cudaMemcpyHostToDevice, stream) != cudaSuccess)
     return SPECGEN_ERR_CUDA;
-  const specgen_status st = specgen_fork_attn_decode(args, lens, cuda_stream);
+  specgen_plan plan;
+  memset(&plan, 0, sizeof(plan));
+  st = plan_impl(args, s, rows_for_decode(lens, s.T, s.F), &plan, cuda_stream, nullptr, 0, true);
   if (st != SPECGEN_OK) return st;
+  if ((st = specgen_fork_attn_run(args, &plan, cuda_stream)) != SPECGEN_OK) return st;
   if (out_bytes > 0 &&
       cudaMemcpyAsync(host_out, dev_out, out_bytes, cudaMemcpyDeviceToHost, stream) != cudaSuccess)
     return SPECGEN_ERR_CUDA;

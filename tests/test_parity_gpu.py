@@ -270,6 +270,44 @@ def test_staged_decode_from_host_buffers(name):
     assert fd.status() == _lib.SPECGEN_OK
 
 
+def test_staged_calls_queued_back_to_back():
+    """Ten staged calls on one stream with no host synchronisation in between,
+    each with other suffix lengths and its own pinned output buffer.  That is
+    more calls than the library's page-locked plan staging ring has slots, so
+    slots are written again behind queued copies; every call must still see
+    its own plan (element-wise against the oracle at its lengths)."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload("tiny_p512_f4")
+    fd = ForkDecode(w)
+    base = np.asarray(w["suffix_lens"], dtype=np.int32)
+    din, hin, (fd.q, fd.prefix_table, fd.prefix_off, fd.suffix_table, fd.suffix_off), _ = \
+        _pack_device([fd.q, fd.prefix_table, fd.prefix_off, fd.suffix_table, fd.suffix_off])
+    dout, _, (fd.out, fd.lse), ooff = _pack_device([fd.out, fd.lse])
+    F, hq, dv = w["total_forks"], w["hq"], w["dv"]
+    stream = torch.cuda.current_stream().cuda_stream
+    torch.cuda.synchronize()
+    houts, cuts = [], []
+    for i in range(10):
+        cut = np.maximum(base - (i * 7) % 19 - np.arange(len(base)) * (i % 4), 0).astype(np.int32)
+        fd.set_suffix_lens(cut)
+        hout = torch.zeros(dout.numel(), dtype=torch.uint8).pin_memory()
+        _lib.specgen_fork_attn_decode_staged(fd.args(), fd.lens, hin, din, din.numel(), dout,
+                                             hout, dout.numel(), stream)
+        houts.append(hout)
+        cuts.append(cut)
+    torch.cuda.synchronize()
+    assert fd.status() == _lib.SPECGEN_OK
+    for cut, hout in zip(cuts, houts):
+        o = hout[ooff[0]:ooff[0] + F * hq * dv * 2].view(torch.bfloat16).float().numpy()
+        lse = hout[ooff[1]:ooff[1] + F * hq * 4].view(torch.float32).numpy()
+        wc = dict(w)
+        wc["suffix_lens"] = cut
+        o_ref, lse_ref = oracle.fork_attn_decode(wc)
+        _compare(o.astype(np.float64).reshape(F, hq, dv), lse.astype(np.float64).reshape(F, hq),
+                 o_ref, lse_ref, f"staged cut {cut.tolist()}")
+
+
 def test_plan_once_run_many_is_deterministic():
     from paper_2606_17518_gb300.fork_attn import ForkDecode
     w = wl.make_workload("fork_p8k_f8")
