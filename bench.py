@@ -745,11 +745,12 @@ def run_decode_steps():
     """--op decode_step: K serving steps of append + attention with growing suffixes.
 
     One plan is made for the lengths after the last step; the kernels cut the
-    suffix items to the current lengths in a device array, which every step
-    advances after its append.  Each step (copy of the step's Q and new K/V
-    rows from pinned host memory, specgen_append_kv with pages from a device
-    free list, length advance, attention, copy of O and LSE back to pinned
-    memory) is captured in CUDA graphs of 16 steps; the K timed steps replay
+    suffix items to the current lengths in a device array, which every step's
+    append advances (writing the next lengths into a second array; the two
+    swap).  Each step (copy of the step's Q and new K/V rows from pinned host
+    memory, specgen_append_kv with pages from a device free list, attention,
+    copy of O and LSE back to pinned memory) is captured in CUDA graphs of 16
+    steps; the K timed steps replay
     them between CUDA events on the stream.  Per-kernel times: graphs of the
     attention stages alone at the final lengths, and a graph of appends into a
     second copy of the state.
@@ -837,8 +838,9 @@ def run_decode_steps():
 
     def step(s):
         d_in.copy_(h_in[s], non_blocking=True)
-        fd.append_kv(d_k, d_v, free[offs[s]:], n_free - offs[s], sp)
-        fd.suffix_lens_dev.add_(1)
+        # the append writes the advanced device lengths (into the other of two
+        # arrays), which this step's attention and the next append read
+        fd.append_kv(d_k, d_v, free[offs[s]:], n_free - offs[s], sp, advance=True)
         fd.run(sp)
         h_out.copy_(d_out, non_blocking=True)
 
@@ -894,6 +896,8 @@ def run_decode_steps():
 
     # attention stages alone at the final lengths
     args, plan = fd.args(), fd.plan_info
+    n_part_kernels = sum(int(x > 0) for x in (plan.n_tc_ctas, plan.n_sfx_ctas,
+                                               plan.n_split_items))
     lib = _lib.load()
     part_ms = graph_ms(lambda i: lib.specgen_fork_attn_run_partials(C.byref(args), C.byref(plan),
                                                                      C.c_void_p(sp)))
@@ -935,7 +939,7 @@ def run_decode_steps():
                              "16 steps incl. per-step H2D/D2H copies; per-kernel times from "
                              "graphs of each kernel alone",
                    "l2": "one resident state (KV stays resident across steps, as in serving)"},
-        "gpu_launches": K * 3,  # append, attention, merge
+        "gpu_launches": K * (2 + n_part_kernels),  # append, partial kernels, merge
         "kernels": {k: {"ms_per_launch": v, "share": v / sum(kern.values())}
                     for k, v in kern.items()},
         "roofline": roof,

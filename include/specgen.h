@@ -347,7 +347,13 @@ specgen_status specgen_fork_cascade_plan_host(const specgen_fork_attn_args* args
  * and the id is written into the fork's block table.  All inputs are device
  * memory and nothing is planned on the host, so the call can be captured in a
  * CUDA graph; the caller then adds 1 to every suffix length (host and device
- * copies) and drops the j ids taken from the front of its free list.
+ * copies) and drops the j ids taken from the front of its free list.  With
+ * suffix_lens_next the kernel writes the advanced device lengths itself, into
+ * a second array (another fork's count still reads the first one), which the
+ * step's attention and the next append then take as their suffix_lens; the
+ * two arrays swap roles every step.  The kernel is launched as a programmatic
+ * dependent of the stream's previous kernel (it reads nothing before that
+ * kernel has completed) and lets the next kernel start its prologue early.
  * A fork whose block table has no room (n / page_size >= its CSR capacity),
  * whose free-list entry does not exist, or whose page id is outside
  * [0, num_pages) writes nothing and ORs SPECGEN_ERR_INDEX's bit (1) into
@@ -367,13 +373,18 @@ typedef struct {
   const int32_t* free_pages;        /* [num_free] page ids handed out in fork order */
   int num_free;
   uint32_t* status;                 /* device status word, or NULL */
+  int32_t* suffix_lens_next;        /* optional [total_forks]: receives the lengths after
+                                       this call (suffix_lens[f] + 1 where fork f appended,
+                                       suffix_lens[f] where it could not); NULL: not
+                                       written.  Must not be suffix_lens itself. */
 } specgen_append_args;
 
 /* Head dims must be multiples of 8 (rows move in 16-byte pieces); page_size a power of
  * two <= 1024; the tiled layout needs page_size % 8 == 0 and a value pool.
  * Returns SPECGEN_OK after launching (asynchronous on cuda_stream),
  * SPECGEN_ERR_NULL / _SHAPE / _UNSUPPORTED on bad arguments (nothing
- * launched), SPECGEN_ERR_CUDA if the launch fails. */
+ * launched; SPECGEN_ERR_UNSUPPORTED for suffix_lens_next == suffix_lens),
+ * SPECGEN_ERR_CUDA if the launch fails. */
 specgen_status specgen_append_kv(const specgen_append_args* args, void* cuda_stream);
 
 /* ---- Prefix page pack / unpack ----------------------------------------------

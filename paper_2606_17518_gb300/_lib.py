@@ -81,6 +81,7 @@ class AppendArgs(C.Structure):
         ("v_pages", C.c_void_p), ("suffix_block_table", C.c_void_p),
         ("suffix_bt_offsets", C.c_void_p), ("suffix_lens", C.c_void_p),
         ("free_pages", C.c_void_p), ("num_free", C.c_int), ("status", C.c_void_p),
+        ("suffix_lens_next", C.c_void_p),
     ]
 
 
@@ -243,12 +244,12 @@ def make_args(*, num_traces, total_forks, hq, hkv, head_dim_qk, head_dim_v, page
 def make_append_args(*, total_forks, hkv, head_dim_qk, head_dim_v, page_size, num_pages,
                      k_new, v_new, k_pages, v_pages, suffix_block_table, suffix_bt_offsets,
                      suffix_lens, free_pages, num_free, status=None,
-                     kv_layout=KV_ROWS) -> AppendArgs:
+                     kv_layout=KV_ROWS, suffix_lens_next=None) -> AppendArgs:
     return AppendArgs(
         int(total_forks), int(hkv), int(head_dim_qk), int(head_dim_v), int(page_size),
         int(num_pages), int(kv_layout), _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages),
         _ptr(suffix_block_table), _ptr(suffix_bt_offsets), _ptr(suffix_lens), _ptr(free_pages),
-        int(num_free), _ptr(status))
+        int(num_free), _ptr(status), _ptr(suffix_lens_next))
 
 
 def specgen_append_kv(args: AppendArgs, stream: int = 0) -> None:

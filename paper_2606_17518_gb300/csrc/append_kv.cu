@@ -9,7 +9,12 @@
 // per fork: the lanes count those earlier forks, then copy the fork's rows
 // (all kv heads) 16 bytes a lane.  A fork whose table is full, whose free-list
 // entry does not exist or whose page id is outside the pool writes nothing and
-// raises the index bit of the status word.
+// raises the index bit of the status word.  With lens_next, lane 0 of a fork's
+// warp also writes the fork's length after the call there (a separate array:
+// the counts of other forks still read lens).  The kernel waits for the
+// stream's previous kernel before it reads anything and lets the next kernel
+// launch at once (that kernel waits for this one's completion before it reads
+// the pools, tables or lengths).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -37,6 +42,8 @@ __device__ __forceinline__ void copy_rows(__nv_bfloat16* pool, const __nv_bfloat
 }
 
 __global__ void __launch_bounds__(32 * kWarps) append_kv_kernel(const AppendParams p) {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int f = blockIdx.x * kWarps + warp;
   if (f >= p.F) return;
@@ -53,6 +60,7 @@ __global__ void __launch_bounds__(32 * kWarps) append_kv_kernel(const AppendPara
     page = slot == 0 ? (j < p.num_free ? p.free_pages[j] : -1) : p.table[off + pidx];
     bad = page < 0 || page >= p.num_pages;
   }
+  if (lane == 0 && p.lens_next) p.lens_next[f] = bad ? n : n + 1;
   if (bad) {
     if (lane == 0 && p.status) atomicOr(p.status, kStatusIndex);
     return;
@@ -66,8 +74,16 @@ __global__ void __launch_bounds__(32 * kWarps) append_kv_kernel(const AppendPara
 
 cudaError_t launch_append_kv(const AppendParams& p, cudaStream_t stream) {
   if (p.F == 0) return cudaSuccess;
-  append_kv_kernel<<<(p.F + kWarps - 1) / kWarps, 32 * kWarps, 0, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((p.F + kWarps - 1) / kWarps));
+  cfg.blockDim = dim3(32 * kWarps);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, append_kv_kernel, p);
 }
 
 }  // namespace specgen

@@ -14,6 +14,7 @@ struct AppendParams {
   int32_t* table;              // suffix block table (CSR, capacity per fork)
   const int32_t* offs;         // [F + 1]
   const int32_t* lens;         // [F] tokens already in each suffix
+  int32_t* lens_next;          // [F] lengths after the call, or nullptr (never lens itself)
   const int32_t* free_pages;
   uint32_t* status;            // or nullptr
   int F, hkv, dqk, dv, B, num_pages, num_free;

@@ -1502,6 +1502,8 @@ specgen_status specgen_append_kv(const specgen_append_args* a, void* cuda_stream
   if (!a->k_new || !a->k_pages || !a->suffix_block_table || !a->suffix_bt_offsets ||
       !a->suffix_lens || (a->num_free > 0 && !a->free_pages))
     return SPECGEN_ERR_NULL;
+  if (a->suffix_lens_next != nullptr && a->suffix_lens_next == a->suffix_lens)
+    return SPECGEN_ERR_UNSUPPORTED;
   const void* rows[4] = {a->k_new, a->v_new, a->k_pages, a->v_pages};
   for (const void* r : rows)
     if (reinterpret_cast<uintptr_t>(r) % 16 != 0) return SPECGEN_ERR_SHAPE;
@@ -1513,6 +1515,7 @@ specgen_status specgen_append_kv(const specgen_append_args* a, void* cuda_stream
   p.table = a->suffix_block_table;
   p.offs = a->suffix_bt_offsets;
   p.lens = a->suffix_lens;
+  p.lens_next = a->suffix_lens_next;
   p.free_pages = a->free_pages;
   p.status = a->status;
   p.F = a->total_forks;

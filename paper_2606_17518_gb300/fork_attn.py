@@ -47,6 +47,9 @@ class ForkDecode:
         self.suffix_table = _i32(w["suffix_table"], device)
         self.suffix_off = _i32(w["suffix_bt_offsets"], device)
         self.suffix_lens_dev = _i32(w["suffix_lens"], device)  # read by specgen_append_kv
+        # the other device length array of an advancing append (made here, not
+        # inside a graph capture)
+        self._lens_alt = torch.empty_like(self.suffix_lens_dev)
         F, hq, dv = w["total_forks"], w["hq"], w["dv"]
         self.out = torch.empty((F, hq, dv), dtype=torch.bfloat16, device=device)
         self.lse = torch.empty((F, hq), dtype=torch.float32, device=device)
@@ -84,19 +87,25 @@ class ForkDecode:
             self.suffix_lens_dev.copy_(torch.from_numpy(w["suffix_lens"]))
         self.plan_info = None
 
-    def append_kv(self, k_new, v_new, free_pages, num_free: int, stream: int = 0):
+    def append_kv(self, k_new, v_new, free_pages, num_free: int, stream: int = 0,
+                  advance: bool = False):
         """One decode step's K/V rows (device bf16 [F][Hkv][D]) into the suffixes,
         taking pages from ``free_pages`` (device int32); status bits go to the
-        workspace status word.  The caller then advances the lengths."""
+        workspace status word.  Without ``advance`` the caller then advances the
+        device lengths; with it the kernel writes them into a second device
+        array, which becomes ``suffix_lens_dev`` (the two swap every step)."""
         w = self.w
+        nxt = self._lens_alt if advance else None
         args = _lib.make_append_args(
             total_forks=w["total_forks"], hkv=w["hkv"], head_dim_qk=w["dqk"],
             head_dim_v=w["dv"], page_size=w["page_size"], num_pages=w["num_pages"],
             k_new=k_new, v_new=v_new, k_pages=self.k_pages, v_pages=self.v_pages,
             suffix_block_table=self.suffix_table, suffix_bt_offsets=self.suffix_off,
             suffix_lens=self.suffix_lens_dev, free_pages=free_pages, num_free=num_free,
-            status=self.workspace, kv_layout=self.kv_layout)
+            status=self.workspace, kv_layout=self.kv_layout, suffix_lens_next=nxt)
         _lib.specgen_append_kv(args, stream)
+        if advance:
+            self.suffix_lens_dev, self._lens_alt = self._lens_alt, self.suffix_lens_dev
 
     def args(self, with_ws: bool = True, **override) -> _lib.ForkAttnArgs:
         w = self.w

@@ -232,6 +232,7 @@ def test_append_host_checks():
     assert st(suffix_lens=None) == S.SPECGEN_ERR_NULL
     assert st(free_pages=None) == S.SPECGEN_ERR_NULL
     assert st(k_new=fake + 8) == S.SPECGEN_ERR_SHAPE            # not 16-byte aligned
+    assert st(suffix_lens_next=fake) == S.SPECGEN_ERR_UNSUPPORTED  # in place: races
 
 
 def test_pack_host_checks():

@@ -109,12 +109,15 @@ def test_append_reports_exhausted_free_list_and_full_table():
     v_new = torch.from_numpy(st["v_new"][0].view(np.int16)).cuda().view(torch.bfloat16)
     free = torch.from_numpy(st["free_pages"]).cuda()
     before = fd.suffix_table.cpu().numpy().copy()
-    fd.append_kv(k_new, v_new, free, 2)          # four forks need a page, two exist
+    lens0 = fd.suffix_lens_dev.cpu().numpy().copy()
+    fd.append_kv(k_new, v_new, free, 2, advance=True)  # four forks need a page, two exist
     assert fd.status() == _lib.SPECGEN_ERR_INDEX
     t = fd.suffix_table.cpu().numpy()
     changed = np.nonzero(t != before)[0]
     assert len(changed) == 2                      # forks 0 and 1 got pages, 2 and 3 wrote nothing
     assert sorted(t[changed].tolist()) == sorted(st["free_pages"][:2].tolist())
+    # the advanced lengths: +1 only where the fork appended
+    assert np.array_equal(fd.suffix_lens_dev.cpu().numpy(), lens0 + np.array([1, 1, 0, 0]))
     # a table with no room: length already at capacity
     st2 = dict(st)
     st2["suffix_lens"] = (st["suffix_bt_offsets"][1:] - st["suffix_bt_offsets"][:-1]) * 16
@@ -157,11 +160,13 @@ def test_plan_ahead_cut_to_device_lengths(name, ahead):
     assert float(np.max(np.abs(lse[fin] - lse_ref[fin]))) <= TOL_LSE
 
 
+@pytest.mark.parametrize("advance", ["torch", "append"])
 @pytest.mark.parametrize("name", ["fork_p8k_f8", "mla_p16k_f8"])
-def test_one_plan_many_decode_steps_in_a_graph(name):
+def test_one_plan_many_decode_steps_in_a_graph(name, advance):
     """One plan for 12 steps ahead; 12 steps of (append, advance the device
     lengths, attention) captured in one CUDA graph; the last step's output and
-    the pools match the oracle."""
+    the pools match the oracle.  The lengths advance either by a torch add on
+    the device or by the append itself (into the other of two arrays)."""
     import torch
     from paper_2606_17518_gb300.fork_attn import ForkDecode
     steps = 12
@@ -192,13 +197,15 @@ def test_one_plan_many_decode_steps_in_a_graph(name):
     with torch.cuda.graph(graph, stream=stream):
         for s in range(steps):
             fd.append_kv(k_new[s], None if v_new is None else v_new[s], free[offs[s]:],
-                         len(st["free_pages"]) - offs[s], sp)
-            fd.suffix_lens_dev.add_(1)
+                         len(st["free_pages"]) - offs[s], sp, advance=advance == "append")
+            if advance == "torch":
+                fd.suffix_lens_dev.add_(1)
             fd.run(sp)
     graph.replay()
     torch.cuda.synchronize()
     o, lse = fd.results()
     assert fd.status() == _lib.SPECGEN_OK
+    assert np.array_equal(fd.suffix_lens_dev.cpu().numpy(), lens0 + steps)
     ref_k, ref_v, ref_t, lens = st["k_pages"], st["v_pages"], st["suffix_table"], lens0.copy()
     used = 0
     for s in range(steps):

@@ -51,6 +51,31 @@ def test_static_matches_workspace_entry_point_twice(name):
         assert _lib.specgen_static_workspace_status() == _lib.SPECGEN_OK
 
 
+def test_static_with_the_suffix_stage_and_the_largest_workload():
+    """Plans that run the suffix-stage kernel beside the prefix kernel (ragged_t8,
+    the largest workload, 9.5 MB of scratch, and a 16-fork call with G = 16)
+    through the scratch array: the same bits as the workspace entry point."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    spec = wl.WorkloadSpec(name="static_sfx_g16", num_traces=2, prefix_len=(8192, 8192),
+                           forks=(16, 16), suffix_len=(300, 900), hq=64, hkv=4, dqk=128,
+                           dv=128, page_size=16, seed=516)
+    for w in (wl.make_workload("ragged_t8"), wl.make_workload(spec)):
+        fd = ForkDecode(w, kv_layout=_lib.KV_TILED)
+        fd.plan()
+        assert fd.plan_info.n_sfx_ctas > 0 and fd.plan_info.ws_end <= (16 << 20)
+        fd.run()
+        torch.cuda.synchronize()
+        o_ref, l_ref = fd.results()
+        fd.out.zero_()
+        fd.lse.zero_()
+        _lib.specgen_fork_attn_decode_static(fd.args(with_ws=False), fd.lens)
+        torch.cuda.synchronize()
+        assert _lib.specgen_static_workspace_status() == _lib.SPECGEN_OK
+        o, lse = fd.results()
+        assert np.array_equal(o, o_ref) and np.array_equal(lse, l_ref)
+
+
 def test_static_status_reports_a_bad_page_id():
     """A page id outside the pool is skipped by the kernels and reported in the
     scratch array's status word; the next clean call resets it."""
