@@ -619,9 +619,7 @@ def measure_suffix_steady(stream, dev, kv_layout):
 
     from paper_2606_17518_gb300 import _lib, workloads as wl
     from paper_2606_17518_gb300.fork_attn import ForkDecode
-    spec = wl.WorkloadSpec(name="suffix_only_f64_s2048", num_traces=1, prefix_len=(0, 0),
-                           forks=(64, 64), suffix_len=(2048, 2048), hq=64, hkv=8, dqk=128,
-                           dv=128, page_size=16, seed=5)
+    spec = wl.DIAGNOSTIC["suffix_only_f64_s2048"]
     w = wl.make_workload(spec)
     fd = ForkDecode(w, device=dev, kv_layout=kv_layout)
     sp = stream.cuda_stream

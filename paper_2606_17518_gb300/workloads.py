@@ -76,6 +76,20 @@ WORKLOADS = {
 }
 WORKLOAD_ORDER = list(WORKLOADS)
 
+# Diagnostic workloads (not benchmark configurations): the suffix-stage kernel
+# alone on a call large enough that its fixed per-call latency is amortised,
+# 64 forks of one trace with 2048-token suffixes and no prefix (538 MB of KV).
+DIAGNOSTIC = {
+    "suffix_only_f64_s2048": WorkloadSpec(
+        "suffix_only_f64_s2048", 1, (0, 0), (64, 64), (2048, 2048), hq=64, hkv=8, dqk=128,
+        dv=128, page_size=16, seed=5),
+}
+
+
+def spec_of(name: str) -> WorkloadSpec:
+    """A benchmark workload or a diagnostic one, by name."""
+    return WORKLOADS[name] if name in WORKLOADS else DIAGNOSTIC[name]
+
 
 def round_to_bf16_bits(x: np.ndarray) -> np.ndarray:
     """float32 -> bf16 bit patterns, round-to-nearest-even (finite inputs)."""
@@ -105,7 +119,7 @@ def workload_lengths(spec: WorkloadSpec | str, seed: int | None = None):
     """(prefix_lens, fork_offsets, suffix_lens) of make_workload(spec, seed), as int32,
     without drawing the KV pools and queries."""
     if isinstance(spec, str):
-        spec = WORKLOADS[spec]
+        spec = spec_of(spec)
     rng = np.random.default_rng(spec.seed if seed is None else seed)
     prefix_lens, forks, suffix_lens = _draw_lengths(rng, spec)
     fork_offsets = np.concatenate([[0], np.cumsum(forks)])
@@ -123,7 +137,7 @@ def make_workload(spec: WorkloadSpec | str, seed: int | None = None,
     hq, hkv, dqk, dv, page_size, scale, name, sentinel_ids.
     """
     if isinstance(spec, str):
-        spec = WORKLOADS[spec]
+        spec = spec_of(spec)
     if overrides:
         spec = WorkloadSpec(**{**asdict(spec), **overrides})
     rng = np.random.default_rng(spec.seed if seed is None else seed)
