@@ -552,8 +552,9 @@ def run_ours():
 
 def measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes):
     """The suffix stage alone: the same forks, queries and suffix pages with empty
-    prefixes, so that the partial-attention kernel reads only the suffix KV (a
-    diagnostic plan; the step itself always runs both stages in one kernel).
+    prefixes, so that the partial-attention kernels read only the suffix KV (a
+    diagnostic plan: the suffix-stage kernel alone on every SM, where the plan
+    splits; the step itself runs the prefix and suffix stages together).
     GB/s = (suffix KV + Q bytes) / the kernel's time, against the nominal 8 TB/s
     and the measured copy bandwidth."""
     import ctypes as C
@@ -665,15 +666,22 @@ def measure_suffix_steady(stream, dev, kv_layout):
 
 
 def measure_e2e(w, reps, stream, dev, K, W):
-    """tokens/s through specgen_fork_attn_decode_staged with host-resident inputs.
+    """tokens/s through specgen_fork_attn_decode_staged_inline with host-resident inputs.
 
-    Every step is one library call that copies that step's queries and block
-    tables from pinned host memory, plans (host) and runs the attention, and
-    reads O and LSE back into pinned host memory.  The KV pools are the serving
-    cache and stay resident.  A step's inputs travel as one packed buffer (Q,
-    then the four table arrays, each at a 256-byte boundary) and its outputs as
-    another (O, then LSE): one copy each way, as a serving loop stages them; the
-    library reads the views inside the packed device buffers.
+    Every step is one library call that plans on the host, copies that step's
+    queries, block tables and plan from pinned host memory (in one copy while
+    the GPU is still busy with earlier steps; inputs first and plan after the
+    planning when it is idle), runs the attention, and reads O and LSE back
+    into pinned host memory.  The KV pools
+    are the serving cache and stay resident.  A step's inputs travel as one
+    packed buffer (Q, then the four table arrays, each at a 256-byte boundary,
+    then room for the plan region) and its outputs as another (O, then LSE).
+    The call writes the plan into the pinned input buffer, so the loop keeps a
+    ring of them (at least 16, a multiple of the replicas) in two halves, and
+    before it starts a half it waits for an event recorded after the last call
+    that used that half: a buffer is reused only once the call that last read
+    it has finished, and the host runs up to one and a half halves ahead of the
+    GPU (one event call per half, none per step).
     """
     import ctypes as C
 
@@ -683,45 +691,69 @@ def measure_e2e(w, reps, stream, dev, K, W):
     replicas = len(reps)
     sp = stream.cuda_stream
     align = lambda n: (n + 255) // 256 * 256
+    n_host = 2 * replicas * max(1, -(-8 // replicas))
+    half = n_host // 2
 
-    def pack(tensors):
-        """One device buffer holding copies of `tensors` (256-byte aligned views) and a
-        pinned host twin; returns (device bytes, host bytes, views)."""
+    def pack(tensors, extra=0):
+        """One device buffer holding copies of `tensors` (256-byte aligned views,
+        then `extra` bytes); returns (device bytes, bytes used, views)."""
         offs, n = [], 0
         for t in tensors:
             offs.append(n)
             n = align(n + t.numel() * t.element_size())
-        dbuf = torch.empty(n, dtype=torch.uint8, device=dev)
+        dbuf = torch.zeros(n + extra, dtype=torch.uint8, device=dev)
         views = []
         for t, o in zip(tensors, offs):
             v = dbuf[o:o + t.numel() * t.element_size()].view(t.dtype).view(t.shape)
             v.copy_(t)
             views.append(v)
-        hbuf = torch.empty(n, dtype=torch.uint8).pin_memory()
-        hbuf.copy_(dbuf)
-        return dbuf, hbuf, views
+        return dbuf, n, views
 
     staged = []
     for r in reps:
-        din, hin, (r.q, r.prefix_table, r.prefix_off, r.suffix_table, r.suffix_off) = pack(
-            [r.q, r.prefix_table, r.prefix_off, r.suffix_table, r.suffix_off])
-        dout, hout, (r.out, r.lse) = pack([r.out, r.lse])
-        staged.append((din, hin, dout, hout, r.args()))
+        region = int(r.plan_info.ws_plan_off + r.plan_info.plan_bytes)
+        din, in_bytes, (r.q, r.prefix_table, r.prefix_off, r.suffix_table, r.suffix_off) = pack(
+            [r.q, r.prefix_table, r.prefix_off, r.suffix_table, r.suffix_off], region + 4096)
+        dout, _, (r.out, r.lse) = pack([r.out, r.lse])
+        staged.append((din, in_bytes, dout, r.args()))
+    hosts = []
+    for j in range(n_host):
+        din = staged[j % replicas][0]
+        hin = torch.empty(din.numel(), dtype=torch.uint8).pin_memory()
+        hin.copy_(din)
+        hout = torch.empty(staged[j % replicas][2].numel(), dtype=torch.uint8).pin_memory()
+        hosts.append((hin, hout))
     torch.cuda.synchronize(dev)
-    bi = staged[0][0].numel() + int(reps[0].plan_info.plan_bytes)
+    in_bytes0 = staged[0][1]
+    region0 = int(reps[0].plan_info.ws_plan_off + reps[0].plan_info.plan_bytes)
+    bi = align(in_bytes0) + region0
     bo = staged[0][2].numel()
 
     lib = _lib.load()
-    staged_call = lib.specgen_fork_attn_decode_staged
-    calls = [(C.byref(args), C.byref(r.lens), C.c_void_p(hin.data_ptr()),
-              C.c_void_p(din.data_ptr()), C.c_size_t(din.numel()), C.c_void_p(dout.data_ptr()),
-              C.c_void_p(hout.data_ptr()), C.c_size_t(dout.numel()), C.c_void_p(sp))
-             for r, (din, hin, dout, hout, args) in zip(reps, staged)]
+    call = lib.specgen_fork_attn_decode_staged_inline
+    calls = []
+    for j in range(n_host):
+        r = reps[j % replicas]
+        din, in_bytes, dout, args = staged[j % replicas]
+        hin, hout = hosts[j]
+        calls.append((C.byref(args), C.byref(r.lens), C.c_void_p(hin.data_ptr()),
+                      C.c_void_p(din.data_ptr()), C.c_size_t(in_bytes), C.c_size_t(din.numel()),
+                      C.c_void_p(dout.data_ptr()), C.c_void_p(hout.data_ptr()),
+                      C.c_size_t(dout.numel()), C.c_void_p(sp)))
+    done = [None, None]  # per half: an event after the last call that used it
 
     def step(i):
-        st = staged_call(*calls[i % replicas])
+        j = i % n_host
+        h = j // half
+        if j % half == 0 and done[h] is not None:
+            done[h].synchronize()  # every call that last used this half is done
+        st = call(*calls[j])
         if st != 0:
             raise RuntimeError(_lib.status_string(st))
+        if j % half == half - 1:
+            ev = torch.cuda.Event()
+            ev.record(stream)
+            done[h] = ev
 
     for i in range(W):
         step(i)
@@ -731,12 +763,17 @@ def measure_e2e(w, reps, stream, dev, K, W):
         step(i)
     torch.cuda.synchronize(dev)
     dt = time.perf_counter() - t0
-    for r in reps:  # the per-step plan left every replica planned and consistent
+    for r, (din, in_bytes, _, _) in zip(reps, staged):
+        st = _lib.specgen_workspace_status(din[align(in_bytes):], sp)
+        if st != 0:
+            raise RuntimeError(f"status {_lib.status_string(st)}")
+        # the per-step plan left every replica planned and consistent
         r.plan_info = None
         r.plan(sp)
     torch.cuda.synchronize(dev)
     return {"value": w["total_forks"] * K / dt, "unit": "tokens/s", "h2d_bytes_per_step": bi,
-            "d2h_bytes_per_step": bo, "steps": K}
+            "d2h_bytes_per_step": bo, "steps": K,
+            "api": "specgen_fork_attn_decode_staged_inline"}
 
 
 def run_decode_steps():

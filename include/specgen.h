@@ -222,6 +222,36 @@ specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* arg
                                                void* host_out, size_t out_bytes,
                                                void* cuda_stream);
 
+/* specgen_fork_attn_decode_staged with the plan in the caller's input
+ * buffers (no counterpart in the paper: a serving convenience).  host_in and
+ * dev_in are in_capacity bytes long (dev_in 256-byte aligned); the caller's
+ * packed inputs occupy their first in_bytes, as for
+ * specgen_fork_attn_decode_staged.  The call plans on the host, writes the
+ * plan region (a zeroed status header, then the plan:
+ * specgen_plan.ws_plan_off + plan_bytes bytes, as the workspace would hold
+ * it) into host_in at offset r (in_bytes rounded up to 256) and sends the
+ * first r + region bytes of host_in to dev_in: in one copy after the planning
+ * when the stream still has work queued, or, when the stream is idle (the
+ * GPU is waiting for this host), the inputs at once, overlapping the
+ * planning, and the plan region after it.  The kernels read the plan there,
+ * and keep their partials in args->workspace (still
+ * specgen_fork_attn_workspace_size bytes).  The call's status word is the
+ * first word at dev_in + r: read it with specgen_workspace_status(dev_in + r,
+ * stream).  host_in is written by the call, so, as for the inputs the caller
+ * stores there, no copy still queued may read it (reuse it only after the
+ * stream has passed the previous call's copy).  Returns SPECGEN_ERR_WORKSPACE
+ * when r + region > in_capacity (the inputs may have been copied to dev_in
+ * already; nothing else is queued), the checks of specgen_fork_attn_decode
+ * and SPECGEN_ERR_SHAPE for a dev_in not 256-byte aligned (nothing queued),
+ * SPECGEN_ERR_NULL for a missing buffer, SPECGEN_ERR_CUDA if a copy or
+ * launch cannot be queued. */
+specgen_status specgen_fork_attn_decode_staged_inline(const specgen_fork_attn_args* args,
+                                                      const specgen_host_lens* lens,
+                                                      void* host_in, void* dev_in,
+                                                      size_t in_bytes, size_t in_capacity,
+                                                      const void* dev_out, void* host_out,
+                                                      size_t out_bytes, void* cuda_stream);
+
 /* specgen_fork_attn_decode for callers that cannot allocate device memory.
  * (No counterpart in the paper: this is a deployment convenience.)  Some
  * callers cannot call cudaMalloc at all -- for example a plugin inside a host

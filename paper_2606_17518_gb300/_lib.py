@@ -41,6 +41,7 @@ EXPORTED = [
     "specgen_fork_prefill_plan_host",
     "specgen_fork_attn_decode",
     "specgen_fork_attn_decode_staged",
+    "specgen_fork_attn_decode_staged_inline",
     "specgen_fork_attn_decode_static",
     "specgen_lse_merge",
     "specgen_append_kv",
@@ -184,6 +185,10 @@ def load() -> C.CDLL:
     lib.specgen_fork_attn_decode_staged.argtypes = [
         P(ForkAttnArgs), P(HostLens), C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p,
         C.c_void_p, C.c_size_t, C.c_void_p]
+    lib.specgen_fork_attn_decode_staged_inline.restype = C.c_int
+    lib.specgen_fork_attn_decode_staged_inline.argtypes = [
+        P(ForkAttnArgs), P(HostLens), C.c_void_p, C.c_void_p, C.c_size_t, C.c_size_t,
+        C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]
     lib.specgen_fork_attn_decode_static.restype = C.c_int
     lib.specgen_fork_attn_decode_static.argtypes = [P(ForkAttnArgs), P(HostLens), C.c_void_p]
     lib.specgen_lse_merge.restype = C.c_int
@@ -401,6 +406,16 @@ def specgen_fork_attn_decode_staged(args: ForkAttnArgs, lens: HostLens, host_in,
         C.byref(args), C.byref(lens), _ptr(host_in), _ptr(dev_in), C.c_size_t(in_bytes),
         _ptr(dev_out), _ptr(host_out), C.c_size_t(out_bytes), C.c_void_p(stream)),
         "specgen_fork_attn_decode_staged")
+
+
+def specgen_fork_attn_decode_staged_inline(args: ForkAttnArgs, lens: HostLens, host_in, dev_in,
+                                           in_bytes: int, in_capacity: int, dev_out, host_out,
+                                           out_bytes: int, stream: int = 0) -> None:
+    """One decode step from host memory with the plan in the same host-to-device copy."""
+    _check(load().specgen_fork_attn_decode_staged_inline(
+        C.byref(args), C.byref(lens), _ptr(host_in), _ptr(dev_in), C.c_size_t(in_bytes),
+        C.c_size_t(in_capacity), _ptr(dev_out), _ptr(host_out), C.c_size_t(out_bytes),
+        C.c_void_p(stream)), "specgen_fork_attn_decode_staged_inline")
 
 
 def specgen_fork_attn_decode_static(args: ForkAttnArgs, lens: HostLens, stream: int = 0) -> None:

@@ -1266,8 +1266,11 @@ struct Marks {
 };
 
 // stages: bit 0 the partial-attention kernels, bit 1 the merge.
+// region: where the plan region (status header, then the plan) was uploaded,
+// when not at the start of args->workspace (the partials stay there)
 specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* plan,
-                        void* cuda_stream, Marks& marks, int stages = 3);
+                        void* cuda_stream, Marks& marks, int stages = 3,
+                        unsigned char* region = nullptr);
 
 }  // namespace
 
@@ -1306,7 +1309,7 @@ specgen_status specgen_fork_attn_run_profiled(const specgen_fork_attn_args* args
 namespace {
 
 specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* plan,
-                        void* cuda_stream, Marks& marks, int stages) {
+                        void* cuda_stream, Marks& marks, int stages, unsigned char* region) {
   if (!args || !plan) return SPECGEN_ERR_NULL;
   if (!plan->valid) return SPECGEN_ERR_SHAPE;
   specgen_status st = check_pointers(args);
@@ -1316,7 +1319,8 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   if ((args->kv_layout == SPECGEN_KV_TILED) != ((plan->flags & 2) != 0)) return SPECGEN_ERR_SHAPE;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   unsigned char* ws = static_cast<unsigned char*>(args->workspace);
-  unsigned char* pl = ws + plan->ws_plan_off;
+  unsigned char* hdr = region ? region : ws;  // status word, then the plan
+  unsigned char* pl = hdr + plan->ws_plan_off;
   float* part_o = reinterpret_cast<float*>(ws + plan->ws_part_o_off);
   float* part_lse = reinterpret_cast<float*>(ws + plan->ws_part_lse_off);
 
@@ -1331,7 +1335,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   sp.items = reinterpret_cast<const SplitItem*>(pl + plan->offsets[0]);
   sp.part_o = part_o;
   sp.part_lse = part_lse;
-  sp.status = reinterpret_cast<uint32_t*>(ws);
+  sp.status = reinterpret_cast<uint32_t*>(hdr);
   sp.hq = args->hq;
   sp.hkv = args->hkv;
   sp.dqk = args->head_dim_qk;
@@ -1479,6 +1483,56 @@ specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* arg
   st = plan_impl(args, s, rows_for_decode(lens, s.T, s.F), &plan, cuda_stream, nullptr, 0, true);
   if (st != SPECGEN_OK) return st;
   if ((st = specgen_fork_attn_run(args, &plan, cuda_stream)) != SPECGEN_OK) return st;
+  if (out_bytes > 0 &&
+      cudaMemcpyAsync(host_out, dev_out, out_bytes, cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  return SPECGEN_OK;
+}
+
+specgen_status specgen_fork_attn_decode_staged_inline(const specgen_fork_attn_args* args,
+                                                      const specgen_host_lens* lens,
+                                                      void* host_in, void* dev_in,
+                                                      size_t in_bytes, size_t in_capacity,
+                                                      const void* dev_out, void* host_out,
+                                                      size_t out_bytes, void* cuda_stream) {
+  if (!args || !lens || !host_in || !dev_in) return SPECGEN_ERR_NULL;
+  if (out_bytes > 0 && (!dev_out || !host_out)) return SPECGEN_ERR_NULL;
+  if (reinterpret_cast<uintptr_t>(dev_in) % 256 != 0) return SPECGEN_ERR_SHAPE;
+  // everything that can refuse the call is checked before anything is queued
+  Shape s;
+  specgen_status st = check_shape(args, lens, &s);
+  if (st != SPECGEN_OK) return st;
+  if ((st = check_pointers(args)) != SPECGEN_OK) return st;
+  const size_t off = align_up(in_bytes, 256);
+  if (off > in_capacity) return SPECGEN_ERR_WORKSPACE;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  unsigned char* hin = static_cast<unsigned char*>(host_in);
+  unsigned char* din = static_cast<unsigned char*>(dev_in);
+  // A stream with nothing left to run is waiting for this host: its inputs
+  // then go up at once, overlapping the planning, and the plan follows in a
+  // second copy.  A busy stream gets inputs and plan in one copy after the
+  // planning (the copy would wait behind the queued work anyway).  A stream
+  // that cannot be queried counts as busy (its copy then reports the error).
+  const cudaError_t q = cudaStreamQuery(stream);
+  if (q != cudaSuccess) (void)cudaGetLastError();  // "not ready" is not an error
+  const bool idle = q == cudaSuccess;
+  if (idle && in_bytes > 0 &&
+      cudaMemcpyAsync(dev_in, host_in, in_bytes, cudaMemcpyHostToDevice, stream) != cudaSuccess)
+    return SPECGEN_ERR_CUDA;
+  specgen_plan plan;
+  memset(&plan, 0, sizeof(plan));
+  if ((st = plan_build(args, s, rows_for_decode(lens, s.T, s.F), &plan)) != SPECGEN_OK) return st;
+  const size_t region = t_plan_bytes.size();
+  if (off + region > in_capacity) return SPECGEN_ERR_WORKSPACE;
+  memcpy(hin + off, t_plan_bytes.data(), region);
+  const cudaError_t e =
+      idle ? cudaMemcpyAsync(din + off, hin + off, region, cudaMemcpyHostToDevice, stream)
+           : cudaMemcpyAsync(dev_in, host_in, off + region, cudaMemcpyHostToDevice, stream);
+  if (e != cudaSuccess) return SPECGEN_ERR_CUDA;
+  Marks marks{nullptr, 0};
+  if ((st = run_impl(args, &plan, cuda_stream, marks, 3,
+                     static_cast<unsigned char*>(dev_in) + off)) != SPECGEN_OK)
+    return st;
   if (out_bytes > 0 &&
       cudaMemcpyAsync(host_out, dev_out, out_bytes, cudaMemcpyDeviceToHost, stream) != cudaSuccess)
     return SPECGEN_ERR_CUDA;

@@ -350,3 +350,31 @@ def test_static_decode_plans_once():
     t_plan = np.median([one_plan() for _ in range(300)])
     t_static = np.median([static_call() for _ in range(300)])
     assert t_static < 1.5 * t_plan, (t_static, t_plan)
+
+
+def test_staged_inline_refuses_on_the_host():
+    """The one-copy staged decode checks everything that can refuse the call
+    (buffers, alignment, shapes, the room left for the plan region after the
+    inputs) on the host, before anything is queued, and writes the plan region
+    into the host buffer at the 256-byte boundary after the inputs only then."""
+    lib = _lib.load()
+    w = wl.make_workload("tiny_p512_f4")
+    args = _fake_args(w)
+    lens, keep = _lens(w)
+    plan_buf = np.zeros(1 << 20, np.uint8)
+    plan = _lib.specgen_fork_attn_plan_host(args, lens, plan_buf)
+    region = int(plan.ws_plan_off + plan.plan_bytes)
+    in_bytes = 1000
+    off = 1024
+    host = np.full(off + region, 7, np.uint8)
+    dev = 0x100000
+    call = lambda h, d, cap, **kw: lib.specgen_fork_attn_decode_staged_inline(
+        C.byref(kw.get("args", args)), C.byref(lens), h, C.c_void_p(d), C.c_size_t(in_bytes),
+        C.c_size_t(cap), None, None, C.c_size_t(0), None)
+    hp = host.ctypes.data_as(C.c_void_p)
+    assert call(None, dev, len(host)) == _lib.SPECGEN_ERR_NULL
+    assert call(hp, dev + 16, len(host)) == _lib.SPECGEN_ERR_SHAPE       # dev_in not 256-aligned
+    assert call(hp, dev, off + region - 1) == _lib.SPECGEN_ERR_WORKSPACE  # no room for the plan
+    bad = _fake_args(w, hkv=3)
+    assert call(hp, dev, len(host), args=bad) == _lib.SPECGEN_ERR_SHAPE
+    assert np.all(host == 7)                                              # nothing written

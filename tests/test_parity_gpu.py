@@ -308,6 +308,103 @@ def test_staged_calls_queued_back_to_back():
                  o_ref, lse_ref, f"staged cut {cut.tolist()}")
 
 
+def _inline_buffers(fd, extra):
+    """The step's packed inputs with `extra` bytes of room after them (for the
+    plan region), on the device and in a pinned host twin."""
+    import torch
+    din, hin, views, _ = _pack_device([fd.q, fd.prefix_table, fd.prefix_off, fd.suffix_table,
+                                       fd.suffix_off])
+    in_bytes = din.numel()
+    r = (in_bytes + 255) // 256 * 256
+    d2 = torch.zeros(r + extra, dtype=torch.uint8, device="cuda")
+    d2[:in_bytes].copy_(din)
+    h2 = torch.zeros(r + extra, dtype=torch.uint8).pin_memory()
+    h2[:in_bytes].copy_(hin)
+    # views into the new device buffer at the same offsets
+    out = []
+    for v in views:
+        o = v.data_ptr() - din.data_ptr()
+        n = v.numel() * v.element_size()
+        out.append(d2[o:o + n].view(v.dtype).view(v.shape))
+    return d2, h2, in_bytes, r, out
+
+
+@pytest.mark.parametrize("name", ["tiny_p512_f4", "fork_p8k_f8", "ragged_t8"])
+def test_staged_inline_decode_from_host_buffers(name):
+    """specgen_fork_attn_decode_staged_inline on an idle stream (the inputs go up
+    at once, the plan region after the planning): its outputs equal the plain
+    call's bits, call after call, and its status word sits after the inputs."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload(name)
+    fd = ForkDecode(w)
+    fd.plan()
+    fd.run()
+    o_ref, l_ref = fd.results()
+    region = int(fd.plan_info.ws_plan_off + fd.plan_info.plan_bytes)
+    din, hin, in_bytes, r, views = _inline_buffers(fd, region + 4096)
+    fd.q, fd.prefix_table, fd.prefix_off, fd.suffix_table, fd.suffix_off = views
+    dout, hout, (fd.out, fd.lse), ooff = _pack_device([fd.out, fd.lse])
+    F, hq, dv = w["total_forks"], w["hq"], w["dv"]
+    for _ in range(2):
+        din.zero_()
+        dout.zero_()
+        hout.zero_()
+        torch.cuda.synchronize()
+        _lib.specgen_fork_attn_decode_staged_inline(fd.args(), fd.lens, hin, din, in_bytes,
+                                                    din.numel(), dout, hout, dout.numel())
+        torch.cuda.synchronize()
+        o = hout[ooff[0]:ooff[0] + F * hq * dv * 2].view(torch.bfloat16).float().numpy()
+        lse = hout[ooff[1]:ooff[1] + F * hq * 4].view(torch.float32).numpy()
+        assert np.array_equal(o.astype(np.float64).reshape(F, hq, dv), o_ref)
+        assert np.array_equal(lse.astype(np.float64).reshape(F, hq), l_ref)
+        assert _lib.specgen_workspace_status(din[r:]) == _lib.SPECGEN_OK
+        # the plan region went up with the inputs
+        assert np.array_equal(din[r:r + region].cpu().numpy(), hin[r:r + region].numpy())
+
+
+def test_staged_inline_calls_queued_back_to_back():
+    """Ten staged calls with the plan in the input buffers, queued without a host
+    synchronisation (the stream is busy, so inputs and plan go up in one copy),
+    each with other suffix lengths, its own pinned input buffer (the call writes
+    its plan there) and its own output buffer: every call sees its own plan."""
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload("tiny_p512_f4")
+    fd = ForkDecode(w)
+    fd.plan()
+    region = int(fd.plan_info.ws_plan_off + fd.plan_info.plan_bytes)
+    din, hin0, in_bytes, r, views = _inline_buffers(fd, region + 4096)
+    fd.q, fd.prefix_table, fd.prefix_off, fd.suffix_table, fd.suffix_off = views
+    dout, _, (fd.out, fd.lse), ooff = _pack_device([fd.out, fd.lse])
+    F, hq, dv = w["total_forks"], w["hq"], w["dv"]
+    base = np.asarray(w["suffix_lens"], dtype=np.int32)
+    stream = torch.cuda.current_stream().cuda_stream
+    torch.cuda.synchronize()
+    houts, cuts, hins = [], [], []
+    for i in range(10):
+        cut = np.maximum(base - (i * 5) % 13 - np.arange(len(base)) * (i % 3), 0).astype(np.int32)
+        fd.set_suffix_lens(cut)
+        hin = torch.zeros_like(hin0).pin_memory()
+        hin[:in_bytes].copy_(hin0[:in_bytes])
+        hout = torch.zeros(dout.numel(), dtype=torch.uint8).pin_memory()
+        _lib.specgen_fork_attn_decode_staged_inline(fd.args(), fd.lens, hin, din, in_bytes,
+                                                    din.numel(), dout, hout, dout.numel(), stream)
+        hins.append(hin)
+        houts.append(hout)
+        cuts.append(cut)
+    torch.cuda.synchronize()
+    assert _lib.specgen_workspace_status(din[r:]) == _lib.SPECGEN_OK
+    for cut, hout in zip(cuts, houts):
+        o = hout[ooff[0]:ooff[0] + F * hq * dv * 2].view(torch.bfloat16).float().numpy()
+        lse = hout[ooff[1]:ooff[1] + F * hq * 4].view(torch.float32).numpy()
+        wc = dict(w)
+        wc["suffix_lens"] = cut
+        o_ref, lse_ref = oracle.fork_attn_decode(wc)
+        _compare(o.astype(np.float64).reshape(F, hq, dv), lse.astype(np.float64).reshape(F, hq),
+                 o_ref, lse_ref, f"inline cut {cut.tolist()}")
+
+
 def test_plan_once_run_many_is_deterministic():
     from paper_2606_17518_gb300.fork_attn import ForkDecode
     w = wl.make_workload("fork_p8k_f8")
