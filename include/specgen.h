@@ -240,11 +240,11 @@ specgen_status specgen_fork_attn_decode_staged(const specgen_fork_attn_args* arg
  * stream).  host_in is written by the call, so, as for the inputs the caller
  * stores there, no copy still queued may read it (reuse it only after the
  * stream has passed the previous call's copy).  Returns SPECGEN_ERR_WORKSPACE
- * when r + region > in_capacity (the inputs may have been copied to dev_in
- * already; nothing else is queued), the checks of specgen_fork_attn_decode
- * and SPECGEN_ERR_SHAPE for a dev_in not 256-byte aligned (nothing queued),
- * SPECGEN_ERR_NULL for a missing buffer, SPECGEN_ERR_CUDA if a copy or
- * launch cannot be queued. */
+ * when r + region > in_capacity or args->workspace_bytes is too small (the
+ * inputs may have been copied to dev_in already; nothing else is queued), the
+ * shape and pointer checks of specgen_fork_attn_decode and SPECGEN_ERR_SHAPE
+ * for a dev_in not 256-byte aligned (nothing queued), SPECGEN_ERR_NULL for a
+ * missing buffer, SPECGEN_ERR_CUDA if a copy or launch cannot be queued. */
 specgen_status specgen_fork_attn_decode_staged_inline(const specgen_fork_attn_args* args,
                                                       const specgen_host_lens* lens,
                                                       void* host_in, void* dev_in,
