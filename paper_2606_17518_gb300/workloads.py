@@ -83,6 +83,14 @@ DIAGNOSTIC = {
     "suffix_only_f64_s2048": WorkloadSpec(
         "suffix_only_f64_s2048", 1, (0, 0), (64, 64), (2048, 2048), hq=64, hkv=8, dqk=128,
         dv=128, page_size=16, seed=5),
+    # the latent kernel's prefix chunks are shared by the forks' items through L2:
+    # four times the forks, and a prefix larger than L2 (151 MB of latent KV)
+    "mla_p16k_f32": WorkloadSpec(
+        "mla_p16k_f32", 1, (16384, 16384), (32, 32), (128, 1024), hq=128, hkv=1, dqk=576,
+        dv=512, page_size=64, separate_v=False, seed=6),
+    "mla_p128k_f8": WorkloadSpec(
+        "mla_p128k_f8", 1, (131072, 131072), (8, 8), (128, 1024), hq=128, hkv=1, dqk=576,
+        dv=512, page_size=64, separate_v=False, seed=7),
 }
 
 
