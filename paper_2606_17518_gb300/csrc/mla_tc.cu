@@ -13,7 +13,8 @@
 // shared memory next to two 64-token K tiles (72 KB each), so its first 256
 // columns live in tensor memory (the A operand of the first 16 k-steps) and
 // the other 320 in shared memory.  Per 64-token tile t (one page):
-//   warp 0 (TMA)   nine boxes of 64 rows x 64 columns (128B swizzle) -> 2-stage ring
+//   warp 0 (TMA)   the page as one box (nine panels of 64 rows x 64 columns,
+//                  128B swizzle) -> 2-stage ring
 //   warp 1 (MMA)   S_t = Q K_t^T (36 k-steps, N = 64; A from TMEM, then shared
 //                  memory), then O += P_t V_t[:, dv0:dv0+256] (A = P in TMEM, N = 256)
 //   warps 2-5      one thread per head: the tile's scores, masked, online
@@ -85,6 +86,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto sK = [&](int s) { return base + kOffKV + s * kStage; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // the merge (a programmatic dependent) may be launched now: it waits for this
+  // grid's completion before it reads any partial
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
   auto table_of = [&](const TcItem& it) {
     const int32_t* bt = it.table_kind == 0 ? p.prefix_bt : p.suffix_bt;
@@ -115,6 +119,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_relinquish();
   }
   tc_fence_before();
+  // Launched as a programmatic dependent, the grid may start while the stream's
+  // previous kernel is still running: everything above touches only this CTA's
+  // own resources and the plan (written by a host copy).  Inputs (lengths,
+  // tables, Q, the pool) and the partial buffers are used only after this wait.
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
@@ -122,7 +131,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     // A tile is one page; page ids are fetched 32 at a time by the warp, one
-    // batch ahead.  Lanes 0..8 each issue one 64-column box.
+    // batch ahead.  Lane 0 issues the tile as one box: all nine 64-column
+    // panels of the page, landing panel after panel.
     int t = 0;
     bool ok = true;
     for (int ii = it_begin; ok && ii < it_end; ++ii) {
@@ -151,8 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
-        if (lane < kPanels)
-          tma_load_4d(sK(s) + lane * kKPanel, &tmk, lane * 64, slot0, 0, page, full(s));
+        if (lane == 0) tma_load_4d(sK(s), &tmk, 0, slot0, 0, page, full(s));
         if (lane == 0 && (page < 0 || page >= p.num_pages)) atomicOr(p.status, kStatusIndex);
       }
     }
@@ -488,13 +497,13 @@ cudaError_t launch_mla_tc(const MlaParams& p, const void* k_pages, int grid, cud
   if (grid == 0) return cudaSuccess;
   EncodeTiledFn enc = encode_fn();
   if (!enc || !k_pages || p.num_pages < 1) return cudaErrorInvalidValue;
-  // latent pool [num_pages][1][64][576] as a 4-D tensor (576, 64, 1, pages);
-  // one box = 64 columns x 64 rows (one page)
+  // latent pool [num_pages][64][576] as a 4-D tensor (64 columns, 64 rows, 9
+  // panels, pages) with the panel stride (128 B) inside the row stride: one box
+  // is a whole page, landing as [panel][row][128 B], 128-byte swizzled
   CUtensorMap mk;
-  const cuuint64_t dims[4] = {(cuuint64_t)kDqk, (cuuint64_t)kPage, 1, (cuuint64_t)p.num_pages};
-  const cuuint64_t strides[3] = {(cuuint64_t)kDqk * 2, (cuuint64_t)kPage * kDqk * 2,
-                                 (cuuint64_t)kPage * kDqk * 2};
-  const cuuint32_t box[4] = {64, kTT, 1, 1};
+  const cuuint64_t dims[4] = {64, (cuuint64_t)kPage, (cuuint64_t)kPanels, (cuuint64_t)p.num_pages};
+  const cuuint64_t strides[3] = {(cuuint64_t)kDqk * 2, 128, (cuuint64_t)kPage * kDqk * 2};
+  const cuuint32_t box[4] = {64, kTT, (cuuint32_t)kPanels, 1};
   const cuuint32_t estr[4] = {1, 1, 1, 1};
   if (enc(&mk, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(k_pages), dims, strides,
           box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -513,8 +522,18 @@ cudaError_t launch_mla_tc(const MlaParams& p, const void* k_pages, int grid, cud
     if (e != cudaSuccess) return e;
     configured = dev;
   }
-  mla_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(p, mk);
-  return cudaGetLastError();
+  // programmatic dependent launch: the prologue overlaps the previous kernel
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = (size_t)kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, mla_tc_kernel, p, mk);
 }
 
 }  // namespace specgen
