@@ -7,7 +7,9 @@
 // are block copies: buffer word w belongs to section s (K, then V), page i and
 // offset o, and pairs with word o of block table[i] of that section's pool.
 // Grid-stride over the buffer's 16-byte words, four independent words per
-// thread in flight; a page id outside the pool is skipped and reported.
+// thread in flight; a page id outside the pool is skipped and reported.  The
+// kernel is a programmatic dependent: it waits for the stream's previous
+// kernel before it reads anything and lets the next one launch at once.
 #include <cuda_runtime.h>
 
 #include "pack_pages.h"
@@ -21,6 +23,8 @@ constexpr int kThreads = 256;
 constexpr int kUnroll = 4;
 
 __global__ void __launch_bounds__(kThreads) pack_pages_kernel(const PackParams p) {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   const size_t nk = (size_t)p.n_pages * p.k_block16;
   const size_t total = nk + (p.v_pages ? (size_t)p.n_pages * p.v_block16 : 0);
   const size_t stride = (size_t)gridDim.x * kThreads * kUnroll;
@@ -68,8 +72,16 @@ cudaError_t launch_pack_pages(const PackParams& p, int n_sm, cudaStream_t stream
   size_t grid = (total + per_cta - 1) / per_cta;
   const size_t cap = (size_t)n_sm * 8;  // enough CTAs in flight to cover HBM latency
   if (grid > cap) grid = cap;
-  pack_pages_kernel<<<(unsigned)grid, kThreads, 0, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, pack_pages_kernel, p);
 }
 
 }  // namespace specgen
