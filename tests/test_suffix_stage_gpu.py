@@ -200,3 +200,34 @@ def test_suffix_stage_repeatable(G, hkv, layout, mode):
     o2, l2 = fd.results()
     assert np.array_equal(o1, o2) and np.array_equal(l1, l2)
     assert fd.status() == _lib.SPECGEN_OK
+
+
+def _ragged_fuzz_spec(case):
+    """Random multi-trace calls large enough that the planner runs the suffix
+    stage beside the prefix kernel: 3-4 traces, 12-20 forks each, prefixes of
+    0.5k-5k tokens and suffixes of 150-800, G from 1 to 16 (with G = 3, 6 and
+    12 filling their n-tiles partly), head dims 64 and 128."""
+    rng = np.random.default_rng(4200 + case)
+    G = [1, 2, 4, 8, 12, 16, 3, 6][case]
+    hkv = [8, 8, 8, 4, 8, 4, 8, 8][case]
+    dqk = [64, 128][case % 2]
+    return wl.WorkloadSpec(
+        name=f"ragged_fuzz{case}", num_traces=int(rng.integers(3, 5)),
+        prefix_len=(int(rng.integers(500, 2000)), int(rng.integers(2000, 5000))),
+        forks=(int(rng.integers(12, 15)), int(rng.integers(15, 21))),
+        suffix_len=(int(rng.integers(150, 400)), int(rng.integers(500, 800))),
+        hq=G * hkv, hkv=hkv, dqk=dqk, dv=dqk, page_size=16, seed=int(rng.integers(1 << 30)))
+
+
+@pytest.mark.parametrize("case", range(8))
+def test_ragged_calls_with_the_suffix_stage_every_row(case):
+    """Every (fork, head) row of random ragged calls that split the SMs between
+    the prefix kernel and the suffix-stage kernel, against the oracle; the pool
+    layout alternates between cases."""
+    w = wl.make_workload(_ragged_fuzz_spec(case))
+    kv = _lib.KV_TILED if case % 2 else _lib.KV_ROWS
+    o, lse, fd = _run(w, kv)
+    assert fd.plan_info.n_tc_ctas > 0
+    assert fd.status() == _lib.SPECGEN_OK
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(o, lse, o_ref, lse_ref, f"ragged fuzz {case}")
