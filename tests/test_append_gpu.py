@@ -160,17 +160,26 @@ def test_plan_ahead_cut_to_device_lengths(name, ahead):
     assert float(np.max(np.abs(lse[fin] - lse_ref[fin]))) <= TOL_LSE
 
 
+# a ragged call whose plan runs the suffix-stage kernel beside the prefix kernel
+SPLIT_SPEC = wl.WorkloadSpec(name="split_g8", num_traces=3, prefix_len=(800, 4000),
+                             forks=(14, 20), suffix_len=(200, 700), hq=32, hkv=4, dqk=128,
+                             dv=128, page_size=16, seed=4321)
+
+
 @pytest.mark.parametrize("advance", ["torch", "append"])
-@pytest.mark.parametrize("name", ["fork_p8k_f8", "mla_p16k_f8"])
+@pytest.mark.parametrize("name", ["fork_p8k_f8", "mla_p16k_f8", "split_g8"])
 def test_one_plan_many_decode_steps_in_a_graph(name, advance):
     """One plan for 12 steps ahead; 12 steps of (append, advance the device
     lengths, attention) captured in one CUDA graph; the last step's output and
     the pools match the oracle.  The lengths advance either by a torch add on
-    the device or by the append itself (into the other of two arrays)."""
+    the device or by the append itself (into the other of two arrays).  With
+    split_g8 the plan runs the suffix-stage kernel, whose items the device
+    lengths cut every step."""
     import torch
     from paper_2606_17518_gb300.fork_attn import ForkDecode
     steps = 12
-    st = wl.make_decode_state(wl.make_workload(name), steps)
+    base = wl.make_workload(SPLIT_SPEC if name == "split_g8" else name)
+    st = wl.make_decode_state(base, steps)
     fd = ForkDecode(st)
     fd.use_device_lens = True
     lens0 = st["suffix_lens"].copy()
@@ -180,6 +189,8 @@ def test_one_plan_many_decode_steps_in_a_graph(name, advance):
     sp = stream.cuda_stream
     fd.plan(sp)
     torch.cuda.synchronize()
+    if name == "split_g8":
+        assert fd.plan_info.n_sfx_ctas > 0 and fd.plan_info.n_tc_ctas > 0
     free = torch.from_numpy(st["free_pages"]).cuda()
     k_new = torch.from_numpy(st["k_new"].view(np.int16)).cuda().view(torch.bfloat16)
     v_new = (None if st["v_new"] is None else
