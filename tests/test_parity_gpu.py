@@ -515,3 +515,45 @@ def test_back_to_back_plans_with_changing_lengths():
         o_ref, lse_ref = oracle.fork_attn_decode(wc)
         _compare(o.float().cpu().numpy().astype(np.float64), lse.cpu().numpy().astype(np.float64),
                  o_ref, lse_ref, f"cut {cut.tolist()}")
+
+
+@pytest.mark.parametrize("name,layout", [("ragged_t8", "tiled"), ("fork_p8k_f8", "rows"),
+                                         ("mla_p16k_f8", "rows")])
+def test_alternating_calls_sharing_a_workspace(name, layout):
+    """Two calls with different queries share one workspace (plan and partials)
+    and are queued back to back, five pairs between host synchronisations: each
+    call's own output keeps its single-call bits.  A call whose kernels wrote
+    partials while the previous call's merge still read them (the
+    grid-dependency waits of the chained launches) would show here."""
+    import copy
+    import torch
+    from paper_2606_17518_gb300.fork_attn import ForkDecode
+    w = wl.make_workload(name)
+    kv = _lib.KV_TILED if layout == "tiled" else _lib.KV_ROWS
+    a = ForkDecode(w, kv_layout=kv)
+    b = copy.copy(a)  # the same pools, tables and workspace
+    b.q = a.q.flip(0).contiguous()  # other queries: the forks' rows in reverse order
+    b.out, b.lse = torch.empty_like(a.out), torch.empty_like(a.lse)
+    a.plan()
+    b.plan_info = a.plan_info  # the same plan, in the same workspace
+    a.run()
+    torch.cuda.synchronize()
+    ra = (a.out.clone(), a.lse.clone())
+    b.run()
+    torch.cuda.synchronize()
+    rb = (b.out.clone(), b.lse.clone())
+    a.out.zero_()
+    b.out.zero_()
+    for i in range(100):
+        a.run()
+        b.run()
+        if i % 5 == 4:
+            assert torch.equal(a.out, ra[0]) and torch.equal(a.lse, ra[1]), i
+            assert torch.equal(b.out, rb[0]) and torch.equal(b.lse, rb[1]), i
+            a.out.zero_()
+            b.out.zero_()
+    assert a.status() == _lib.SPECGEN_OK
+    # and the references themselves are right
+    o_ref, lse_ref = oracle.fork_attn_decode(w)
+    _compare(ra[0].float().cpu().numpy().astype(np.float64),
+             ra[1].cpu().numpy().astype(np.float64), o_ref, lse_ref, name)
