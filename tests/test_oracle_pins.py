@@ -100,6 +100,42 @@ def test_two_key_golden_fixture():
     np.testing.assert_allclose(lse[0], vals["lse"][0], rtol=0, atol=1e-15)
 
 
+def test_fork_decode_golden_fixture():
+    """A shared paged prefix and two private suffixes, worked by hand
+    (tests/golden/fork_decode_small.txt): pins the prefix/suffix concatenation,
+    the page and slot lookup and the per-fork independence of the suffixes."""
+    vals, kv = {}, []
+    with open(os.path.join(GOLDEN, "fork_decode_small.txt")) as fh:
+        for line in fh:
+            if not line.strip() or line.startswith("#"):
+                continue
+            name, *nums = line.split()
+            if name in ("k", "v"):
+                kv.append((name, [float(x) for x in nums]))
+            else:
+                vals[name] = [float(x) for x in nums]
+    B, P = int(vals["page_size"][0]), int(vals["num_pages"][0])
+    pools = {n: np.full((P, 1, B, 2), wl.BF16_QNAN, dtype=np.uint16) for n in ("k", "v")}
+    for name, (page, slot, x, y) in kv:
+        pools[name][int(page), 0, int(slot)] = wl.round_to_bf16_bits(np.array([x, y]))
+    q = wl.round_to_bf16_bits(np.array([vals["q"], vals["q"]])).reshape(2, 1, 2)
+    w = dict(q=q, k_pages=pools["k"], v_pages=pools["v"],
+             prefix_table=np.array(vals["prefix_table"], np.int32),
+             prefix_bt_offsets=np.array([0, 1], np.int32),
+             prefix_lens=np.array(vals["prefix_len"], np.int32),
+             fork_offsets=np.array([0, 2], np.int32),
+             suffix_table=np.array(vals["suffix_table"], np.int32),
+             suffix_bt_offsets=np.array([0, 1, 2], np.int32),
+             suffix_lens=np.array(vals["suffix_lens"], np.int32),
+             num_traces=1, total_forks=2, num_pages=P, hq=1, hkv=1, dqk=2, dv=2,
+             page_size=B, scale=math.log(vals["scale_log_of"][0]))
+    o, lse = oracle.fork_attn_decode(w)
+    np.testing.assert_allclose(o[0, 0], vals["o0"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(o[1, 0], vals["o1"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(lse[:, 0], [vals["lse0"][0], vals["lse1"][0]], rtol=0, atol=1e-14)
+    assert abs(vals["lse0"][0] - math.log(7)) < 1e-15 and abs(vals["lse1"][0] - math.log(4)) < 1e-15
+
+
 def test_empty_key_set():
     o, lse = attention_rows(np.ones((2, 4)), np.zeros((0, 4)), np.zeros((0, 3)), 1.0)
     assert np.array_equal(o, np.zeros((2, 3)))
