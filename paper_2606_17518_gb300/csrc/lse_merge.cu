@@ -65,6 +65,29 @@ __global__ void __launch_bounds__(kMergeThreads, MIN_BLOCKS) merge_parts_kernel(
   store_merged(mr, p.out + (size_t)row * p.dv, c4, p.lse + row, c4 == 0);
 }
 
+// merge_parts_kernel with two 4-column slices per thread (c4 = 2 k and 2 k + 1
+// of the same head): the form for grids of many waves.
+template <int BATCH, int MIN_BLOCKS>
+__global__ void __launch_bounds__(kMergeThreads, MIN_BLOCKS) merge_parts2_kernel(const MergeParams p) {
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  const int c4n = p.dv / 4, c2n = c4n / 2;
+  const int gid = blockIdx.x * kMergeThreads + threadIdx.x;
+  const bool live = gid < p.n_rows * c2n;
+  const int h = gid % p.hq, rest = gid / p.hq;
+  const int c4 = 2 * (rest % c2n), f = rest / c2n;
+  const int row = f * p.hq + h;
+  const int base = live ? p.part_base[f] : 0;
+  const int n = live ? p.n_parts[f * p.n_groups + h / (p.hq / p.n_groups)] : 0;
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  if (!live) return;
+  RowMerge r0, r1;
+  merge_row2<BATCH>(p.part_lse + (size_t)base * p.hq + h, (size_t)p.hq,
+                    reinterpret_cast<const float4*>(p.part_o) + part_o_f4(base, h, c4, p.hq, p.dv),
+                    (size_t)c4n * p.hq, (size_t)p.hq, n, &r0, &r1);
+  store_merged(r0, p.out + (size_t)row * p.dv, c4, p.lse + row, c4 == 0);
+  store_merged(r1, p.out + (size_t)row * p.dv, c4 + 1, p.lse + row, false);
+}
+
 template <typename T>
 __device__ __forceinline__ float ld_as_float(const T* p, size_t i);
 template <>
@@ -120,9 +143,10 @@ cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool a
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (configured != dev) {
-    const void* kernels[3] = {reinterpret_cast<const void*>(merge_parts_kernel<16, 1>),
+    const void* kernels[4] = {reinterpret_cast<const void*>(merge_parts_kernel<16, 1>),
                               reinterpret_cast<const void*>(merge_parts_kernel<8, 4>),
-                              reinterpret_cast<const void*>(merge_parts_kernel<4, 8>)};
+                              reinterpret_cast<const void*>(merge_parts_kernel<4, 8>),
+                              reinterpret_cast<const void*>(merge_parts2_kernel<4, 4>)};
     // keep the SMs in the shared-memory-heavy configuration of the kernels
     // around this one, so that no L1/shared-memory reconfiguration is needed
     for (const void* k : kernels) {
@@ -135,8 +159,15 @@ cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool a
     configured = dev;
   }
   const long long threads = (long long)p.n_rows * (p.dv / 4);
-  const long long blocks = (threads + kMergeThreads - 1) / kMergeThreads;
-  const int form = blocks > 3LL * sms ? 2 : (p.max_parts <= 8 ? 1 : 0);
+  long long blocks = (threads + kMergeThreads - 1) / kMergeThreads;
+  int form = blocks > 3LL * sms ? 2 : (p.max_parts <= 8 ? 1 : 0);
+  // grids of many waves over rows of few parts: two slices per thread (half
+  // the threads, twice the bytes in flight each; with many parts per row the
+  // one-slice form keeps more rows in flight)
+  if (form == 2 && p.max_parts <= 8 && (p.dv / 4) % 2 == 0) {
+    form = 3;
+    blocks = (threads / 2 + kMergeThreads - 1) / kMergeThreads;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)blocks);
   cfg.blockDim = dim3(kMergeThreads);
@@ -147,6 +178,7 @@ cudaError_t launch_merge_parts(const MergeParams& p, cudaStream_t stream, bool a
   attr[0].val.programmaticStreamSerializationAllowed = after_dependent ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  if (form == 3) return cudaLaunchKernelEx(&cfg, merge_parts2_kernel<4, 4>, p);
   if (form == 2) return cudaLaunchKernelEx(&cfg, merge_parts_kernel<4, 8>, p);
   if (form == 1) return cudaLaunchKernelEx(&cfg, merge_parts_kernel<8, 4>, p);
   return cudaLaunchKernelEx(&cfg, merge_parts_kernel<16, 1>, p);
