@@ -199,9 +199,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = p.cta_offsets[blockIdx.x], it_end = p.cta_offsets[blockIdx.x + 1];
   const int n_items = it_end - it_begin;
-  // dependents released at the start (see late_trigger)
-  if (!p.late_trigger && threadIdx.x == 0)
-    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  // dependents (the merge) released at the start: they wait for this grid's
+  // completion before they read anything it writes
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
   // the CTA's first items, one per lane (40-byte records): the plan is written
   // by a host copy, never by a kernel, so it is read before the wait below
@@ -243,7 +243,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   // kernel of the stream is still running: everything above touches only this
   // CTA's own resources and the plan.  The inputs (device lengths, block tables,
   // Q, K/V, possibly written by that kernel) and the partial buffers (possibly
-  // still read by it) are used only after this wait.  Before it, the two copy
+  // still read by it) are used only after this wait.  (Behind the suffix stage
+  // there is no wait here: see wait_at_end.)  Before it, the two copy
   // warps only ask L2 for the first item's first two tiles: the page ids they
   // read here serve as prefetch addresses (in-range ids only) and nothing else,
   // so a table the previous kernel rewrites costs bandwidth, never correctness.
@@ -263,13 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
-  asm volatile("griddepcontrol.wait;\n" ::: "memory");
-  // With the suffix stage behind it, the next kernel of the stream may be
-  // launched only once every CTA is past this wait, i.e. once the previous
-  // kernel has finished: the suffix stage runs beside this grid and relies on
-  // that ordering for its inputs.
-  if (p.late_trigger && threadIdx.x == 0)
-    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  if (!p.wait_at_end) asm volatile("griddepcontrol.wait;\n" ::: "memory");
   if (warp == 0) {
     __syncwarp();
     for (int k = lane; k < n_cached; k += 32) items[k] = clamp_item(items[k], p.suffix_lens);
@@ -804,6 +799,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  // behind the suffix stage: complete only after it has (see wait_at_end)
+  if (p.wait_at_end) asm volatile("griddepcontrol.wait;\n" ::: "memory");
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,

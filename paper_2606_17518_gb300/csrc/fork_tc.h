@@ -26,11 +26,12 @@ struct TcParams {
   const int32_t* suffix_lens;  // device lengths that clamp suffix items, or nullptr
   int hq, hkv, G, dv, num_pages;
   float scale_log2;            // softmax scale * log2(e), > 0
-  // 1: the suffix-stage kernel follows this grid in the stream and runs beside
-  // it, so its dependents are released only once every CTA has passed the wait
-  // for the previous kernel; 0: they are released at the start (the merge
-  // waits for this grid's completion anyway)
-  int late_trigger;
+  // 1: this grid follows the suffix-stage kernel in the stream and runs beside
+  // it.  It is launched only once every suffix-stage CTA has passed its wait for
+  // the kernel before both, so it starts without a wait of its own; it waits for
+  // the suffix-stage grid at its end instead, so that the merge, which waits for
+  // this grid, sees the suffix partials too.
+  int wait_at_end;
 };
 
 bool fork_tc_supported(int dqk, int dv, bool latent, int page_size, int G);

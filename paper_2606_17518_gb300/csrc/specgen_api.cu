@@ -1345,7 +1345,15 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
   sp.scale_log2 = args->scale * 1.4426950408889634f;
   sp.suffix_lens = args->suffix_lens;
   if (!marks.mark(stream, 0)) return SPECGEN_ERR_CUDA;
-  if ((stages & 1) && plan->n_tc_ctas > 0) {
+  // With both partial kernels the suffix stage goes first: it waits for the
+  // stream's previous kernel, then lets the prefix kernel launch beside it on
+  // the SMs it leaves free; the prefix kernel, which usually ends last, waits
+  // for the suffix-stage grid only at its end, and the merge waits for the
+  // prefix kernel.  (The other order makes the suffix stage hold its CTAs
+  // until the prefix kernel completes: two grid completions in a row at the
+  // end of every call.)
+  const bool both = (stages & 1) && plan->n_tc_ctas > 0 && plan->n_sfx_ctas > 0;
+  auto launch_tc = [&]() -> specgen_status {
     TcParams tp;
     tp.q = sp.q;
     tp.prefix_bt = args->prefix_block_table;
@@ -1365,7 +1373,7 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     tp.num_pages = args->num_pages;
     tp.scale_log2 = sp.scale_log2;
     tp.suffix_lens = args->suffix_lens;
-    tp.late_trigger = plan->n_sfx_ctas > 0 ? 1 : 0;
+    tp.wait_at_end = both ? 1 : 0;
     cudaError_t e;
     if (args->v_pages == nullptr) {
       MlaParams mp;
@@ -1393,8 +1401,9 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     }
     if (e != cudaSuccess) return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
-  }
-  if ((stages & 1) && plan->n_sfx_ctas > 0) {
+    return SPECGEN_OK;
+  };
+  auto launch_sfx = [&]() -> specgen_status {
     SfxParams xp;
     xp.q = sp.q;
     xp.k_pages = static_cast<const __nv_bfloat16*>(args->k_pages);
@@ -1414,11 +1423,20 @@ specgen_status run_impl(const specgen_fork_attn_args* args, const specgen_plan* 
     xp.dv = args->head_dim_v;
     xp.num_pages = args->num_pages;
     xp.scale_log2 = sp.scale_log2;
-    xp.wait_first = plan->n_tc_ctas > 0 ? 0 : 1;
+    xp.late_trigger = both ? 1 : 0;
     if (launch_suffix_stage(xp, args->k_pages, args->v_pages, plan->n_sfx_ctas, args->head_dim_qk,
                             args->kv_layout == SPECGEN_KV_TILED, stream) != cudaSuccess)
       return SPECGEN_ERR_CUDA;
     if (!marks.mark(stream, ++marks.launches)) return SPECGEN_ERR_CUDA;
+    return SPECGEN_OK;
+  };
+  if ((stages & 1) && plan->n_sfx_ctas > 0) {
+    const specgen_status st = launch_sfx();
+    if (st != SPECGEN_OK) return st;
+  }
+  if ((stages & 1) && plan->n_tc_ctas > 0) {
+    const specgen_status st = launch_tc();
+    if (st != SPECGEN_OK) return st;
   }
   if ((stages & 1) && plan->n_split_items > 0) {
     if (launch_split_decode(sp, plan->n_split_items, args->v_pages == nullptr, stream) !=

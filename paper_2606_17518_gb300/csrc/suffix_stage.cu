@@ -1,6 +1,7 @@
 // Suffix stage of fork decode: a split-K, bandwidth-bound paged decode kernel
-// that runs beside the tensor-core prefix kernel, on the SMs that kernel leaves
-// free.
+// that runs beside the tensor-core prefix kernel, each on its own share of the
+// SMs (launched first, this grid takes its share; the prefix kernel, launched
+// once every CTA here has passed the wait for the previous kernel, the rest).
 //
 // The suffix of one fork is private to that fork, so its keys serve only the
 // G = hq / hkv query heads of one kv head: a 128-row tensor-core tile would
@@ -130,13 +131,13 @@ __device__ __forceinline__ void suffix_warp(const SfxParams& p, const CUtensorMa
     for (int x = lane; x < n_cached * kWords; x += 32) dst[x] = src[x];
   }
   __syncwarp();
-  // Alone (waiting for the previous kernel below), the warp first asks L2 for
+  // Before waiting for the previous kernel (below), the warp asks L2 for
   // its first item's first pages and query rows, read with the item as
   // planned: only plans with host-resolved table offsets take part, so every
   // read here is of the plan or of table entries at positions the plan was made
   // for.  A prefetch moves nothing into this CTA: a table or length the previous
   // kernel still rewrites can at worst warm the wrong pages.
-  if (p.wait_first && n_cached > 0 && cache[0].table_off >= 0) {
+  if (n_cached > 0 && cache[0].table_off >= 0) {
     const TcItem it0 = cache[0];
     const int np0 = (it0.tok_end - it0.tok_begin + kPage - 1) / kPage;
     if (lane < kSlots && lane < np0) {
@@ -158,11 +159,12 @@ __device__ __forceinline__ void suffix_warp(const SfxParams& p, const CUtensorMa
     }
   }
   // Inputs (device lengths, tables, Q, K/V) may be written by the stream's
-  // previous kernel, and the partial buffers still read by it.  Alone, this
-  // grid waits for it here.  Behind the prefix kernel, this grid starts only
-  // after every prefix CTA has passed its own wait for that kernel, so the
-  // inputs are ready (the wait comes at the end, see there).
-  if (p.wait_first) asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  // previous kernel, and the partial buffers still read by it: this grid waits
+  // for it here.  With the prefix kernel behind it, that kernel is released
+  // only now (so it needs no wait of its own for the inputs).
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  if (p.late_trigger && threadIdx.x == 0)
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   if (lane < n_cached) cache[lane] = clamp_item(cache[lane], p.suffix_lens);
   __syncwarp();
 
@@ -474,9 +476,6 @@ __device__ __forceinline__ void suffix_warp(const SfxParams& p, const CUtensorMa
     if (q_issued > q_used) mbar_wait_drain(qbar, q_used & 1, p.status);
   }
   __syncwarp();
-  // beside the prefix kernel: complete only after it has, so that the merge
-  // (which waits for this grid) sees the prefix partials too
-  if (!p.wait_first) asm volatile("griddepcontrol.wait;\n" ::: "memory");
 }
 
 template <int D, bool TL, int NT>
@@ -493,9 +492,10 @@ __global__ void __launch_bounds__(kSuffixWarps * 32, kSuffixCtasPerSm)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(gb + L::kAbort);
   if (threadIdx.x == 0) {
     *abort_flag = 0;
-    // the merge (a programmatic dependent) may be launched now: it waits for
-    // this grid's completion before it reads any partial
-    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+    // alone, the merge (a programmatic dependent) may be launched now: it waits
+    // for this grid's completion before it reads any partial (with the prefix
+    // kernel behind this grid, the trigger comes after the wait instead)
+    if (!p.late_trigger) asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   }
   __syncthreads();
   suffix_warp<D, TL, NT>(p, &tmk, &tmv, sb, gb, threadIdx.x >> 5, abort_flag);

@@ -32,12 +32,13 @@ struct SfxParams {
   const int32_t* suffix_lens;    // device lengths that clamp the items, or nullptr
   int hq, hkv, G, dv, num_pages;
   float scale_log2;              // softmax scale * log2(e), > 0
-  // 1: no kernel of this call runs ahead of this one, so it waits for the
-  // stream's previous kernel before it touches anything.  0: it runs beside the
-  // prefix kernel, which is launched first and lets it start only once that
-  // previous kernel has finished; it then waits for the prefix kernel before
-  // it completes, so that the merge after it sees every partial.
-  int wait_first;
+  // This grid is the first partial-attention kernel of a call: it waits for the
+  // stream's previous kernel before it touches anything.  late_trigger 1: the
+  // prefix kernel follows it in the stream and runs beside it, so this grid's
+  // dependents are released only once every CTA has passed that wait (the
+  // prefix kernel then starts without a wait of its own); 0: they (the merge)
+  // are released at the start.
+  int late_trigger;
 };
 
 bool suffix_stage_supported(int dqk, int dv, bool latent, int page_size, int G);
