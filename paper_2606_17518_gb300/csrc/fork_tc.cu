@@ -250,8 +250,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   // so a table the previous kernel rewrites costs bandwidth, never correctness.
   // Only plans with host-resolved table offsets take part: then every read
   // here is of the plan or of table entries at positions the plan was built
-  // for.
-  if ((warp == 0 || warp == kVWarp) && n_items > 0) {
+  // for.  Behind the suffix stage there is no wait to overlap, and the copies
+  // themselves follow at once: no prefetch (measured 0.5 us faster).
+  if (!p.wait_at_end && (warp == 0 || warp == kVWarp) && n_items > 0) {
     const TcItem it = p.items[it_begin];  // from the plan itself, not the cache
     const int npages = (it.tok_end - it.tok_begin + kPB - 1) / kPB;
     if (it.table_off >= 0 && lane < 2 * kPagesPerTile && lane < npages) {

@@ -136,8 +136,10 @@ __device__ __forceinline__ void suffix_warp(const SfxParams& p, const CUtensorMa
   // planned: only plans with host-resolved table offsets take part, so every
   // read here is of the plan or of table entries at positions the plan was made
   // for.  A prefetch moves nothing into this CTA: a table or length the previous
-  // kernel still rewrites can at worst warm the wrong pages.
-  if (n_cached > 0 && cache[0].table_off >= 0) {
+  // kernel still rewrites can at worst warm the wrong pages.  Not with the
+  // prefix kernel behind this grid: there the requests would compete with the
+  // previous call's last prefix CTAs, which are on the critical path.
+  if (!p.late_trigger && n_cached > 0 && cache[0].table_off >= 0) {
     const TcItem it0 = cache[0];
     const int np0 = (it0.tok_end - it0.tok_begin + kPage - 1) / kPage;
     if (lane < kSlots && lane < np0) {
