@@ -62,6 +62,8 @@ def parse_args():
                          "page and head, the faster layout on the default workload) or "
                          "token-major rows; latent (MLA) pools are always rows")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-secondary", action="store_true",
+                    help="skip the other configurations' summary lines (`secondary`)")
     ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
     return ap.parse_args()
 
@@ -549,11 +551,44 @@ def run_ours():
                 ARGS.workload, ARGS.cpu_sample_seconds / 2, nbytes["total"])
         except Exception as exc:  # reported, never silently dropped
             line["cpu_baseline"] = {"error": repr(exc)[:200]}
+    if rank == 0 and world == 1 and not ARGS.no_secondary:
+        line["secondary"] = secondary_workloads(K, W)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+# the other configurations of the benchmark: c2 (8k prefix, 8 forks), c3 (32k
+# prefix, 16 forks) and c5 (latent KV)
+SECONDARY = ("fork_p8k_f8", "long_p32k_f16", "mla_p16k_f8")
+
+
+def secondary_workloads(K, W):
+    """The other configurations, each measured by this script in a child process
+    of its own (`--workload NAME`, same steps and warm-up, no CPU baseline) after
+    the main measurement, and summarised here: their rates, per-kernel times,
+    rooflines and end-to-end rates, so that one default run records every
+    configuration.  A child that fails is reported with its error."""
+    out = {}
+    for name in SECONDARY:
+        if name == ARGS.workload:
+            continue
+        cmd = [sys.executable, os.path.abspath(__file__), "--workload", name, "--no-cpu-baseline",
+               "--no-secondary", "--steps", str(K), "--warmup", str(W)]
+        try:
+            r = subprocess.run(cmd, capture_output=True, text=True, timeout=600, cwd=ROOT)
+            if r.returncode != 0:
+                raise RuntimeError(f"exit {r.returncode}: {r.stderr.strip()[-160:]}")
+            d = json.loads(r.stdout.strip().splitlines()[-1])
+            out[name] = {k: d.get(k) for k in ("value", "unit", "ms_per_step", "kernels",
+                                                "roofline", "tensor_pipe_pct", "clocks")}
+            out[name]["e2e"] = (d.get("e2e") or {}).get("value")
+            out[name]["config"] = d.get("config")
+        except Exception as exc:  # reported, never silently dropped
+            out[name] = {"error": repr(exc)[:240]}
+    return out
 
 
 def measure_suffix_stage(w, reps, kv_layout, stream, dev, per_graph, nbytes):

@@ -45,3 +45,36 @@ def test_oracle_children_and_cpu_model(monkeypatch):
     line = bench.cpu_baseline_all_cores("tiny_p512_f4", 0.2, 1 << 20)
     assert line["cores"] == min(16, os.cpu_count() or 1) and line["value"] > 0
     assert bench.cpu_baseline_all_cores("tiny_p512_f4", 0.2, 2 << 30) is None
+
+
+def test_secondary_summaries_from_child_lines(monkeypatch):
+    """The default line's `secondary` block: one child run per other configuration,
+    summarised from the child's own JSON line; a child that fails is reported with
+    its error instead of being dropped."""
+    monkeypatch.setattr(sys, "argv", ["bench.py"])
+    import bench
+    calls = []
+
+    class Done:
+        def __init__(self, rc, out, err=""):
+            self.returncode, self.stdout, self.stderr = rc, out, err
+
+    def fake_run(cmd, **kw):
+        calls.append(cmd)
+        name = cmd[cmd.index("--workload") + 1]
+        if name == "mla_p16k_f8":
+            return Done(1, "", "RuntimeError: boom")
+        line = {"value": 1.5, "unit": "tokens/s", "ms_per_step": 0.01, "kernels": {},
+                "roofline": {"frac": 0.5}, "tensor_pipe_pct": None, "clocks": {},
+                "e2e": {"value": 1.0}, "config": {"workload": name}}
+        return Done(0, "noise\n" + json.dumps(line) + "\n")
+
+    monkeypatch.setattr(bench.subprocess, "run", fake_run)
+    out = bench.secondary_workloads(7, 3)
+    assert set(out) == set(bench.SECONDARY) - {bench.ARGS.workload}
+    assert out["fork_p8k_f8"]["value"] == 1.5 and out["fork_p8k_f8"]["e2e"] == 1.0
+    assert out["fork_p8k_f8"]["config"]["workload"] == "fork_p8k_f8"
+    assert "boom" in out["mla_p16k_f8"]["error"]
+    for cmd in calls:  # same steps and warm-up, no CPU baseline, no recursion
+        assert cmd[cmd.index("--steps") + 1] == "7" and cmd[cmd.index("--warmup") + 1] == "3"
+        assert "--no-cpu-baseline" in cmd and "--no-secondary" in cmd
